@@ -1,0 +1,8 @@
+"""fp64 CPU oracle for the Qwen3-architecture decoder forward pass.
+
+TEST INFRASTRUCTURE ONLY.  Only ``tests/``, ``__graft_entry__.smoke()`` and
+``bench.py``'s CPU-baseline / reference arm may import this package.  The
+product path (``paper_2609_12471_gb300``) never imports it and shares no code
+with it; the two meet only in the seeded inputs of ``synth``.
+"""
+from .qwen3 import *  # noqa: F401,F403

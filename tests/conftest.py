@@ -1,0 +1,26 @@
+"""Shared pytest configuration: the `gpu` marker and small fixtures."""
+import os
+import sys
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+
+def pytest_configure(config):
+    config.addinivalue_line("markers", "gpu: needs a CUDA GPU (GB300, sm_103a)")
+    config.addinivalue_line("markers", "slow: long-running (full-size model) case")
+
+
+@pytest.fixture(scope="session")
+def tiny_shape():
+    import synth
+    return synth.shape("tiny_fp32")
+
+
+@pytest.fixture(scope="session")
+def tiny_weights(tiny_shape):
+    import synth
+    return synth.LazyWeights(tiny_shape)

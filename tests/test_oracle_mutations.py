@@ -1,0 +1,45 @@
+"""Plant plausible mistakes in a temporary copy of the oracle and check that the pins fail.
+
+Each mutation is applied to a copy of ``oracle/`` in a temporary directory;
+the real oracle is never modified.  The pins in ``test_oracle_pins.py`` are
+run against the mutated copy in a subprocess and must fail.
+"""
+import os
+import shutil
+import subprocess
+import sys
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+MUTATIONS = {
+    "rope_sign": ("a * c - b * s, b * c + a * s", "a * c + b * s, b * c - a * s"),
+    "rope_inverse_frequency": ("theta ** (-2.0 * i / head_dim)", "theta ** (-1.0 * i / head_dim)"),
+    "dropped_attention_residual": ('x = x + o @ Lw["wo"].T', 'x = o @ Lw["wo"].T'),
+    "transposed_wo": ('x = x + o @ Lw["wo"].T', 'x = x + o @ Lw["wo"]'),
+    "gqa_head_index": ("g = h // group", "g = h % n_kv"),
+    "eps_outside_sqrt": ("x / np.sqrt(ms + eps) * g", "x / (np.sqrt(ms) + eps) * g"),
+    "dropped_q_norm": ('q = rms_norm(q, Lw["q_norm"], eps)', "q = q"),
+    "attention_scale": ("/ np.sqrt(d)", "/ d"),
+    "causal_mask_off_by_one": ("k_pos[None, :] <= q_pos[:, None]", "k_pos[None, :] < q_pos[:, None] + 2"),
+    "gate_up_swapped": ('silu(u @ Lw["wg"].T) * (u @ Lw["wu"].T)', 'silu(u @ Lw["wu"].T) * (u @ Lw["wg"].T)'),
+    "dropped_final_norm": ('return rms_norm(x, widen(W["final_norm"]), cfg.rms_eps)', "return x"),
+    "log_softmax_sign": ("z - (m + np.log", "z + (m + np.log"),
+}
+
+
+@pytest.mark.parametrize("name", sorted(MUTATIONS))
+def test_pins_catch_planted_mistake(name, tmp_path):
+    before, after = MUTATIONS[name]
+    shutil.copytree(os.path.join(ROOT, "oracle"), tmp_path / "oracle",
+                    ignore=shutil.ignore_patterns("__pycache__"))
+    p = tmp_path / "oracle" / "qwen3.py"
+    src = p.read_text()
+    assert src.count(before) == 1, f"mutation anchor for {name} not found"
+    p.write_text(src.replace(before, after))
+    env = dict(os.environ, PYTHONPATH=os.pathsep.join([str(tmp_path), ROOT]))
+    r = subprocess.run([sys.executable, "-m", "pytest", "-q", "-x", "-p", "no:cacheprovider",
+                        os.path.join(ROOT, "tests", "test_oracle_pins.py")],
+                       cwd=str(tmp_path), env=env, capture_output=True, text=True, timeout=600)
+    assert r.returncode != 0, f"pins did not catch {name}:\n{r.stdout[-2000:]}"
