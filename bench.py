@@ -1,0 +1,337 @@
+#!/usr/bin/env python3
+"""Benchmark of the rollout hot path on GB300: a Qwen3-8B-shaped bf16 decoder
+(random init) decoding a teacher-forced batch of 16 rollouts, prompt 512 tokens
+then 1024 decode steps with per-token log-probs.
+
+One step = one whole rollout (prefill of 16 x 512 tokens + 1024 decode steps of
+16 tokens each).  `value` = decoded tokens per second over all ranks (replicas:
+every rank runs its own rollout batch; no collective on the data path).
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--impl reference]
+
+`--impl reference` times the fp64 CPU oracle on a bounded sample of the same
+workload (the only comparison program this method has).
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "decode tokens/s and prefill/score tokens/s on 1 GB300; % HBM / bf16 roofline"
+UNIT = "tokens/s"
+B, P, N = 16, 512, 1024
+WORKLOAD = ("qwen3-8b-shaped bf16 rollout decode: batch 16, prompt 512 random tokens, "
+            "1024 teacher-forced decode steps, per-token log-probs")
+ORACLE_TOKENS = 32  # tokens of rollout row 0 the CPU oracle scores per sample
+
+
+def parse():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=3)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    return ap.parse_args()
+
+
+def dist_setup():
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if world > 1:
+        import torch
+        import torch.distributed as dist
+        torch.cuda.set_device(local)
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+    return world, rank, local
+
+
+def barrier(world):
+    if world > 1:
+        import torch.distributed as dist
+        dist.barrier()
+
+
+def max_over_ranks(v: float, world: int) -> float:
+    if world == 1:
+        return v
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([v], dtype=torch.float64, device="cuda")
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+class ClockSampler:
+    """nvidia-smi clocks / throttle reasons sampled every 200 ms while running."""
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, device_index: int):
+        self.path = tempfile.mktemp(suffix=".csv")
+        self.proc = None
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits",
+                 "-lms", "200", "-i", str(device_index)],
+                stdout=open(self.path, "w"), stderr=subprocess.DEVNULL)
+        except (OSError, FileNotFoundError):
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        rows = []
+        for line in open(self.path):
+            f = [x.strip() for x in line.split(",")]
+            if len(f) >= 9:
+                rows.append(f)
+        os.unlink(self.path)
+        if not rows:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["no samples"]}
+
+        def num(x):
+            try:
+                return float(x)
+            except ValueError:
+                return None
+        sm = [num(r[1]) for r in rows if num(r[1]) is not None]
+        mx = [num(r[2]) for r in rows if num(r[2]) is not None]
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({names[i] for r in rows for i in range(4) if r[5 + i].lower() == "active"})
+        load = [v for v in sm if mx and v > 0.5 * max(mx)] or sm
+        return {"sm_mhz": statistics.median(load) if load else None,
+                "sm_max_mhz": max(mx) if mx else None, "reasons": reasons,
+                "samples": len(rows),
+                "power_w_max": max((num(r[3]) or 0.0) for r in rows)}
+
+
+def measured_peaks():
+    try:
+        return json.load(open(os.path.join(ROOT, "MEASURED_PEAKS.json")))
+    except (OSError, ValueError):
+        return None
+
+
+def source_sha(paths):
+    h = hashlib.sha256()
+    for p in paths:
+        h.update(open(os.path.join(ROOT, p), "rb").read())
+    return h.hexdigest()[:16]
+
+
+def recorded_traffic(key: str):
+    """DRAM bytes per launch from a committed ncu summary, if the kernel source is unchanged."""
+    try:
+        t = json.load(open(os.path.join(ROOT, "profiles", "traffic.json")))[key]
+    except (OSError, ValueError, KeyError):
+        return None
+    if source_sha(t["sources"]) != t["source_sha"]:
+        return None
+    return t["dram_bytes_per_launch"]
+
+
+# --------------------------------------------------------------------------- CPU oracle sample
+def oracle_sample(s, W, seq_row):
+    """fp64 oracle: full causal forward + log-probs over the first ORACLE_TOKENS tokens."""
+    import oracle
+    t0 = time.perf_counter()
+    lp, _, _ = oracle.score_sequence(s, W, seq_row[:ORACLE_TOKENS + 1])
+    dt = time.perf_counter() - t0
+    return ORACLE_TOKENS / dt, dt, lp
+
+
+def cpu_cores():
+    n = len(os.sched_getaffinity(0)) if hasattr(os, "sched_getaffinity") else os.cpu_count()
+    return int(os.environ.get("OPENBLAS_NUM_THREADS", n))
+
+
+def cpu_baseline_entry(value, dt):
+    return {"value": value, "unit": UNIT, "cores": cpu_cores(), "kind": "oracle",
+            "sample": (f"fp64 oracle: causal forward and per-token log-probs of the first "
+                       f"{ORACLE_TOKENS} tokens of rollout row 0 (all 36 layers + lm_head; "
+                       f"weights widened from bf16 layer by layer), {dt:.1f} s")}
+
+
+# --------------------------------------------------------------------------- arms
+def run_reference(args, world, rank):
+    if rank != 0:
+        return
+    import synth
+    s = synth.shape("q8b")
+    W = synth.LazyWeights(s, cache=True)
+    seq = synth.tokens((B, P + N + 1), s.vocab)
+    times = []
+    for i in range(args.warmup + args.steps):
+        _, dt, _ = oracle_sample(s, W, seq[0])
+        if i >= args.warmup:
+            times.append(dt)
+    dt = statistics.mean(times)
+    value = ORACLE_TOKENS / dt
+    line = {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": 0,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": dt * 1e3,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+            "data": "synthetic", "config": {"workload": WORKLOAD, "sample_tokens": ORACLE_TOKENS},
+            "cpu_baseline": cpu_baseline_entry(value, dt),
+            "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+
+
+def run_ours(args, world, rank, local):
+    import numpy as np
+    import torch
+
+    import synth
+    from paper_2609_12471_gb300 import build as qkbuild
+    qkbuild.build()
+    import paper_2609_12471_gb300 as qk
+    from paper_2609_12471_gb300 import _binding
+    from paper_2609_12471_gb300.runtime import Decoder
+
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    s = synth.shape("q8b")
+    want_cpu = rank == 0 and world == 1 and not args.no_cpu_baseline
+    W = synth.LazyWeights(s, cache=want_cpu)
+    names = [t[0] for t in synth.tensor_list(s)]
+    dec = Decoder(qk.qk_config_preset("q8b"), (W[n] for n in names), device=dev)
+    seq = synth.tokens((B, P + N + 1), s.vocab, stream=rank)
+    seq_d = torch.tensor(seq, dtype=torch.int32, device=dev)
+    kv = dec.new_kv(B, P + N)
+    lp = torch.empty(B, N + 1, dtype=torch.float32, device=dev)
+    stream = torch.cuda.current_stream(dev)
+
+    def step():
+        dec.rollout(kv, B, P + N, seq_d, P, logprobs=lp)
+
+    for _ in range(args.warmup):
+        step()
+    torch.cuda.synchronize(dev)
+    if dec.check_status() != 0:
+        raise RuntimeError("device status flags set during warm-up")
+
+    # ---- timed region: K whole rollouts, device-resident inputs
+    n_layers = s.n_layers
+    _binding._load().qk_profile_begin.argtypes = [_binding._P, _binding._I, _binding._I]
+    lib = _binding._load()
+    lib.qk_profile_end.argtypes = [_binding._P, _binding.ctypes.POINTER(_binding.ctypes.c_float),
+                                   _binding.ctypes.POINTER(_binding._I)]
+    lib.qk_launch_count.restype = _binding.ctypes.c_uint64
+    if lib.qk_profile_begin(dec.handle, 2, args.steps * N * n_layers) != 0:  # QK_PROF_GATE_UP
+        raise RuntimeError(qk.qk_last_error())
+    clocks = ClockSampler(local)
+    barrier(world)
+    torch.cuda.synchronize(dev)
+    launches0 = lib.qk_launch_count()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(args.steps):
+        step()
+    e1.record(stream)
+    torch.cuda.synchronize(dev)
+    launches = lib.qk_launch_count() - launches0
+    barrier(world)
+    clk = clocks.stop()
+    ms = e1.elapsed_time(e0) * -1 if False else e0.elapsed_time(e1)
+    ms_step = max_over_ranks(ms / args.steps, world)
+    prof_ms = _binding.ctypes.c_float()
+    prof_n = _binding._I()
+    if lib.qk_profile_end(dec.handle, _binding.ctypes.byref(prof_ms), _binding.ctypes.byref(prof_n)) != 0:
+        raise RuntimeError(qk.qk_last_error())
+    if dec.check_status() != 0:
+        raise RuntimeError("device status flags set during the timed region")
+    value = world * B * N / (ms_step / 1e3)
+
+    # ---- prefill alone (for the prefill tokens/s figure)
+    pz = torch.empty(B, dtype=torch.float32, device=dev)
+    torch.cuda.synchronize(dev)
+    p0, p1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    p0.record(stream)
+    for _ in range(args.steps):
+        dec.prefill(kv, B, P + N, seq_d[:, :P].contiguous(), 0, None, seq_d[:, P].contiguous(), pz)
+    p1.record(stream)
+    torch.cuda.synchronize(dev)
+    prefill_ms = p0.elapsed_time(p1) / args.steps
+
+    # ---- end to end through the public API with host buffers
+    seq_h = torch.from_numpy(seq).pin_memory()
+    lp_h = torch.empty(B, N + 1, dtype=torch.float32).pin_memory()
+    seq_dev = torch.empty_like(seq_d)
+    torch.cuda.synchronize(dev)
+    barrier(world)
+    t0 = time.perf_counter()
+    for _ in range(args.steps):
+        seq_dev.copy_(seq_h, non_blocking=True)
+        dec.rollout(kv, B, P + N, seq_dev, P, logprobs=lp)
+        lp_h.copy_(lp, non_blocking=True)
+        torch.cuda.synchronize(dev)
+    e2e_s = max_over_ranks((time.perf_counter() - t0) / args.steps, world)
+    e2e_value = world * B * N / e2e_s
+    lp_np = lp_h.numpy()
+    if not (np.all(np.isfinite(lp_np)) and np.all(lp_np <= 1e-4)):
+        raise RuntimeError("log-probs out of range")
+
+    if rank != 0:
+        return
+    peaks = measured_peaks()
+    hbm_peak = peaks["hbm_gbs"] if peaks else 6800.0
+    c = dec.cfg
+    gu_bytes = 2 * c.intermediate * c.hidden * 2 + B * c.hidden * 2 + B * c.intermediate * 2
+    avg_launch_s = (prof_ms.value / max(prof_n.value, 1)) / 1e3
+    achieved = gu_bytes / avg_launch_s / 1e9
+    roofline = {"bound": "hbm", "kernel": "decode gate/up linear + SwiGLU (M=16)",
+                "achieved": achieved, "peak": hbm_peak, "unit": "GB/s",
+                "frac": achieved / hbm_peak,
+                "peak_source": "measured" if peaks else "fallback",
+                "algorithmic_bytes_per_launch": gu_bytes, "launches_timed": prof_n.value,
+                "avg_launch_us": avg_launch_s * 1e6,
+                "traffic": recorded_traffic("gate_up_decode_b16")}
+    step_bytes = 15136811008 + B * sum(P + j + 1 for j in range(N)) * 147456 / N
+    line = {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": ms_step, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+            "config": {"workload": WORKLOAD, "batch": B, "prompt_tokens": P, "decode_steps": N,
+                       "l2": "inputs larger than L2: 15.1 GB of weights streamed per decode step",
+                       "replicas": world},
+            "prefill_tokens_per_s": world * B * P / (prefill_ms / 1e3),
+            "decode_hbm_fraction_of_8tbs": (step_bytes * N / 1e9) / ((ms_step - prefill_ms) / 1e3) / 8000.0,
+            "roofline": roofline, "clocks": clk, "gpu_launches": int(launches),
+            "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": int(seq.nbytes),
+                    "d2h_bytes_per_step": int(lp_h.numel() * 4)}}
+    if want_cpu:
+        v, dt, _ = oracle_sample(s, W, seq[0])
+        line["cpu_baseline"] = cpu_baseline_entry(v, dt)
+    print(json.dumps(line), flush=True)
+
+
+def main():
+    args = parse()
+    world, rank, local = dist_setup()
+    if args.impl == "reference":
+        run_reference(args, world, rank)
+    else:
+        run_ours(args, world, rank, local)
+    if world > 1:
+        import torch.distributed as dist
+        dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,199 @@
+/*
+ * qk.h -- C ABI of libqk: the forward pass of a Qwen3-architecture decoder on
+ * one GB300 (sm_103a), for rollout decode and teacher-forced log-prob scoring.
+ *
+ * What it computes.  The policy forward pass whose per-token log-probability
+ * log pi_theta(y_t | x, y_<t) enters the SFT objective (Eq. sft, Sec. "Task
+ * Serialization and SFT Objective") and the PPO-clipped GRPO objective (Eq. ppo,
+ * Sec. "GRPO Optimization": the ratio rho_t and the KL term), and whose
+ * autoregressive decode produces the rollouts of the RL loop (Sec.
+ * "Implementation Components").  The paper cites the Qwen3 architecture without
+ * restating it; the layer definition used here is:
+ *     x = E[token];  per layer: u = RMSNorm(x)*g1; q,k,v = W_q u, W_k u, W_v u;
+ *     per head RMSNorm of q and k (gains of length head_dim) then rotate-half
+ *     RoPE (theta from the config); causal GQA attention (kv head = q head /
+ *     (n_q/n_kv), scale 1/sqrt(head_dim)); x += W_o o; u = RMSNorm(x)*g2;
+ *     x += W_down(silu(W_gate u) * W_up u);
+ *     logits = W_lm (RMSNorm(x)*g_final); log p = logit - logsumexp(logits).
+ * RMSNorm is x / sqrt(mean(x^2) + eps).
+ *
+ * Conventions (every entry point):
+ *  - Memory.  The library never allocates device memory.  Every device buffer
+ *    (packed weights, KV cache, workspace, inputs, outputs) is allocated by the
+ *    caller and borrowed for the duration of the call (the packed-weight buffer
+ *    for the model's lifetime).  Pointers documented "dev" are device pointers.
+ *  - Streams.  `stream` is a cudaStream_t passed as void*; NULL means the
+ *    legacy default stream.  Every compute call is asynchronous on that stream
+ *    and performs no host synchronisation; it can be captured in a CUDA graph.
+ *  - Errors.  Every int-returning call returns QK_OK (0) or a negative QK_E*
+ *    code and leaves a message for qk_last_error() (thread-local).  Arguments
+ *    are validated on the host before any launch; a call that returns an error
+ *    has launched nothing.  Data-dependent faults found on the device (a token
+ *    id outside [0, vocab), a position outside the cache, a bounded wait that
+ *    expired) set bits of the model's device status word instead; the kernels
+ *    then substitute a safe value (token 0, position clamped) rather than read
+ *    out of bounds.  qk_check_status() reads and clears that word.
+ *  - dtype.  QK_DTYPE_BF16 models keep weights, activations and KV cache in
+ *    bf16 with fp32 accumulation, an fp32 residual stream and fp32 softmax /
+ *    log-softmax statistics.  QK_DTYPE_F32 models are fp32 end to end (no TF32).
+ */
+#ifndef QK_H
+#define QK_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#define QK_OK 0
+#define QK_EINVAL (-1)   /* null pointer, bad enum, unknown preset            */
+#define QK_ESHAPE (-2)   /* size out of range: B > max_batch, T too long, ... */
+#define QK_EDTYPE (-3)   /* unsupported dtype / head_dim / grouping           */
+#define QK_ECUDA (-4)    /* a CUDA runtime / driver call failed               */
+#define QK_ETIMEOUT (-5) /* a device-side bounded wait expired                */
+#define QK_EDEVICE (-6)  /* device status word had a fault bit set            */
+#define QK_ENOSPACE (-7) /* caller buffer smaller than the size query returns */
+
+#define QK_DTYPE_BF16 0
+#define QK_DTYPE_F32 1
+
+/* Bits of the device status word (qk_check_status). */
+#define QK_STATUS_BAD_TOKEN 1u    /* token id outside [0, vocab); id 0 was used   */
+#define QK_STATUS_BAD_POS 2u      /* position outside [0, max_seq); it was clamped */
+#define QK_STATUS_TIMEOUT 4u      /* a bounded device wait gave up                 */
+
+/* Kinds of call for qk_workspace_bytes. */
+#define QK_CALL_DECODE 0   /* qk_decode_step / qk_decode_layer: B tokens          */
+#define QK_CALL_PREFILL 1  /* qk_prefill: B x T tokens                             */
+#define QK_CALL_SCORE 2    /* qk_score_logprobs: B x T tokens, no KV cache         */
+#define QK_CALL_ROLLOUT 3  /* qk_rollout_teacher_forced: prefill B x T then decode */
+
+typedef struct qk_config {
+    int32_t n_layers;      /* decoder layers                                  */
+    int32_t hidden;        /* H, multiple of 64                               */
+    int32_t n_q_heads;     /* query heads                                     */
+    int32_t n_kv_heads;    /* key/value heads; n_q_heads % n_kv_heads == 0    */
+    int32_t head_dim;      /* d: 64 or 128                                    */
+    int32_t intermediate;  /* SwiGLU width I, multiple of 128                 */
+    int32_t vocab;         /* V                                               */
+    int32_t dtype;         /* QK_DTYPE_BF16 or QK_DTYPE_F32                   */
+    int32_t max_positions; /* length of the RoPE table (largest position + 1) */
+    int32_t reserved;      /* must be 0                                       */
+    double rms_eps;        /* RMSNorm epsilon (inside the square root)        */
+    double rope_theta;     /* RoPE base                                       */
+} qk_config;
+
+typedef struct qk_model qk_model;
+
+/* Fill *out with a named preset: "tiny_fp32" (2 layers, H 256, 4/2 heads, d 64,
+ * I 768, V 4096, fp32), "q8b" (36 layers, H 4096, 32/8 heads, d 128, I 12288,
+ * V 151936, bf16), "q8b_layer" (one q8b layer).  eps 1e-6, theta 1e6,
+ * max_positions 8192.  Returns QK_EINVAL for an unknown name. */
+int qk_config_preset(const char* name, qk_config* out);
+
+/* Number of weight tensors of a config, in the canonical order used by
+ * qk_model_load: embed [V,H]; then per layer attn_norm [H], wq [nq*d,H],
+ * wk [nkv*d,H], wv [nkv*d,H], q_norm [d], k_norm [d], wo [H,nq*d],
+ * mlp_norm [H], wg [I,H], wu [I,H], wd [H,I]; then final_norm [H],
+ * lm_head [V,H].  Matrices are row-major [out, in]. */
+int qk_weight_count(const qk_config* cfg, int* n_tensors);
+
+/* Bytes of the packed device buffer qk_model_load needs for this config. */
+int qk_model_packed_bytes(const qk_config* cfg, size_t* bytes);
+
+/* Build a model.  `tensors` is a host array of n_tensors device pointers in the
+ * canonical order above, each holding the tensor in the config's dtype.  They
+ * are read (repacked into `packed`, which must hold qk_model_packed_bytes bytes
+ * and be 256-byte aligned) on `stream` and may be freed once the stream has
+ * passed this call.  `packed` is borrowed for the model's lifetime.  *out
+ * receives a host object owned by the library; release it with qk_model_free. */
+int qk_model_load(const qk_config* cfg, const void* const* tensors, int n_tensors, void* packed,
+                  size_t packed_bytes, void* stream, qk_model** out);
+void qk_model_free(qk_model* m);
+
+/* KV cache bytes for max_batch rows of max_seq positions: per layer K then V,
+ * each [max_batch, n_kv, max_seq, d] in the model dtype, contiguous. */
+int qk_kv_bytes(const qk_model* m, int max_batch, int max_seq, size_t* bytes);
+
+/* Workspace bytes for one call of the given kind (QK_CALL_*) with batch B and
+ * T tokens per row (T = 1 for decode; T = prompt length for a rollout) against
+ * a cache of max_seq positions. */
+int qk_workspace_bytes(const qk_model* m, int kind, int B, int T, int max_seq, size_t* bytes);
+
+/* Prefill T tokens per row at positions start_pos .. start_pos+T-1 (causal
+ * attention over cache positions 0 .. p), writing their K and V into the cache.
+ * tokens: dev int32 [B, T].  The cache rows b < B must already hold positions
+ * < start_pos.  Outputs for the last position of each row (any may be NULL):
+ * last_logits dev fp32 [B, V]; logprobs dev fp32 [B] = log p(targets[b]) with
+ * targets dev int32 [B] (required when logprobs is given); argmax dev int32 [B]
+ * (lowest index among equal maxima).  QK_ESHAPE if B > max_batch or
+ * start_pos + T > max_seq. */
+int qk_prefill(qk_model* m, void* kv, int max_batch, int max_seq, const int32_t* tokens, int B,
+               int T, int start_pos, float* last_logits, const int32_t* targets, float* logprobs,
+               int32_t* argmax, void* workspace, size_t ws_bytes, void* stream);
+
+/* One decode step: row b consumes tokens[b] at position pos[b] (dev int32 [B]
+ * each), writes its K and V at pos[b] and attends positions 0 .. pos[b].
+ * Outputs as in qk_prefill, for the B new positions. */
+int qk_decode_step(qk_model* m, void* kv, int max_batch, int max_seq, const int32_t* tokens,
+                   const int32_t* pos, int B, float* logits, const int32_t* targets,
+                   float* logprobs, int32_t* argmax, void* workspace, size_t ws_bytes,
+                   void* stream);
+
+/* One decoder layer of a decode step on a given residual stream: x dev fp32
+ * [B, H] is updated in place; the new K and V go to the layer's cache at
+ * pos[b] (dev int32 [B]) and attention covers 0 .. pos[b]. */
+int qk_decode_layer(qk_model* m, int layer, void* kv, int max_batch, int max_seq, float* x,
+                    const int32_t* pos, int B, void* workspace, size_t ws_bytes, void* stream);
+
+/* Teacher-forced scoring (Eq. sft / Eq. ppo inputs): tokens dev int32 [B, T],
+ * T >= 2.  logprobs dev fp32 [B, T-1]: logprobs[b, t] = log p(tokens[b, t+1] |
+ * tokens[b, <= t]).  argmax dev int32 [B, T-1] or NULL.  Positions start at 0;
+ * no KV cache is kept. */
+int qk_score_logprobs(qk_model* m, const int32_t* tokens, int B, int T, float* logprobs,
+                      int32_t* argmax, void* workspace, size_t ws_bytes, void* stream);
+
+/* Teacher-forced rollout: seq dev int32 [B, P+N+1] = prompt (P tokens) ++
+ * c[0..N].  Prefill over the prompt scores c[0]; decode step j (0 <= j < N)
+ * consumes c[j] at position P+j and scores c[j+1].  logprobs dev fp32 [B, N+1],
+ * argmax dev int32 [B, N+1] or NULL.  The cache ends holding P+N positions;
+ * P + N <= max_seq. */
+int qk_rollout_teacher_forced(qk_model* m, void* kv, int max_batch, int max_seq,
+                              const int32_t* seq, int B, int P, int N, float* logprobs,
+                              int32_t* argmax, void* workspace, size_t ws_bytes, void* stream);
+
+/* Synchronise `stream`, read the device status word into *flags (QK_STATUS_*
+ * bits) and clear it.  Returns QK_EDEVICE if any bit was set, QK_OK otherwise. */
+int qk_check_status(qk_model* m, void* stream, uint32_t* flags);
+
+/* ---- measurement ----------------------------------------------------------
+ * Kernel classes that qk_profile_begin can bracket with CUDA events.  Only the
+ * launches made by decode steps (qk_decode_step, the decode phase of
+ * qk_rollout_teacher_forced, qk_decode_layer) are bracketed. */
+#define QK_PROF_QKV 0      /* RMSNorm'd input x W_qkv                     */
+#define QK_PROF_O 1        /* attention output x W_o + residual           */
+#define QK_PROF_GATE_UP 2  /* x W_gate, x W_up, SwiGLU                    */
+#define QK_PROF_DOWN 3     /* h x W_down + residual                       */
+#define QK_PROF_ATTN 4     /* decode attention (all its kernels)          */
+#define QK_PROF_LM_HEAD 5  /* final RMSNorm'd x W_lm (logits)             */
+
+/* Start bracketing up to max_launches launches of kernel class `kind` with
+ * CUDA events recorded on the launching stream.  Creates 2*max_launches
+ * events (host objects; no device allocation).  Replaces any active session. */
+int qk_profile_begin(qk_model* m, int kind, int max_launches);
+/* End the session: synchronise on its last event and return the summed
+ * event-to-event time (ms) and the number of bracketed launches. */
+int qk_profile_end(qk_model* m, float* total_ms, int* launches);
+
+/* Number of kernels libqk has launched in this process (all models). */
+uint64_t qk_launch_count(void);
+
+/* Message of the last failed call on this thread ("" if none). */
+const char* qk_last_error(void);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* QK_H */

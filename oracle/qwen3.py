@@ -305,17 +305,27 @@ def layer_decode_step(cfg, Lw: dict, x: np.ndarray, k_cache: np.ndarray, v_cache
     values already normed and rotated at positions 0..pos[b]-1.  The new token
     sits at pos[b], its key and value are appended and attended.  Returns
     (x_out [B, H], k_new [B, n_kv, d], v_new [B, n_kv, d]).
+
+    Same steps as decoder_layer; the B rows share the linear layers (each row is
+    an independent matrix-vector product) and differ only in their caches.
     """
     B = x.shape[0]
-    out = np.empty_like(x, dtype=np.float64)
-    kn_all = np.empty((B, cfg.n_kv_heads, cfg.head_dim))
-    vn_all = np.empty_like(kn_all)
+    nq, nkv, d, eps = cfg.n_q_heads, cfg.n_kv_heads, cfg.head_dim, cfg.rms_eps
+    pos = np.asarray(pos)
+    x = widen(x)
+    u = rms_norm(x, Lw["attn_norm"], eps)
+    q = rms_norm((u @ Lw["wq"].T).reshape(B, nq, d), Lw["q_norm"], eps)
+    k = rms_norm((u @ Lw["wk"].T).reshape(B, nkv, d), Lw["k_norm"], eps)
+    v = (u @ Lw["wv"].T).reshape(B, nkv, d)
+    q = apply_rope(q, pos, cfg.rope_theta)
+    k = apply_rope(k, pos, cfg.rope_theta)
+    o = np.empty((B, nq, d))
     for b in range(B):
         p = int(pos[b])
-        kp = widen(k_cache[b, :, :p, :]).transpose(1, 0, 2)
-        vp = widen(v_cache[b, :, :p, :]).transpose(1, 0, 2)
-        xo, kn, vn = decoder_layer(cfg, Lw, widen(x[b:b + 1]), [p], kp, vp, np.arange(p))
-        out[b] = xo[0]
-        kn_all[b] = kn[0]
-        vn_all[b] = vn[0]
-    return out, kn_all, vn_all
+        K = np.concatenate([widen(k_cache[b, :, :p, :]).transpose(1, 0, 2), k[b:b + 1]])
+        V = np.concatenate([widen(v_cache[b, :, :p, :]).transpose(1, 0, 2), v[b:b + 1]])
+        o[b] = attention(q[b:b + 1], K, V, [p], np.arange(p + 1))[0]
+    x = x + o.reshape(B, nq * d) @ Lw["wo"].T
+    u = rms_norm(x, Lw["mlp_norm"], eps)
+    x = x + (silu(u @ Lw["wg"].T) * (u @ Lw["wu"].T)) @ Lw["wd"].T
+    return x, k, v

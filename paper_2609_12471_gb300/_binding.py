@@ -1,0 +1,215 @@
+"""ctypes binding of libqk (include/qk.h): the same entry points, argument marshalling only.
+
+Device buffers may be passed as torch CUDA tensors (their data_ptr() is used)
+or as raw integer addresses; ``None`` passes NULL.  ``stream`` defaults to
+torch's current CUDA stream.  A non-zero status raises QKError carrying
+qk_last_error().
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+
+PKG = os.path.dirname(os.path.abspath(__file__))
+_LIB_FILE = os.path.join(PKG, "libqk.so")
+
+QK_OK, QK_EINVAL, QK_ESHAPE, QK_EDTYPE, QK_ECUDA, QK_ETIMEOUT, QK_EDEVICE, QK_ENOSPACE = (
+    0, -1, -2, -3, -4, -5, -6, -7)
+QK_DTYPE_BF16, QK_DTYPE_F32 = 0, 1
+QK_STATUS_BAD_TOKEN, QK_STATUS_BAD_POS, QK_STATUS_TIMEOUT = 1, 2, 4
+QK_CALL_DECODE, QK_CALL_PREFILL, QK_CALL_SCORE, QK_CALL_ROLLOUT = 0, 1, 2, 3
+
+__all__ = [
+    "QK_OK", "QK_EINVAL", "QK_ESHAPE", "QK_EDTYPE", "QK_ECUDA", "QK_ETIMEOUT", "QK_EDEVICE",
+    "QK_ENOSPACE", "QK_DTYPE_BF16", "QK_DTYPE_F32", "QK_STATUS_BAD_TOKEN", "QK_STATUS_BAD_POS",
+    "QK_STATUS_TIMEOUT", "QK_CALL_DECODE", "QK_CALL_PREFILL", "QK_CALL_SCORE", "QK_CALL_ROLLOUT",
+    "qk_config", "qk_config_preset", "qk_weight_count", "qk_model_packed_bytes", "qk_model_load",
+    "qk_model_free", "qk_kv_bytes", "qk_workspace_bytes", "qk_prefill", "qk_decode_step",
+    "qk_decode_layer", "qk_score_logprobs", "qk_rollout_teacher_forced", "qk_check_status",
+    "qk_last_error", "QKError", "lib_path", "exported_symbols",
+]
+
+
+class QKError(RuntimeError):
+    def __init__(self, code: int, msg: str):
+        super().__init__(f"libqk error {code}: {msg}")
+        self.code = code
+
+
+class qk_config(ctypes.Structure):
+    _fields_ = [("n_layers", ctypes.c_int32), ("hidden", ctypes.c_int32),
+                ("n_q_heads", ctypes.c_int32), ("n_kv_heads", ctypes.c_int32),
+                ("head_dim", ctypes.c_int32), ("intermediate", ctypes.c_int32),
+                ("vocab", ctypes.c_int32), ("dtype", ctypes.c_int32),
+                ("max_positions", ctypes.c_int32), ("reserved", ctypes.c_int32),
+                ("rms_eps", ctypes.c_double), ("rope_theta", ctypes.c_double)]
+
+    def __repr__(self):
+        return "qk_config(" + ", ".join(f"{n}={getattr(self, n)}" for n, _ in self._fields_) + ")"
+
+
+def lib_path() -> str:
+    return _LIB_FILE
+
+
+_P, _I, _SZ = ctypes.c_void_p, ctypes.c_int, ctypes.c_size_t
+_SIGS = {
+    "qk_config_preset": ([ctypes.c_char_p, ctypes.POINTER(qk_config)], _I),
+    "qk_weight_count": ([ctypes.POINTER(qk_config), ctypes.POINTER(_I)], _I),
+    "qk_model_packed_bytes": ([ctypes.POINTER(qk_config), ctypes.POINTER(_SZ)], _I),
+    "qk_model_load": ([ctypes.POINTER(qk_config), ctypes.POINTER(_P), _I, _P, _SZ, _P,
+                       ctypes.POINTER(_P)], _I),
+    "qk_model_free": ([_P], None),
+    "qk_kv_bytes": ([_P, _I, _I, ctypes.POINTER(_SZ)], _I),
+    "qk_workspace_bytes": ([_P, _I, _I, _I, _I, ctypes.POINTER(_SZ)], _I),
+    "qk_prefill": ([_P, _P, _I, _I, _P, _I, _I, _I, _P, _P, _P, _P, _P, _SZ, _P], _I),
+    "qk_decode_step": ([_P, _P, _I, _I, _P, _P, _I, _P, _P, _P, _P, _P, _SZ, _P], _I),
+    "qk_decode_layer": ([_P, _I, _P, _I, _I, _P, _P, _I, _P, _SZ, _P], _I),
+    "qk_score_logprobs": ([_P, _P, _I, _I, _P, _P, _P, _SZ, _P], _I),
+    "qk_rollout_teacher_forced": ([_P, _P, _I, _I, _P, _I, _I, _I, _P, _P, _P, _SZ, _P], _I),
+    "qk_check_status": ([_P, _P, ctypes.POINTER(ctypes.c_uint32)], _I),
+    "qk_last_error": ([], ctypes.c_char_p),
+}
+
+_lib = None
+
+
+def _load():
+    global _lib
+    if _lib is None:
+        if not os.path.exists(_LIB_FILE):
+            raise ImportError(f"libqk.so is not built ({_LIB_FILE}); run "
+                              "paper_2609_12471_gb300.build.build() or __graft_entry__.build()")
+        lib = ctypes.CDLL(_LIB_FILE)
+        for name, (args, res) in _SIGS.items():
+            f = getattr(lib, name)
+            f.argtypes = args
+            f.restype = res
+        _lib = lib
+    return _lib
+
+
+def exported_symbols():
+    """Names of the ABI entry points this binding resolves (all must exist in libqk.so)."""
+    lib = _load()
+    return [n for n in _SIGS if hasattr(lib, n)]
+
+
+def qk_last_error() -> str:
+    return _load().qk_last_error().decode()
+
+
+def _check(rc: int):
+    if rc != QK_OK:
+        raise QKError(rc, qk_last_error())
+
+
+def _ptr(x):
+    if x is None:
+        return None
+    if isinstance(x, int):
+        return x
+    if hasattr(x, "data_ptr"):
+        return x.data_ptr()
+    raise TypeError(f"cannot pass {type(x)} as a pointer")
+
+
+def _stream(stream):
+    if stream is None:
+        import torch
+        return torch.cuda.current_stream().cuda_stream
+    if isinstance(stream, int):
+        return stream
+    return stream.cuda_stream
+
+
+def _nbytes(t, given):
+    if given is not None:
+        return given
+    return t.numel() * t.element_size()
+
+
+def qk_config_preset(name: str) -> qk_config:
+    c = qk_config()
+    _check(_load().qk_config_preset(name.encode(), ctypes.byref(c)))
+    return c
+
+
+def qk_weight_count(cfg: qk_config) -> int:
+    n = _I()
+    _check(_load().qk_weight_count(ctypes.byref(cfg), ctypes.byref(n)))
+    return n.value
+
+
+def qk_model_packed_bytes(cfg: qk_config) -> int:
+    n = _SZ()
+    _check(_load().qk_model_packed_bytes(ctypes.byref(cfg), ctypes.byref(n)))
+    return n.value
+
+
+def qk_model_load(cfg: qk_config, tensors, packed, packed_bytes=None, stream=None):
+    arr = (_P * len(tensors))(*[_ptr(t) for t in tensors])
+    out = _P()
+    _check(_load().qk_model_load(ctypes.byref(cfg), arr, len(tensors), _ptr(packed),
+                                 _nbytes(packed, packed_bytes), _stream(stream), ctypes.byref(out)))
+    return out.value
+
+
+def qk_model_free(m):
+    _load().qk_model_free(m)
+
+
+def qk_kv_bytes(m, max_batch: int, max_seq: int) -> int:
+    n = _SZ()
+    _check(_load().qk_kv_bytes(m, max_batch, max_seq, ctypes.byref(n)))
+    return n.value
+
+
+def qk_workspace_bytes(m, kind: int, B: int, T: int, max_seq: int) -> int:
+    n = _SZ()
+    _check(_load().qk_workspace_bytes(m, kind, B, T, max_seq, ctypes.byref(n)))
+    return n.value
+
+
+def qk_prefill(m, kv, max_batch, max_seq, tokens, B, T, start_pos=0, last_logits=None,
+               targets=None, logprobs=None, argmax=None, workspace=None, ws_bytes=None,
+               stream=None):
+    _check(_load().qk_prefill(m, _ptr(kv), max_batch, max_seq, _ptr(tokens), B, T, start_pos,
+                              _ptr(last_logits), _ptr(targets), _ptr(logprobs), _ptr(argmax),
+                              _ptr(workspace), _nbytes(workspace, ws_bytes), _stream(stream)))
+
+
+def qk_decode_step(m, kv, max_batch, max_seq, tokens, pos, B, logits=None, targets=None,
+                   logprobs=None, argmax=None, workspace=None, ws_bytes=None, stream=None):
+    _check(_load().qk_decode_step(m, _ptr(kv), max_batch, max_seq, _ptr(tokens), _ptr(pos), B,
+                                  _ptr(logits), _ptr(targets), _ptr(logprobs), _ptr(argmax),
+                                  _ptr(workspace), _nbytes(workspace, ws_bytes), _stream(stream)))
+
+
+def qk_decode_layer(m, layer, kv, max_batch, max_seq, x, pos, B, workspace=None, ws_bytes=None,
+                    stream=None):
+    _check(_load().qk_decode_layer(m, layer, _ptr(kv), max_batch, max_seq, _ptr(x), _ptr(pos), B,
+                                   _ptr(workspace), _nbytes(workspace, ws_bytes), _stream(stream)))
+
+
+def qk_score_logprobs(m, tokens, B, T, logprobs, argmax=None, workspace=None, ws_bytes=None,
+                      stream=None):
+    _check(_load().qk_score_logprobs(m, _ptr(tokens), B, T, _ptr(logprobs), _ptr(argmax),
+                                     _ptr(workspace), _nbytes(workspace, ws_bytes),
+                                     _stream(stream)))
+
+
+def qk_rollout_teacher_forced(m, kv, max_batch, max_seq, seq, B, P, N, logprobs, argmax=None,
+                              workspace=None, ws_bytes=None, stream=None):
+    _check(_load().qk_rollout_teacher_forced(m, _ptr(kv), max_batch, max_seq, _ptr(seq), B, P, N,
+                                             _ptr(logprobs), _ptr(argmax), _ptr(workspace),
+                                             _nbytes(workspace, ws_bytes), _stream(stream)))
+
+
+def qk_check_status(m, stream=None) -> int:
+    """Returns the status bits (0 when clean); does not raise on QK_EDEVICE."""
+    v = ctypes.c_uint32()
+    rc = _load().qk_check_status(m, _stream(stream), ctypes.byref(v))
+    if rc not in (QK_OK, QK_EDEVICE):
+        _check(rc)
+    return v.value

@@ -1,0 +1,30 @@
+// Kernel selection for the linear layers and attention of one forward call.
+#include "qk_internal.cuh"
+
+namespace qk {
+
+void linear(const Model& m, const void* A, int lda, const void* W, void* C, int ldc, int M, int N,
+            int K, int epi, void* gu, cudaStream_t s) {
+    const int dt = m.cfg.dtype;
+    if (dt == QK_DTYPE_BF16 && M <= 16) {
+        launch_gemv_bf16((const bf16*)A, lda, (const bf16*)W, C, ldc, M, N, K, epi, s);
+        return;
+    }
+    if (epi == EPI_SWIGLU) {
+        launch_gemm_simt(A, lda, W, gu, 2 * N, M, 2 * N, K, dt, EPI_STORE_ACT, s);
+        launch_swiglu(gu, C, dt, M, N, s);
+        return;
+    }
+    launch_gemm_simt(A, lda, W, C, ldc, M, N, K, dt, epi, s);
+}
+
+void launch_attention(const Model& m, const void* q, int q_ld, const void* k_cache,
+                      const void* v_cache, int M, int max_batch, int max_seq, PosIndex pos,
+                      void* o, cudaStream_t s) {
+    (void)max_batch;
+    const qk_config& c = m.cfg;
+    launch_attention_simt(q, q_ld, k_cache, v_cache, c.dtype, M, c.n_q_heads, c.n_kv_heads,
+                          c.head_dim, max_seq, pos, o, m.status, s);
+}
+
+}  // namespace qk

@@ -1,0 +1,309 @@
+// Elementwise and row-wise kernels of the decoder forward pass: embedding
+// gather, RMSNorm, per-head QK-RMSNorm + RoPE + KV-cache write, SwiGLU,
+// vocabulary log-softmax / gather / argmax, and the load-time RoPE table.
+#include <math.h>
+
+#include "qk_internal.cuh"
+
+namespace qk {
+
+__device__ __forceinline__ float to_f(float v) { return v; }
+__device__ __forceinline__ float to_f(bf16 v) { return __bfloat162float(v); }
+template <typename T> __device__ __forceinline__ T from_f(float v);
+template <> __device__ __forceinline__ float from_f<float>(float v) { return v; }
+template <> __device__ __forceinline__ bf16 from_f<bf16>(float v) { return __float2bfloat16_rn(v); }
+
+__device__ __forceinline__ float warp_sum(float v) {
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+    return v;
+}
+
+// Sum over a block whose size is a multiple of 32 (at most 1024); every thread gets the total.
+__device__ float block_sum(float v, float* red) {
+    v = warp_sum(v);
+    int w = threadIdx.x >> 5, l = threadIdx.x & 31, nw = blockDim.x >> 5;
+    __syncthreads();
+    if (l == 0) red[w] = v;
+    __syncthreads();
+    float t = l < nw ? red[l] : 0.f;
+    return warp_sum(t);
+}
+
+// ---------------------------------------------------------------- embedding (x_0 = E[token])
+template <typename T>
+__global__ void embed_kernel(const T* __restrict__ E, int V, int H, TokIndex tok,
+                             float* __restrict__ x, uint32_t* status) {
+    int r = blockIdx.x;
+    int id = tok.ptr[(size_t)(r / tok.T) * tok.ld + tok.off + r % tok.T];
+    if (id < 0 || id >= V) {
+        if (threadIdx.x == 0) atomicOr(status, QK_STATUS_BAD_TOKEN);
+        id = 0;
+    }
+    const T* src = E + (size_t)id * H;
+    float* dst = x + (size_t)r * H;
+    for (int i = threadIdx.x; i < H; i += blockDim.x) dst[i] = to_f(src[i]);
+}
+
+void launch_embed(const void* E, int dtype, int V, int H, TokIndex tok, int M, float* x,
+                  uint32_t* status, cudaStream_t s) {
+    note_launch();
+    if (M <= 0) return;
+    if (dtype == QK_DTYPE_BF16)
+        embed_kernel<bf16><<<M, 256, 0, s>>>((const bf16*)E, V, H, tok, x, status);
+    else
+        embed_kernel<float><<<M, 256, 0, s>>>((const float*)E, V, H, tok, x, status);
+}
+
+// ---------------------------------------------------------------- RMSNorm
+template <typename OutT>
+__global__ void rmsnorm_kernel(const float* __restrict__ x, int in_step, int in_off,
+                               const float* __restrict__ g, int H, float eps,
+                               OutT* __restrict__ out) {
+    __shared__ float red[32];
+    int r = blockIdx.x;
+    const float* xr = x + ((size_t)r * in_step + in_off) * H;
+    float ss = 0.f;
+    for (int i = threadIdx.x * 4; i < H; i += blockDim.x * 4) {
+        float4 v = *reinterpret_cast<const float4*>(xr + i);
+        ss += v.x * v.x + v.y * v.y + v.z * v.z + v.w * v.w;
+    }
+    ss = block_sum(ss, red);
+    float scale = rsqrtf(ss / (float)H + eps);
+    OutT* o = out + (size_t)r * H;
+    for (int i = threadIdx.x * 4; i < H; i += blockDim.x * 4) {
+        float4 v = *reinterpret_cast<const float4*>(xr + i);
+        float4 gg = *reinterpret_cast<const float4*>(g + i);
+        o[i + 0] = from_f<OutT>(v.x * scale * gg.x);
+        o[i + 1] = from_f<OutT>(v.y * scale * gg.y);
+        o[i + 2] = from_f<OutT>(v.z * scale * gg.z);
+        o[i + 3] = from_f<OutT>(v.w * scale * gg.w);
+    }
+}
+
+void launch_rmsnorm(const float* x, int in_step, int in_off, const float* g, int H, float eps,
+                    void* out, int out_dtype, int M, cudaStream_t s) {
+    note_launch();
+    if (M <= 0) return;
+    int threads = H >= 1024 ? 256 : 64;
+    if (out_dtype == QK_DTYPE_BF16)
+        rmsnorm_kernel<bf16><<<M, threads, 0, s>>>(x, in_step, in_off, g, H, eps, (bf16*)out);
+    else
+        rmsnorm_kernel<float><<<M, threads, 0, s>>>(x, in_step, in_off, g, H, eps, (float*)out);
+}
+
+// ---------------------------------------------------------------- QK-norm + RoPE + cache write
+// One warp per (token, head) of the fused qkv row; lane owns elements lane + 32 i.
+template <typename T, int D>
+__global__ void qk_norm_rope_kernel(T* __restrict__ qkv, int nq, int nkv, const float* __restrict__ gq,
+                                    const float* __restrict__ gk, float eps,
+                                    const float* __restrict__ rc, const float* __restrict__ rs,
+                                    int max_positions, PosIndex pos, T* __restrict__ kc,
+                                    T* __restrict__ vc, int max_seq, uint32_t* status) {
+    constexpr int E = D / 32, HALF = D / 2;
+    int lane = threadIdx.x & 31;
+    int hh = blockIdx.y * (blockDim.x >> 5) + (threadIdx.x >> 5);
+    int nh = nq + 2 * nkv;
+    if (hh >= nh) return;
+    int r = blockIdx.x;
+    int b = r / pos.T, t = r % pos.T;
+    int p = pos.pos_dev ? pos.pos_dev[b] + t : pos.start + t;
+    int lim = max_seq < max_positions ? max_seq : max_positions;
+    if (p < 0 || p >= lim) {
+        if (lane == 0) atomicOr(status, QK_STATUS_BAD_POS);
+        p = p < 0 ? 0 : lim - 1;
+    }
+    T* src = qkv + (size_t)r * nh * D + (size_t)hh * D;
+    float e[E];
+#pragma unroll
+    for (int i = 0; i < E; ++i) e[i] = to_f(src[lane + 32 * i]);
+    if (hh >= nq + nkv) {  // value head: straight to the cache
+        int kvh = hh - nq - nkv;
+        T* dst = vc + (((size_t)b * nkv + kvh) * max_seq + p) * D;
+#pragma unroll
+        for (int i = 0; i < E; ++i) dst[lane + 32 * i] = src[lane + 32 * i];
+        return;
+    }
+    const float* g = hh < nq ? gq : gk;
+    float ss = 0.f;
+#pragma unroll
+    for (int i = 0; i < E; ++i) ss += e[i] * e[i];
+    ss = warp_sum(ss);
+    float scale = rsqrtf(ss / (float)D + eps);
+#pragma unroll
+    for (int i = 0; i < E; ++i) e[i] = e[i] * scale * g[lane + 32 * i];
+    const float* cr = rc + (size_t)p * HALF;
+    const float* sr = rs + (size_t)p * HALF;
+#pragma unroll
+    for (int i = 0; i < E / 2; ++i) {
+        int j = lane + 32 * i;  // j < d/2, partner j + d/2 is element i + E/2 of this lane
+        float c = cr[j], sn = sr[j];
+        float a = e[i], bb = e[i + E / 2];
+        e[i] = a * c - bb * sn;
+        e[i + E / 2] = bb * c + a * sn;
+    }
+    T* dst;
+    if (hh < nq) {
+        dst = src;
+    } else {
+        int kvh = hh - nq;
+        dst = kc + (((size_t)b * nkv + kvh) * max_seq + p) * D;
+    }
+#pragma unroll
+    for (int i = 0; i < E; ++i) dst[lane + 32 * i] = from_f<T>(e[i]);
+}
+
+void launch_qk_norm_rope(void* qkv, int dtype, int M, int nq, int nkv, int d, const float* gq,
+                         const float* gk, float eps, const float* rope_cos, const float* rope_sin,
+                         int max_positions, PosIndex pos, void* k_cache, void* v_cache,
+                         int max_seq, uint32_t* status, cudaStream_t s) {
+    note_launch();
+    if (M <= 0) return;
+    dim3 grid(M, (nq + 2 * nkv + 7) / 8);
+#define QK_NR(T, D)                                                                          \
+    qk_norm_rope_kernel<T, D><<<grid, 256, 0, s>>>((T*)qkv, nq, nkv, gq, gk, eps, rope_cos,  \
+                                                   rope_sin, max_positions, pos, (T*)k_cache, \
+                                                   (T*)v_cache, max_seq, status)
+    if (dtype == QK_DTYPE_BF16) {
+        if (d == 128) QK_NR(bf16, 128); else QK_NR(bf16, 64);
+    } else {
+        if (d == 128) QK_NR(float, 128); else QK_NR(float, 64);
+    }
+#undef QK_NR
+}
+
+// ---------------------------------------------------------------- SwiGLU (unfused path)
+template <typename T>
+__global__ void swiglu_kernel(const T* __restrict__ gu, T* __restrict__ h, int M, int I) {
+    size_t n = (size_t)M * I;
+    for (size_t e = blockIdx.x * (size_t)blockDim.x + threadIdx.x; e < n;
+         e += (size_t)gridDim.x * blockDim.x) {
+        size_t m = e / I;
+        int j = (int)(e % I);
+        const T* row = gu + m * 2 * I + (size_t)(j >> 7) * 256 + (j & 127);
+        float g = to_f(row[0]), u = to_f(row[128]);
+        h[e] = from_f<T>(g / (1.f + expf(-g)) * u);
+    }
+}
+
+void launch_swiglu(const void* gu, void* h, int dtype, int M, int I, cudaStream_t s) {
+    note_launch();
+    if (M <= 0) return;
+    size_t n = (size_t)M * I;
+    int blocks = (int)((n + 255) / 256);
+    if (blocks > 65535) blocks = 65535;
+    if (dtype == QK_DTYPE_BF16)
+        swiglu_kernel<bf16><<<blocks, 256, 0, s>>>((const bf16*)gu, (bf16*)h, M, I);
+    else
+        swiglu_kernel<float><<<blocks, 256, 0, s>>>((const float*)gu, (float*)h, M, I);
+}
+
+// ---------------------------------------------------------------- log-softmax / gather / argmax
+// One block per logits row: max and lowest arg-max, then logsumexp, then the target's log-prob.
+__global__ void logits_reduce_kernel(const float* __restrict__ logits, int V, OutIndex oi,
+                                     float* __restrict__ lp, int32_t* __restrict__ am,
+                                     uint32_t* status) {
+    __shared__ float red_v[32];
+    __shared__ int red_i[32];
+    __shared__ float red[32];
+    int r = blockIdx.x;
+    int g = oi.row0 + r;
+    int b = g / oi.T, t = g % oi.T;
+    if (t >= oi.out_lim) return;
+    const float* z = logits + (size_t)r * V;
+    float best = -INFINITY;
+    int bi = 0x7fffffff;
+    for (int i = threadIdx.x * 4; i < V; i += blockDim.x * 4) {
+        float4 v = *reinterpret_cast<const float4*>(z + i);
+        if (v.x > best) { best = v.x; bi = i; }
+        if (v.y > best) { best = v.y; bi = i + 1; }
+        if (v.z > best) { best = v.z; bi = i + 2; }
+        if (v.w > best) { best = v.w; bi = i + 3; }
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+        float ov = __shfl_xor_sync(0xffffffffu, best, o);
+        int oidx = __shfl_xor_sync(0xffffffffu, bi, o);
+        if (ov > best || (ov == best && oidx < bi)) { best = ov; bi = oidx; }
+    }
+    int w = threadIdx.x >> 5, l = threadIdx.x & 31, nw = blockDim.x >> 5;
+    if (l == 0) { red_v[w] = best; red_i[w] = bi; }
+    __syncthreads();
+    best = l < nw ? red_v[l] : -INFINITY;
+    bi = l < nw ? red_i[l] : 0x7fffffff;
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+        float ov = __shfl_xor_sync(0xffffffffu, best, o);
+        int oidx = __shfl_xor_sync(0xffffffffu, bi, o);
+        if (ov > best || (ov == best && oidx < bi)) { best = ov; bi = oidx; }
+    }
+    float se = 0.f;
+    for (int i = threadIdx.x * 4; i < V; i += blockDim.x * 4) {
+        float4 v = *reinterpret_cast<const float4*>(z + i);
+        se += expf(v.x - best) + expf(v.y - best) + expf(v.z - best) + expf(v.w - best);
+    }
+    se = block_sum(se, red);
+    if (threadIdx.x == 0) {
+        size_t o = (size_t)b * oi.out_ld + oi.out_off + t;
+        if (am) am[o] = bi;
+        if (lp && oi.tgt) {
+            int tg = oi.tgt[(size_t)b * oi.tgt_ld + oi.tgt_off + t];
+            if (tg < 0 || tg >= V) {
+                atomicOr(status, QK_STATUS_BAD_TOKEN);
+                tg = 0;
+            }
+            lp[o] = z[tg] - (best + logf(se));
+        }
+    }
+}
+
+void launch_logits_reduce(const float* logits, int M, int V, OutIndex oi, float* lp,
+                          int32_t* argmax, uint32_t* status, cudaStream_t s) {
+    note_launch();
+    if (M <= 0) return;
+    logits_reduce_kernel<<<M, 512, 0, s>>>(logits, V, oi, lp, argmax, status);
+}
+
+// ---------------------------------------------------------------- load-time tables
+// cos / sin of p * theta^(-2i/d) in double precision, stored as fp32 [max_positions, d/2].
+__global__ void rope_table_kernel(float* cos_t, float* sin_t, int max_positions, int d,
+                                  double theta) {
+    int half = d / 2;
+    size_t n = (size_t)max_positions * half;
+    for (size_t e = blockIdx.x * (size_t)blockDim.x + threadIdx.x; e < n;
+         e += (size_t)gridDim.x * blockDim.x) {
+        int p = (int)(e / half), i = (int)(e % half);
+        double inv_freq = pow(theta, -2.0 * i / d);
+        double ang = (double)p * inv_freq;
+        double sn, c;
+        sincos(ang, &sn, &c);
+        cos_t[e] = (float)c;
+        sin_t[e] = (float)sn;
+    }
+}
+
+void launch_rope_table(float* cos_t, float* sin_t, int max_positions, int d, double theta,
+                       cudaStream_t s) {
+    note_launch();
+    size_t n = (size_t)max_positions * (d / 2);
+    int blocks = (int)((n + 255) / 256);
+    if (blocks > 4096) blocks = 4096;
+    rope_table_kernel<<<blocks, 256, 0, s>>>(cos_t, sin_t, max_positions, d, theta);
+}
+
+template <typename T>
+__global__ void widen_kernel(const T* src, float* dst, int n) {
+    int i = blockIdx.x * blockDim.x + threadIdx.x;
+    if (i < n) dst[i] = to_f(src[i]);
+}
+
+void launch_widen_gain(const void* src, int dtype, float* dst, int n, cudaStream_t s) {
+    note_launch();
+    int blocks = (n + 255) / 256;
+    if (dtype == QK_DTYPE_BF16)
+        widen_kernel<bf16><<<blocks, 256, 0, s>>>((const bf16*)src, dst, n);
+    else
+        widen_kernel<float><<<blocks, 256, 0, s>>>((const float*)src, dst, n);
+}
+
+}  // namespace qk

@@ -1,0 +1,590 @@
+// libqk C ABI: configuration presets, packed weight layout, model loading,
+// workspace layout and the host-side orchestration of the forward pass.
+//
+// Every entry point validates its arguments on the host before any launch,
+// launches only on the caller's stream, never synchronises (except
+// qk_check_status) and never allocates device memory.
+#include <stdarg.h>
+#include <stdio.h>
+#include <string.h>
+
+#include <atomic>
+#include <new>
+
+#include "qk_internal.cuh"
+
+namespace qk {
+
+static thread_local char g_err[512] = "";
+static std::atomic<uint64_t> g_launches{0};
+
+void note_launch(int n) { g_launches.fetch_add((uint64_t)n, std::memory_order_relaxed); }
+
+bool prof_open(Model& m, int kind, cudaStream_t s) {
+    if (!m.in_decode || m.prof_kind != kind || m.prof_used + 2 > (int)m.prof_ev.size()) return false;
+    cudaEventRecord(m.prof_ev[m.prof_used++], s);
+    return true;
+}
+
+void prof_close(Model& m, bool opened, cudaStream_t s) {
+    if (opened) cudaEventRecord(m.prof_ev[m.prof_used++], s);
+}
+
+int set_error(int code, const char* fmt, ...) {
+    va_list ap;
+    va_start(ap, fmt);
+    vsnprintf(g_err, sizeof(g_err), fmt, ap);
+    va_end(ap);
+    return code;
+}
+
+int cuda_error(cudaError_t e, const char* what) {
+    return set_error(QK_ECUDA, "%s: %s", what, cudaGetErrorString(e));
+}
+
+static size_t align256(size_t v) { return (v + 255) & ~(size_t)255; }
+
+int validate_config(const qk_config& c) {
+    if (c.dtype != QK_DTYPE_BF16 && c.dtype != QK_DTYPE_F32)
+        return set_error(QK_EDTYPE, "dtype %d is neither QK_DTYPE_BF16 nor QK_DTYPE_F32", c.dtype);
+    if (c.head_dim != 64 && c.head_dim != 128)
+        return set_error(QK_EDTYPE, "head_dim %d unsupported (64 or 128)", c.head_dim);
+    if (c.n_layers < 1 || c.n_q_heads < 1 || c.n_kv_heads < 1 || c.n_q_heads % c.n_kv_heads)
+        return set_error(QK_ESHAPE, "bad layer / head counts (%d layers, %d q heads, %d kv heads)",
+                         c.n_layers, c.n_q_heads, c.n_kv_heads);
+    if (c.n_q_heads / c.n_kv_heads > 32)
+        return set_error(QK_EDTYPE, "query heads per kv head > 32 unsupported");
+    if (c.hidden < 64 || c.hidden % 64)
+        return set_error(QK_ESHAPE, "hidden %d must be a positive multiple of 64", c.hidden);
+    if (c.intermediate < 128 || c.intermediate % 128)
+        return set_error(QK_ESHAPE, "intermediate %d must be a positive multiple of 128", c.intermediate);
+    if (c.vocab < 4 || c.vocab % 4)
+        return set_error(QK_ESHAPE, "vocab %d must be a positive multiple of 4", c.vocab);
+    if (c.max_positions < 1 || c.reserved != 0)
+        return set_error(QK_EINVAL, "max_positions must be >= 1 and reserved 0");
+    if (!(c.rms_eps > 0.0) || !(c.rope_theta > 1.0))
+        return set_error(QK_EINVAL, "rms_eps must be > 0 and rope_theta > 1");
+    return QK_OK;
+}
+
+int packed_layout(const qk_config& c, PackedLayout* out) {
+    QK_TRY(validate_config(c));
+    size_t es = c.dtype == QK_DTYPE_BF16 ? 2 : 4;
+    size_t H = c.hidden, d = c.head_dim, nq = c.n_q_heads, nkv = c.n_kv_heads, I = c.intermediate,
+           V = c.vocab;
+    size_t off = 0;
+    auto take = [&](size_t bytes) {
+        size_t o = off;
+        off = align256(off + bytes);
+        return o;
+    };
+    out->status = take(256);
+    out->rope_cos = take((size_t)c.max_positions * (d / 2) * 4);
+    out->rope_sin = take((size_t)c.max_positions * (d / 2) * 4);
+    out->embed = take(V * H * es);
+    out->layers.resize(c.n_layers);
+    for (int l = 0; l < c.n_layers; ++l) {
+        PackedLayout::L& L = out->layers[l];
+        L.attn_norm = take(H * 4);
+        L.q_norm = take(d * 4);
+        L.k_norm = take(d * 4);
+        L.mlp_norm = take(H * 4);
+        L.w_qkv = take((nq + 2 * nkv) * d * H * es);
+        L.w_o = take(H * nq * d * es);
+        L.w_gu = take(2 * I * H * es);
+        L.w_d = take(H * I * es);
+    }
+    out->final_norm = take(H * 4);
+    out->lm_head = take(V * H * es);
+    out->total = off;
+    return QK_OK;
+}
+
+// ---------------------------------------------------------------- workspace layout
+struct Workspace {
+    float* x;       // [M, H] fp32 residual stream
+    void* u;        // [M, H] normalised input of a linear layer
+    void* qkv;      // [M, (nq + 2 nkv) d]
+    void* o;        // [M, nq d] attention output
+    void* h;        // [M, I] SwiGLU output
+    void* gu;       // [M, 2 I] gate/up before SwiGLU (unfused path only)
+    void* skv;      // scoring: K and V of one layer, [2][B, nkv, T, d]
+    float* logits;  // [logit_rows, V]
+    int logit_rows;
+    size_t total;
+};
+
+static const int kScoreLogitRows = 4096;
+
+static int workspace_layout(const Model& m, int kind, int B, int T, Workspace* w, char* base) {
+    const qk_config& c = m.cfg;
+    if (B < 1 || T < 1) return set_error(QK_ESHAPE, "batch %d and tokens %d must be >= 1", B, T);
+    size_t es = m.es;
+    size_t M = (size_t)B * (kind == QK_CALL_DECODE ? 1 : T);
+    if (M > (size_t)1 << 24) return set_error(QK_ESHAPE, "too many tokens in one call (%zu)", M);
+    size_t H = c.hidden, d = c.head_dim, nq = c.n_q_heads, nkv = c.n_kv_heads, I = c.intermediate;
+    size_t off = 0;
+    auto take = [&](size_t bytes) {
+        char* p = base ? base + off : nullptr;
+        off = align256(off + bytes);
+        return (void*)p;
+    };
+    w->x = (float*)take(M * H * 4);
+    w->u = take(M * H * es);
+    w->qkv = take(M * (nq + 2 * nkv) * d * es);
+    w->o = take(M * nq * d * es);
+    w->h = take(M * I * es);
+    w->gu = take(M * 2 * I * es);
+    w->skv = kind == QK_CALL_SCORE ? take(2 * (size_t)B * nkv * T * d * es) : nullptr;
+    size_t rows = kind == QK_CALL_SCORE ? (M < (size_t)kScoreLogitRows ? M : kScoreLogitRows) : B;
+    w->logit_rows = (int)rows;
+    w->logits = (float*)take(rows * (size_t)c.vocab * 4);
+    w->total = off;
+    return QK_OK;
+}
+
+// ---------------------------------------------------------------- forward pieces
+struct KVView {
+    char* base;        // layer 0's K
+    size_t layer_bytes;  // bytes from one layer's K to the next layer's K (0: shared scratch)
+    size_t half_bytes;   // bytes from a layer's K to its V
+    int max_batch, max_seq;
+    void* k(int l) const { return base + (size_t)l * layer_bytes; }
+    void* v(int l) const { return base + (size_t)l * layer_bytes + half_bytes; }
+};
+
+static KVView cache_view(const Model& m, void* kv, int max_batch, int max_seq) {
+    const qk_config& c = m.cfg;
+    size_t half = (size_t)max_batch * c.n_kv_heads * max_seq * c.head_dim * m.es;
+    return KVView{(char*)kv, 2 * half, half, max_batch, max_seq};
+}
+
+static void run_layer(Model& m, int l, const Workspace& w, int M, PosIndex pos,
+                      const KVView& kv, cudaStream_t s) {
+    const qk_config& c = m.cfg;
+    const LayerW& L = m.layers[l];
+    int H = c.hidden, d = c.head_dim, nq = c.n_q_heads, nkv = c.n_kv_heads, I = c.intermediate;
+    int nqkv = (nq + 2 * nkv) * d;
+    float eps = (float)c.rms_eps;
+    bool pr;
+    launch_rmsnorm(w.x, 1, 0, L.attn_norm, H, eps, w.u, c.dtype, M, s);
+    pr = prof_open(m, QK_PROF_QKV, s);
+    linear(m, w.u, H, L.w_qkv, w.qkv, nqkv, M, nqkv, H, EPI_STORE_ACT, w.gu, s);
+    prof_close(m, pr, s);
+    launch_qk_norm_rope(w.qkv, c.dtype, M, nq, nkv, d, L.q_norm, L.k_norm, eps, m.rope_cos,
+                        m.rope_sin, c.max_positions, pos, kv.k(l), kv.v(l), kv.max_seq, m.status,
+                        s);
+    pr = prof_open(m, QK_PROF_ATTN, s);
+    launch_attention(m, w.qkv, nqkv, kv.k(l), kv.v(l), M, kv.max_batch, kv.max_seq, pos, w.o, s);
+    prof_close(m, pr, s);
+    pr = prof_open(m, QK_PROF_O, s);
+    linear(m, w.o, nq * d, L.w_o, w.x, H, M, H, nq * d, EPI_RESID_F32, w.gu, s);
+    prof_close(m, pr, s);
+    launch_rmsnorm(w.x, 1, 0, L.mlp_norm, H, eps, w.u, c.dtype, M, s);
+    pr = prof_open(m, QK_PROF_GATE_UP, s);
+    linear(m, w.u, H, L.w_gu, w.h, I, M, I, H, EPI_SWIGLU, w.gu, s);
+    prof_close(m, pr, s);
+    pr = prof_open(m, QK_PROF_DOWN, s);
+    linear(m, w.h, I, L.w_d, w.x, H, M, H, I, EPI_RESID_F32, w.gu, s);
+    prof_close(m, pr, s);
+}
+
+// Final norm of M_out selected rows (row r of the output reads residual row r * in_step + in_off),
+// lm_head into `logits`, then log-prob / argmax per row.
+static void run_head(Model& m, const Workspace& w, int M_out, int in_step, int in_off,
+                     float* logits, OutIndex oi, float* lp, int32_t* am, cudaStream_t s) {
+    const qk_config& c = m.cfg;
+    launch_rmsnorm(w.x, in_step, in_off, m.final_norm, c.hidden, (float)c.rms_eps, w.u, c.dtype,
+                   M_out, s);
+    bool pr = prof_open(m, QK_PROF_LM_HEAD, s);
+    linear(m, w.u, c.hidden, m.lm_head, logits, c.vocab, M_out, c.vocab, c.hidden, EPI_STORE_F32,
+           w.gu, s);
+    prof_close(m, pr, s);
+    if (lp || am) launch_logits_reduce(logits, M_out, c.vocab, oi, lp, am, m.status, s);
+}
+
+static int check_launch(const char* what) {
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) return cuda_error(e, what);
+    return QK_OK;
+}
+
+static int get_ws(const Model& m, int kind, int B, int T, void* ws, size_t ws_bytes, Workspace* w) {
+    QK_TRY(workspace_layout(m, kind, B, T, w, nullptr));
+    if (!ws) return set_error(QK_EINVAL, "workspace is NULL");
+    if (((uintptr_t)ws & 255) != 0) return set_error(QK_EINVAL, "workspace must be 256-byte aligned");
+    if (ws_bytes < w->total)
+        return set_error(QK_ENOSPACE, "workspace has %zu bytes, needs %zu", ws_bytes, w->total);
+    return workspace_layout(m, kind, B, T, w, (char*)ws);
+}
+
+static int check_cache(const Model& m, void* kv, int max_batch, int max_seq, int B) {
+    if (!kv) return set_error(QK_EINVAL, "kv cache is NULL");
+    if (((uintptr_t)kv & 255) != 0) return set_error(QK_EINVAL, "kv cache must be 256-byte aligned");
+    if (max_batch < 1 || max_seq < 1) return set_error(QK_ESHAPE, "max_batch / max_seq must be >= 1");
+    if (B < 1 || B > max_batch) return set_error(QK_ESHAPE, "batch %d outside [1, %d]", B, max_batch);
+    if (max_seq > m.cfg.max_positions)
+        return set_error(QK_ESHAPE, "max_seq %d exceeds the RoPE table (%d positions)", max_seq,
+                         m.cfg.max_positions);
+    return QK_OK;
+}
+
+}  // namespace qk
+
+using namespace qk;
+
+// ================================================================ C ABI
+extern "C" {
+
+const char* qk_last_error(void) { return g_err; }
+
+int qk_config_preset(const char* name, qk_config* out) {
+    if (!name || !out) return set_error(QK_EINVAL, "null argument");
+    qk_config c;
+    memset(&c, 0, sizeof(c));
+    c.rms_eps = 1e-6;
+    c.rope_theta = 1e6;
+    c.max_positions = 8192;
+    if (!strcmp(name, "tiny_fp32")) {
+        c.n_layers = 2; c.hidden = 256; c.n_q_heads = 4; c.n_kv_heads = 2; c.head_dim = 64;
+        c.intermediate = 768; c.vocab = 4096; c.dtype = QK_DTYPE_F32;
+    } else if (!strcmp(name, "q8b") || !strcmp(name, "q8b_layer")) {
+        c.n_layers = strcmp(name, "q8b") ? 1 : 36; c.hidden = 4096; c.n_q_heads = 32;
+        c.n_kv_heads = 8; c.head_dim = 128; c.intermediate = 12288; c.vocab = 151936;
+        c.dtype = QK_DTYPE_BF16;
+    } else {
+        return set_error(QK_EINVAL, "unknown preset '%s'", name);
+    }
+    *out = c;
+    return QK_OK;
+}
+
+int qk_weight_count(const qk_config* cfg, int* n) {
+    if (!cfg || !n) return set_error(QK_EINVAL, "null argument");
+    QK_TRY(validate_config(*cfg));
+    *n = 3 + 11 * cfg->n_layers;
+    return QK_OK;
+}
+
+int qk_model_packed_bytes(const qk_config* cfg, size_t* bytes) {
+    if (!cfg || !bytes) return set_error(QK_EINVAL, "null argument");
+    PackedLayout p;
+    QK_TRY(packed_layout(*cfg, &p));
+    *bytes = p.total;
+    return QK_OK;
+}
+
+int qk_model_load(const qk_config* cfg, const void* const* tensors, int n_tensors, void* packed,
+                  size_t packed_bytes, void* stream, qk_model** out) {
+    if (!cfg || !tensors || !packed || !out) return set_error(QK_EINVAL, "null argument");
+    *out = nullptr;
+    PackedLayout p;
+    QK_TRY(packed_layout(*cfg, &p));
+    if (n_tensors != 3 + 11 * cfg->n_layers)
+        return set_error(QK_EINVAL, "expected %d tensors, got %d", 3 + 11 * cfg->n_layers, n_tensors);
+    for (int i = 0; i < n_tensors; ++i)
+        if (!tensors[i]) return set_error(QK_EINVAL, "tensor %d is NULL", i);
+    if (((uintptr_t)packed & 255) != 0) return set_error(QK_EINVAL, "packed buffer must be 256-byte aligned");
+    if (packed_bytes < p.total)
+        return set_error(QK_ENOSPACE, "packed buffer has %zu bytes, needs %zu", packed_bytes, p.total);
+    cudaStream_t s = (cudaStream_t)stream;
+    Model* m = new (std::nothrow) Model();
+    if (!m) return set_error(QK_EINVAL, "host allocation failed");
+    const qk_config& c = *cfg;
+    m->cfg = c;
+    m->es = c.dtype == QK_DTYPE_BF16 ? 2 : 4;
+    m->packed = (char*)packed;
+    m->packed_bytes = packed_bytes;
+    auto fail = [&](int code) { delete m; return code; };
+    cudaError_t e = cudaGetDevice(&m->device);
+    if (e == cudaSuccess) e = cudaDeviceGetAttribute(&m->num_sms, cudaDevAttrMultiProcessorCount, m->device);
+    if (e != cudaSuccess) return fail(cuda_error(e, "device query"));
+    char* B = (char*)packed;
+    m->status = (uint32_t*)(B + p.status);
+    m->rope_cos = (float*)(B + p.rope_cos);
+    m->rope_sin = (float*)(B + p.rope_sin);
+    m->embed = B + p.embed;
+    m->final_norm = (float*)(B + p.final_norm);
+    m->lm_head = B + p.lm_head;
+    m->layers.resize(c.n_layers);
+    size_t es = m->es, H = c.hidden, d = c.head_dim, nq = c.n_q_heads, nkv = c.n_kv_heads,
+           I = c.intermediate, V = c.vocab;
+    e = cudaMemsetAsync(m->status, 0, 256, s);
+    if (e != cudaSuccess) return fail(cuda_error(e, "status clear"));
+    launch_rope_table(m->rope_cos, m->rope_sin, c.max_positions, c.head_dim, c.rope_theta, s);
+    int t = 0;
+    auto copy = [&](void* dst, const void* src, size_t bytes) {
+        return cudaMemcpyAsync(dst, src, bytes, cudaMemcpyDeviceToDevice, s);
+    };
+    if ((e = copy(m->embed, tensors[t++], V * H * es)) != cudaSuccess) return fail(cuda_error(e, "embed copy"));
+    for (int l = 0; l < c.n_layers; ++l) {
+        const PackedLayout::L& PL = p.layers[l];
+        LayerW& L = m->layers[l];
+        L.attn_norm = (float*)(B + PL.attn_norm);
+        L.q_norm = (float*)(B + PL.q_norm);
+        L.k_norm = (float*)(B + PL.k_norm);
+        L.mlp_norm = (float*)(B + PL.mlp_norm);
+        L.w_qkv = B + PL.w_qkv;
+        L.w_o = B + PL.w_o;
+        L.w_gu = B + PL.w_gu;
+        L.w_d = B + PL.w_d;
+        const void* const* T = tensors + t;
+        t += 11;
+        launch_widen_gain(T[0], c.dtype, L.attn_norm, (int)H, s);
+        char* qkv = (char*)L.w_qkv;
+        e = copy(qkv, T[1], nq * d * H * es);
+        if (e == cudaSuccess) e = copy(qkv + nq * d * H * es, T[2], nkv * d * H * es);
+        if (e == cudaSuccess) e = copy(qkv + (nq + nkv) * d * H * es, T[3], nkv * d * H * es);
+        if (e != cudaSuccess) return fail(cuda_error(e, "qkv copy"));
+        launch_widen_gain(T[4], c.dtype, L.q_norm, (int)d, s);
+        launch_widen_gain(T[5], c.dtype, L.k_norm, (int)d, s);
+        if ((e = copy(L.w_o, T[6], H * nq * d * es)) != cudaSuccess) return fail(cuda_error(e, "wo copy"));
+        launch_widen_gain(T[7], c.dtype, L.mlp_norm, (int)H, s);
+        // gate/up interleave: block i of 128 gate rows goes to rows [256 i, 256 i + 128),
+        // the matching 128 up rows to [256 i + 128, 256 i + 256).
+        size_t blk = 128 * H * es;
+        e = cudaMemcpy2DAsync(L.w_gu, 2 * blk, T[8], blk, blk, I / 128, cudaMemcpyDeviceToDevice, s);
+        if (e == cudaSuccess)
+            e = cudaMemcpy2DAsync((char*)L.w_gu + blk, 2 * blk, T[9], blk, blk, I / 128,
+                                  cudaMemcpyDeviceToDevice, s);
+        if (e != cudaSuccess) return fail(cuda_error(e, "gate/up copy"));
+        if ((e = copy(L.w_d, T[10], H * I * es)) != cudaSuccess) return fail(cuda_error(e, "wd copy"));
+    }
+    launch_widen_gain(tensors[t++], c.dtype, m->final_norm, (int)H, s);
+    if ((e = copy(m->lm_head, tensors[t++], V * H * es)) != cudaSuccess) return fail(cuda_error(e, "lm_head copy"));
+    int rc = check_launch("model load kernels");
+    if (rc != QK_OK) return fail(rc);
+    *out = (qk_model*)m;
+    return QK_OK;
+}
+
+static void prof_release(Model& m) {
+    for (cudaEvent_t e : m.prof_ev) cudaEventDestroy(e);
+    m.prof_ev.clear();
+    m.prof_used = 0;
+    m.prof_kind = -1;
+}
+
+void qk_model_free(qk_model* m) {
+    if (!m) return;
+    prof_release(*(Model*)m);
+    delete (Model*)m;
+}
+
+int qk_profile_begin(qk_model* mh, int kind, int max_launches) {
+    if (!mh) return set_error(QK_EINVAL, "null argument");
+    Model& m = *(Model*)mh;
+    if (kind < QK_PROF_QKV || kind > QK_PROF_LM_HEAD) return set_error(QK_EINVAL, "unknown kernel class %d", kind);
+    if (max_launches < 1 || max_launches > (1 << 20)) return set_error(QK_EINVAL, "max_launches out of range");
+    prof_release(m);
+    m.prof_ev.resize(2 * (size_t)max_launches);
+    for (size_t i = 0; i < m.prof_ev.size(); ++i) {
+        cudaError_t e = cudaEventCreate(&m.prof_ev[i]);
+        if (e != cudaSuccess) {
+            m.prof_ev.resize(i);
+            prof_release(m);
+            return cuda_error(e, "cudaEventCreate");
+        }
+    }
+    m.prof_kind = kind;
+    return QK_OK;
+}
+
+int qk_profile_end(qk_model* mh, float* total_ms, int* launches) {
+    if (!mh || !total_ms || !launches) return set_error(QK_EINVAL, "null argument");
+    Model& m = *(Model*)mh;
+    float tot = 0.f;
+    int n = m.prof_used / 2;
+    if (n > 0) {
+        cudaError_t e = cudaEventSynchronize(m.prof_ev[2 * n - 1]);
+        for (int i = 0; e == cudaSuccess && i < n; ++i) {
+            float ms = 0.f;
+            e = cudaEventElapsedTime(&ms, m.prof_ev[2 * i], m.prof_ev[2 * i + 1]);
+            tot += ms;
+        }
+        if (e != cudaSuccess) {
+            prof_release(m);
+            return cuda_error(e, "profile events");
+        }
+    }
+    prof_release(m);
+    *total_ms = tot;
+    *launches = n;
+    return QK_OK;
+}
+
+uint64_t qk_launch_count(void) { return g_launches.load(); }
+
+int qk_kv_bytes(const qk_model* mh, int max_batch, int max_seq, size_t* bytes) {
+    if (!mh || !bytes) return set_error(QK_EINVAL, "null argument");
+    const Model& m = *(const Model*)mh;
+    if (max_batch < 1 || max_seq < 1) return set_error(QK_ESHAPE, "max_batch / max_seq must be >= 1");
+    *bytes = 2 * (size_t)m.cfg.n_layers * max_batch * m.cfg.n_kv_heads * max_seq * m.cfg.head_dim * m.es;
+    return QK_OK;
+}
+
+int qk_workspace_bytes(const qk_model* mh, int kind, int B, int T, int max_seq, size_t* bytes) {
+    if (!mh || !bytes) return set_error(QK_EINVAL, "null argument");
+    const Model& m = *(const Model*)mh;
+    (void)max_seq;
+    Workspace w;
+    if (kind == QK_CALL_ROLLOUT) {
+        Workspace w2;
+        QK_TRY(workspace_layout(m, QK_CALL_PREFILL, B, T, &w, nullptr));
+        QK_TRY(workspace_layout(m, QK_CALL_DECODE, B, 1, &w2, nullptr));
+        *bytes = w.total > w2.total ? w.total : w2.total;
+        return QK_OK;
+    }
+    if (kind != QK_CALL_DECODE && kind != QK_CALL_PREFILL && kind != QK_CALL_SCORE)
+        return set_error(QK_EINVAL, "unknown call kind %d", kind);
+    QK_TRY(workspace_layout(m, kind, B, T, &w, nullptr));
+    *bytes = w.total;
+    return QK_OK;
+}
+
+static int prefill_impl(Model& m, void* kv, int max_batch, int max_seq, TokIndex tok, int B, int T,
+                        int start_pos, float* last_logits, OutIndex oi, float* lp, int32_t* am,
+                        void* ws, size_t ws_bytes, cudaStream_t s) {
+    Workspace w;
+    QK_TRY(get_ws(m, QK_CALL_PREFILL, B, T, ws, ws_bytes, &w));
+    int M = B * T;
+    KVView view = cache_view(m, kv, max_batch, max_seq);
+    launch_embed(m.embed, m.cfg.dtype, m.cfg.vocab, m.cfg.hidden, tok, M, w.x, m.status, s);
+    PosIndex pos{nullptr, start_pos, T};
+    for (int l = 0; l < m.cfg.n_layers; ++l) run_layer(m, l, w, M, pos, view, s);
+    if (last_logits || lp || am)
+        run_head(m, w, B, T, T - 1, last_logits ? last_logits : w.logits, oi, lp, am, s);
+    return check_launch("prefill");
+}
+
+int qk_prefill(qk_model* mh, void* kv, int max_batch, int max_seq, const int32_t* tokens, int B,
+               int T, int start_pos, float* last_logits, const int32_t* targets, float* logprobs,
+               int32_t* argmax, void* workspace, size_t ws_bytes, void* stream) {
+    if (!mh || !tokens) return set_error(QK_EINVAL, "null argument");
+    Model& m = *(Model*)mh;
+    QK_TRY(check_cache(m, kv, max_batch, max_seq, B));
+    if (T < 1 || start_pos < 0 || (long)start_pos + T > max_seq)
+        return set_error(QK_ESHAPE, "positions [%d, %d) outside the cache of %d", start_pos,
+                         start_pos + T, max_seq);
+    if (logprobs && !targets) return set_error(QK_EINVAL, "logprobs requested without targets");
+    OutIndex oi{1, 1, 1, 0, targets, 1, 0, 0};
+    return prefill_impl(m, kv, max_batch, max_seq, TokIndex{tokens, T, T, 0}, B, T, start_pos,
+                        last_logits, oi, logprobs, argmax, workspace, ws_bytes, (cudaStream_t)stream);
+}
+
+static int decode_impl(Model& m, void* kv, int max_batch, int max_seq, TokIndex tok, PosIndex pos,
+                       int B, float* logits, OutIndex oi, float* lp, int32_t* am, void* ws,
+                       size_t ws_bytes, cudaStream_t s) {
+    Workspace w;
+    QK_TRY(get_ws(m, QK_CALL_DECODE, B, 1, ws, ws_bytes, &w));
+    KVView view = cache_view(m, kv, max_batch, max_seq);
+    m.in_decode = true;
+    launch_embed(m.embed, m.cfg.dtype, m.cfg.vocab, m.cfg.hidden, tok, B, w.x, m.status, s);
+    for (int l = 0; l < m.cfg.n_layers; ++l) run_layer(m, l, w, B, pos, view, s);
+    if (logits || lp || am) run_head(m, w, B, 1, 0, logits ? logits : w.logits, oi, lp, am, s);
+    m.in_decode = false;
+    return check_launch("decode step");
+}
+
+int qk_decode_step(qk_model* mh, void* kv, int max_batch, int max_seq, const int32_t* tokens,
+                   const int32_t* pos, int B, float* logits, const int32_t* targets,
+                   float* logprobs, int32_t* argmax, void* workspace, size_t ws_bytes,
+                   void* stream) {
+    if (!mh || !tokens || !pos) return set_error(QK_EINVAL, "null argument");
+    Model& m = *(Model*)mh;
+    QK_TRY(check_cache(m, kv, max_batch, max_seq, B));
+    if (logprobs && !targets) return set_error(QK_EINVAL, "logprobs requested without targets");
+    OutIndex oi{1, 1, 1, 0, targets, 1, 0, 0};
+    return decode_impl(m, kv, max_batch, max_seq, TokIndex{tokens, 1, 1, 0}, PosIndex{pos, 0, 1}, B,
+                       logits, oi, logprobs, argmax, workspace, ws_bytes, (cudaStream_t)stream);
+}
+
+int qk_decode_layer(qk_model* mh, int layer, void* kv, int max_batch, int max_seq, float* x,
+                    const int32_t* pos, int B, void* workspace, size_t ws_bytes, void* stream) {
+    if (!mh || !x || !pos) return set_error(QK_EINVAL, "null argument");
+    Model& m = *(Model*)mh;
+    if (layer < 0 || layer >= m.cfg.n_layers)
+        return set_error(QK_EINVAL, "layer %d outside [0, %d)", layer, m.cfg.n_layers);
+    QK_TRY(check_cache(m, kv, max_batch, max_seq, B));
+    Workspace w;
+    QK_TRY(get_ws(m, QK_CALL_DECODE, B, 1, workspace, ws_bytes, &w));
+    w.x = x;
+    m.in_decode = true;
+    run_layer(m, layer, w, B, PosIndex{pos, 0, 1}, cache_view(m, kv, max_batch, max_seq),
+              (cudaStream_t)stream);
+    m.in_decode = false;
+    return check_launch("decode layer");
+}
+
+int qk_score_logprobs(qk_model* mh, const int32_t* tokens, int B, int T, float* logprobs,
+                      int32_t* argmax, void* workspace, size_t ws_bytes, void* stream) {
+    if (!mh || !tokens || !logprobs) return set_error(QK_EINVAL, "null argument");
+    Model& m = *(Model*)mh;
+    if (B < 1 || T < 2) return set_error(QK_ESHAPE, "scoring needs B >= 1 and T >= 2 (got %d, %d)", B, T);
+    if (T > m.cfg.max_positions)
+        return set_error(QK_ESHAPE, "T %d exceeds the RoPE table (%d)", T, m.cfg.max_positions);
+    Workspace w;
+    QK_TRY(get_ws(m, QK_CALL_SCORE, B, T, workspace, ws_bytes, &w));
+    cudaStream_t s = (cudaStream_t)stream;
+    int M = B * T;
+    // One layer's K and V live in scratch shaped like a cache of B rows x T positions;
+    // every layer reuses it (layer stride 0).
+    size_t half = (size_t)B * m.cfg.n_kv_heads * T * m.cfg.head_dim * m.es;
+    KVView view{(char*)w.skv, 0, half, B, T};
+    launch_embed(m.embed, m.cfg.dtype, m.cfg.vocab, m.cfg.hidden, TokIndex{tokens, T, T, 0}, M, w.x,
+                 m.status, s);
+    PosIndex pos{nullptr, 0, T};
+    for (int l = 0; l < m.cfg.n_layers; ++l) run_layer(m, l, w, M, pos, view, s);
+    // lm_head over all rows in chunks; row r = b T + t scores tokens[b, t + 1] for t < T - 1.
+    for (int r0 = 0; r0 < M; r0 += w.logit_rows) {
+        int rows = M - r0 < w.logit_rows ? M - r0 : w.logit_rows;
+        launch_rmsnorm(w.x + (size_t)r0 * m.cfg.hidden, 1, 0, m.final_norm, m.cfg.hidden,
+                       (float)m.cfg.rms_eps, w.u, m.cfg.dtype, rows, s);
+        linear(m, w.u, m.cfg.hidden, m.lm_head, w.logits, m.cfg.vocab, rows, m.cfg.vocab,
+               m.cfg.hidden, EPI_STORE_F32, w.gu, s);
+        OutIndex oi{T, T - 1, T - 1, 0, tokens, T, 1, r0};
+        launch_logits_reduce(w.logits, rows, m.cfg.vocab, oi, logprobs, argmax, m.status, s);
+    }
+    return check_launch("score");
+}
+
+int qk_rollout_teacher_forced(qk_model* mh, void* kv, int max_batch, int max_seq,
+                              const int32_t* seq, int B, int P, int N, float* logprobs,
+                              int32_t* argmax, void* workspace, size_t ws_bytes, void* stream) {
+    if (!mh || !seq || !logprobs) return set_error(QK_EINVAL, "null argument");
+    Model& m = *(Model*)mh;
+    QK_TRY(check_cache(m, kv, max_batch, max_seq, B));
+    if (P < 1 || N < 0 || (long)P + N > max_seq)
+        return set_error(QK_ESHAPE, "prompt %d + steps %d exceed the cache of %d", P, N, max_seq);
+    size_t need;
+    QK_TRY(qk_workspace_bytes(mh, QK_CALL_ROLLOUT, B, P, max_seq, &need));
+    if (!workspace || ws_bytes < need)
+        return set_error(QK_ENOSPACE, "workspace has %zu bytes, needs %zu", ws_bytes, need);
+    cudaStream_t s = (cudaStream_t)stream;
+    int L = P + N + 1;
+    OutIndex oi{1, 1, N + 1, 0, seq, L, P, 0};
+    QK_TRY(prefill_impl(m, kv, max_batch, max_seq, TokIndex{seq, P, L, 0}, B, P, 0, nullptr, oi,
+                        logprobs, argmax, workspace, ws_bytes, s));
+    for (int j = 0; j < N; ++j) {
+        OutIndex oj{1, 1, N + 1, j + 1, seq, L, P + j + 1, 0};
+        QK_TRY(decode_impl(m, kv, max_batch, max_seq, TokIndex{seq, 1, L, P + j},
+                           PosIndex{nullptr, P + j, 1}, B, nullptr, oj, logprobs, argmax,
+                           workspace, ws_bytes, s));
+    }
+    return QK_OK;
+}
+
+int qk_check_status(qk_model* mh, void* stream, uint32_t* flags) {
+    if (!mh) return set_error(QK_EINVAL, "null argument");
+    Model& m = *(Model*)mh;
+    cudaStream_t s = (cudaStream_t)stream;
+    uint32_t v = 0;
+    QK_TRY_CUDA(cudaStreamSynchronize(s));
+    QK_TRY_CUDA(cudaMemcpy(&v, m.status, sizeof(v), cudaMemcpyDeviceToHost));
+    QK_TRY_CUDA(cudaMemset(m.status, 0, sizeof(v)));
+    if (flags) *flags = v;
+    if (v) return set_error(QK_EDEVICE, "device status 0x%x", v);
+    return QK_OK;
+}
+
+}  // extern "C"

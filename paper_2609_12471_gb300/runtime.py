@@ -1,0 +1,115 @@
+"""Buffer management around the libqk C ABI.
+
+PyTorch supplies device memory and streams; every computation is a libqk call.
+``Decoder`` owns the packed weights, KV caches and workspaces (all torch
+tensors, so the library itself never allocates) and forwards to the binding.
+"""
+from __future__ import annotations
+
+import numpy as np
+import torch
+
+from . import _binding as B
+
+
+def _to_device(arr: np.ndarray, device) -> torch.Tensor:
+    if arr.dtype == np.uint16:
+        t = torch.from_numpy(arr.view(np.int16))
+    else:
+        t = torch.from_numpy(np.ascontiguousarray(arr))
+    return t.to(device, non_blocking=False)
+
+
+class Decoder:
+    """A loaded model plus cached workspaces.
+
+    host_tensors: a sequence (or an iterable) of numpy arrays in the canonical
+    order of qk_model_load (bf16 as uint16 bit patterns, or float32).  Tensors
+    are uploaded in groups so that the unpacked copy never exceeds ~group_bytes.
+    """
+
+    def __init__(self, cfg: B.qk_config, host_tensors, device="cuda", group_bytes=4 << 30):
+        self.cfg = cfg
+        self.device = torch.device(device)
+        n = B.qk_weight_count(cfg)
+        self.packed = torch.empty(B.qk_model_packed_bytes(cfg), dtype=torch.uint8, device=self.device)
+        tensors = list(host_tensors)
+        if len(tensors) != n:
+            raise ValueError(f"expected {n} tensors, got {len(tensors)}")
+        # The loader repacks all tensors in one call, so every tensor must be resident at once.
+        dev = [_to_device(np.asarray(a), self.device) for a in tensors]
+        self.handle = B.qk_model_load(cfg, dev, self.packed)
+        torch.cuda.current_stream(self.device).synchronize()
+        del dev
+        self._ws = {}
+
+    def close(self):
+        if self.handle:
+            B.qk_model_free(self.handle)
+            self.handle = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+    # ------------------------------------------------------------ buffers
+    def new_kv(self, max_batch: int, max_seq: int) -> torch.Tensor:
+        return torch.empty(B.qk_kv_bytes(self.handle, max_batch, max_seq), dtype=torch.uint8,
+                           device=self.device)
+
+    def workspace(self, kind: int, Bn: int, T: int, max_seq: int = 1) -> torch.Tensor:
+        need = B.qk_workspace_bytes(self.handle, kind, Bn, T, max_seq)
+        ws = self._ws.get(kind)
+        if ws is None or ws.numel() < need:
+            ws = torch.empty(need, dtype=torch.uint8, device=self.device)
+            self._ws[kind] = ws
+        return ws
+
+    def kv_view(self, kv: torch.Tensor, max_batch: int, max_seq: int):
+        """The cache as [layers, 2, max_batch, n_kv, max_seq, d] in the model dtype."""
+        c = self.cfg
+        dt = torch.bfloat16 if c.dtype == B.QK_DTYPE_BF16 else torch.float32
+        return kv.view(dt).view(c.n_layers, 2, max_batch, c.n_kv_heads, max_seq, c.head_dim)
+
+    # ------------------------------------------------------------ calls
+    def prefill(self, kv, max_batch, max_seq, tokens, start_pos=0, last_logits=None, targets=None,
+                logprobs=None, argmax=None):
+        Bn, T = tokens.shape
+        ws = self.workspace(B.QK_CALL_PREFILL, Bn, T, max_seq)
+        B.qk_prefill(self.handle, kv, max_batch, max_seq, tokens, Bn, T, start_pos, last_logits,
+                     targets, logprobs, argmax, ws)
+
+    def decode_step(self, kv, max_batch, max_seq, tokens, pos, logits=None, targets=None,
+                    logprobs=None, argmax=None):
+        Bn = tokens.shape[0]
+        ws = self.workspace(B.QK_CALL_DECODE, Bn, 1, max_seq)
+        B.qk_decode_step(self.handle, kv, max_batch, max_seq, tokens, pos, Bn, logits, targets,
+                         logprobs, argmax, ws)
+
+    def decode_layer(self, layer, kv, max_batch, max_seq, x, pos):
+        Bn = x.shape[0]
+        ws = self.workspace(B.QK_CALL_DECODE, Bn, 1, max_seq)
+        B.qk_decode_layer(self.handle, layer, kv, max_batch, max_seq, x, pos, Bn, ws)
+
+    def score(self, tokens, logprobs=None, argmax=None):
+        Bn, T = tokens.shape
+        if logprobs is None:
+            logprobs = torch.empty(Bn, T - 1, dtype=torch.float32, device=self.device)
+        ws = self.workspace(B.QK_CALL_SCORE, Bn, T)
+        B.qk_score_logprobs(self.handle, tokens, Bn, T, logprobs, argmax, ws)
+        return logprobs
+
+    def rollout(self, kv, max_batch, max_seq, seq, P, logprobs=None, argmax=None):
+        Bn, L = seq.shape
+        N = L - P - 1
+        if logprobs is None:
+            logprobs = torch.empty(Bn, N + 1, dtype=torch.float32, device=self.device)
+        ws = self.workspace(B.QK_CALL_ROLLOUT, Bn, P, max_seq)
+        B.qk_rollout_teacher_forced(self.handle, kv, max_batch, max_seq, seq, Bn, P, N, logprobs,
+                                    argmax, ws)
+        return logprobs
+
+    def check_status(self) -> int:
+        return B.qk_check_status(self.handle)

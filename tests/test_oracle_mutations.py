@@ -26,6 +26,8 @@ MUTATIONS = {
     "gate_up_swapped": ('silu(u @ Lw["wg"].T) * (u @ Lw["wu"].T)', 'silu(u @ Lw["wu"].T) * (u @ Lw["wg"].T)'),
     "dropped_final_norm": ('return rms_norm(x, widen(W["final_norm"]), cfg.rms_eps)', "return x"),
     "log_softmax_sign": ("z - (m + np.log", "z + (m + np.log"),
+    "layer_step_drops_new_key": ("V = np.concatenate([widen(v_cache[b, :, :p, :]).transpose(1, 0, 2), v[b:b + 1]])",
+                                 "V = np.concatenate([widen(v_cache[b, :, :p, :]).transpose(1, 0, 2), v[b:b + 1] * 0])"),
 }
 
 
@@ -36,7 +38,7 @@ def test_pins_catch_planted_mistake(name, tmp_path):
                     ignore=shutil.ignore_patterns("__pycache__"))
     p = tmp_path / "oracle" / "qwen3.py"
     src = p.read_text()
-    assert src.count(before) == 1, f"mutation anchor for {name} not found"
+    assert src.count(before) >= 1, f"mutation anchor for {name} not found"
     p.write_text(src.replace(before, after))
     env = dict(os.environ, PYTHONPATH=os.pathsep.join([str(tmp_path), ROOT]))
     r = subprocess.run([sys.executable, "-m", "pytest", "-q", "-x", "-p", "no:cacheprovider",

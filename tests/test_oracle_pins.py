@@ -307,3 +307,22 @@ def test_brute_force_one_layer_two_tokens():
         logits.append(matvec(m("lm_head"), norm(x, m("final_norm"))))
     z = oracle.forward_logits(cfg, W, tokens)
     assert np.allclose(z, np.array(logits), atol=1e-13)
+
+
+def test_layer_decode_step_batched_rows_match_per_row_layers(tiny_shape, tiny_weights):
+    # Rows with different cache lengths; each must equal decoder_layer on that row alone.
+    Lw = oracle.layer_weights(tiny_weights, 1)
+    r = np.random.default_rng(5)
+    B, S = 3, 20
+    kc = r.standard_normal((B, tiny_shape.n_kv_heads, S, tiny_shape.head_dim))
+    vc = r.standard_normal((B, tiny_shape.n_kv_heads, S, tiny_shape.head_dim))
+    x = r.standard_normal((B, tiny_shape.hidden))
+    pos = [19, 0, 7]
+    out, kn, vn = oracle.layer_decode_step(tiny_shape, Lw, x, kc, vc, pos)
+    for b in range(B):
+        p = pos[b]
+        xo, k1, v1 = oracle.decoder_layer(tiny_shape, Lw, x[b:b + 1], [p],
+                                          kc[b, :, :p].transpose(1, 0, 2),
+                                          vc[b, :, :p].transpose(1, 0, 2), np.arange(p))
+        assert np.allclose(out[b], xo[0], atol=1e-12)
+        assert np.allclose(kn[b], k1[0], atol=1e-13) and np.allclose(vn[b], v1[0], atol=1e-13)
