@@ -202,7 +202,6 @@ def run_ours(args, world, rank, local):
     from paper_2609_12471_gb300 import build as qkbuild
     qkbuild.build()
     import paper_2609_12471_gb300 as qk
-    from paper_2609_12471_gb300 import _binding
     from paper_2609_12471_gb300.runtime import Decoder
 
     torch.cuda.set_device(local)
@@ -229,32 +228,23 @@ def run_ours(args, world, rank, local):
 
     # ---- timed region: K whole rollouts, device-resident inputs
     n_layers = s.n_layers
-    _binding._load().qk_profile_begin.argtypes = [_binding._P, _binding._I, _binding._I]
-    lib = _binding._load()
-    lib.qk_profile_end.argtypes = [_binding._P, _binding.ctypes.POINTER(_binding.ctypes.c_float),
-                                   _binding.ctypes.POINTER(_binding._I)]
-    lib.qk_launch_count.restype = _binding.ctypes.c_uint64
-    if lib.qk_profile_begin(dec.handle, 2, args.steps * N * n_layers) != 0:  # QK_PROF_GATE_UP
-        raise RuntimeError(qk.qk_last_error())
+    qk.qk_profile_begin(dec.handle, qk.QK_PROF_GATE_UP, args.steps * N * n_layers)
     clocks = ClockSampler(local)
     barrier(world)
     torch.cuda.synchronize(dev)
-    launches0 = lib.qk_launch_count()
+    launches0 = qk.qk_launch_count()
     e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     e0.record(stream)
     for _ in range(args.steps):
         step()
     e1.record(stream)
     torch.cuda.synchronize(dev)
-    launches = lib.qk_launch_count() - launches0
+    launches = qk.qk_launch_count() - launches0
     barrier(world)
     clk = clocks.stop()
-    ms = e1.elapsed_time(e0) * -1 if False else e0.elapsed_time(e1)
+    ms = e0.elapsed_time(e1)
     ms_step = max_over_ranks(ms / args.steps, world)
-    prof_ms = _binding.ctypes.c_float()
-    prof_n = _binding._I()
-    if lib.qk_profile_end(dec.handle, _binding.ctypes.byref(prof_ms), _binding.ctypes.byref(prof_n)) != 0:
-        raise RuntimeError(qk.qk_last_error())
+    prof_ms, prof_n = qk.qk_profile_end(dec.handle)
     if dec.check_status() != 0:
         raise RuntimeError("device status flags set during the timed region")
     value = world * B * N / (ms_step / 1e3)
@@ -294,13 +284,13 @@ def run_ours(args, world, rank, local):
     hbm_peak = peaks["hbm_gbs"] if peaks else 6800.0
     c = dec.cfg
     gu_bytes = 2 * c.intermediate * c.hidden * 2 + B * c.hidden * 2 + B * c.intermediate * 2
-    avg_launch_s = (prof_ms.value / max(prof_n.value, 1)) / 1e3
+    avg_launch_s = (prof_ms / max(prof_n, 1)) / 1e3
     achieved = gu_bytes / avg_launch_s / 1e9
     roofline = {"bound": "hbm", "kernel": "decode gate/up linear + SwiGLU (M=16)",
                 "achieved": achieved, "peak": hbm_peak, "unit": "GB/s",
                 "frac": achieved / hbm_peak,
                 "peak_source": "measured" if peaks else "fallback",
-                "algorithmic_bytes_per_launch": gu_bytes, "launches_timed": prof_n.value,
+                "algorithmic_bytes_per_launch": gu_bytes, "launches_timed": prof_n,
                 "avg_launch_us": avg_launch_s * 1e6,
                 "traffic": recorded_traffic("gate_up_decode_b16")}
     step_bytes = 15136811008 + B * sum(P + j + 1 for j in range(N)) * 147456 / N

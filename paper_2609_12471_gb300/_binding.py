@@ -18,6 +18,8 @@ QK_OK, QK_EINVAL, QK_ESHAPE, QK_EDTYPE, QK_ECUDA, QK_ETIMEOUT, QK_EDEVICE, QK_EN
 QK_DTYPE_BF16, QK_DTYPE_F32 = 0, 1
 QK_STATUS_BAD_TOKEN, QK_STATUS_BAD_POS, QK_STATUS_TIMEOUT = 1, 2, 4
 QK_CALL_DECODE, QK_CALL_PREFILL, QK_CALL_SCORE, QK_CALL_ROLLOUT = 0, 1, 2, 3
+QK_PROF_QKV, QK_PROF_O, QK_PROF_GATE_UP, QK_PROF_DOWN, QK_PROF_ATTN, QK_PROF_LM_HEAD = range(6)
+QK_EPI_STORE, QK_EPI_STORE_F32, QK_EPI_RESID_F32, QK_EPI_SWIGLU = 0, 1, 2, 3
 
 __all__ = [
     "QK_OK", "QK_EINVAL", "QK_ESHAPE", "QK_EDTYPE", "QK_ECUDA", "QK_ETIMEOUT", "QK_EDEVICE",
@@ -26,7 +28,10 @@ __all__ = [
     "qk_config", "qk_config_preset", "qk_weight_count", "qk_model_packed_bytes", "qk_model_load",
     "qk_model_free", "qk_kv_bytes", "qk_workspace_bytes", "qk_prefill", "qk_decode_step",
     "qk_decode_layer", "qk_score_logprobs", "qk_rollout_teacher_forced", "qk_check_status",
-    "qk_last_error", "QKError", "lib_path", "exported_symbols",
+    "qk_last_error", "QKError", "lib_path", "exported_symbols", "qk_profile_begin",
+    "qk_profile_end", "qk_launch_count", "qk_op_linear", "QK_PROF_QKV", "QK_PROF_O",
+    "QK_PROF_GATE_UP", "QK_PROF_DOWN", "QK_PROF_ATTN", "QK_PROF_LM_HEAD", "QK_EPI_STORE",
+    "QK_EPI_STORE_F32", "QK_EPI_RESID_F32", "QK_EPI_SWIGLU",
 ]
 
 
@@ -69,6 +74,10 @@ _SIGS = {
     "qk_rollout_teacher_forced": ([_P, _P, _I, _I, _P, _I, _I, _I, _P, _P, _P, _SZ, _P], _I),
     "qk_check_status": ([_P, _P, ctypes.POINTER(ctypes.c_uint32)], _I),
     "qk_last_error": ([], ctypes.c_char_p),
+    "qk_profile_begin": ([_P, _I, _I], _I),
+    "qk_profile_end": ([_P, ctypes.POINTER(ctypes.c_float), ctypes.POINTER(_I)], _I),
+    "qk_launch_count": ([], ctypes.c_uint64),
+    "qk_op_linear": ([_P, _P, _I, _P, _P, _I, _I, _I, _I, _I, _P, _SZ, _P], _I),
 }
 
 _lib = None
@@ -213,3 +222,26 @@ def qk_check_status(m, stream=None) -> int:
     if rc not in (QK_OK, QK_EDEVICE):
         _check(rc)
     return v.value
+
+
+def qk_profile_begin(m, kind: int, max_launches: int):
+    _check(_load().qk_profile_begin(m, kind, max_launches))
+
+
+def qk_profile_end(m):
+    """Returns (total_ms, launches) of the bracketed kernel class."""
+    ms = ctypes.c_float()
+    n = _I()
+    _check(_load().qk_profile_end(m, ctypes.byref(ms), ctypes.byref(n)))
+    return ms.value, n.value
+
+
+def qk_launch_count() -> int:
+    return int(_load().qk_launch_count())
+
+
+def qk_op_linear(m, A, lda, W, C, ldc, M, N, K, epilogue, scratch=None, scratch_bytes=None,
+                 stream=None):
+    sb = 0 if scratch is None else _nbytes(scratch, scratch_bytes)
+    _check(_load().qk_op_linear(m, _ptr(A), lda, _ptr(W), _ptr(C), ldc, M, N, K, epilogue,
+                                _ptr(scratch), sb, _stream(stream)))

@@ -3,11 +3,20 @@
 
 namespace qk {
 
-void linear(const Model& m, const void* A, int lda, const void* W, void* C, int ldc, int M, int N,
+// bf16: up to 16 token rows stream the weights through the CUDA-core GEMV (the
+// layer is bound by reading W; tensor cores would idle), more rows go to the
+// tcgen05 GEMM.  fp32: CUDA-core GEMM (no TF32).
+void linear(Model& m, const void* A, int lda, const void* W, void* C, int ldc, int M, int N,
             int K, int epi, void* gu, cudaStream_t s) {
     const int dt = m.cfg.dtype;
     if (dt == QK_DTYPE_BF16 && M <= 16) {
         launch_gemv_bf16((const bf16*)A, lda, (const bf16*)W, C, ldc, M, N, K, epi, s);
+        return;
+    }
+    if (dt == QK_DTYPE_BF16 && gemm_tc_supported(A, lda, N, K)) {
+        int rc = launch_gemm_tc((const bf16*)A, lda, (const bf16*)W, C, ldc, M, N, K, epi,
+                                m.num_sms, m.status, s);
+        if (rc != QK_OK && !m.deferred_error) m.deferred_error = rc;
         return;
     }
     if (epi == EPI_SWIGLU) {

@@ -209,6 +209,15 @@ static int check_launch(const char* what) {
     return QK_OK;
 }
 
+static int check_launch(Model& m, const char* what) {
+    int rc = check_launch(what);
+    if (rc == QK_OK && m.deferred_error) {
+        rc = set_error(m.deferred_error, "%s: a tensor-map encode or kernel attribute call failed", what);
+    }
+    m.deferred_error = 0;
+    return rc;
+}
+
 static int get_ws(const Model& m, int kind, int B, int T, void* ws, size_t ws_bytes, Workspace* w) {
     QK_TRY(workspace_layout(m, kind, B, T, w, nullptr));
     if (!ws) return set_error(QK_EINVAL, "workspace is NULL");
@@ -415,6 +424,22 @@ int qk_profile_end(qk_model* mh, float* total_ms, int* launches) {
 
 uint64_t qk_launch_count(void) { return g_launches.load(); }
 
+int qk_op_linear(qk_model* mh, const void* A, int lda, const void* W, void* C, int ldc, int M,
+                 int N, int K, int epilogue, void* scratch, size_t scratch_bytes, void* stream) {
+    if (!mh || !A || !W || !C) return set_error(QK_EINVAL, "null argument");
+    Model& m = *(Model*)mh;
+    if (M < 1 || N < 1 || K < 16 || K % 16 || lda < K || (epilogue == QK_EPI_SWIGLU && N % 128))
+        return set_error(QK_ESHAPE, "bad linear shape M %d N %d K %d lda %d", M, N, K, lda);
+    if (epilogue < QK_EPI_STORE || epilogue > QK_EPI_SWIGLU)
+        return set_error(QK_EINVAL, "unknown epilogue %d", epilogue);
+    if (ldc < N) return set_error(QK_ESHAPE, "ldc %d < N %d", ldc, N);
+    size_t need = epilogue == QK_EPI_SWIGLU ? (size_t)M * 2 * N * m.es : 0;
+    if (need && (!scratch || scratch_bytes < need))
+        return set_error(QK_ENOSPACE, "linear scratch has %zu bytes, needs %zu", scratch_bytes, need);
+    linear(m, A, lda, W, C, ldc, M, N, K, epilogue, scratch, (cudaStream_t)stream);
+    return check_launch(m, "linear");
+}
+
 int qk_kv_bytes(const qk_model* mh, int max_batch, int max_seq, size_t* bytes) {
     if (!mh || !bytes) return set_error(QK_EINVAL, "null argument");
     const Model& m = *(const Model*)mh;
@@ -454,7 +479,7 @@ static int prefill_impl(Model& m, void* kv, int max_batch, int max_seq, TokIndex
     for (int l = 0; l < m.cfg.n_layers; ++l) run_layer(m, l, w, M, pos, view, s);
     if (last_logits || lp || am)
         run_head(m, w, B, T, T - 1, last_logits ? last_logits : w.logits, oi, lp, am, s);
-    return check_launch("prefill");
+    return check_launch(m, "prefill");
 }
 
 int qk_prefill(qk_model* mh, void* kv, int max_batch, int max_seq, const int32_t* tokens, int B,
@@ -483,7 +508,7 @@ static int decode_impl(Model& m, void* kv, int max_batch, int max_seq, TokIndex 
     for (int l = 0; l < m.cfg.n_layers; ++l) run_layer(m, l, w, B, pos, view, s);
     if (logits || lp || am) run_head(m, w, B, 1, 0, logits ? logits : w.logits, oi, lp, am, s);
     m.in_decode = false;
-    return check_launch("decode step");
+    return check_launch(m, "decode step");
 }
 
 int qk_decode_step(qk_model* mh, void* kv, int max_batch, int max_seq, const int32_t* tokens,
@@ -513,7 +538,7 @@ int qk_decode_layer(qk_model* mh, int layer, void* kv, int max_batch, int max_se
     run_layer(m, layer, w, B, PosIndex{pos, 0, 1}, cache_view(m, kv, max_batch, max_seq),
               (cudaStream_t)stream);
     m.in_decode = false;
-    return check_launch("decode layer");
+    return check_launch(m, "decode layer");
 }
 
 int qk_score_logprobs(qk_model* mh, const int32_t* tokens, int B, int T, float* logprobs,
@@ -545,7 +570,7 @@ int qk_score_logprobs(qk_model* mh, const int32_t* tokens, int B, int T, float* 
         OutIndex oi{T, T - 1, T - 1, 0, tokens, T, 1, r0};
         launch_logits_reduce(w.logits, rows, m.cfg.vocab, oi, logprobs, argmax, m.status, s);
     }
-    return check_launch("score");
+    return check_launch(m, "score");
 }
 
 int qk_rollout_teacher_forced(qk_model* mh, void* kv, int max_batch, int max_seq,

@@ -9,6 +9,7 @@
 #include <vector>
 
 #include "qk.h"
+#include "qk_ops.h"
 
 namespace qk {
 
@@ -59,6 +60,9 @@ struct Model {
     bool in_decode = false;
     std::vector<cudaEvent_t> prof_ev;
     int prof_used = 0;
+    // First host-side failure of a launch inside an orchestration (0 = none);
+    // reported and cleared by the entry point that made the launches.
+    int deferred_error = 0;
 };
 
 // Records the opening event of a bracketed launch; returns whether it did.
@@ -137,11 +141,15 @@ void launch_gemm_simt(const void* A, int lda, const void* W, void* C, int ldc, i
                       int K, int dtype, int epi, cudaStream_t s);
 void launch_gemv_bf16(const bf16* A, int lda, const bf16* W, void* C, int ldc, int M, int N,
                       int K, int epi, cudaStream_t s);
+// tcgen05 path (k_gemm_tc.cu): N % 128 == 0, K % 64 == 0, A 16-byte aligned, lda % 8 == 0.
+bool gemm_tc_supported(const void* A, int lda, int N, int K);
+int launch_gemm_tc(const bf16* A, int lda, const bf16* W, void* C, int ldc, int M, int N, int K,
+                   int epi, int num_sms, uint32_t* status, cudaStream_t s);
 
 // Kernel selection (k_dispatch.cu).  linear: C = A W^T with epilogue `epi`; for
 // EPI_SWIGLU, N is the SwiGLU width I and W holds 2 I interleaved rows; `gu` is
 // scratch [M, 2 I] for paths that cannot fuse the SwiGLU epilogue.
-void linear(const Model& m, const void* A, int lda, const void* W, void* C, int ldc, int M, int N,
+void linear(Model& m, const void* A, int lda, const void* W, void* C, int ldc, int M, int N,
             int K, int epi, void* gu, cudaStream_t s);
 void launch_attention(const Model& m, const void* q, int q_ld, const void* k_cache,
                       const void* v_cache, int M, int max_batch, int max_seq, PosIndex pos,
