@@ -33,6 +33,31 @@ extern "C" {
 int qk_op_linear(qk_model* m, const void* A, int lda, const void* W, void* C, int ldc, int M,
                  int N, int K, int epilogue, void* scratch, size_t scratch_bytes, void* stream);
 
+/* The QK_EPI_SWIGLU linear step on the CUDA-core path (the one that stages the
+ * [M, 2N] gate/up product in scratch before applying SwiGLU), for callers that
+ * cannot hand the library a scratch buffer: e.g. a process that reserved its
+ * whole device memory budget up front, or code embedded in a runtime that owns
+ * the allocator and forbids side allocations.  The paper has no counterpart;
+ * this is a service entry point of the library.
+ *
+ * It allocates nothing: the gate/up product lives in a file-scope device array
+ * of QK_STATIC_SCRATCH_BYTES (8 MiB) that every GPU loading libqk holds until
+ * the process exits.  Inputs and outputs are the caller's, as in qk_op_linear
+ * with QK_EPI_SWIGLU: A [M, K] (row stride lda), W [2N, K] (128-row gate/up
+ * blocks), C [M, N] with ldc == N, all in the model's dtype.
+ *  - Limit: M * 2N * element size must not exceed QK_STATIC_SCRATCH_BYTES;
+ *    larger calls return QK_ESHAPE and launch nothing.
+ *  - Set-up: the first call on each device looks up the array's device address
+ *    (cudaGetSymbolAddress, with that device current) and caches it; make that
+ *    first call before any stream capture.
+ *  - Sharing: every call on a device uses the same array and it keeps the last
+ *    call's contents (each call overwrites all of the part it reads, so nothing
+ *    needs clearing).  Calls that overlap on the GPU (other streams, other host
+ *    threads) race on the array; serialise them. */
+#define QK_STATIC_SCRATCH_BYTES (8u << 20)
+int qk_op_linear_swiglu_static(qk_model* m, const void* A, int lda, const void* W, void* C,
+                               int ldc, int M, int N, int K, void* stream);
+
 #ifdef __cplusplus
 }
 #endif

@@ -20,6 +20,7 @@ QK_STATUS_BAD_TOKEN, QK_STATUS_BAD_POS, QK_STATUS_TIMEOUT = 1, 2, 4
 QK_CALL_DECODE, QK_CALL_PREFILL, QK_CALL_SCORE, QK_CALL_ROLLOUT = 0, 1, 2, 3
 QK_PROF_QKV, QK_PROF_O, QK_PROF_GATE_UP, QK_PROF_DOWN, QK_PROF_ATTN, QK_PROF_LM_HEAD = range(6)
 QK_EPI_STORE, QK_EPI_STORE_F32, QK_EPI_RESID_F32, QK_EPI_SWIGLU = 0, 1, 2, 3
+QK_STATIC_SCRATCH_BYTES = 8 << 20
 
 __all__ = [
     "QK_OK", "QK_EINVAL", "QK_ESHAPE", "QK_EDTYPE", "QK_ECUDA", "QK_ETIMEOUT", "QK_EDEVICE",
@@ -31,7 +32,8 @@ __all__ = [
     "qk_last_error", "QKError", "lib_path", "exported_symbols", "qk_profile_begin",
     "qk_profile_end", "qk_launch_count", "qk_op_linear", "QK_PROF_QKV", "QK_PROF_O",
     "QK_PROF_GATE_UP", "QK_PROF_DOWN", "QK_PROF_ATTN", "QK_PROF_LM_HEAD", "QK_EPI_STORE",
-    "QK_EPI_STORE_F32", "QK_EPI_RESID_F32", "QK_EPI_SWIGLU",
+    "QK_EPI_STORE_F32", "QK_EPI_RESID_F32", "QK_EPI_SWIGLU", "qk_op_linear_swiglu_static",
+    "QK_STATIC_SCRATCH_BYTES",
 ]
 
 
@@ -78,6 +80,7 @@ _SIGS = {
     "qk_profile_end": ([_P, ctypes.POINTER(ctypes.c_float), ctypes.POINTER(_I)], _I),
     "qk_launch_count": ([], ctypes.c_uint64),
     "qk_op_linear": ([_P, _P, _I, _P, _P, _I, _I, _I, _I, _I, _P, _SZ, _P], _I),
+    "qk_op_linear_swiglu_static": ([_P, _P, _I, _P, _P, _I, _I, _I, _I, _P], _I),
 }
 
 _lib = None
@@ -245,3 +248,9 @@ def qk_op_linear(m, A, lda, W, C, ldc, M, N, K, epilogue, scratch=None, scratch_
     sb = 0 if scratch is None else _nbytes(scratch, scratch_bytes)
     _check(_load().qk_op_linear(m, _ptr(A), lda, _ptr(W), _ptr(C), ldc, M, N, K, epilogue,
                                 _ptr(scratch), sb, _stream(stream)))
+
+
+def qk_op_linear_swiglu_static(m, A, lda, W, C, ldc, M, N, K, stream=None):
+    """SwiGLU linear step with its gate/up intermediate in the library's static device array."""
+    _check(_load().qk_op_linear_swiglu_static(m, _ptr(A), lda, _ptr(W), _ptr(C), ldc, M, N, K,
+                                              _stream(stream)))
