@@ -33,6 +33,10 @@ B, P, N = 16, 512, 1024
 WORKLOAD = ("qwen3-8b-shaped bf16 rollout decode: batch 16, prompt 512 random tokens, "
             "1024 teacher-forced decode steps, per-token log-probs")
 ORACLE_TOKENS = 32  # tokens of rollout row 0 the CPU oracle scores per sample
+# Scoring 32 x 4096 (all 36 layers): linear layers 2 * 131072 * 6.946e9 params, lm_head over
+# 4095 scored positions per row (the kernel evaluates all 4096), causal attention.
+SCORE_FLOPS = (2 * 32 * 4096 * (36 * 192937984) + 2 * 32 * 4096 * 151936 * 4096
+               + 36 * 32 * 32 * 2 * 2 * 128 * (4096 * 4097 // 2))
 
 
 def parse():
@@ -64,13 +68,21 @@ def barrier(world):
 
 
 def max_over_ranks(v: float, world: int) -> float:
+    """Largest value over the ranks (the job's time is its slowest replica's)."""
     if world == 1:
         return v
     import torch
     import torch.distributed as dist
-    t = torch.tensor([v], dtype=torch.float64, device="cuda")
+    dev = "cuda" if dist.get_backend() == "nccl" else "cpu"
+    t = torch.tensor([v], dtype=torch.float64, device=dev)
     dist.all_reduce(t, op=dist.ReduceOp.MAX)
     return float(t.item())
+
+
+def replica_tokens(vocab: int, rank: int):
+    """Rollout batch of replica `rank`: its own seeded token stream (weights are shared)."""
+    import synth
+    return synth.tokens((B, P + N + 1), vocab, stream=rank)
 
 
 class ClockSampler:
@@ -211,7 +223,7 @@ def run_ours(args, world, rank, local):
     W = synth.LazyWeights(s, cache=want_cpu)
     names = [t[0] for t in synth.tensor_list(s)]
     dec = Decoder(qk.qk_config_preset("q8b"), (W[n] for n in names), device=dev)
-    seq = synth.tokens((B, P + N + 1), s.vocab, stream=rank)
+    seq = replica_tokens(s.vocab, rank)
     seq_d = torch.tensor(seq, dtype=torch.int32, device=dev)
     kv = dec.new_kv(B, P + N)
     lp = torch.empty(B, N + 1, dtype=torch.float32, device=dev)
@@ -278,15 +290,37 @@ def run_ours(args, world, rank, local):
     if not (np.all(np.isfinite(lp_np)) and np.all(lp_np <= 1e-4)):
         raise RuntimeError("log-probs out of range")
 
+    # ---- scoring pass (teacher-forced log-probs of 32 x 4096 tokens): secondary figure
+    SB, ST = 32, 4096
+    score_tok = torch.tensor(synth.tokens((SB, ST), s.vocab, stream=100 + rank), dtype=torch.int32,
+                             device=dev)
+    score_lp = torch.empty(SB, ST - 1, dtype=torch.float32, device=dev)
+    dec.score(score_tok, logprobs=score_lp)  # warm-up
+    torch.cuda.synchronize(dev)
+    s0, s1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    n_score = 2
+    s0.record(stream)
+    for _ in range(n_score):
+        dec.score(score_tok, logprobs=score_lp)
+    s1.record(stream)
+    torch.cuda.synchronize(dev)
+    score_s = max_over_ranks(s0.elapsed_time(s1) / n_score / 1e3, world)
+    if dec.check_status() != 0 or not torch.isfinite(score_lp).all():
+        raise RuntimeError("scoring produced invalid output")
+    del score_tok, score_lp
+
     if rank != 0:
         return
     peaks = measured_peaks()
     hbm_peak = peaks["hbm_gbs"] if peaks else 6800.0
+    bf16_peak = peaks["bf16_tflops"] if peaks else 1900.0
     c = dec.cfg
     gu_bytes = 2 * c.intermediate * c.hidden * 2 + B * c.hidden * 2 + B * c.intermediate * 2
     avg_launch_s = (prof_ms / max(prof_n, 1)) / 1e3
     achieved = gu_bytes / avg_launch_s / 1e9
-    roofline = {"bound": "hbm", "kernel": "decode gate/up linear + SwiGLU (M=16)",
+    roofline = {"bound": "hbm", "kernel": "decode gate/up linear (tcgen05 split-K GEMM, 16 token rows)",
+                "timed_launches": "the gate/up launches of each timed rollout's first decode step "
+                                  "(later steps replay a captured CUDA graph without event nodes)",
                 "achieved": achieved, "peak": hbm_peak, "unit": "GB/s",
                 "frac": achieved / hbm_peak,
                 "peak_source": "measured" if peaks else "fallback",
@@ -301,8 +335,16 @@ def run_ours(args, world, rank, local):
                        "l2": "inputs larger than L2: 15.1 GB of weights streamed per decode step",
                        "replicas": world},
             "prefill_tokens_per_s": world * B * P / (prefill_ms / 1e3),
+            "score_tokens_per_s": world * SB * ST / score_s,
+            "score_roofline": {"bound": "tensor", "workload": "scoring 32 x 4096 tokens",
+                               "flops_per_call": SCORE_FLOPS,
+                               "achieved": SCORE_FLOPS / score_s / 1e12,
+                               "peak": bf16_peak, "unit": "TFLOP/s",
+                               "frac": SCORE_FLOPS / score_s / 1e12 / bf16_peak,
+                               "peak_source": "measured (burst)" if peaks else "fallback"},
             "decode_hbm_fraction_of_8tbs": (step_bytes * N / 1e9) / ((ms_step - prefill_ms) / 1e3) / 8000.0,
             "roofline": roofline, "clocks": clk, "gpu_launches": int(launches),
+            "launches_before_timed": int(launches0),
             "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": int(seq.nbytes),
                     "d2h_bytes_per_step": int(lp_h.numel() * 4)}}
     if want_cpu:

@@ -174,7 +174,7 @@ int qk_check_status(qk_model* m, void* stream, uint32_t* flags);
  * qk_rollout_teacher_forced, qk_decode_layer) are bracketed. */
 #define QK_PROF_QKV 0      /* RMSNorm'd input x W_qkv                     */
 #define QK_PROF_O 1        /* attention output x W_o + residual           */
-#define QK_PROF_GATE_UP 2  /* x W_gate, x W_up, SwiGLU                    */
+#define QK_PROF_GATE_UP 2  /* x W_gate, x W_up (with SwiGLU when fused)    */
 #define QK_PROF_DOWN 3     /* h x W_down + residual                       */
 #define QK_PROF_ATTN 4     /* decode attention (all its kernels)          */
 #define QK_PROF_LM_HEAD 5  /* final RMSNorm'd x W_lm (logits)             */

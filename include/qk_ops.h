@@ -28,7 +28,7 @@ extern "C" {
  * for QK_EPI_SWIGLU), C [M, ldc].  This is the step the Qwen3 layer uses for its
  * QKV, output, gate/up and down projections and for the lm_head (logits =
  * W_lm h).  scratch: device buffer of M * 2N elements of the model dtype, needed
- * only for QK_EPI_SWIGLU on the fp32 model (else may be NULL).  K must be a
+ * only for QK_EPI_SWIGLU on the fp32 model (else may be NULL and is ignored).  K must be a
  * multiple of 16, N of 128 for QK_EPI_SWIGLU. */
 int qk_op_linear(qk_model* m, const void* A, int lda, const void* W, void* C, int ldc, int M,
                  int N, int K, int epilogue, void* scratch, size_t scratch_bytes, void* stream);

@@ -42,6 +42,7 @@ __global__ void attention_simt_kernel(const T* __restrict__ q, int q_ld, const T
                                       PosIndex pos, T* __restrict__ o, uint32_t* status) {
     constexpr int E = D / 32;
     extern __shared__ float qs[];  // [warps][D]
+    pdl_wait();
     int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     int group = nq / nkv;
     int r = blockIdx.x, kvh = blockIdx.y, h = kvh * group + warp;
@@ -104,9 +105,8 @@ void launch_attention_simt(const void* q, int q_ld, const void* k_cache, const v
     int threads = 32 * group;
     size_t smem = (size_t)group * d * sizeof(float);
 #define QK_ATT(T, D)                                                                           \
-    attention_simt_kernel<T, D><<<grid, threads, smem, s>>>((const T*)q, q_ld, (const T*)k_cache,    \
-                                                            (const T*)v_cache, nq, nkv,       \
-                                                            max_seq, pos, (T*)o, status)
+    launch_k(attention_simt_kernel<T, D>, grid, dim3(threads), smem, s, (const T*)q, q_ld,    \
+             (const T*)k_cache, (const T*)v_cache, nq, nkv, max_seq, pos, (T*)o, status)
     if (dtype == QK_DTYPE_BF16) {
         if (d == 128) QK_ATT(bf16, 128); else QK_ATT(bf16, 64);
     } else {

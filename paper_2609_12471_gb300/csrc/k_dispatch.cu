@@ -3,13 +3,13 @@
 
 namespace qk {
 
-// bf16: up to 16 token rows stream the weights through the CUDA-core GEMV (the
-// layer is bound by reading W; tensor cores would idle), more rows go to the
-// tcgen05 GEMM.  fp32: CUDA-core GEMM (no TF32).
+// bf16: up to kGemvMaxRows token rows stream the weights through the CUDA-core
+// GEMV (bound by reading W), more rows go to the tcgen05 GEMM.  fp32: CUDA-core
+// GEMM (no TF32).
 void linear(Model& m, const void* A, int lda, const void* W, void* C, int ldc, int M, int N,
             int K, int epi, void* gu, cudaStream_t s) {
     const int dt = m.cfg.dtype;
-    if (dt == QK_DTYPE_BF16 && M <= 16) {
+    if (dt == QK_DTYPE_BF16 && M <= kGemvMaxRows) {
         launch_gemv_bf16((const bf16*)A, lda, (const bf16*)W, C, ldc, M, N, K, epi, s);
         return;
     }
@@ -27,11 +27,30 @@ void linear(Model& m, const void* A, int lda, const void* W, void* C, int ldc, i
     launch_gemm_simt(A, lda, W, C, ldc, M, N, K, dt, epi, s);
 }
 
-void launch_attention(const Model& m, const void* q, int q_ld, const void* k_cache,
-                      const void* v_cache, int M, int max_batch, int max_seq, PosIndex pos,
-                      void* o, cudaStream_t s) {
-    (void)max_batch;
+void launch_attention(Model& m, const void* q, int q_ld, const void* k_cache, const void* v_cache,
+                      int M, int max_batch, int max_seq, PosIndex pos, void* o, void* scratch,
+                      cudaStream_t s) {
     const qk_config& c = m.cfg;
+    if (c.dtype == QK_DTYPE_BF16 && pos.T == 1 && scratch &&
+        attn_decode_supported(c.head_dim, c.n_q_heads, c.n_kv_heads) &&
+        (const char*)v_cache == (const char*)k_cache + (size_t)max_batch * c.n_kv_heads * max_seq *
+                                                            c.head_dim * 2) {
+        int rc = launch_attn_decode((const bf16*)q, q_ld, k_cache, c.n_q_heads, c.n_kv_heads,
+                                    max_batch, max_seq, M, pos, scratch, (bf16*)o, m.num_sms,
+                                    m.status, s);
+        if (rc != QK_OK && !m.deferred_error) m.deferred_error = rc;
+        return;
+    }
+    if (c.dtype == QK_DTYPE_BF16 && pos.T > 1 && !pos.pos_dev &&
+        attn_prefill_supported(c.head_dim, c.n_q_heads, c.n_kv_heads) &&
+        (const char*)v_cache == (const char*)k_cache + (size_t)max_batch * c.n_kv_heads * max_seq *
+                                                            c.head_dim * 2) {
+        int rc = launch_attn_prefill((const bf16*)q, q_ld, k_cache, c.n_q_heads, c.n_kv_heads,
+                                     max_batch, max_seq, M / pos.T, pos.T, pos.start, (bf16*)o,
+                                     m.status, s);
+        if (rc != QK_OK && !m.deferred_error) m.deferred_error = rc;
+        return;
+    }
     launch_attention_simt(q, q_ld, k_cache, v_cache, c.dtype, M, c.n_q_heads, c.n_kv_heads,
                           c.head_dim, max_seq, pos, o, m.status, s);
 }

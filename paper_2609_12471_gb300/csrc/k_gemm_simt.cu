@@ -38,6 +38,7 @@ __global__ void __launch_bounds__(256) gemm_simt_kernel(const T* __restrict__ A,
     constexpr int BM = 64, BN = 64, BK = 16;
     __shared__ float As[BK][BM + 4];
     __shared__ float Ws[BK][BN + 4];
+    pdl_wait();
     int tid = threadIdx.x;
     int tx = tid % 16, ty = tid / 16;
     int m0 = blockIdx.y * BM, n0 = blockIdx.x * BN;
@@ -110,6 +111,7 @@ __global__ void __launch_bounds__(256) gemv_bf16_kernel(const bf16* __restrict__
                                                         int K, int epi) {
     constexpr int NR = SW ? 2 * R : R;
     constexpr int U = 2;
+    pdl_wait();
     int lane = threadIdx.x & 31;
     int f0 = (blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5)) * R;
     if (f0 >= N) return;
@@ -190,9 +192,11 @@ void gemv_dispatch(const bf16* A, int lda, const bf16* W, void* C, int ldc, int 
     int warps = (N + R - 1) / R;
     int blocks = (warps + 7) / 8;
     if (epi == EPI_SWIGLU)
-        gemv_bf16_kernel<MT, R, true><<<blocks, 256, 0, s>>>(A, lda, W, C, ldc, N, K, epi);
+        launch_k(gemv_bf16_kernel<MT, R, true>, dim3(blocks), dim3(256), 0, s, A, lda, W, C, ldc, N,
+                 K, epi);
     else
-        gemv_bf16_kernel<MT, R, false><<<blocks, 256, 0, s>>>(A, lda, W, C, ldc, N, K, epi);
+        launch_k(gemv_bf16_kernel<MT, R, false>, dim3(blocks), dim3(256), 0, s, A, lda, W, C, ldc, N,
+                 K, epi);
 }
 
 }  // namespace
@@ -203,14 +207,14 @@ void launch_gemm_simt(const void* A, int lda, const void* W, void* C, int ldc, i
     if (M <= 0 || N <= 0) return;
     dim3 grid((N + 63) / 64, (M + 63) / 64);
     if (dtype == QK_DTYPE_BF16)
-        gemm_simt_kernel<bf16><<<grid, 256, 0, s>>>((const bf16*)A, lda, (const bf16*)W, C, ldc,
-                                                     M, N, K, epi);
+        launch_k(gemm_simt_kernel<bf16>, grid, dim3(256), 0, s, (const bf16*)A, lda,
+                 (const bf16*)W, C, ldc, M, N, K, epi);
     else
-        gemm_simt_kernel<float><<<grid, 256, 0, s>>>((const float*)A, lda, (const float*)W, C,
-                                                      ldc, M, N, K, epi);
+        launch_k(gemm_simt_kernel<float>, grid, dim3(256), 0, s, (const float*)A, lda,
+                 (const float*)W, C, ldc, M, N, K, epi);
 }
 
-// M <= 16 token rows; N output features (I for SwiGLU).
+// M <= 16 token rows (the model uses it up to kGemvMaxRows); N output features (I for SwiGLU).
 void launch_gemv_bf16(const bf16* A, int lda, const bf16* W, void* C, int ldc, int M, int N,
                       int K, int epi, cudaStream_t s) {
     note_launch();

@@ -57,7 +57,7 @@ __device__ __forceinline__ float silu(float g) { return g / (1.f + __expf(-g)); 
 template <int BN, bool SWIGLU, int STAGES>
 __global__ void __launch_bounds__(kThreads, 1)
     gemm_tc_kernel(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ CUtensorMap tmX,
-                   void* __restrict__ C, int ldc, int M, int N, int K, int epi,
+                   void* __restrict__ C, int ldc, int M, int N, int K, int epi, int n_split,
                    uint32_t* __restrict__ status) {
     using G = Cfg<BN, SWIGLU, STAGES>;
     extern __shared__ uint8_t smem_raw[];
@@ -75,7 +75,9 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int n_feat = N / 128;
     const int n_tok = (M + BN - 1) / BN;
-    const int num_tiles = n_feat * n_tok;
+    // Work unit t = ((feat * n_tok) + tok) * n_split + split; a split covers k-blocks
+    // [split * kblocks / n_split, (split + 1) * kblocks / n_split).
+    const int num_tiles = n_feat * n_tok * n_split;
     const int kblocks = K / kBK;
 
     if (threadIdx.x == 0) {
@@ -98,6 +100,10 @@ __global__ void __launch_bounds__(kThreads, 1)
     __syncthreads();
     tc::fence_after_sync();
     const uint32_t tmem_base = *tmem_slot;
+    // Everything above touched only shared memory and TMEM.  The producer thread
+    // waits for the previous kernel after it has issued the first ring of weight
+    // tiles (weights are never written by a kernel); every other thread waits now.
+    if (!(warp == 0 && lane == 0)) pdl_wait();
 
     if (warp == 0) {
         if (lane == 0) {
@@ -107,9 +113,23 @@ __global__ void __launch_bounds__(kThreads, 1)
             int armed[STAGES];
             for (int s = 0; s < STAGES; ++s) armed[s] = -1;
             bool ok = true;
+            // activation loads held back until the dependency wait: (stage, x, y)
+            int pend_stage[STAGES], pend_x[STAGES], pend_y[STAGES];
+            int npend = 0;
+            bool waited = false;
+            auto release_pending = [&]() {
+                pdl_wait();
+                waited = true;
+                for (int i = 0; i < npend; ++i)
+                    tc::tma_load_2d(sB + pend_stage[i] * G::B_BYTES, &tmX, pend_x[i], pend_y[i],
+                                    &full[pend_stage[i]]);
+                npend = 0;
+            };
             for (int t = blockIdx.x; ok && t < num_tiles; t += gridDim.x) {
-                const int feat = t / n_tok, tok = t % n_tok;
-                for (int kb = 0; kb < kblocks; ++kb) {
+                const int split = t % n_split, rest = t / n_split;
+                const int feat = rest / n_tok, tok = rest % n_tok;
+                const int kb0 = split * kblocks / n_split, kb1 = (split + 1) * kblocks / n_split;
+                for (int kb = kb0; kb < kb1; ++kb) {
                     if (!tc::mbar_wait(&empty[stage], phase ^ 1, abort_flag)) {
                         ok = false;
                         break;
@@ -117,7 +137,15 @@ __global__ void __launch_bounds__(kThreads, 1)
                     tc::mbar_expect_tx(&full[stage], G::A_BYTES + G::B_BYTES);
                     tc::tma_load_2d(sA + stage * G::A_BYTES, &tmW, kb * kBK, feat * G::A_ROWS,
                                     &full[stage]);
-                    tc::tma_load_2d(sB + stage * G::B_BYTES, &tmX, kb * kBK, tok * BN, &full[stage]);
+                    if (waited) {
+                        tc::tma_load_2d(sB + stage * G::B_BYTES, &tmX, kb * kBK, tok * BN,
+                                        &full[stage]);
+                    } else {
+                        pend_stage[npend] = stage;
+                        pend_x[npend] = kb * kBK;
+                        pend_y[npend] = tok * BN;
+                        if (++npend == STAGES) release_pending();
+                    }
                     armed[stage] = (int)phase;
                     if (++stage == STAGES) {
                         stage = 0;
@@ -125,6 +153,8 @@ __global__ void __launch_bounds__(kThreads, 1)
                     }
                 }
             }
+            if (!waited) release_pending();
+            pdl_trigger();  // every load of this CTA is issued: the next kernel may be scheduled
             if (!ok) {  // abort path: let every copy this thread issued land before exit
                 for (int s = 0; s < STAGES; ++s)
                     if (armed[s] >= 0) tc::mbar_wait_drain(&full[s], (uint32_t)armed[s]);
@@ -140,13 +170,15 @@ __global__ void __launch_bounds__(kThreads, 1)
             uint32_t acc_phase = 0;
             bool ok = true, issued = false;
             for (int t = blockIdx.x; ok && t < num_tiles; t += gridDim.x) {
+                const int split = t % n_split;
+                const int kb0 = split * kblocks / n_split, kb1 = (split + 1) * kblocks / n_split;
                 if (!tc::mbar_wait(&tempty[acc], acc_phase ^ 1, abort_flag)) {
                     ok = false;
                     break;
                 }
                 tc::fence_after_sync();
                 const uint32_t d = tmem_base + (uint32_t)(acc * G::ACC_COLS);
-                for (int kb = 0; kb < kblocks; ++kb) {
+                for (int kb = kb0; kb < kb1; ++kb) {
                     if (!tc::mbar_wait(&full[stage], phase, abort_flag)) {
                         ok = false;
                         break;
@@ -157,7 +189,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
                     for (int k = 0; k < kBK / 16; ++k) {
                         const uint64_t bd = tc::sw128_desc(b0 + k * 32);
-                        const uint32_t accum = (kb | k) ? 1u : 0u;
+                        const uint32_t accum = (kb != kb0 || k) ? 1u : 0u;
                         tc::mma_bf16(d, tc::sw128_desc(a0 + k * 32), bd, idesc, accum);
                         if (SWIGLU)
                             tc::mma_bf16(d + BN, tc::sw128_desc(a0 + 128 * 128 + k * 32), bd, idesc,
@@ -186,7 +218,8 @@ __global__ void __launch_bounds__(kThreads, 1)
         int acc = 0;
         uint32_t acc_phase = 0;
         for (int t = blockIdx.x; t < num_tiles; t += gridDim.x) {
-            const int feat = t / n_tok, tok = t % n_tok;
+            const int split = t % n_split, rest = t / n_split;
+            const int feat = rest / n_tok, tok = rest % n_tok;
             bool ok = tc::mbar_wait(&tfull[acc], acc_phase, abort_flag);
             ok = __all_sync(0xffffffffu, ok);
             if (!ok) break;
@@ -209,6 +242,8 @@ __global__ void __launch_bounds__(kThreads, 1)
                     const float v = __uint_as_float(r[j]);
                     if (SWIGLU) {
                         ((bf16*)C)[o] = __float2bfloat16_rn(silu(v) * __uint_as_float(u[j]));
+                    } else if (epi == EPI_PARTIAL_F32) {
+                        ((float*)C)[(size_t)split * M * ldc + o] = v;
                     } else if (epi == EPI_STORE_ACT) {
                         ((bf16*)C)[o] = __float2bfloat16_rn(v);
                     } else if (epi == EPI_STORE_F32) {
@@ -272,7 +307,7 @@ bool make_map(CUtensorMap* map, const void* base, int inner, int rows, int ld, i
 
 template <int BN, bool SWIGLU, int STAGES>
 int launch_cfg(const bf16* A, int lda, const bf16* W, void* C, int ldc, int M, int N, int K,
-               int epi, int num_sms, uint32_t* status, cudaStream_t s) {
+               int epi, int n_split, int num_sms, uint32_t* status, cudaStream_t s) {
     using G = Cfg<BN, SWIGLU, STAGES>;
     static bool attr_set = false;
     if (!attr_set) {
@@ -285,10 +320,10 @@ int launch_cfg(const bf16* A, int lda, const bf16* W, void* C, int ldc, int M, i
     const int w_rows = SWIGLU ? 2 * N : N;
     if (!make_map(&tmW, W, K, w_rows, K, G::A_ROWS) || !make_map(&tmX, A, K, M, lda, BN))
         return QK_ECUDA;
-    const int tiles = (N / 128) * ((M + BN - 1) / BN);
+    const int tiles = (N / 128) * ((M + BN - 1) / BN) * n_split;
     const int grid = tiles < num_sms ? tiles : num_sms;
-    gemm_tc_kernel<BN, SWIGLU, STAGES>
-        <<<grid, kThreads, G::SMEM, s>>>(tmW, tmX, C, ldc, M, N, K, epi, status);
+    launch_k(gemm_tc_kernel<BN, SWIGLU, STAGES>, dim3(grid), dim3(kThreads), G::SMEM, s, tmW, tmX, C,
+             ldc, M, N, K, epi, n_split, status);
     note_launch();
     return QK_OK;
 }
@@ -305,14 +340,51 @@ int launch_gemm_tc(const bf16* A, int lda, const bf16* W, void* C, int ldc, int 
                    int epi, int num_sms, uint32_t* status, cudaStream_t s) {
     if (M <= 0) return QK_OK;
     if (epi == EPI_SWIGLU) {
-        if (M <= 32) return launch_cfg<32, true, 6>(A, lda, W, C, ldc, M, N, K, epi, num_sms, status, s);
-        if (M <= 64) return launch_cfg<64, true, 5>(A, lda, W, C, ldc, M, N, K, epi, num_sms, status, s);
-        return launch_cfg<128, true, 4>(A, lda, W, C, ldc, M, N, K, epi, num_sms, status, s);
+        if (M <= 16) return launch_cfg<16, true, 6>(A, lda, W, C, ldc, M, N, K, epi, 1, num_sms, status, s);
+        if (M <= 32) return launch_cfg<32, true, 6>(A, lda, W, C, ldc, M, N, K, epi, 1, num_sms, status, s);
+        if (M <= 64) return launch_cfg<64, true, 5>(A, lda, W, C, ldc, M, N, K, epi, 1, num_sms, status, s);
+        return launch_cfg<128, true, 4>(A, lda, W, C, ldc, M, N, K, epi, 1, num_sms, status, s);
     }
-    if (M <= 32) return launch_cfg<32, false, 8>(A, lda, W, C, ldc, M, N, K, epi, num_sms, status, s);
-    if (M <= 64) return launch_cfg<64, false, 8>(A, lda, W, C, ldc, M, N, K, epi, num_sms, status, s);
-    if (M <= 128) return launch_cfg<128, false, 6>(A, lda, W, C, ldc, M, N, K, epi, num_sms, status, s);
-    return launch_cfg<256, false, 4>(A, lda, W, C, ldc, M, N, K, epi, num_sms, status, s);
+    if (M <= 16) return launch_cfg<16, false, 8>(A, lda, W, C, ldc, M, N, K, epi, 1, num_sms, status, s);
+    if (M <= 32) return launch_cfg<32, false, 8>(A, lda, W, C, ldc, M, N, K, epi, 1, num_sms, status, s);
+    if (M <= 64) return launch_cfg<64, false, 8>(A, lda, W, C, ldc, M, N, K, epi, 1, num_sms, status, s);
+    if (M <= 128) return launch_cfg<128, false, 6>(A, lda, W, C, ldc, M, N, K, epi, 1, num_sms, status, s);
+    return launch_cfg<256, false, 4>(A, lda, W, C, ldc, M, N, K, epi, 1, num_sms, status, s);
+}
+
+// Split count for a decode-sized GEMM (one token tile): the smallest S whose
+// N/128 * S work units fill the persistent grid to >= 90 % of its last round,
+// with at least 4 k-blocks per unit; the best S found otherwise.
+int gemm_tc_split(int N, int K, int num_sms) {
+    const int n_feat = N / 128, kblocks = K / kBK;
+    int best = 1;
+    double best_eff = 0.0;
+    for (int S = 1; S <= 32 && kblocks / S >= 4; ++S) {
+        const int units = n_feat * S;
+        const int rounds = (units + num_sms - 1) / num_sms;
+        const double eff = (double)units / ((double)rounds * num_sms);
+        if (eff >= 0.9) return S;
+        if (eff > best_eff + 1e-9) {
+            best_eff = eff;
+            best = S;
+        }
+    }
+    return best;
+}
+
+// Decode-sized linear (M <= 64 rows) split over K: unit `split` writes its fp32 partial
+// product to part[split][M][N]; consumers add the n_split partials in order.
+int launch_gemm_tc_splitk(const bf16* A, int lda, const bf16* W, float* part, int M, int N, int K,
+                          int n_split, int num_sms, uint32_t* status, cudaStream_t s) {
+    if (M <= 0) return QK_OK;
+    if (M <= 16)
+        return launch_cfg<16, false, 8>(A, lda, W, part, N, M, N, K, EPI_PARTIAL_F32, n_split,
+                                        num_sms, status, s);
+    if (M <= 32)
+        return launch_cfg<32, false, 8>(A, lda, W, part, N, M, N, K, EPI_PARTIAL_F32, n_split,
+                                        num_sms, status, s);
+    return launch_cfg<64, false, 8>(A, lda, W, part, N, M, N, K, EPI_PARTIAL_F32, n_split,
+                                    num_sms, status, s);
 }
 
 }  // namespace qk

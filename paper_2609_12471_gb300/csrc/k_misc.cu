@@ -1,6 +1,7 @@
 // Elementwise and row-wise kernels of the decoder forward pass: embedding
 // gather, RMSNorm, per-head QK-RMSNorm + RoPE + KV-cache write, SwiGLU,
 // vocabulary log-softmax / gather / argmax, and the load-time RoPE table.
+#include <cooperative_groups.h>
 #include <math.h>
 
 #include "qk_internal.cuh"
@@ -34,6 +35,7 @@ __device__ float block_sum(float v, float* red) {
 template <typename T>
 __global__ void embed_kernel(const T* __restrict__ E, int V, int H, TokIndex tok,
                              float* __restrict__ x, uint32_t* status) {
+    pdl_wait();
     int r = blockIdx.x;
     int id = tok.ptr[(size_t)(r / tok.T) * tok.ld + tok.off + r % tok.T];
     if (id < 0 || id >= V) {
@@ -50,9 +52,9 @@ void launch_embed(const void* E, int dtype, int V, int H, TokIndex tok, int M, f
     note_launch();
     if (M <= 0) return;
     if (dtype == QK_DTYPE_BF16)
-        embed_kernel<bf16><<<M, 256, 0, s>>>((const bf16*)E, V, H, tok, x, status);
+        launch_k(embed_kernel<bf16>, dim3(M), dim3(256), 0, s, (const bf16*)E, V, H, tok, x, status);
     else
-        embed_kernel<float><<<M, 256, 0, s>>>((const float*)E, V, H, tok, x, status);
+        launch_k(embed_kernel<float>, dim3(M), dim3(256), 0, s, (const float*)E, V, H, tok, x, status);
 }
 
 // ---------------------------------------------------------------- RMSNorm
@@ -61,6 +63,7 @@ __global__ void rmsnorm_kernel(const float* __restrict__ x, int in_step, int in_
                                const float* __restrict__ g, int H, float eps,
                                OutT* __restrict__ out) {
     __shared__ float red[32];
+    pdl_wait();
     int r = blockIdx.x;
     const float* xr = x + ((size_t)r * in_step + in_off) * H;
     float ss = 0.f;
@@ -81,26 +84,130 @@ __global__ void rmsnorm_kernel(const float* __restrict__ x, int in_step, int in_
     }
 }
 
+// x[r] += sum_{s < S} part[s][r] (fixed order), written back; then out[r] = RMSNorm(x[r]) * g.
+// Folds the residual add of a split-K linear into the norm that reads the residual next.
+// A row is spread over a cluster of CL CTAs (128 threads, 4 consecutive elements per
+// thread and pass); each CTA reduces the sum of squares of its slice and the CTAs of
+// the cluster exchange those sums through distributed shared memory.
+__global__ void __launch_bounds__(128)
+    rmsnorm_resid_kernel(float* __restrict__ x, const float* __restrict__ part, int S,
+                         size_t split_stride, const float* __restrict__ g, int H, float eps,
+                         bf16* __restrict__ out) {
+    namespace cg = cooperative_groups;
+    cg::cluster_group cluster = cg::this_cluster();
+    __shared__ float red[4];
+    __shared__ float slice_ss;
+    pdl_wait();
+    const int CL = (int)cluster.num_blocks();
+    const int rank = (int)cluster.block_rank();
+    const int r = blockIdx.y;
+    const int slice = H / CL;
+    float* xr = x + (size_t)r * H + (size_t)rank * slice;
+    const float* pr = part + (size_t)r * H + (size_t)rank * slice;
+    float ss = 0.f;
+    for (int i = threadIdx.x * 4; i < slice; i += blockDim.x * 4) {
+        float4 v = *reinterpret_cast<const float4*>(xr + i);
+        for (int sp = 0; sp < S; ++sp) {
+            float4 a = *reinterpret_cast<const float4*>(pr + sp * split_stride + i);
+            v.x += a.x; v.y += a.y; v.z += a.z; v.w += a.w;
+        }
+        if (S > 0) *reinterpret_cast<float4*>(xr + i) = v;
+        ss += v.x * v.x + v.y * v.y + v.z * v.z + v.w * v.w;
+    }
+    ss = warp_sum(ss);
+    if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = ss;
+    __syncthreads();
+    if (threadIdx.x == 0) slice_ss = red[0] + red[1] + red[2] + red[3];
+    cluster.sync();
+    float tot = 0.f;
+    for (int c = 0; c < CL; ++c) tot += *cluster.map_shared_rank(&slice_ss, c);
+    const float scale = rsqrtf(tot / (float)H + eps);
+    bf16* o = out + (size_t)r * H + (size_t)rank * slice;
+    const float* gg = g + (size_t)rank * slice;
+    for (int i = threadIdx.x * 4; i < slice; i += blockDim.x * 4) {
+        float4 v = *reinterpret_cast<const float4*>(xr + i);
+        float4 w = *reinterpret_cast<const float4*>(gg + i);
+        o[i + 0] = __float2bfloat16_rn(v.x * scale * w.x);
+        o[i + 1] = __float2bfloat16_rn(v.y * scale * w.y);
+        o[i + 2] = __float2bfloat16_rn(v.z * scale * w.z);
+        o[i + 3] = __float2bfloat16_rn(v.w * scale * w.w);
+    }
+    cluster.sync();  // keep this CTA's slice_ss alive until every peer has read it
+}
+
+// Cluster size: up to 8 CTAs, each slice a multiple of 512 elements.
+static int resid_cluster(int H) {
+    int cl = 8;
+    while (cl > 1 && (H % (cl * 512) != 0)) cl >>= 1;
+    return cl;
+}
+
+void launch_rmsnorm_resid(float* x, const float* part, int S, const float* g, int H, float eps,
+                          bf16* out, int M, cudaStream_t s) {
+    note_launch();
+    if (M <= 0) return;
+    const int cl = resid_cluster(H);
+    launch_k_cluster(rmsnorm_resid_kernel, dim3(cl, M), dim3(128), 0, s, cl, x, part, S,
+                     (size_t)M * H, g, H, eps, out);
+}
+
+// h[r, j] = silu(sum_s gate) * (sum_s up) from split-K partials of the packed gate/up linear
+// (part[s][r][2I], blocks of 128 gate columns each followed by the matching 128 up columns).
+__global__ void swiglu_partials_kernel(const float* __restrict__ part, int S, size_t split_stride,
+                                       bf16* __restrict__ h, int M, int I) {
+    pdl_wait();
+    size_t n = (size_t)M * I;
+    for (size_t e = blockIdx.x * (size_t)blockDim.x + threadIdx.x; e < n;
+         e += (size_t)gridDim.x * blockDim.x) {
+        size_t m = e / I;
+        int j = (int)(e % I);
+        size_t c = m * 2 * I + (size_t)(j >> 7) * 256 + (j & 127);
+        float gs = 0.f, us = 0.f;
+        for (int sp = 0; sp < S; ++sp) {
+            gs += part[sp * split_stride + c];
+            us += part[sp * split_stride + c + 128];
+        }
+        h[e] = __float2bfloat16_rn(gs / (1.f + expf(-gs)) * us);
+    }
+}
+
+void launch_swiglu_partials(const float* part, int S, bf16* h, int M, int I, cudaStream_t s) {
+    note_launch();
+    if (M <= 0) return;
+    size_t n = (size_t)M * I;
+    int blocks = (int)((n + 255) / 256);
+    if (blocks > 65535) blocks = 65535;
+    launch_k(swiglu_partials_kernel, dim3(blocks), dim3(256), 0, s, part, S, (size_t)M * 2 * I, h,
+             M, I);
+}
+
 void launch_rmsnorm(const float* x, int in_step, int in_off, const float* g, int H, float eps,
                     void* out, int out_dtype, int M, cudaStream_t s) {
     note_launch();
     if (M <= 0) return;
     int threads = H >= 1024 ? 256 : 64;
     if (out_dtype == QK_DTYPE_BF16)
-        rmsnorm_kernel<bf16><<<M, threads, 0, s>>>(x, in_step, in_off, g, H, eps, (bf16*)out);
+        launch_k(rmsnorm_kernel<bf16>, dim3(M), dim3(threads), 0, s, x, in_step, in_off, g, H, eps,
+                 (bf16*)out);
     else
-        rmsnorm_kernel<float><<<M, threads, 0, s>>>(x, in_step, in_off, g, H, eps, (float*)out);
+        launch_k(rmsnorm_kernel<float>, dim3(M), dim3(threads), 0, s, x, in_step, in_off, g, H, eps,
+                 (float*)out);
 }
 
 // ---------------------------------------------------------------- QK-norm + RoPE + cache write
 // One warp per (token, head) of the fused qkv row; lane owns elements lane + 32 i.
+// With part != nullptr the projections come from S fp32 split-K partials
+// part[s][r][(nq + 2 nkv) D] (summed in fixed order) instead of the qkv buffer;
+// q is still written to the qkv buffer, k and v to the cache.
 template <typename T, int D>
 __global__ void qk_norm_rope_kernel(T* __restrict__ qkv, int nq, int nkv, const float* __restrict__ gq,
                                     const float* __restrict__ gk, float eps,
                                     const float* __restrict__ rc, const float* __restrict__ rs,
                                     int max_positions, PosIndex pos, T* __restrict__ kc,
-                                    T* __restrict__ vc, int max_seq, uint32_t* status) {
+                                    T* __restrict__ vc, int max_seq, uint32_t* status,
+                                    const float* __restrict__ part, int S, size_t split_stride) {
     constexpr int E = D / 32, HALF = D / 2;
+    pdl_wait();
     int lane = threadIdx.x & 31;
     int hh = blockIdx.y * (blockDim.x >> 5) + (threadIdx.x >> 5);
     int nh = nq + 2 * nkv;
@@ -115,13 +222,23 @@ __global__ void qk_norm_rope_kernel(T* __restrict__ qkv, int nq, int nkv, const 
     }
     T* src = qkv + (size_t)r * nh * D + (size_t)hh * D;
     float e[E];
+    if (part) {
+        const float* pp = part + (size_t)r * nh * D + (size_t)hh * D;
 #pragma unroll
-    for (int i = 0; i < E; ++i) e[i] = to_f(src[lane + 32 * i]);
+        for (int i = 0; i < E; ++i) {
+            float v = 0.f;
+            for (int sp = 0; sp < S; ++sp) v += pp[sp * split_stride + lane + 32 * i];
+            e[i] = v;
+        }
+    } else {
+#pragma unroll
+        for (int i = 0; i < E; ++i) e[i] = to_f(src[lane + 32 * i]);
+    }
     if (hh >= nq + nkv) {  // value head: straight to the cache
         int kvh = hh - nq - nkv;
         T* dst = vc + (((size_t)b * nkv + kvh) * max_seq + p) * D;
 #pragma unroll
-        for (int i = 0; i < E; ++i) dst[lane + 32 * i] = src[lane + 32 * i];
+        for (int i = 0; i < E; ++i) dst[lane + 32 * i] = from_f<T>(e[i]);
         return;
     }
     const float* g = hh < nq ? gq : gk;
@@ -156,14 +273,15 @@ __global__ void qk_norm_rope_kernel(T* __restrict__ qkv, int nq, int nkv, const 
 void launch_qk_norm_rope(void* qkv, int dtype, int M, int nq, int nkv, int d, const float* gq,
                          const float* gk, float eps, const float* rope_cos, const float* rope_sin,
                          int max_positions, PosIndex pos, void* k_cache, void* v_cache,
-                         int max_seq, uint32_t* status, cudaStream_t s) {
+                         int max_seq, uint32_t* status, cudaStream_t s, const float* part,
+                         int S) {
     note_launch();
     if (M <= 0) return;
     dim3 grid(M, (nq + 2 * nkv + 7) / 8);
 #define QK_NR(T, D)                                                                          \
-    qk_norm_rope_kernel<T, D><<<grid, 256, 0, s>>>((T*)qkv, nq, nkv, gq, gk, eps, rope_cos,  \
-                                                   rope_sin, max_positions, pos, (T*)k_cache, \
-                                                   (T*)v_cache, max_seq, status)
+    launch_k(qk_norm_rope_kernel<T, D>, grid, dim3(256), 0, s, (T*)qkv, nq, nkv, gq, gk, eps,  \
+             rope_cos, rope_sin, max_positions, pos, (T*)k_cache, (T*)v_cache, max_seq, status, \
+             part, S, (size_t)M * (nq + 2 * nkv) * d)
     if (dtype == QK_DTYPE_BF16) {
         if (d == 128) QK_NR(bf16, 128); else QK_NR(bf16, 64);
     } else {
@@ -175,6 +293,7 @@ void launch_qk_norm_rope(void* qkv, int dtype, int M, int nq, int nkv, int d, co
 // ---------------------------------------------------------------- SwiGLU (unfused path)
 template <typename T>
 __global__ void swiglu_kernel(const T* __restrict__ gu, T* __restrict__ h, int M, int I) {
+    pdl_wait();
     size_t n = (size_t)M * I;
     for (size_t e = blockIdx.x * (size_t)blockDim.x + threadIdx.x; e < n;
          e += (size_t)gridDim.x * blockDim.x) {
@@ -193,9 +312,10 @@ void launch_swiglu(const void* gu, void* h, int dtype, int M, int I, cudaStream_
     int blocks = (int)((n + 255) / 256);
     if (blocks > 65535) blocks = 65535;
     if (dtype == QK_DTYPE_BF16)
-        swiglu_kernel<bf16><<<blocks, 256, 0, s>>>((const bf16*)gu, (bf16*)h, M, I);
+        launch_k(swiglu_kernel<bf16>, dim3(blocks), dim3(256), 0, s, (const bf16*)gu, (bf16*)h, M, I);
     else
-        swiglu_kernel<float><<<blocks, 256, 0, s>>>((const float*)gu, (float*)h, M, I);
+        launch_k(swiglu_kernel<float>, dim3(blocks), dim3(256), 0, s, (const float*)gu, (float*)h, M,
+                 I);
 }
 
 // ---------------------------------------------------------------- log-softmax / gather / argmax
@@ -206,6 +326,7 @@ __global__ void logits_reduce_kernel(const float* __restrict__ logits, int V, Ou
     __shared__ float red_v[32];
     __shared__ int red_i[32];
     __shared__ float red[32];
+    pdl_wait();
     int r = blockIdx.x;
     int g = oi.row0 + r;
     int b = g / oi.T, t = g % oi.T;
@@ -244,7 +365,7 @@ __global__ void logits_reduce_kernel(const float* __restrict__ logits, int V, Ou
     }
     se = block_sum(se, red);
     if (threadIdx.x == 0) {
-        size_t o = (size_t)b * oi.out_ld + oi.out_off + t;
+        size_t o = (size_t)b * oi.out_ld + oi.out_off + t + (oi.dyn_off ? *oi.dyn_off : 0);
         if (am) am[o] = bi;
         if (lp && oi.tgt) {
             int tg = oi.tgt[(size_t)b * oi.tgt_ld + oi.tgt_off + t];
@@ -261,7 +382,32 @@ void launch_logits_reduce(const float* logits, int M, int V, OutIndex oi, float*
                           int32_t* argmax, uint32_t* status, cudaStream_t s) {
     note_launch();
     if (M <= 0) return;
-    logits_reduce_kernel<<<M, 512, 0, s>>>(logits, V, oi, lp, argmax, status);
+    launch_k(logits_reduce_kernel, dim3(M), dim3(512), 0, s, logits, V, oi, lp, argmax, status);
+}
+
+// ---------------------------------------------------------------- rollout cursor
+__global__ void rollout_prepare_kernel(const int32_t* __restrict__ seq, int L, int P, int B,
+                                       int32_t* step, int32_t* pos, int32_t* tok, int32_t* tgt,
+                                       int32_t* out_off) {
+    pdl_wait();
+    const int s = *step;
+    __syncthreads();  // every thread has read the step before it advances
+    for (int b = threadIdx.x; b < B; b += blockDim.x) {
+        pos[b] = P + s;
+        tok[b] = seq[(size_t)b * L + P + s];
+        tgt[b] = seq[(size_t)b * L + P + s + 1];
+    }
+    if (threadIdx.x == 0) {
+        *out_off = s + 1;
+        *step = s + 1;
+    }
+}
+
+void launch_rollout_prepare(const int32_t* seq, int L, int P, int B, int32_t* step, int32_t* pos,
+                            int32_t* tok, int32_t* tgt, int32_t* out_off, cudaStream_t s) {
+    note_launch();
+    launch_k(rollout_prepare_kernel, dim3(1), dim3(256), 0, s, seq, L, P, B, step, pos, tok, tgt,
+             out_off);
 }
 
 // ---------------------------------------------------------------- load-time tables

@@ -39,6 +39,7 @@ int set_error(int code, const char* fmt, ...) {
 }
 
 int cuda_error(cudaError_t e, const char* what) {
+    (void)cudaGetLastError();  // do not leave the error for the next call's launch check
     return set_error(QK_ECUDA, "%s: %s", what, cudaGetErrorString(e));
 }
 
@@ -109,6 +110,8 @@ struct Workspace {
     void* h;        // [M, I] SwiGLU output
     void* gu;       // [M, 2 I] gate/up before SwiGLU (unfused path only)
     void* skv;      // scoring: K and V of one layer, [2][B, nkv, T, d]
+    void* attn;     // decode: split-attention partials (bf16 models)
+    float* part;    // decode: split-K partial products of the linear layers (bf16 models)
     float* logits;  // [logit_rows, V]
     int logit_rows;
     size_t total;
@@ -116,7 +119,48 @@ struct Workspace {
 
 static const int kScoreLogitRows = 4096;
 
-static int workspace_layout(const Model& m, int kind, int B, int T, Workspace* w, char* base) {
+// The rollout keeps a cursor (step counter, per-row position / token / target,
+// output slot) in 256-byte-aligned slots after the prefill/decode workspace.
+static size_t rollout_cursor_bytes(int B) { return 5 * align256((size_t)(B > 1 ? B : 1) * 4); }
+
+// Decode batches of bf16 models with more than kGemvMaxRows and at most
+// kSplitMaxRows rows run their linear layers as split-K tcgen05 GEMMs whose fp32
+// partials are summed (in a fixed order) by the kernel that consumes them;
+// smaller batches stream the weights through the CUDA-core GEMV.
+static const int kSplitMaxRows = 64;
+
+struct Splits {
+    int qkv, o, gu, d;
+};
+
+static bool use_splitk(const Model& m, int M) {
+    const qk_config& c = m.cfg;
+    return c.dtype == QK_DTYPE_BF16 && M > kGemvMaxRows && M <= kSplitMaxRows && c.hidden % 128 == 0 &&
+           (c.n_q_heads * c.head_dim) % 128 == 0 && ((c.n_q_heads + 2 * c.n_kv_heads) * c.head_dim) % 128 == 0;
+}
+
+static Splits decode_splits(const Model& m) {
+    const qk_config& c = m.cfg;
+    const int nqkv = (c.n_q_heads + 2 * c.n_kv_heads) * c.head_dim;
+    return Splits{gemm_tc_split(nqkv, c.hidden, m.num_sms),
+                  gemm_tc_split(c.hidden, c.n_q_heads * c.head_dim, m.num_sms),
+                  gemm_tc_split(2 * c.intermediate, c.hidden, m.num_sms),
+                  gemm_tc_split(c.hidden, c.intermediate, m.num_sms)};
+}
+
+static size_t splitk_part_floats(const Model& m, int M) {
+    const qk_config& c = m.cfg;
+    const Splits sp = decode_splits(m);
+    const size_t nqkv = (size_t)(c.n_q_heads + 2 * c.n_kv_heads) * c.head_dim;
+    size_t f = (size_t)sp.qkv * M * nqkv;
+    f = f > (size_t)sp.o * M * c.hidden ? f : (size_t)sp.o * M * c.hidden;
+    f = f > (size_t)sp.gu * M * 2 * c.intermediate ? f : (size_t)sp.gu * M * 2 * c.intermediate;
+    f = f > (size_t)sp.d * M * c.hidden ? f : (size_t)sp.d * M * c.hidden;
+    return f;
+}
+
+static int workspace_layout(const Model& m, int kind, int B, int T, int max_seq, Workspace* w,
+                            char* base) {
     const qk_config& c = m.cfg;
     if (B < 1 || T < 1) return set_error(QK_ESHAPE, "batch %d and tokens %d must be >= 1", B, T);
     size_t es = m.es;
@@ -134,8 +178,16 @@ static int workspace_layout(const Model& m, int kind, int B, int T, Workspace* w
     w->qkv = take(M * (nq + 2 * nkv) * d * es);
     w->o = take(M * nq * d * es);
     w->h = take(M * I * es);
-    w->gu = take(M * 2 * I * es);
+    w->gu = c.dtype == QK_DTYPE_F32 ? take(M * 2 * I * es) : nullptr;  // unfused SwiGLU path only
     w->skv = kind == QK_CALL_SCORE ? take(2 * (size_t)B * nkv * T * d * es) : nullptr;
+    w->part = kind == QK_CALL_DECODE && use_splitk(m, B) ? (float*)take(splitk_part_floats(m, B) * 4)
+                                                         : nullptr;
+    w->attn = nullptr;
+    if (kind == QK_CALL_DECODE && c.dtype == QK_DTYPE_BF16 &&
+        attn_decode_supported(c.head_dim, c.n_q_heads, c.n_kv_heads)) {
+        if (max_seq < 1) return set_error(QK_ESHAPE, "max_seq must be >= 1");
+        w->attn = take(attn_decode_scratch_bytes(B, c.n_q_heads, c.n_kv_heads, max_seq, m.num_sms));
+    }
     size_t rows = kind == QK_CALL_SCORE ? (M < (size_t)kScoreLogitRows ? M : kScoreLogitRows) : B;
     w->logit_rows = (int)rows;
     w->logits = (float*)take(rows * (size_t)c.vocab * 4);
@@ -175,7 +227,8 @@ static void run_layer(Model& m, int l, const Workspace& w, int M, PosIndex pos,
                         m.rope_sin, c.max_positions, pos, kv.k(l), kv.v(l), kv.max_seq, m.status,
                         s);
     pr = prof_open(m, QK_PROF_ATTN, s);
-    launch_attention(m, w.qkv, nqkv, kv.k(l), kv.v(l), M, kv.max_batch, kv.max_seq, pos, w.o, s);
+    launch_attention(m, w.qkv, nqkv, kv.k(l), kv.v(l), M, kv.max_batch, kv.max_seq, pos, w.o,
+                     w.attn, s);
     prof_close(m, pr, s);
     pr = prof_open(m, QK_PROF_O, s);
     linear(m, w.o, nq * d, L.w_o, w.x, H, M, H, nq * d, EPI_RESID_F32, w.gu, s);
@@ -189,18 +242,76 @@ static void run_layer(Model& m, int l, const Workspace& w, int M, PosIndex pos,
     prof_close(m, pr, s);
 }
 
+// One decoder layer of a decode step with split-K linear layers.  The down
+// projection's partials are left in w.part for the next consumer (the next
+// layer's input norm, the final norm, or flush_residual); `pending` says whether
+// the previous layer left such partials.
+static void run_layer_splitk(Model& m, int l, const Workspace& w, int M, PosIndex pos,
+                             const KVView& kv, bool pending, cudaStream_t s) {
+    const qk_config& c = m.cfg;
+    const LayerW& L = m.layers[l];
+    const Splits sp = decode_splits(m);
+    int H = c.hidden, d = c.head_dim, nq = c.n_q_heads, nkv = c.n_kv_heads, I = c.intermediate;
+    int nqkv = (nq + 2 * nkv) * d;
+    float eps = (float)c.rms_eps;
+    bf16* u = (bf16*)w.u;
+    bool pr;
+    auto gemm = [&](const void* A, int lda, const void* W, int N, int K, int S) {
+        int rc = launch_gemm_tc_splitk((const bf16*)A, lda, (const bf16*)W, w.part, M, N, K, S,
+                                       m.num_sms, m.status, s);
+        if (rc != QK_OK && !m.deferred_error) m.deferred_error = rc;
+    };
+    if (pending)
+        launch_rmsnorm_resid(w.x, w.part, sp.d, L.attn_norm, H, eps, u, M, s);
+    else
+        launch_rmsnorm(w.x, 1, 0, L.attn_norm, H, eps, u, c.dtype, M, s);
+    pr = prof_open(m, QK_PROF_QKV, s);
+    gemm(u, H, L.w_qkv, nqkv, H, sp.qkv);
+    prof_close(m, pr, s);
+    launch_qk_norm_rope(w.qkv, c.dtype, M, nq, nkv, d, L.q_norm, L.k_norm, eps, m.rope_cos,
+                        m.rope_sin, c.max_positions, pos, kv.k(l), kv.v(l), kv.max_seq, m.status, s,
+                        w.part, sp.qkv);
+    pr = prof_open(m, QK_PROF_ATTN, s);
+    launch_attention(m, w.qkv, nqkv, kv.k(l), kv.v(l), M, kv.max_batch, kv.max_seq, pos, w.o,
+                     w.attn, s);
+    prof_close(m, pr, s);
+    pr = prof_open(m, QK_PROF_O, s);
+    gemm(w.o, nq * d, L.w_o, H, nq * d, sp.o);
+    prof_close(m, pr, s);
+    launch_rmsnorm_resid(w.x, w.part, sp.o, L.mlp_norm, H, eps, u, M, s);
+    pr = prof_open(m, QK_PROF_GATE_UP, s);
+    gemm(u, H, L.w_gu, 2 * I, H, sp.gu);
+    prof_close(m, pr, s);
+    launch_swiglu_partials(w.part, sp.gu, (bf16*)w.h, M, I, s);
+    pr = prof_open(m, QK_PROF_DOWN, s);
+    gemm(w.h, I, L.w_d, H, I, sp.d);
+    prof_close(m, pr, s);
+}
+
 // Final norm of M_out selected rows (row r of the output reads residual row r * in_step + in_off),
 // lm_head into `logits`, then log-prob / argmax per row.
 static void run_head(Model& m, const Workspace& w, int M_out, int in_step, int in_off,
-                     float* logits, OutIndex oi, float* lp, int32_t* am, cudaStream_t s) {
+                     float* logits, OutIndex oi, float* lp, int32_t* am, cudaStream_t s,
+                     bool normed = false) {
     const qk_config& c = m.cfg;
-    launch_rmsnorm(w.x, in_step, in_off, m.final_norm, c.hidden, (float)c.rms_eps, w.u, c.dtype,
-                   M_out, s);
+    if (!normed)
+        launch_rmsnorm(w.x, in_step, in_off, m.final_norm, c.hidden, (float)c.rms_eps, w.u,
+                       c.dtype, M_out, s);
     bool pr = prof_open(m, QK_PROF_LM_HEAD, s);
     linear(m, w.u, c.hidden, m.lm_head, logits, c.vocab, M_out, c.vocab, c.hidden, EPI_STORE_F32,
            w.gu, s);
     prof_close(m, pr, s);
     if (lp || am) launch_logits_reduce(logits, M_out, c.vocab, oi, lp, am, m.status, s);
+}
+
+// The split decode attention merges through tickets in its scratch that must be
+// zero at the start of a step (each layer leaves them zero again).
+static int clear_attn_tickets(const Model& m, const Workspace& w, int B, int max_seq, cudaStream_t s) {
+    if (!w.attn) return QK_OK;
+    const qk_config& c = m.cfg;
+    int* t = attn_decode_tickets(w.attn, B, c.n_q_heads, c.n_kv_heads, max_seq, m.num_sms);
+    QK_TRY_CUDA(cudaMemsetAsync(t, 0, (size_t)B * c.n_kv_heads * sizeof(int), s));
+    return QK_OK;
 }
 
 static int check_launch(const char* what) {
@@ -218,13 +329,14 @@ static int check_launch(Model& m, const char* what) {
     return rc;
 }
 
-static int get_ws(const Model& m, int kind, int B, int T, void* ws, size_t ws_bytes, Workspace* w) {
-    QK_TRY(workspace_layout(m, kind, B, T, w, nullptr));
+static int get_ws(const Model& m, int kind, int B, int T, int max_seq, void* ws, size_t ws_bytes,
+                  Workspace* w) {
+    QK_TRY(workspace_layout(m, kind, B, T, max_seq, w, nullptr));
     if (!ws) return set_error(QK_EINVAL, "workspace is NULL");
     if (((uintptr_t)ws & 255) != 0) return set_error(QK_EINVAL, "workspace must be 256-byte aligned");
     if (ws_bytes < w->total)
         return set_error(QK_ENOSPACE, "workspace has %zu bytes, needs %zu", ws_bytes, w->total);
-    return workspace_layout(m, kind, B, T, w, (char*)ws);
+    return workspace_layout(m, kind, B, T, max_seq, w, (char*)ws);
 }
 
 static int check_cache(const Model& m, void* kv, int max_batch, int max_seq, int B) {
@@ -377,6 +489,8 @@ static void prof_release(Model& m) {
 void qk_model_free(qk_model* m) {
     if (!m) return;
     prof_release(*(Model*)m);
+    for (auto& g : ((Model*)m)->graphs) cudaGraphExecDestroy(g.exec);
+    if (((Model*)m)->capture_stream) cudaStreamDestroy(((Model*)m)->capture_stream);
     delete (Model*)m;
 }
 
@@ -433,7 +547,8 @@ int qk_op_linear(qk_model* mh, const void* A, int lda, const void* W, void* C, i
     if (epilogue < QK_EPI_STORE || epilogue > QK_EPI_SWIGLU)
         return set_error(QK_EINVAL, "unknown epilogue %d", epilogue);
     if (ldc < N) return set_error(QK_ESHAPE, "ldc %d < N %d", ldc, N);
-    size_t need = epilogue == QK_EPI_SWIGLU ? (size_t)M * 2 * N * m.es : 0;
+    // Only the CUDA-core path (fp32 models) stages the gate/up product in scratch.
+    size_t need = epilogue == QK_EPI_SWIGLU && m.cfg.dtype == QK_DTYPE_F32 ? (size_t)M * 2 * N * m.es : 0;
     if (need && (!scratch || scratch_bytes < need))
         return set_error(QK_ENOSPACE, "linear scratch has %zu bytes, needs %zu", scratch_bytes, need);
     linear(m, A, lda, W, C, ldc, M, N, K, epilogue, scratch, (cudaStream_t)stream);
@@ -451,18 +566,17 @@ int qk_kv_bytes(const qk_model* mh, int max_batch, int max_seq, size_t* bytes) {
 int qk_workspace_bytes(const qk_model* mh, int kind, int B, int T, int max_seq, size_t* bytes) {
     if (!mh || !bytes) return set_error(QK_EINVAL, "null argument");
     const Model& m = *(const Model*)mh;
-    (void)max_seq;
     Workspace w;
     if (kind == QK_CALL_ROLLOUT) {
         Workspace w2;
-        QK_TRY(workspace_layout(m, QK_CALL_PREFILL, B, T, &w, nullptr));
-        QK_TRY(workspace_layout(m, QK_CALL_DECODE, B, 1, &w2, nullptr));
-        *bytes = w.total > w2.total ? w.total : w2.total;
+        QK_TRY(workspace_layout(m, QK_CALL_PREFILL, B, T, max_seq, &w, nullptr));
+        QK_TRY(workspace_layout(m, QK_CALL_DECODE, B, 1, max_seq, &w2, nullptr));
+        *bytes = (w.total > w2.total ? w.total : w2.total) + rollout_cursor_bytes(B);
         return QK_OK;
     }
     if (kind != QK_CALL_DECODE && kind != QK_CALL_PREFILL && kind != QK_CALL_SCORE)
         return set_error(QK_EINVAL, "unknown call kind %d", kind);
-    QK_TRY(workspace_layout(m, kind, B, T, &w, nullptr));
+    QK_TRY(workspace_layout(m, kind, B, T, max_seq, &w, nullptr));
     *bytes = w.total;
     return QK_OK;
 }
@@ -471,7 +585,7 @@ static int prefill_impl(Model& m, void* kv, int max_batch, int max_seq, TokIndex
                         int start_pos, float* last_logits, OutIndex oi, float* lp, int32_t* am,
                         void* ws, size_t ws_bytes, cudaStream_t s) {
     Workspace w;
-    QK_TRY(get_ws(m, QK_CALL_PREFILL, B, T, ws, ws_bytes, &w));
+    QK_TRY(get_ws(m, QK_CALL_PREFILL, B, T, max_seq, ws, ws_bytes, &w));
     int M = B * T;
     KVView view = cache_view(m, kv, max_batch, max_seq);
     launch_embed(m.embed, m.cfg.dtype, m.cfg.vocab, m.cfg.hidden, tok, M, w.x, m.status, s);
@@ -501,12 +615,22 @@ static int decode_impl(Model& m, void* kv, int max_batch, int max_seq, TokIndex 
                        int B, float* logits, OutIndex oi, float* lp, int32_t* am, void* ws,
                        size_t ws_bytes, cudaStream_t s) {
     Workspace w;
-    QK_TRY(get_ws(m, QK_CALL_DECODE, B, 1, ws, ws_bytes, &w));
+    QK_TRY(get_ws(m, QK_CALL_DECODE, B, 1, max_seq, ws, ws_bytes, &w));
     KVView view = cache_view(m, kv, max_batch, max_seq);
+    QK_TRY(clear_attn_tickets(m, w, B, max_seq, s));
     m.in_decode = true;
     launch_embed(m.embed, m.cfg.dtype, m.cfg.vocab, m.cfg.hidden, tok, B, w.x, m.status, s);
-    for (int l = 0; l < m.cfg.n_layers; ++l) run_layer(m, l, w, B, pos, view, s);
-    if (logits || lp || am) run_head(m, w, B, 1, 0, logits ? logits : w.logits, oi, lp, am, s);
+    if (w.part) {
+        for (int l = 0; l < m.cfg.n_layers; ++l) run_layer_splitk(m, l, w, B, pos, view, l > 0, s);
+        // the last layer's down-projection partials join the residual in the final norm's pass
+        launch_rmsnorm_resid(w.x, w.part, decode_splits(m).d, m.final_norm, m.cfg.hidden,
+                             (float)m.cfg.rms_eps, (bf16*)w.u, B, s);
+        if (logits || lp || am)
+            run_head(m, w, B, 1, 0, logits ? logits : w.logits, oi, lp, am, s, /*normed=*/true);
+    } else {
+        for (int l = 0; l < m.cfg.n_layers; ++l) run_layer(m, l, w, B, pos, view, s);
+        if (logits || lp || am) run_head(m, w, B, 1, 0, logits ? logits : w.logits, oi, lp, am, s);
+    }
     m.in_decode = false;
     return check_launch(m, "decode step");
 }
@@ -532,11 +656,20 @@ int qk_decode_layer(qk_model* mh, int layer, void* kv, int max_batch, int max_se
         return set_error(QK_EINVAL, "layer %d outside [0, %d)", layer, m.cfg.n_layers);
     QK_TRY(check_cache(m, kv, max_batch, max_seq, B));
     Workspace w;
-    QK_TRY(get_ws(m, QK_CALL_DECODE, B, 1, workspace, ws_bytes, &w));
+    QK_TRY(get_ws(m, QK_CALL_DECODE, B, 1, max_seq, workspace, ws_bytes, &w));
     w.x = x;
+    cudaStream_t s = (cudaStream_t)stream;
+    QK_TRY(clear_attn_tickets(m, w, B, max_seq, s));
     m.in_decode = true;
-    run_layer(m, layer, w, B, PosIndex{pos, 0, 1}, cache_view(m, kv, max_batch, max_seq),
-              (cudaStream_t)stream);
+    if (w.part) {
+        run_layer_splitk(m, layer, w, B, PosIndex{pos, 0, 1}, cache_view(m, kv, max_batch, max_seq),
+                         false, s);
+        // add the down projection's partials to x (the normed output is not needed)
+        launch_rmsnorm_resid(w.x, w.part, decode_splits(m).d, m.final_norm, m.cfg.hidden,
+                             (float)m.cfg.rms_eps, (bf16*)w.u, B, s);
+    } else {
+        run_layer(m, layer, w, B, PosIndex{pos, 0, 1}, cache_view(m, kv, max_batch, max_seq), s);
+    }
     m.in_decode = false;
     return check_launch(m, "decode layer");
 }
@@ -549,7 +682,7 @@ int qk_score_logprobs(qk_model* mh, const int32_t* tokens, int B, int T, float* 
     if (T > m.cfg.max_positions)
         return set_error(QK_ESHAPE, "T %d exceeds the RoPE table (%d)", T, m.cfg.max_positions);
     Workspace w;
-    QK_TRY(get_ws(m, QK_CALL_SCORE, B, T, workspace, ws_bytes, &w));
+    QK_TRY(get_ws(m, QK_CALL_SCORE, B, T, T, workspace, ws_bytes, &w));
     cudaStream_t s = (cudaStream_t)stream;
     int M = B * T;
     // One layer's K and V live in scratch shaped like a cache of B rows x T positions;
@@ -586,15 +719,80 @@ int qk_rollout_teacher_forced(qk_model* mh, void* kv, int max_batch, int max_seq
     if (!workspace || ws_bytes < need)
         return set_error(QK_ENOSPACE, "workspace has %zu bytes, needs %zu", ws_bytes, need);
     cudaStream_t s = (cudaStream_t)stream;
-    int L = P + N + 1;
+    const int L = P + N + 1;
     OutIndex oi{1, 1, N + 1, 0, seq, L, P, 0};
     QK_TRY(prefill_impl(m, kv, max_batch, max_seq, TokIndex{seq, P, L, 0}, B, P, 0, nullptr, oi,
                         logprobs, argmax, workspace, ws_bytes, s));
-    for (int j = 0; j < N; ++j) {
-        OutIndex oj{1, 1, N + 1, j + 1, seq, L, P + j + 1, 0};
-        QK_TRY(decode_impl(m, kv, max_batch, max_seq, TokIndex{seq, 1, L, P + j},
-                           PosIndex{nullptr, P + j, 1}, B, nullptr, oj, logprobs, argmax,
-                           workspace, ws_bytes, s));
+    if (N == 0) return QK_OK;
+    // cursor slots
+    const size_t slot = align256((size_t)B * 4);
+    char* cur = (char*)workspace + (need - rollout_cursor_bytes(B));
+    int32_t* step = (int32_t*)cur;
+    int32_t* pos = (int32_t*)(cur + slot);
+    int32_t* tok = (int32_t*)(cur + 2 * slot);
+    int32_t* tgt = (int32_t*)(cur + 3 * slot);
+    int32_t* off = (int32_t*)(cur + 4 * slot);
+    QK_TRY_CUDA(cudaMemsetAsync(step, 0, sizeof(int32_t), s));
+    OutIndex od{1, 1, N + 1, 0, tgt, 1, 0, 0, off};
+    auto one_step = [&]() -> int {
+        launch_rollout_prepare(seq, L, P, B, step, pos, tok, tgt, off, s);
+        return decode_impl(m, kv, max_batch, max_seq, TokIndex{tok, 1, 1, 0}, PosIndex{pos, 0, 1},
+                           B, nullptr, od, logprobs, argmax, workspace, ws_bytes, s);
+    };
+    // Step 0 runs directly (it also performs any one-time kernel set-up).
+    QK_TRY(one_step());
+    if (N == 1) return QK_OK;
+    cudaStreamCaptureStatus cs = cudaStreamCaptureStatusNone;
+    QK_TRY_CUDA(cudaStreamIsCapturing(s, &cs));
+    if (cs != cudaStreamCaptureStatusNone) {  // already inside the caller's capture: no nesting
+        for (int j = 1; j < N; ++j) QK_TRY(one_step());
+        return QK_OK;
+    }
+    const uint64_t key[12] = {(uint64_t)(uintptr_t)kv, (uint64_t)max_batch, (uint64_t)max_seq,
+                              (uint64_t)(uintptr_t)seq, (uint64_t)B, (uint64_t)P, (uint64_t)N,
+                              (uint64_t)(uintptr_t)logprobs, (uint64_t)(uintptr_t)argmax,
+                              (uint64_t)(uintptr_t)workspace, (uint64_t)ws_bytes, 0};
+    cudaGraphExec_t exec = nullptr;
+    int kernels = 0;
+    for (auto& g : m.graphs)
+        if (!memcmp(g.key, key, sizeof(key))) {
+            exec = g.exec;
+            kernels = g.kernels;
+        }
+    if (!exec) {
+        if (!m.capture_stream)
+            QK_TRY_CUDA(cudaStreamCreateWithFlags(&m.capture_stream, cudaStreamNonBlocking));
+        cudaStream_t cs_stream = m.capture_stream;
+        QK_TRY_CUDA(cudaStreamBeginCapture(cs_stream, cudaStreamCaptureModeThreadLocal));
+        const uint64_t before = g_launches.load();
+        launch_rollout_prepare(seq, L, P, B, step, pos, tok, tgt, off, cs_stream);
+        int rc = decode_impl(m, kv, max_batch, max_seq, TokIndex{tok, 1, 1, 0}, PosIndex{pos, 0, 1},
+                             B, nullptr, od, logprobs, argmax, workspace, ws_bytes, cs_stream);
+        kernels = (int)(g_launches.load() - before);
+        g_launches.fetch_sub((uint64_t)kernels);  // counted again below, once per replay
+        cudaGraph_t graph = nullptr;
+        cudaError_t e = cudaStreamEndCapture(cs_stream, &graph);
+        if (rc != QK_OK) {
+            if (graph) cudaGraphDestroy(graph);
+            return rc;
+        }
+        if (e != cudaSuccess) return cuda_error(e, "rollout step capture");
+        e = cudaGraphInstantiate(&exec, graph, 0);
+        cudaGraphDestroy(graph);
+        if (e != cudaSuccess) return cuda_error(e, "rollout step graph instantiate");
+        if (m.graphs.size() >= 8) {
+            cudaGraphExecDestroy(m.graphs.front().exec);
+            m.graphs.erase(m.graphs.begin());
+        }
+        Model::StepGraph g;
+        memcpy(g.key, key, sizeof(key));
+        g.exec = exec;
+        g.kernels = kernels;
+        m.graphs.push_back(g);
+    }
+    for (int j = 1; j < N; ++j) {
+        QK_TRY_CUDA(cudaGraphLaunch(exec, s));
+        note_launch(kernels);
     }
     return QK_OK;
 }

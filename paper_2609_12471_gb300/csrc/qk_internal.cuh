@@ -6,6 +6,7 @@
 #include <cuda_runtime.h>
 #include <stdint.h>
 
+#include <utility>
 #include <vector>
 
 #include "qk.h"
@@ -14,6 +15,58 @@
 namespace qk {
 
 using bf16 = __nv_bfloat16;
+
+// Programmatic dependent launch: a kernel launched with launch_k may start while
+// the previous kernel on the stream is still running; it must execute
+// pdl_wait() before its first global-memory access (read or write) that can
+// depend on or conflict with earlier kernels.  Launched normally, pdl_wait() is
+// a no-op.
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+// Lets the next kernel on the stream be scheduled (its pdl_wait still waits for this one to finish).
+__device__ __forceinline__ void pdl_trigger() {
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+
+template <typename... KArgs, typename... Args>
+inline void launch_k(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t s,
+                     Args&&... args) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = grid;
+    cfg.blockDim = block;
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = s;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    cudaLaunchKernelEx(&cfg, kernel, std::forward<Args>(args)...);
+}
+
+// As launch_k, with a thread-block cluster of cluster_x CTAs along x.
+template <typename... KArgs, typename... Args>
+inline void launch_k_cluster(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem,
+                             cudaStream_t s, int cluster_x, Args&&... args) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = grid;
+    cfg.blockDim = block;
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = s;
+    cudaLaunchAttribute attr[2];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    attr[1].id = cudaLaunchAttributeClusterDimension;
+    attr[1].val.clusterDim.x = cluster_x;
+    attr[1].val.clusterDim.y = 1;
+    attr[1].val.clusterDim.z = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 2;
+    cudaLaunchKernelEx(&cfg, kernel, std::forward<Args>(args)...);
+}
+
+// bf16 linear layers over at most this many token rows stream the weights through
+// the CUDA-core GEMV (fused epilogues); larger ones run on the tensor cores.
+constexpr int kGemvMaxRows = 4;
 
 // ---------------------------------------------------------------- errors
 int set_error(int code, const char* fmt, ...);
@@ -60,6 +113,17 @@ struct Model {
     bool in_decode = false;
     std::vector<cudaEvent_t> prof_ev;
     int prof_used = 0;
+    // Instantiated decode-step graphs of qk_rollout_teacher_forced, keyed by the call's
+    // pointers and sizes (every kernel parameter of a step is fixed by them).
+    struct StepGraph {
+        uint64_t key[12];
+        cudaGraphExec_t exec;
+        int kernels;  // kernel nodes of one step (for the launch counter)
+    };
+    std::vector<StepGraph> graphs;
+    // Library-owned stream on which step graphs are captured (capture records only;
+    // the graphs are launched on the caller's stream).  Created on first use.
+    cudaStream_t capture_stream = nullptr;
     // First host-side failure of a launch inside an orchestration (0 = none);
     // reported and cleared by the entry point that made the launches.
     int deferred_error = 0;
@@ -88,6 +152,7 @@ enum Epi : int {
     EPI_STORE_F32 = 1,   // C (fp32, ldc) = acc
     EPI_RESID_F32 = 2,   // C (fp32, ldc) += acc
     EPI_SWIGLU = 3,      // W holds gate/up blocks of 128 rows; C[m, j] = silu(gate) * up, N = I
+    EPI_PARTIAL_F32 = 4, // split-K unit s writes its fp32 partial to C[s][m][n] (ldc = N)
 };
 
 // Token id of flattened row r: tokens[(r / T) * ld + off + r % T].
@@ -105,11 +170,13 @@ struct PosIndex {
 // Where the log-prob / argmax of flattened logits row r goes.  b = r / T, t = r % T;
 // the row is skipped when t >= out_lim; target = tgt[b * tgt_ld + tgt_off + t];
 // outputs at index b * out_ld + out_off + t.
-// Rows are numbered from row0 (a chunk of a larger set of rows).
+// Rows are numbered from row0 (a chunk of a larger set of rows).  With dyn_off set,
+// *dyn_off (read on the device) is added to the output index.
 struct OutIndex {
     int T, out_lim, out_ld, out_off;
     const int32_t* tgt;
     int tgt_ld, tgt_off, row0;
+    const int32_t* dyn_off = nullptr;
 };
 
 void launch_embed(const void* E, int dtype, int V, int H, TokIndex tok, int M, float* x,
@@ -118,13 +185,24 @@ void launch_embed(const void* E, int dtype, int V, int H, TokIndex tok, int M, f
 void launch_rmsnorm(const float* x, int in_step, int in_off, const float* g, int H, float eps,
                     void* out, int out_dtype, int M, cudaStream_t s);
 // Per-head RMSNorm of q and k, RoPE of q and k, q written in place, k and v to the cache.
+// part != nullptr: read q/k/v as the sum of S fp32 split-K partials [S][M][(nq+2nkv) d].
 void launch_qk_norm_rope(void* qkv, int dtype, int M, int nq, int nkv, int d, const float* gq,
                          const float* gk, float eps, const float* rope_cos, const float* rope_sin,
                          int max_positions, PosIndex pos, void* k_cache, void* v_cache,
-                         int max_seq, uint32_t* status, cudaStream_t s);
+                         int max_seq, uint32_t* status, cudaStream_t s,
+                         const float* part = nullptr, int S = 0);
+// Residual add of S split-K partials [S][M][H] into x, then RMSNorm -> bf16.
+void launch_rmsnorm_resid(float* x, const float* part, int S, const float* g, int H, float eps,
+                          bf16* out, int M, cudaStream_t s);
+// SwiGLU of the summed gate/up partials [S][M][2I] -> h [M, I] bf16.
+void launch_swiglu_partials(const float* part, int S, bf16* h, int M, int I, cudaStream_t s);
 void launch_swiglu(const void* gu, void* h, int dtype, int M, int I, cudaStream_t s);
 void launch_logits_reduce(const float* logits, int M, int V, OutIndex oi, float* lp,
                           int32_t* argmax, uint32_t* status, cudaStream_t s);
+// Rollout cursor: s = *step; pos[b] = P + s; tok[b] = seq[b, P + s]; tgt[b] = seq[b, P + s + 1];
+// *out_off = s + 1; *step = s + 1.
+void launch_rollout_prepare(const int32_t* seq, int L, int P, int B, int32_t* step, int32_t* pos,
+                            int32_t* tok, int32_t* tgt, int32_t* out_off, cudaStream_t s);
 void launch_rope_table(float* cos_t, float* sin_t, int max_positions, int d, double theta,
                        cudaStream_t s);
 void launch_widen_gain(const void* src, int dtype, float* dst, int n, cudaStream_t s);
@@ -145,14 +223,35 @@ void launch_gemv_bf16(const bf16* A, int lda, const bf16* W, void* C, int ldc, i
 bool gemm_tc_supported(const void* A, int lda, int N, int K);
 int launch_gemm_tc(const bf16* A, int lda, const bf16* W, void* C, int ldc, int M, int N, int K,
                    int epi, int num_sms, uint32_t* status, cudaStream_t s);
+int gemm_tc_split(int N, int K, int num_sms);
+int launch_gemm_tc_splitk(const bf16* A, int lda, const bf16* W, float* part, int M, int N, int K,
+                          int n_split, int num_sms, uint32_t* status, cudaStream_t s);
 
 // Kernel selection (k_dispatch.cu).  linear: C = A W^T with epilogue `epi`; for
 // EPI_SWIGLU, N is the SwiGLU width I and W holds 2 I interleaved rows; `gu` is
 // scratch [M, 2 I] for paths that cannot fuse the SwiGLU epilogue.
 void linear(Model& m, const void* A, int lda, const void* W, void* C, int ldc, int M, int N,
             int K, int epi, void* gu, cudaStream_t s);
-void launch_attention(const Model& m, const void* q, int q_ld, const void* k_cache,
-                      const void* v_cache, int M, int max_batch, int max_seq, PosIndex pos,
-                      void* o, cudaStream_t s);
+// Decode rows (pos.T == 1) of a bf16 model go to the split tensor-core kernel,
+// whose partials use `scratch` (attn_decode_scratch_bytes); other cases run the
+// SIMT kernel.
+void launch_attention(Model& m, const void* q, int q_ld, const void* k_cache, const void* v_cache,
+                      int M, int max_batch, int max_seq, PosIndex pos, void* o, void* scratch,
+                      cudaStream_t s);
+// Causal tensor-core attention for prefill / scoring (k_attn_prefill.cu): M = B x T
+// query rows at positions start .. start+T-1; head_dim 128.
+bool attn_prefill_supported(int d, int nq, int nkv);
+int launch_attn_prefill(const bf16* q, int q_ld, const void* k_layer, int nq, int nkv,
+                        int max_batch, int max_seq, int B, int T, int start, bf16* o,
+                        uint32_t* status, cudaStream_t s);
+// Split tensor-core decode attention (k_attn_decode.cu); head_dim 128, G <= 8.
+void attn_decode_split(int B, int nkv, int max_seq, int num_sms, int* chunk, int* n_split);
+size_t attn_decode_scratch_bytes(int B, int nq, int nkv, int max_seq, int num_sms);
+// Merge tickets inside that scratch; zero them (B * nkv ints) before a decode step.
+int* attn_decode_tickets(void* scratch, int B, int nq, int nkv, int max_seq, int num_sms);
+bool attn_decode_supported(int d, int nq, int nkv);
+int launch_attn_decode(const bf16* q, int q_ld, const void* k_layer, int nq, int nkv,
+                       int max_batch, int max_seq, int B, PosIndex pos, void* scratch, bf16* o,
+                       int num_sms, uint32_t* status, cudaStream_t s);
 
 }  // namespace qk

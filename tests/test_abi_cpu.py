@@ -1,0 +1,82 @@
+"""The C ABI on a machine without a GPU: libqk.so builds, loads, exports every
+function include/*.h declares, and its host-only entry points (presets, tensor
+counts, packed sizes, argument validation, error strings) behave as declared.
+No call here touches a device."""
+import ctypes
+import glob
+import os
+import re
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+@pytest.fixture(scope="module")
+def lib():
+    from paper_2609_12471_gb300 import build
+    path = build.build()
+    return ctypes.CDLL(path)
+
+
+def _declared():
+    names = set()
+    for h in glob.glob(os.path.join(ROOT, "include", "*.h")):
+        src = open(h).read()
+        src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+        names |= set(re.findall(r"^\s*(?:const\s+)?[\w]+\s*\**\s+\**(qk_\w+)\s*\(", src, flags=re.M))
+    return names
+
+
+def test_every_declared_symbol_is_exported(lib):
+    names = _declared()
+    assert len(names) >= 18, names
+    missing = [n for n in sorted(names) if not hasattr(lib, n)]
+    assert not missing, f"declared but not exported: {missing}"
+
+
+def test_binding_covers_the_declared_abi():
+    import paper_2609_12471_gb300 as qk
+    assert set(qk.exported_symbols()) == _declared()
+
+
+def test_presets_and_sizes():
+    import paper_2609_12471_gb300 as qk
+    c = qk.qk_config_preset("q8b")
+    assert (c.n_layers, c.hidden, c.n_q_heads, c.n_kv_heads, c.head_dim, c.intermediate,
+            c.vocab, c.dtype) == (36, 4096, 32, 8, 128, 12288, 151936, qk.QK_DTYPE_BF16)
+    assert c.rms_eps == 1e-6 and c.rope_theta == 1e6
+    assert qk.qk_weight_count(c) == 3 + 11 * 36
+    # bf16 weights (8.19e9 params) + fp32 gains + RoPE tables + alignment
+    nbytes = qk.qk_model_packed_bytes(c)
+    params = 2 * 151936 * 4096 + 36 * (192937984) 
+    assert 2 * params < nbytes < 2 * params + 64 * 2**20
+    t = qk.qk_config_preset("tiny_fp32")
+    assert (t.n_layers, t.hidden, t.dtype) == (2, 256, qk.QK_DTYPE_F32)
+    one = qk.qk_config_preset("q8b_layer")
+    assert one.n_layers == 1 and qk.qk_weight_count(one) == 14
+
+
+@pytest.mark.parametrize("field,value,code", [
+    ("dtype", 7, -3), ("head_dim", 96, -3), ("hidden", 100, -2), ("intermediate", 100, -2),
+    ("vocab", 3, -2), ("n_kv_heads", 3, -2), ("reserved", 1, -1), ("max_positions", 0, -1),
+])
+def test_config_validation_errors(field, value, code):
+    import paper_2609_12471_gb300 as qk
+    c = qk.qk_config_preset("q8b")
+    setattr(c, field, value)
+    with pytest.raises(qk.QKError) as e:
+        qk.qk_model_packed_bytes(c)
+    assert e.value.code == code
+    assert qk.qk_last_error()
+
+
+def test_unknown_preset_and_null_arguments(lib):
+    import paper_2609_12471_gb300 as qk
+    with pytest.raises(qk.QKError) as e:
+        qk.qk_config_preset("nope")
+    assert e.value.code == qk.QK_EINVAL and "nope" in str(e.value)
+    lib.qk_model_packed_bytes.argtypes = [ctypes.c_void_p, ctypes.c_void_p]
+    assert lib.qk_model_packed_bytes(None, None) == qk.QK_EINVAL
+    lib.qk_workspace_bytes.argtypes = [ctypes.c_void_p] + [ctypes.c_int] * 4 + [ctypes.c_void_p]
+    assert lib.qk_workspace_bytes(None, 0, 1, 1, 1, None) == qk.QK_EINVAL

@@ -36,7 +36,7 @@ def _ref(A, W, epi, C0):
 
 
 CASES = [  # (M, N, K)
-    (1, 384, 256), (5, 128, 4096), (16, 640, 192), (17, 384, 256), (31, 128, 64),
+    (1, 384, 256), (4, 256, 512), (5, 128, 4096), (16, 640, 192), (17, 384, 256), (31, 128, 64),
     (33, 256, 4096), (64, 128, 512), (100, 384, 256), (129, 256, 320), (300, 128, 4096),
     (1000, 640, 256),
 ]

@@ -153,3 +153,29 @@ def test_bad_position_sets_status(tiny):
     dec.decode_step(kv, 2, 8, torch.ones(2, dtype=torch.int32, device="cuda"), pos)
     import paper_2609_12471_gb300 as qk
     assert dec.check_status() & qk.QK_STATUS_BAD_POS
+
+
+def test_rollout_inside_caller_graph_capture(tiny):
+    """Inside a caller's own stream capture the rollout launches its steps directly
+    (no nested capture); replaying the caller's graph gives the direct call's numbers."""
+    import torch
+    s, W, dec = tiny
+    B, P, N = 2, 16, 6
+    seq = torch.tensor(synth.tokens((B, P + N + 1), s.vocab, stream=80), dtype=torch.int32,
+                       device="cuda")
+    kv = dec.new_kv(B, P + N)
+    ref = dec.rollout(kv, B, P + N, seq, P).clone()
+    out = torch.empty(B, N + 1, device="cuda")
+    side = torch.cuda.Stream()
+    side.wait_stream(torch.cuda.current_stream())
+    with torch.cuda.stream(side):
+        dec.rollout(kv, B, P + N, seq, P, logprobs=out)  # warm the workspace outside capture
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g, stream=side, capture_error_mode="thread_local"):
+            dec.rollout(kv, B, P + N, seq, P, logprobs=out)
+    torch.cuda.current_stream().wait_stream(side)
+    out.zero_()
+    g.replay()
+    torch.cuda.synchronize()
+    assert dec.check_status() == 0
+    assert torch.equal(out, ref)
