@@ -66,6 +66,7 @@ __global__ void __launch_bounds__(128)
     volatile int* abort_flag = (volatile int*)(full + kStages);
 
     pdl_wait();
+    pdl_trigger();  // the next kernel may launch once every CTA of this grid is resident
     const int split = blockIdx.x;
     const int b = blockIdx.y / nkv, kvh = blockIdx.y % nkv;
     const int G = nq / nkv;
@@ -289,18 +290,28 @@ typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t,
 
 }  // namespace
 
-// Chunking of the key range: about two resident CTAs per SM (two fit in shared
-// memory), chunks of whole 64-key tiles.
+// Chunking of the key range into whole 64-key tiles.  With two resident CTAs
+// per SM, the time is modelled as waves x (tiles per CTA + 1.5 tiles of fixed
+// cost: prologue, pipeline fill, partial write and merge); the chunk with the
+// lowest cost wins (ties go to the longer chunk).
 void attn_decode_split(int B, int nkv, int max_seq, int num_sms, int* chunk, int* n_split) {
     const int pairs = B * nkv;
-    int want = (2 * num_sms + pairs - 1) / pairs;
-    const int max_split = (max_seq + kTileKeys - 1) / kTileKeys;
-    if (want < 1) want = 1;
-    if (want > max_split) want = max_split;
-    int c = (max_seq + want - 1) / want;
-    c = (c + kTileKeys - 1) / kTileKeys * kTileKeys;
-    *chunk = c;
-    *n_split = (max_seq + c - 1) / c;
+    const int n_tiles = (max_seq + kTileKeys - 1) / kTileKeys;
+    const int slots = 2 * num_sms;
+    int best_c = n_tiles;
+    double best = 1e30;
+    for (int c = n_tiles; c >= 1; --c) {
+        const int splits = (n_tiles + c - 1) / c;
+        const long ctas = (long)pairs * splits;
+        const long waves = (ctas + slots - 1) / slots;
+        const double cost = (double)waves * (c + 1.5);
+        if (cost < best - 1e-9) {
+            best = cost;
+            best_c = c;
+        }
+    }
+    *chunk = best_c * kTileKeys;
+    *n_split = (n_tiles + best_c - 1) / best_c;
 }
 
 // Partials [B nq][n_split][128] fp32, (m, l) [B nq][n_split], then the merge tickets

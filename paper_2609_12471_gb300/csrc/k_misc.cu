@@ -36,6 +36,7 @@ template <typename T>
 __global__ void embed_kernel(const T* __restrict__ E, int V, int H, TokIndex tok,
                              float* __restrict__ x, uint32_t* status) {
     pdl_wait();
+    pdl_trigger();  // short kernel: let the next one launch and prefetch now
     int r = blockIdx.x;
     int id = tok.ptr[(size_t)(r / tok.T) * tok.ld + tok.off + r % tok.T];
     if (id < 0 || id >= V) {
@@ -64,6 +65,7 @@ __global__ void rmsnorm_kernel(const float* __restrict__ x, int in_step, int in_
                                OutT* __restrict__ out) {
     __shared__ float red[32];
     pdl_wait();
+    pdl_trigger();  // short kernel: let the next one launch and prefetch now
     int r = blockIdx.x;
     const float* xr = x + ((size_t)r * in_step + in_off) * H;
     float ss = 0.f;
@@ -98,6 +100,7 @@ __global__ void __launch_bounds__(128)
     __shared__ float red[4];
     __shared__ float slice_ss;
     pdl_wait();
+    pdl_trigger();  // short kernel: let the next one launch and prefetch now
     const int CL = (int)cluster.num_blocks();
     const int rank = (int)cluster.block_rank();
     const int r = blockIdx.y;
@@ -156,6 +159,7 @@ void launch_rmsnorm_resid(float* x, const float* part, int S, const float* g, in
 __global__ void swiglu_partials_kernel(const float* __restrict__ part, int S, size_t split_stride,
                                        bf16* __restrict__ h, int M, int I) {
     pdl_wait();
+    pdl_trigger();  // short kernel: let the next one launch and prefetch now
     size_t n = (size_t)M * I;
     for (size_t e = blockIdx.x * (size_t)blockDim.x + threadIdx.x; e < n;
          e += (size_t)gridDim.x * blockDim.x) {
@@ -208,6 +212,7 @@ __global__ void qk_norm_rope_kernel(T* __restrict__ qkv, int nq, int nkv, const 
                                     const float* __restrict__ part, int S, size_t split_stride) {
     constexpr int E = D / 32, HALF = D / 2;
     pdl_wait();
+    pdl_trigger();  // short kernel: let the next one launch and prefetch now
     int lane = threadIdx.x & 31;
     int hh = blockIdx.y * (blockDim.x >> 5) + (threadIdx.x >> 5);
     int nh = nq + 2 * nkv;
@@ -294,6 +299,7 @@ void launch_qk_norm_rope(void* qkv, int dtype, int M, int nq, int nkv, int d, co
 template <typename T>
 __global__ void swiglu_kernel(const T* __restrict__ gu, T* __restrict__ h, int M, int I) {
     pdl_wait();
+    pdl_trigger();  // short kernel: let the next one launch and prefetch now
     size_t n = (size_t)M * I;
     for (size_t e = blockIdx.x * (size_t)blockDim.x + threadIdx.x; e < n;
          e += (size_t)gridDim.x * blockDim.x) {
@@ -327,6 +333,7 @@ __global__ void logits_reduce_kernel(const float* __restrict__ logits, int V, Ou
     __shared__ int red_i[32];
     __shared__ float red[32];
     pdl_wait();
+    pdl_trigger();  // short kernel: let the next one launch and prefetch now
     int r = blockIdx.x;
     int g = oi.row0 + r;
     int b = g / oi.T, t = g % oi.T;
@@ -390,6 +397,7 @@ __global__ void rollout_prepare_kernel(const int32_t* __restrict__ seq, int L, i
                                        int32_t* step, int32_t* pos, int32_t* tok, int32_t* tgt,
                                        int32_t* out_off) {
     pdl_wait();
+    pdl_trigger();  // short kernel: let the next one launch and prefetch now
     const int s = *step;
     __syncthreads();  // every thread has read the step before it advances
     for (int b = threadIdx.x; b < B; b += blockDim.x) {

@@ -1,0 +1,124 @@
+"""Full-size checks of the 36-layer Qwen3-8B-shaped bf16 model, in the launch
+configurations the benchmark times.
+
+At these sizes the fp64 oracle cannot evaluate every output, so each test
+combines (a) properties that hold at any size (finite log-probs, log p <= 0,
+arg-max inside the vocabulary, a clean status word), (b) agreement between two
+independent GPU code paths for the same quantity (decode steps with split-K
+linears and split decode attention vs. teacher-forced scoring with whole GEMMs
+and causal prefill attention), within the bf16 noise tolerance, and (c) oracle
+samples where causality lets a short prefix stand for the whole sequence.
+
+Workloads: rollout batch 16, prompt 512, 1024 teacher-forced decode steps;
+scoring batch 32 x 4096; the long-trajectory endpoint at batch 64 (prefill of
+8191 tokens per row, then one decode step at position 8191, cache 8192).
+"""
+import gc
+
+import numpy as np
+import pytest
+
+import oracle
+import synth
+from _bf16_floor import forward_logits_bf16_activations
+from _gpu import decoder
+
+pytestmark = pytest.mark.gpu
+LP_ABS = 5e-2
+# Two bf16 code paths each carry about the bf16 floor's error (max ~0.1, mean ~0.025
+# in log-prob on the 36-layer model); their difference is bounded by twice that.
+# A structural error (wrong position, layer or row) moves log-probs by O(1).
+TWO_PATH_MAX, TWO_PATH_MEAN = 0.4, 0.06
+
+
+@pytest.fixture(scope="module")
+def q8b():
+    s = synth.shape("q8b")
+    dec, W = decoder(s)
+    yield s, W, dec
+    dec.close()
+
+
+def _props(lp, am, V):
+    assert np.all(np.isfinite(lp)) and np.all(lp <= 1e-4)
+    if am is not None:
+        assert am.min() >= 0 and am.max() < V
+
+
+def _oracle_lp_tol(s, W, toks, n_scored):
+    """Oracle log-probs of the first n_scored positions of toks, and the bf16-floor
+    tolerance for them (max(5e-2, 2 x floor))."""
+    z = oracle.forward_logits(s, W, toks)[:n_scored]
+    zf = forward_logits_bf16_activations(s, W, toks)[:n_scored]
+    lp = oracle.token_logprobs(z, toks[1:n_scored + 1])
+    lpf = oracle.token_logprobs(zf, toks[1:n_scored + 1])
+    return lp, max(LP_ABS, 2 * float(np.max(np.abs(lpf - lp))))
+
+
+def test_rollout_b16_p512_n1024(q8b):
+    import torch
+    s, W, dec = q8b
+    B, P, N = 16, 512, 1024
+    seq = synth.tokens((B, P + N + 1), s.vocab)  # the bench's token batch (stream 0)
+    d = torch.tensor(seq, dtype=torch.int32, device="cuda")
+    kv = dec.new_kv(B, P + N)
+    am = torch.empty(B, N + 1, dtype=torch.int32, device="cuda")
+    lp = dec.rollout(kv, B, P + N, d, P, argmax=am).cpu().numpy()
+    assert dec.check_status() == 0
+    _props(lp, am.cpu().numpy(), s.vocab)
+    del kv
+    # (b) scoring the same sequences: lp_score[b, P - 1 + j] scores c[j] like lp[b, j]
+    lp_s = dec.score(d[:, :P + N + 1].contiguous()).cpu().numpy()
+    assert dec.check_status() == 0
+    diff = np.abs(lp_s[:, P - 1:] - lp)
+    assert diff.max() <= TWO_PATH_MAX and diff.mean() <= TWO_PATH_MEAN, (diff.max(), diff.mean())
+    # (c) oracle on row 0: the log-probs of c[0..3] need positions 0 .. P+3
+    ref, tol = _oracle_lp_tol(s, W, seq[0, :P + 5], P + 4)
+    assert np.max(np.abs(lp[0, :4] - ref[P - 1:P + 3])) <= tol
+
+
+def test_score_b32_t4096(q8b):
+    import torch
+    s, W, dec = q8b
+    B, T = 32, 4096
+    toks = synth.tokens((B, T), s.vocab, stream=100)  # the bench's scoring batch
+    am = torch.empty(B, T - 1, dtype=torch.int32, device="cuda")
+    lp = dec.score(torch.tensor(toks, dtype=torch.int32, device="cuda"), argmax=am).cpu().numpy()
+    assert dec.check_status() == 0
+    _props(lp, am.cpu().numpy(), s.vocab)
+    # (c) causality: positions t < 63 of rows 0 and 31 depend only on their first 64 tokens
+    for b in (0, B - 1):
+        ref, tol = _oracle_lp_tol(s, W, toks[b, :64], 63)
+        assert np.max(np.abs(lp[b, :63] - ref)) <= tol
+
+
+def test_long_trajectory_endpoint_b64_s8192(q8b):
+    import torch
+    s, W, dec = q8b
+    B, S = 64, 8192
+    seq = torch.tensor(synth.tokens((B, S + 1), s.vocab, stream=7), dtype=torch.int32,
+                       device="cuda")
+    # path 1: scoring of all 8192 scored positions
+    lp_s = dec.score(seq).cpu().numpy()
+    assert dec.check_status() == 0
+    dec._ws.clear()
+    gc.collect()
+    torch.cuda.empty_cache()
+    # path 2: prefill of 8191 tokens (scores position 8190), decode step at 8191 (scores 8191)
+    kv = dec.new_kv(B, S)
+    l1 = torch.empty(B, device="cuda")
+    a1 = torch.empty(B, dtype=torch.int32, device="cuda")
+    dec.prefill(kv, B, S, seq[:, :S - 1].contiguous(), 0, None, seq[:, S - 1].contiguous(), l1, a1)
+    l2 = torch.empty(B, device="cuda")
+    a2 = torch.empty(B, dtype=torch.int32, device="cuda")
+    pos = torch.full((B,), S - 1, dtype=torch.int32, device="cuda")
+    dec.decode_step(kv, B, S, seq[:, S - 1].contiguous(), pos, None, seq[:, S].contiguous(), l2, a2)
+    assert dec.check_status() == 0
+    got = np.stack([l1.cpu().numpy(), l2.cpu().numpy()], axis=1)
+    _props(got, np.stack([a1.cpu().numpy(), a2.cpu().numpy()]), s.vocab)
+    diff = np.abs(got - lp_s[:, S - 2:S])
+    assert diff.max() <= TWO_PATH_MAX and diff.mean() <= TWO_PATH_MEAN, (diff.max(), diff.mean())
+    del kv
+    dec._ws.clear()
+    gc.collect()
+    torch.cuda.empty_cache()
