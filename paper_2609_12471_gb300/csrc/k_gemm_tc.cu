@@ -40,26 +40,31 @@ __host__ __device__ constexpr int pow2_at_least(int v) {
     return p;
 }
 
-template <int BN, bool SWIGLU, int STAGES>
+template <int BN, bool SWIGLU, int STAGES, bool FUSED = false>
 struct Cfg {
     static constexpr int A_ROWS = SWIGLU ? 256 : 128;
     static constexpr int A_BYTES = A_ROWS * 128;
     static constexpr int B_BYTES = BN * 128;
     static constexpr int ACC_COLS = SWIGLU ? 2 * BN : BN;
     static constexpr int TMEM_COLS = pow2_at_least(2 * ACC_COLS);
-    static constexpr int SMEM = STAGES * (A_BYTES + B_BYTES) + 1024 /*align*/ + 256 /*barriers*/;
+    // fused epilogue scratch (floats): s_row[64], p_row[64] (int), red[4][64], xch[128][BN], flag
+    static constexpr int FUSE_FLOATS = FUSED ? 64 + 64 + 4 * 64 + 128 * BN + 4 : 0;
+    static constexpr int SMEM =
+        STAGES * (A_BYTES + B_BYTES) + 1024 /*align*/ + 256 /*barriers*/ + FUSE_FLOATS * 4;
     static_assert(TMEM_COLS <= 512, "accumulators exceed TMEM");
     static_assert(BN % 16 == 0 && BN >= 16 && BN <= 256, "invalid MMA N");
 };
 
 __device__ __forceinline__ float silu(float g) { return g / (1.f + __expf(-g)); }
 
-template <int BN, bool SWIGLU, int STAGES>
+__device__ __forceinline__ void epi_bar() { asm volatile("bar.sync 1, 128;" ::: "memory"); }
+
+template <int BN, bool SWIGLU, int STAGES, bool FUSED>
 __global__ void __launch_bounds__(kThreads, 1)
     gemm_tc_kernel(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ CUtensorMap tmX,
                    void* __restrict__ C, int ldc, int M, int N, int K, int epi, int n_split,
-                   uint32_t* __restrict__ status) {
-    using G = Cfg<BN, SWIGLU, STAGES>;
+                   uint32_t* __restrict__ status, const __grid_constant__ Fuse fz) {
+    using G = Cfg<BN, SWIGLU, STAGES, FUSED>;
     extern __shared__ uint8_t smem_raw[];
     uint8_t* smem = (uint8_t*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
     uint8_t* sA = smem;
@@ -71,6 +76,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     uint64_t* drain = tempty + 2;
     uint32_t* tmem_slot = (uint32_t*)(drain + 1);
     volatile int* abort_flag = (volatile int*)(tmem_slot + 1);
+    float* fscr = (float*)(smem + STAGES * (G::A_BYTES + G::B_BYTES) + 256);  // fused scratch
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int n_feat = N / 128;
@@ -212,6 +218,222 @@ __global__ void __launch_bounds__(kThreads, 1)
                 tc::mbar_wait_drain(drain, 0);
             }
         }
+    } else if constexpr (FUSED) {
+        // ---------------------------------------------------- fused epilogue (warps 2..5)
+        // One token tile (M <= BN).  Each unit: TMEM -> registers, release the
+        // accumulator, write the fp32 partial, take the tile's ticket; the last unit
+        // of a tile sums the partials in split order and applies fz.op.
+        const int q = warp & 3;
+        const int e = threadIdx.x - 64;  // 0..127 across the epilogue warps
+        const int row = q * 32 + lane;   // accumulator row (TMEM lane) = feature within the tile
+        // Per-token values used by every unit are computed once: the input-norm scale
+        // s_row and (QKV) the clamped cache position p_row.  Loops over the tile's
+        // tokens are predicated (no early exit) so their independent loads overlap.
+        float* s_row = fscr;                      // [64]
+        int* p_row = (int*)(fscr + 64);           // [64]
+        float* red = fscr + 128;                  // [4][64]
+        float* xch = fscr + 128 + 256;            // [128][BN]
+        volatile int* flag = (volatile int*)(fscr + 128 + 256 + 128 * BN);
+        if (fz.op == FUSE_QKV || fz.op == FUSE_SWIGLU || fz.op == FUSE_COLSCALE) {
+            for (int j = e; j < BN; j += 128) {
+                float t = 0.f;
+                if (j < M)
+                    for (int i = 0; i < fz.n_ssq; ++i) t += fz.ssq_in[(size_t)i * M + j];
+                s_row[j] = j < M ? rsqrtf(t / (float)fz.H + fz.eps) : 0.f;
+            }
+        }
+        if (fz.op == FUSE_QKV) {
+            const int lim = fz.max_seq < fz.max_positions ? fz.max_seq : fz.max_positions;
+            for (int j = e; j < BN; j += 128) {
+                int p = 0;
+                if (j < M) {
+                    p = fz.pos.pos_dev ? fz.pos.pos_dev[j] : fz.pos.start;
+                    if (p < 0 || p >= lim) {
+                        atomicOr(fz.status, QK_STATUS_BAD_POS);
+                        p = p < 0 ? 0 : lim - 1;
+                    }
+                }
+                p_row[j] = p;
+            }
+        }
+        epi_bar();
+        int acc = 0;
+        uint32_t acc_phase = 0;
+        const size_t sstride = (size_t)M * N;
+        for (int t = blockIdx.x; t < num_tiles; t += gridDim.x) {
+            const int split = t % n_split, feat = t / n_split;
+            bool ok = tc::mbar_wait(&tfull[acc], acc_phase, abort_flag);
+            ok = __all_sync(0xffffffffu, ok);
+            if (!ok) break;
+            tc::fence_after_sync();
+            const uint32_t tbase = tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(acc * G::ACC_COLS);
+            float v[BN];
+#pragma unroll
+            for (int j = 0; j < BN; ++j) v[j] = 0.f;
+#pragma unroll
+            for (int c0 = 0; c0 < BN; c0 += 16) {
+                if (c0 < M) {
+                    uint32_t r[16];
+                    tc::tmem_ld16(tbase + c0, r);
+                    tc::tmem_wait_ld();
+#pragma unroll
+                    for (int j = 0; j < 16; ++j) v[c0 + j] = __uint_as_float(r[j]);
+                }
+            }
+            tc::fence_before_sync();
+            __syncwarp();
+            if (lane == 0) tc::mbar_arrive(&tempty[acc]);
+            acc ^= 1;
+            if (acc == 0) acc_phase ^= 1;
+
+            const int f = feat * 128 + row;
+            const bool swiglu = fz.op == FUSE_SWIGLU;
+            const bool ticketed = swiglu || n_split > 1;
+            const int key = swiglu ? feat >> 1 : feat;
+            if (ticketed) {
+#pragma unroll
+                for (int j = 0; j < BN; ++j)
+                    if (j < M) fz.part[split * sstride + (size_t)j * N + f] = v[j];
+                // The barrier orders every epilogue thread's stores before the ticket
+                // thread's fence, which publishes them at GPU scope before the atomic; the
+                // last unit's ticket thread fences again before its peers read (L2 loads).
+                epi_bar();
+                if (e == 0) {
+                    const int need = swiglu ? 2 * n_split : n_split;
+                    __threadfence();
+                    const bool last = atomicAdd(&fz.tickets[key], 1) == need - 1;
+                    if (last) __threadfence();
+                    *flag = last;
+                }
+                epi_bar();
+                const bool last = *flag != 0;
+                if (!last) continue;  // uniform over the four warps
+                if (!swiglu) {
+                    // sum in split order; the loads of one split are independent, so each
+                    // split costs one L2 round trip (this unit's own split is in registers)
+                    float a[BN];
+#pragma unroll
+                    for (int j = 0; j < BN; ++j) a[j] = 0.f;
+                    for (int sp = 0; sp < n_split; ++sp) {
+                        if (sp == split) {
+#pragma unroll
+                            for (int j = 0; j < BN; ++j) a[j] += v[j];
+                        } else {
+                            float ld[BN];
+#pragma unroll
+                            for (int j = 0; j < BN; ++j)
+                                ld[j] = j < M ? __ldcg(&fz.part[sp * sstride + (size_t)j * N + f]) : 0.f;
+#pragma unroll
+                            for (int j = 0; j < BN; ++j) a[j] += ld[j];
+                        }
+                    }
+#pragma unroll
+                    for (int j = 0; j < BN; ++j) v[j] = a[j];
+                }
+            }
+            if (fz.op == FUSE_QKV) {
+                const int hh = feat, nq = fz.nq, nkv = fz.nkv;
+#pragma unroll
+                for (int j = 0; j < BN; ++j) v[j] *= s_row[j];
+                if (hh < nq + nkv) {
+                    // per-head RMSNorm over the 128 rows of the tile, per token
+#pragma unroll
+                    for (int j = 0; j < BN; ++j) {
+                        float sq = v[j] * v[j];
+#pragma unroll
+                        for (int o = 16; o > 0; o >>= 1) sq += __shfl_xor_sync(0xffffffffu, sq, o);
+                        if (lane == 0) red[q * 64 + j] = sq;
+                    }
+                    epi_bar();
+                    const float gain = hh < nq ? fz.gq[row] : fz.gk[row];
+#pragma unroll
+                    for (int j = 0; j < BN; ++j) {
+                        const float tot = red[j] + red[64 + j] + red[128 + j] + red[192 + j];
+                        v[j] = v[j] * rsqrtf(tot / 128.f + fz.eps) * gain;
+                        xch[row * BN + j] = v[j];
+                    }
+                    epi_bar();
+                    // rotate-half RoPE: row i < 64 pairs with row i + 64
+                    const int i = row & 63;
+                    float c[BN], sn[BN];
+#pragma unroll
+                    for (int j = 0; j < BN; ++j) {
+                        c[j] = fz.rope_cos[(size_t)p_row[j] * 64 + i];
+                        sn[j] = fz.rope_sin[(size_t)p_row[j] * 64 + i];
+                    }
+#pragma unroll
+                    for (int j = 0; j < BN; ++j) {
+                        const float partner = xch[(row ^ 64) * BN + j];
+                        const float o = row < 64 ? v[j] * c[j] - partner * sn[j] : v[j] * c[j] + partner * sn[j];
+                        if (j < M) {
+                            if (hh < nq)
+                                fz.q_out[(size_t)j * fz.q_ld + (size_t)hh * 128 + row] = __float2bfloat16_rn(o);
+                            else
+                                fz.k_cache[(((size_t)j * nkv + (hh - nq)) * fz.max_seq + p_row[j]) * 128 + row] =
+                                    __float2bfloat16_rn(o);
+                        }
+                    }
+                } else {
+#pragma unroll
+                    for (int j = 0; j < BN; ++j)
+                        if (j < M)
+                            fz.v_cache[(((size_t)j * nkv + (hh - nq - nkv)) * fz.max_seq + p_row[j]) * 128 + row] =
+                                __float2bfloat16_rn(v[j]);
+                }
+            } else if (fz.op == FUSE_RESID) {
+                const float gn = fz.g_next[f];
+                float xo[BN];
+#pragma unroll
+                for (int j = 0; j < BN; ++j) xo[j] = j < M ? fz.x[(size_t)j * N + f] : 0.f;
+#pragma unroll
+                for (int j = 0; j < BN; ++j) {
+                    const float xn = xo[j] + v[j];
+                    if (j < M) {
+                        fz.x[(size_t)j * N + f] = xn;
+                        fz.xg_out[(size_t)j * N + f] = __float2bfloat16_rn(xn * gn);
+                    }
+                    float sq = j < M ? xn * xn : 0.f;
+#pragma unroll
+                    for (int k = 16; k > 0; k >>= 1) sq += __shfl_xor_sync(0xffffffffu, sq, k);
+                    if (lane == 0) red[q * 64 + j] = sq;
+                }
+                epi_bar();
+                if (e < M) fz.ssq_out[(size_t)feat * M + e] = red[e] + red[64 + e] + red[128 + e] + red[192 + e];
+            } else if (fz.op == FUSE_SWIGLU) {
+                // this unit completed the pair: gate tile 2 jb, up tile 2 jb + 1
+                const int jb = feat >> 1, I = N / 2;
+                const int fg = (2 * jb) * 128 + row, fu = fg + 128;
+                float gs[BN], us[BN];
+#pragma unroll
+                for (int j = 0; j < BN; ++j) gs[j] = us[j] = 0.f;
+                for (int sp = 0; sp < n_split; ++sp) {
+                    float lg[BN], lu[BN];
+#pragma unroll
+                    for (int j = 0; j < BN; ++j) {
+                        lg[j] = j < M ? __ldcg(&fz.part[sp * sstride + (size_t)j * N + fg]) : 0.f;
+                        lu[j] = j < M ? __ldcg(&fz.part[sp * sstride + (size_t)j * N + fu]) : 0.f;
+                    }
+#pragma unroll
+                    for (int j = 0; j < BN; ++j) {
+                        gs[j] += lg[j];
+                        us[j] += lu[j];
+                    }
+                }
+#pragma unroll
+                for (int j = 0; j < BN; ++j) {
+                    const float g = gs[j] * s_row[j], u = us[j] * s_row[j];
+                    if (j < M)
+                        fz.h_out[(size_t)j * I + (size_t)jb * 128 + row] =
+                            __float2bfloat16_rn(g / (1.f + __expf(-g)) * u);
+                }
+            } else if (fz.op == FUSE_COLSCALE) {
+#pragma unroll
+                for (int j = 0; j < BN; ++j)
+                    if (j < M) ((float*)C)[(size_t)j * ldc + f] = v[j] * s_row[j];
+            }
+            if (ticketed && e == 0) fz.tickets[key] = 0;
+            epi_bar();  // scratch (red, xch, flag) is reused by the next unit
+        }
     } else {
         // ---------------------------------------------------- epilogue (warps 2..5)
         const int q = warp & 3;
@@ -305,13 +527,14 @@ bool make_map(CUtensorMap* map, const void* base, int inner, int rows, int ld, i
     return r == CUDA_SUCCESS;
 }
 
-template <int BN, bool SWIGLU, int STAGES>
+template <int BN, bool SWIGLU, int STAGES, bool FUSED = false>
 int launch_cfg(const bf16* A, int lda, const bf16* W, void* C, int ldc, int M, int N, int K,
-               int epi, int n_split, int num_sms, uint32_t* status, cudaStream_t s) {
-    using G = Cfg<BN, SWIGLU, STAGES>;
+               int epi, int n_split, int num_sms, uint32_t* status, cudaStream_t s,
+               const Fuse* fz = nullptr) {
+    using G = Cfg<BN, SWIGLU, STAGES, FUSED>;
     static bool attr_set = false;
     if (!attr_set) {
-        if (cudaFuncSetAttribute(gemm_tc_kernel<BN, SWIGLU, STAGES>,
+        if (cudaFuncSetAttribute(gemm_tc_kernel<BN, SWIGLU, STAGES, FUSED>,
                                  cudaFuncAttributeMaxDynamicSharedMemorySize, G::SMEM) != cudaSuccess)
             return QK_ECUDA;
         attr_set = true;
@@ -322,8 +545,9 @@ int launch_cfg(const bf16* A, int lda, const bf16* W, void* C, int ldc, int M, i
         return QK_ECUDA;
     const int tiles = (N / 128) * ((M + BN - 1) / BN) * n_split;
     const int grid = tiles < num_sms ? tiles : num_sms;
-    launch_k(gemm_tc_kernel<BN, SWIGLU, STAGES>, dim3(grid), dim3(kThreads), G::SMEM, s, tmW, tmX, C,
-             ldc, M, N, K, epi, n_split, status);
+    Fuse none{};
+    launch_k(gemm_tc_kernel<BN, SWIGLU, STAGES, FUSED>, dim3(grid), dim3(kThreads), G::SMEM, s, tmW,
+             tmX, C, ldc, M, N, K, epi, n_split, status, fz ? *fz : none);
     note_launch();
     return QK_OK;
 }
@@ -353,17 +577,18 @@ int launch_gemm_tc(const bf16* A, int lda, const bf16* W, void* C, int ldc, int 
 }
 
 // Split count for a decode-sized GEMM (one token tile): the smallest S whose
-// N/128 * S work units fill the persistent grid to >= 90 % of its last round,
-// with at least 4 k-blocks per unit; the best S found otherwise.
+// N/128 * S work units fill the persistent grid to >= 80 % of its last round,
+// with at least 12 k-blocks per unit (each unit ends in a fused epilogue); the
+// best S found otherwise.
 int gemm_tc_split(int N, int K, int num_sms) {
     const int n_feat = N / 128, kblocks = K / kBK;
     int best = 1;
     double best_eff = 0.0;
-    for (int S = 1; S <= 32 && kblocks / S >= 4; ++S) {
+    for (int S = 1; S <= 32 && kblocks / S >= 12; ++S) {
         const int units = n_feat * S;
         const int rounds = (units + num_sms - 1) / num_sms;
         const double eff = (double)units / ((double)rounds * num_sms);
-        if (eff >= 0.9) return S;
+        if (eff >= 0.8) return S;
         if (eff > best_eff + 1e-9) {
             best_eff = eff;
             best = S;
@@ -372,19 +597,19 @@ int gemm_tc_split(int N, int K, int num_sms) {
     return best;
 }
 
-// Decode-sized linear (M <= 64 rows) split over K: unit `split` writes its fp32 partial
-// product to part[split][M][N]; consumers add the n_split partials in order.
-int launch_gemm_tc_splitk(const bf16* A, int lda, const bf16* W, float* part, int M, int N, int K,
-                          int n_split, int num_sms, uint32_t* status, cudaStream_t s) {
+// Decode linear with a fused epilogue (see Fuse); one token tile of M <= 64 rows.
+int launch_gemm_tc_fused(const bf16* A, int lda, const bf16* W, float* out, int M, int N, int K,
+                         int n_split, const Fuse& f, int num_sms, uint32_t* status, cudaStream_t s) {
     if (M <= 0) return QK_OK;
+    if (M > 64) return QK_ESHAPE;
     if (M <= 16)
-        return launch_cfg<16, false, 8>(A, lda, W, part, N, M, N, K, EPI_PARTIAL_F32, n_split,
-                                        num_sms, status, s);
+        return launch_cfg<16, false, 8, true>(A, lda, W, out, N, M, N, K, EPI_PARTIAL_F32, n_split,
+                                              num_sms, status, s, &f);
     if (M <= 32)
-        return launch_cfg<32, false, 8>(A, lda, W, part, N, M, N, K, EPI_PARTIAL_F32, n_split,
-                                        num_sms, status, s);
-    return launch_cfg<64, false, 8>(A, lda, W, part, N, M, N, K, EPI_PARTIAL_F32, n_split,
-                                    num_sms, status, s);
+        return launch_cfg<32, false, 8, true>(A, lda, W, out, N, M, N, K, EPI_PARTIAL_F32, n_split,
+                                              num_sms, status, s, &f);
+    return launch_cfg<64, false, 7, true>(A, lda, W, out, N, M, N, K, EPI_PARTIAL_F32, n_split,
+                                          num_sms, status, s, &f);
 }
 
 }  // namespace qk

@@ -1,7 +1,6 @@
 // Elementwise and row-wise kernels of the decoder forward pass: embedding
 // gather, RMSNorm, per-head QK-RMSNorm + RoPE + KV-cache write, SwiGLU,
 // vocabulary log-softmax / gather / argmax, and the load-time RoPE table.
-#include <cooperative_groups.h>
 #include <math.h>
 
 #include "qk_internal.cuh"
@@ -58,6 +57,43 @@ void launch_embed(const void* E, int dtype, int V, int H, TokIndex tok, int M, f
         launch_k(embed_kernel<float>, dim3(M), dim3(256), 0, s, (const float*)E, V, H, tok, x, status);
 }
 
+// ---------------------------------------------------------------- embedding + gain (fused decode)
+// One CTA per (128-feature tile, row): x = E[token] (or the given x), xg = bf16(x * g) and
+// the tile's sum of squares ssq[tile][row] (the input-norm statistics of the next linear).
+__global__ void __launch_bounds__(128)
+    embed_gain_kernel(const bf16* __restrict__ E, int V, TokIndex tok, int do_embed,
+                      float* __restrict__ x, const float* __restrict__ g, bf16* __restrict__ xg,
+                      float* __restrict__ ssq, int M, int H, uint32_t* status) {
+    __shared__ float red[4];
+    pdl_wait();
+    const int m = blockIdx.y, f = blockIdx.x * 128 + threadIdx.x;
+    float xv;
+    if (do_embed) {
+        int id = tok.ptr[(size_t)(m / tok.T) * tok.ld + tok.off + m % tok.T];
+        if (id < 0 || id >= V) {
+            if (threadIdx.x == 0 && blockIdx.x == 0) atomicOr(status, QK_STATUS_BAD_TOKEN);
+            id = 0;
+        }
+        xv = __bfloat162float(E[(size_t)id * H + f]);
+        x[(size_t)m * H + f] = xv;
+    } else {
+        xv = x[(size_t)m * H + f];
+    }
+    xg[(size_t)m * H + f] = __float2bfloat16_rn(xv * g[f]);
+    const float sq = warp_sum(xv * xv);
+    if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = sq;
+    __syncthreads();
+    if (threadIdx.x == 0) ssq[(size_t)blockIdx.x * M + m] = red[0] + red[1] + red[2] + red[3];
+}
+
+void launch_embed_gain(const void* E, int V, TokIndex tok, bool do_embed, float* x, const float* g,
+                       bf16* xg, float* ssq, int M, int H, uint32_t* status, cudaStream_t s) {
+    note_launch();
+    if (M <= 0) return;
+    launch_k(embed_gain_kernel, dim3(H / 128, M), dim3(128), 0, s, (const bf16*)E, V, tok,
+             do_embed ? 1 : 0, x, g, xg, ssq, M, H, status);
+}
+
 // ---------------------------------------------------------------- RMSNorm
 template <typename OutT>
 __global__ void rmsnorm_kernel(const float* __restrict__ x, int in_step, int in_off,
@@ -86,105 +122,6 @@ __global__ void rmsnorm_kernel(const float* __restrict__ x, int in_step, int in_
     }
 }
 
-// x[r] += sum_{s < S} part[s][r] (fixed order), written back; then out[r] = RMSNorm(x[r]) * g.
-// Folds the residual add of a split-K linear into the norm that reads the residual next.
-// A row is spread over a cluster of CL CTAs (128 threads, 4 consecutive elements per
-// thread and pass); each CTA reduces the sum of squares of its slice and the CTAs of
-// the cluster exchange those sums through distributed shared memory.
-__global__ void __launch_bounds__(128)
-    rmsnorm_resid_kernel(float* __restrict__ x, const float* __restrict__ part, int S,
-                         size_t split_stride, const float* __restrict__ g, int H, float eps,
-                         bf16* __restrict__ out) {
-    namespace cg = cooperative_groups;
-    cg::cluster_group cluster = cg::this_cluster();
-    __shared__ float red[4];
-    __shared__ float slice_ss;
-    pdl_wait();
-    pdl_trigger();  // short kernel: let the next one launch and prefetch now
-    const int CL = (int)cluster.num_blocks();
-    const int rank = (int)cluster.block_rank();
-    const int r = blockIdx.y;
-    const int slice = H / CL;
-    float* xr = x + (size_t)r * H + (size_t)rank * slice;
-    const float* pr = part + (size_t)r * H + (size_t)rank * slice;
-    float ss = 0.f;
-    for (int i = threadIdx.x * 4; i < slice; i += blockDim.x * 4) {
-        float4 v = *reinterpret_cast<const float4*>(xr + i);
-        for (int sp = 0; sp < S; ++sp) {
-            float4 a = *reinterpret_cast<const float4*>(pr + sp * split_stride + i);
-            v.x += a.x; v.y += a.y; v.z += a.z; v.w += a.w;
-        }
-        if (S > 0) *reinterpret_cast<float4*>(xr + i) = v;
-        ss += v.x * v.x + v.y * v.y + v.z * v.z + v.w * v.w;
-    }
-    ss = warp_sum(ss);
-    if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = ss;
-    __syncthreads();
-    if (threadIdx.x == 0) slice_ss = red[0] + red[1] + red[2] + red[3];
-    cluster.sync();
-    float tot = 0.f;
-    for (int c = 0; c < CL; ++c) tot += *cluster.map_shared_rank(&slice_ss, c);
-    const float scale = rsqrtf(tot / (float)H + eps);
-    bf16* o = out + (size_t)r * H + (size_t)rank * slice;
-    const float* gg = g + (size_t)rank * slice;
-    for (int i = threadIdx.x * 4; i < slice; i += blockDim.x * 4) {
-        float4 v = *reinterpret_cast<const float4*>(xr + i);
-        float4 w = *reinterpret_cast<const float4*>(gg + i);
-        o[i + 0] = __float2bfloat16_rn(v.x * scale * w.x);
-        o[i + 1] = __float2bfloat16_rn(v.y * scale * w.y);
-        o[i + 2] = __float2bfloat16_rn(v.z * scale * w.z);
-        o[i + 3] = __float2bfloat16_rn(v.w * scale * w.w);
-    }
-    cluster.sync();  // keep this CTA's slice_ss alive until every peer has read it
-}
-
-// Cluster size: up to 8 CTAs, each slice a multiple of 512 elements.
-static int resid_cluster(int H) {
-    int cl = 8;
-    while (cl > 1 && (H % (cl * 512) != 0)) cl >>= 1;
-    return cl;
-}
-
-void launch_rmsnorm_resid(float* x, const float* part, int S, const float* g, int H, float eps,
-                          bf16* out, int M, cudaStream_t s) {
-    note_launch();
-    if (M <= 0) return;
-    const int cl = resid_cluster(H);
-    launch_k_cluster(rmsnorm_resid_kernel, dim3(cl, M), dim3(128), 0, s, cl, x, part, S,
-                     (size_t)M * H, g, H, eps, out);
-}
-
-// h[r, j] = silu(sum_s gate) * (sum_s up) from split-K partials of the packed gate/up linear
-// (part[s][r][2I], blocks of 128 gate columns each followed by the matching 128 up columns).
-__global__ void swiglu_partials_kernel(const float* __restrict__ part, int S, size_t split_stride,
-                                       bf16* __restrict__ h, int M, int I) {
-    pdl_wait();
-    pdl_trigger();  // short kernel: let the next one launch and prefetch now
-    size_t n = (size_t)M * I;
-    for (size_t e = blockIdx.x * (size_t)blockDim.x + threadIdx.x; e < n;
-         e += (size_t)gridDim.x * blockDim.x) {
-        size_t m = e / I;
-        int j = (int)(e % I);
-        size_t c = m * 2 * I + (size_t)(j >> 7) * 256 + (j & 127);
-        float gs = 0.f, us = 0.f;
-        for (int sp = 0; sp < S; ++sp) {
-            gs += part[sp * split_stride + c];
-            us += part[sp * split_stride + c + 128];
-        }
-        h[e] = __float2bfloat16_rn(gs / (1.f + expf(-gs)) * us);
-    }
-}
-
-void launch_swiglu_partials(const float* part, int S, bf16* h, int M, int I, cudaStream_t s) {
-    note_launch();
-    if (M <= 0) return;
-    size_t n = (size_t)M * I;
-    int blocks = (int)((n + 255) / 256);
-    if (blocks > 65535) blocks = 65535;
-    launch_k(swiglu_partials_kernel, dim3(blocks), dim3(256), 0, s, part, S, (size_t)M * 2 * I, h,
-             M, I);
-}
-
 void launch_rmsnorm(const float* x, int in_step, int in_off, const float* g, int H, float eps,
                     void* out, int out_dtype, int M, cudaStream_t s) {
     note_launch();
@@ -200,16 +137,12 @@ void launch_rmsnorm(const float* x, int in_step, int in_off, const float* g, int
 
 // ---------------------------------------------------------------- QK-norm + RoPE + cache write
 // One warp per (token, head) of the fused qkv row; lane owns elements lane + 32 i.
-// With part != nullptr the projections come from S fp32 split-K partials
-// part[s][r][(nq + 2 nkv) D] (summed in fixed order) instead of the qkv buffer;
-// q is still written to the qkv buffer, k and v to the cache.
 template <typename T, int D>
 __global__ void qk_norm_rope_kernel(T* __restrict__ qkv, int nq, int nkv, const float* __restrict__ gq,
                                     const float* __restrict__ gk, float eps,
                                     const float* __restrict__ rc, const float* __restrict__ rs,
                                     int max_positions, PosIndex pos, T* __restrict__ kc,
-                                    T* __restrict__ vc, int max_seq, uint32_t* status,
-                                    const float* __restrict__ part, int S, size_t split_stride) {
+                                    T* __restrict__ vc, int max_seq, uint32_t* status) {
     constexpr int E = D / 32, HALF = D / 2;
     pdl_wait();
     pdl_trigger();  // short kernel: let the next one launch and prefetch now
@@ -227,23 +160,13 @@ __global__ void qk_norm_rope_kernel(T* __restrict__ qkv, int nq, int nkv, const 
     }
     T* src = qkv + (size_t)r * nh * D + (size_t)hh * D;
     float e[E];
-    if (part) {
-        const float* pp = part + (size_t)r * nh * D + (size_t)hh * D;
 #pragma unroll
-        for (int i = 0; i < E; ++i) {
-            float v = 0.f;
-            for (int sp = 0; sp < S; ++sp) v += pp[sp * split_stride + lane + 32 * i];
-            e[i] = v;
-        }
-    } else {
-#pragma unroll
-        for (int i = 0; i < E; ++i) e[i] = to_f(src[lane + 32 * i]);
-    }
+    for (int i = 0; i < E; ++i) e[i] = to_f(src[lane + 32 * i]);
     if (hh >= nq + nkv) {  // value head: straight to the cache
         int kvh = hh - nq - nkv;
         T* dst = vc + (((size_t)b * nkv + kvh) * max_seq + p) * D;
 #pragma unroll
-        for (int i = 0; i < E; ++i) dst[lane + 32 * i] = from_f<T>(e[i]);
+        for (int i = 0; i < E; ++i) dst[lane + 32 * i] = src[lane + 32 * i];
         return;
     }
     const float* g = hh < nq ? gq : gk;
@@ -278,15 +201,13 @@ __global__ void qk_norm_rope_kernel(T* __restrict__ qkv, int nq, int nkv, const 
 void launch_qk_norm_rope(void* qkv, int dtype, int M, int nq, int nkv, int d, const float* gq,
                          const float* gk, float eps, const float* rope_cos, const float* rope_sin,
                          int max_positions, PosIndex pos, void* k_cache, void* v_cache,
-                         int max_seq, uint32_t* status, cudaStream_t s, const float* part,
-                         int S) {
+                         int max_seq, uint32_t* status, cudaStream_t s) {
     note_launch();
     if (M <= 0) return;
     dim3 grid(M, (nq + 2 * nkv + 7) / 8);
 #define QK_NR(T, D)                                                                          \
     launch_k(qk_norm_rope_kernel<T, D>, grid, dim3(256), 0, s, (T*)qkv, nq, nkv, gq, gk, eps,  \
-             rope_cos, rope_sin, max_positions, pos, (T*)k_cache, (T*)v_cache, max_seq, status, \
-             part, S, (size_t)M * (nq + 2 * nkv) * d)
+             rope_cos, rope_sin, max_positions, pos, (T*)k_cache, (T*)v_cache, max_seq, status)
     if (dtype == QK_DTYPE_BF16) {
         if (d == 128) QK_NR(bf16, 128); else QK_NR(bf16, 64);
     } else {

@@ -112,6 +112,9 @@ struct Workspace {
     void* skv;      // scoring: K and V of one layer, [2][B, nkv, T, d]
     void* attn;     // decode: split-attention partials (bf16 models)
     float* part;    // decode: split-K partial products of the linear layers (bf16 models)
+    bf16* xg;       // decode: bf16(x * g) for the next linear's input (fused path)
+    float* ssq;     // decode: per-128-feature-tile sums of squares of x [H/128, M]
+    int* tickets;   // decode: last-unit tickets of the fused linears
     float* logits;  // [logit_rows, V]
     int logit_rows;
     size_t total;
@@ -133,10 +136,16 @@ struct Splits {
     int qkv, o, gu, d;
 };
 
+// Decode steps of bf16 models with head_dim 128 and up to kSplitMaxRows rows run the
+// fused path: split-K tcgen05 linears whose last unit per tile applies QK-norm + RoPE,
+// the residual add (with the next norm's statistics) or SwiGLU in its epilogue.
+static const int kTicketSlots = 1024;
+
 static bool use_splitk(const Model& m, int M) {
     const qk_config& c = m.cfg;
-    return c.dtype == QK_DTYPE_BF16 && M > kGemvMaxRows && M <= kSplitMaxRows && c.hidden % 128 == 0 &&
-           (c.n_q_heads * c.head_dim) % 128 == 0 && ((c.n_q_heads + 2 * c.n_kv_heads) * c.head_dim) % 128 == 0;
+    return c.dtype == QK_DTYPE_BF16 && M >= 1 && M <= kSplitMaxRows && c.head_dim == 128 &&
+           c.hidden % 128 == 0 && (2 * c.intermediate) / 128 <= 2 * kTicketSlots &&
+           ((c.n_q_heads + 2 * c.n_kv_heads) * c.head_dim) / 128 <= kTicketSlots;
 }
 
 static Splits decode_splits(const Model& m) {
@@ -180,8 +189,11 @@ static int workspace_layout(const Model& m, int kind, int B, int T, int max_seq,
     w->h = take(M * I * es);
     w->gu = c.dtype == QK_DTYPE_F32 ? take(M * 2 * I * es) : nullptr;  // unfused SwiGLU path only
     w->skv = kind == QK_CALL_SCORE ? take(2 * (size_t)B * nkv * T * d * es) : nullptr;
-    w->part = kind == QK_CALL_DECODE && use_splitk(m, B) ? (float*)take(splitk_part_floats(m, B) * 4)
-                                                         : nullptr;
+    const bool fused = kind == QK_CALL_DECODE && use_splitk(m, B);
+    w->part = fused ? (float*)take(splitk_part_floats(m, B) * 4) : nullptr;
+    w->xg = fused ? (bf16*)take(M * H * 2) : nullptr;
+    w->ssq = fused ? (float*)take((H / 128) * M * 4) : nullptr;
+    w->tickets = fused ? (int*)take(kTicketSlots * 4) : nullptr;
     w->attn = nullptr;
     if (kind == QK_CALL_DECODE && c.dtype == QK_DTYPE_BF16 &&
         attn_decode_supported(c.head_dim, c.n_q_heads, c.n_kv_heads)) {
@@ -242,49 +254,71 @@ static void run_layer(Model& m, int l, const Workspace& w, int M, PosIndex pos,
     prof_close(m, pr, s);
 }
 
-// One decoder layer of a decode step with split-K linear layers.  The down
-// projection's partials are left in w.part for the next consumer (the next
-// layer's input norm, the final norm, or flush_residual); `pending` says whether
-// the previous layer left such partials.
-static void run_layer_splitk(Model& m, int l, const Workspace& w, int M, PosIndex pos,
-                             const KVView& kv, bool pending, cudaStream_t s) {
+// One decoder layer of a fused decode step.  On entry w.x holds the residual,
+// w.xg = bf16(x * g_attn) and w.ssq its tile sums of squares; on exit the same for
+// the layer's output with gain g_next (the next layer's input norm or the final norm).
+static void run_layer_fused(Model& m, int l, const Workspace& w, int M, PosIndex pos,
+                            const KVView& kv, const float* g_next, cudaStream_t s) {
     const qk_config& c = m.cfg;
     const LayerW& L = m.layers[l];
     const Splits sp = decode_splits(m);
-    int H = c.hidden, d = c.head_dim, nq = c.n_q_heads, nkv = c.n_kv_heads, I = c.intermediate;
-    int nqkv = (nq + 2 * nkv) * d;
-    float eps = (float)c.rms_eps;
-    bf16* u = (bf16*)w.u;
-    bool pr;
-    auto gemm = [&](const void* A, int lda, const void* W, int N, int K, int S) {
-        int rc = launch_gemm_tc_splitk((const bf16*)A, lda, (const bf16*)W, w.part, M, N, K, S,
-                                       m.num_sms, m.status, s);
+    const int H = c.hidden, d = c.head_dim, nq = c.n_q_heads, nkv = c.n_kv_heads, I = c.intermediate;
+    const int nqkv = (nq + 2 * nkv) * d;
+    Fuse f{};
+    f.tickets = w.tickets;
+    f.part = w.part;
+    f.ssq_in = w.ssq;
+    f.n_ssq = H / 128;
+    f.H = H;
+    f.eps = (float)c.rms_eps;
+    f.status = m.status;
+    auto gemm = [&](const void* A, int lda, const void* W, int N, int K, int S, const Fuse& fz) {
+        int rc = launch_gemm_tc_fused((const bf16*)A, lda, (const bf16*)W, nullptr, M, N, K, S, fz,
+                                      m.num_sms, m.status, s);
         if (rc != QK_OK && !m.deferred_error) m.deferred_error = rc;
     };
-    if (pending)
-        launch_rmsnorm_resid(w.x, w.part, sp.d, L.attn_norm, H, eps, u, M, s);
-    else
-        launch_rmsnorm(w.x, 1, 0, L.attn_norm, H, eps, u, c.dtype, M, s);
+    bool pr;
+    Fuse fq = f;
+    fq.op = FUSE_QKV;
+    fq.nq = nq;
+    fq.nkv = nkv;
+    fq.gq = L.q_norm;
+    fq.gk = L.k_norm;
+    fq.rope_cos = m.rope_cos;
+    fq.rope_sin = m.rope_sin;
+    fq.max_positions = c.max_positions;
+    fq.pos = pos;
+    fq.q_out = (bf16*)w.qkv;
+    fq.q_ld = nqkv;
+    fq.k_cache = (bf16*)kv.k(l);
+    fq.v_cache = (bf16*)kv.v(l);
+    fq.max_seq = kv.max_seq;
     pr = prof_open(m, QK_PROF_QKV, s);
-    gemm(u, H, L.w_qkv, nqkv, H, sp.qkv);
+    gemm(w.xg, H, L.w_qkv, nqkv, H, sp.qkv, fq);
     prof_close(m, pr, s);
-    launch_qk_norm_rope(w.qkv, c.dtype, M, nq, nkv, d, L.q_norm, L.k_norm, eps, m.rope_cos,
-                        m.rope_sin, c.max_positions, pos, kv.k(l), kv.v(l), kv.max_seq, m.status, s,
-                        w.part, sp.qkv);
     pr = prof_open(m, QK_PROF_ATTN, s);
     launch_attention(m, w.qkv, nqkv, kv.k(l), kv.v(l), M, kv.max_batch, kv.max_seq, pos, w.o,
                      w.attn, s);
     prof_close(m, pr, s);
+    Fuse fo = f;
+    fo.op = FUSE_RESID;
+    fo.x = w.x;
+    fo.g_next = L.mlp_norm;
+    fo.xg_out = w.xg;
+    fo.ssq_out = w.ssq;
     pr = prof_open(m, QK_PROF_O, s);
-    gemm(w.o, nq * d, L.w_o, H, nq * d, sp.o);
+    gemm(w.o, nq * d, L.w_o, H, nq * d, sp.o, fo);
     prof_close(m, pr, s);
-    launch_rmsnorm_resid(w.x, w.part, sp.o, L.mlp_norm, H, eps, u, M, s);
+    Fuse fg = f;
+    fg.op = FUSE_SWIGLU;
+    fg.h_out = (bf16*)w.h;
     pr = prof_open(m, QK_PROF_GATE_UP, s);
-    gemm(u, H, L.w_gu, 2 * I, H, sp.gu);
+    gemm(w.xg, H, L.w_gu, 2 * I, H, sp.gu, fg);
     prof_close(m, pr, s);
-    launch_swiglu_partials(w.part, sp.gu, (bf16*)w.h, M, I, s);
+    Fuse fd = fo;
+    fd.g_next = g_next;
     pr = prof_open(m, QK_PROF_DOWN, s);
-    gemm(w.h, I, L.w_d, H, I, sp.d);
+    gemm(w.h, I, L.w_d, H, I, sp.d, fd);
     prof_close(m, pr, s);
 }
 
@@ -621,12 +655,29 @@ static int decode_impl(Model& m, void* kv, int max_batch, int max_seq, TokIndex 
     m.in_decode = true;
     launch_embed(m.embed, m.cfg.dtype, m.cfg.vocab, m.cfg.hidden, tok, B, w.x, m.status, s);
     if (w.part) {
-        for (int l = 0; l < m.cfg.n_layers; ++l) run_layer_splitk(m, l, w, B, pos, view, l > 0, s);
-        // the last layer's down-projection partials join the residual in the final norm's pass
-        launch_rmsnorm_resid(w.x, w.part, decode_splits(m).d, m.final_norm, m.cfg.hidden,
-                             (float)m.cfg.rms_eps, (bf16*)w.u, B, s);
-        if (logits || lp || am)
-            run_head(m, w, B, 1, 0, logits ? logits : w.logits, oi, lp, am, s, /*normed=*/true);
+        const qk_config& c = m.cfg;
+        QK_TRY_CUDA(cudaMemsetAsync(w.tickets, 0, kTicketSlots * sizeof(int), s));
+        launch_embed_gain(m.embed, c.vocab, tok, true, w.x, m.layers[0].attn_norm, w.xg, w.ssq, B,
+                          c.hidden, m.status, s);
+        for (int l = 0; l < c.n_layers; ++l)
+            run_layer_fused(m, l, w, B, pos, view,
+                            l + 1 < c.n_layers ? m.layers[l + 1].attn_norm : m.final_norm, s);
+        if (logits || lp || am) {
+            // logits = s_m * (W_lm (x g_final)), s_m the final RMSNorm scale of row m
+            float* z = logits ? logits : w.logits;
+            Fuse fl{};
+            fl.op = FUSE_COLSCALE;
+            fl.ssq_in = w.ssq;
+            fl.n_ssq = c.hidden / 128;
+            fl.H = c.hidden;
+            fl.eps = (float)c.rms_eps;
+            bool pr = prof_open(m, QK_PROF_LM_HEAD, s);
+            int rc = launch_gemm_tc_fused(w.xg, c.hidden, (const bf16*)m.lm_head, z, B, c.vocab,
+                                          c.hidden, 1, fl, m.num_sms, m.status, s);
+            prof_close(m, pr, s);
+            if (rc != QK_OK && !m.deferred_error) m.deferred_error = rc;
+            if (lp || am) launch_logits_reduce(z, B, c.vocab, oi, lp, am, m.status, s);
+        }
     } else {
         for (int l = 0; l < m.cfg.n_layers; ++l) run_layer(m, l, w, B, pos, view, s);
         if (logits || lp || am) run_head(m, w, B, 1, 0, logits ? logits : w.logits, oi, lp, am, s);
@@ -662,11 +713,12 @@ int qk_decode_layer(qk_model* mh, int layer, void* kv, int max_batch, int max_se
     QK_TRY(clear_attn_tickets(m, w, B, max_seq, s));
     m.in_decode = true;
     if (w.part) {
-        run_layer_splitk(m, layer, w, B, PosIndex{pos, 0, 1}, cache_view(m, kv, max_batch, max_seq),
-                         false, s);
-        // add the down projection's partials to x (the normed output is not needed)
-        launch_rmsnorm_resid(w.x, w.part, decode_splits(m).d, m.final_norm, m.cfg.hidden,
-                             (float)m.cfg.rms_eps, (bf16*)w.u, B, s);
+        const LayerW& L = m.layers[layer];
+        QK_TRY_CUDA(cudaMemsetAsync(w.tickets, 0, kTicketSlots * sizeof(int), s));
+        launch_embed_gain(nullptr, m.cfg.vocab, TokIndex{}, false, w.x, L.attn_norm, w.xg, w.ssq, B,
+                          m.cfg.hidden, m.status, s);
+        run_layer_fused(m, layer, w, B, PosIndex{pos, 0, 1}, cache_view(m, kv, max_batch, max_seq),
+                        L.attn_norm, s);
     } else {
         run_layer(m, layer, w, B, PosIndex{pos, 0, 1}, cache_view(m, kv, max_batch, max_seq), s);
     }

@@ -43,27 +43,6 @@ inline void launch_k(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t sme
     cudaLaunchKernelEx(&cfg, kernel, std::forward<Args>(args)...);
 }
 
-// As launch_k, with a thread-block cluster of cluster_x CTAs along x.
-template <typename... KArgs, typename... Args>
-inline void launch_k_cluster(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem,
-                             cudaStream_t s, int cluster_x, Args&&... args) {
-    cudaLaunchConfig_t cfg = {};
-    cfg.gridDim = grid;
-    cfg.blockDim = block;
-    cfg.dynamicSmemBytes = smem;
-    cfg.stream = s;
-    cudaLaunchAttribute attr[2];
-    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-    attr[0].val.programmaticStreamSerializationAllowed = 1;
-    attr[1].id = cudaLaunchAttributeClusterDimension;
-    attr[1].val.clusterDim.x = cluster_x;
-    attr[1].val.clusterDim.y = 1;
-    attr[1].val.clusterDim.z = 1;
-    cfg.attrs = attr;
-    cfg.numAttrs = 2;
-    cudaLaunchKernelEx(&cfg, kernel, std::forward<Args>(args)...);
-}
-
 // bf16 linear layers over at most this many token rows stream the weights through
 // the CUDA-core GEMV (fused epilogues); larger ones run on the tensor cores.
 constexpr int kGemvMaxRows = 4;
@@ -185,17 +164,10 @@ void launch_embed(const void* E, int dtype, int V, int H, TokIndex tok, int M, f
 void launch_rmsnorm(const float* x, int in_step, int in_off, const float* g, int H, float eps,
                     void* out, int out_dtype, int M, cudaStream_t s);
 // Per-head RMSNorm of q and k, RoPE of q and k, q written in place, k and v to the cache.
-// part != nullptr: read q/k/v as the sum of S fp32 split-K partials [S][M][(nq+2nkv) d].
 void launch_qk_norm_rope(void* qkv, int dtype, int M, int nq, int nkv, int d, const float* gq,
                          const float* gk, float eps, const float* rope_cos, const float* rope_sin,
                          int max_positions, PosIndex pos, void* k_cache, void* v_cache,
-                         int max_seq, uint32_t* status, cudaStream_t s,
-                         const float* part = nullptr, int S = 0);
-// Residual add of S split-K partials [S][M][H] into x, then RMSNorm -> bf16.
-void launch_rmsnorm_resid(float* x, const float* part, int S, const float* g, int H, float eps,
-                          bf16* out, int M, cudaStream_t s);
-// SwiGLU of the summed gate/up partials [S][M][2I] -> h [M, I] bf16.
-void launch_swiglu_partials(const float* part, int S, bf16* h, int M, int I, cudaStream_t s);
+                         int max_seq, uint32_t* status, cudaStream_t s);
 void launch_swiglu(const void* gu, void* h, int dtype, int M, int I, cudaStream_t s);
 void launch_logits_reduce(const float* logits, int M, int V, OutIndex oi, float* lp,
                           int32_t* argmax, uint32_t* status, cudaStream_t s);
@@ -224,8 +196,61 @@ bool gemm_tc_supported(const void* A, int lda, int N, int K);
 int launch_gemm_tc(const bf16* A, int lda, const bf16* W, void* C, int ldc, int M, int N, int K,
                    int epi, int num_sms, uint32_t* status, cudaStream_t s);
 int gemm_tc_split(int N, int K, int num_sms);
-int launch_gemm_tc_splitk(const bf16* A, int lda, const bf16* W, float* part, int M, int N, int K,
-                          int n_split, int num_sms, uint32_t* status, cudaStream_t s);
+
+
+// Fused epilogue of a decode-sized split-K linear (one token tile, M <= 64 rows).
+// Every work unit writes its fp32 partial to part[split][M][N]; the last unit of a
+// tile (the last of a gate/up tile pair for FUSE_SWIGLU) takes the tile's ticket,
+// sums the partials in split order and applies `op`.  Tickets must be zero on
+// entry and are zero again on exit.  The linear's input is x * g (bf16, not yet
+// normalised); the RMSNorm scale s_m = rsqrt(sum_t ssq_in[t][m] / H + eps) of
+// token row m is applied after the product (W (x g s) = s W (x g)).
+enum FuseOp : int {
+    FUSE_NONE = 0,
+    FUSE_QKV = 1,       // tile = one head: s, per-head RMSNorm + RoPE for q/k, q -> q_out, k/v -> cache
+    FUSE_RESID = 2,     // x += sum; xg_out = bf16(x * g_next); ssq_out[tile][m] = sum of x^2 over the tile
+    FUSE_SWIGLU = 3,    // tiles 2j (gate) and 2j+1 (up): h[m, 128 j + r] = silu(s g) * (s u)
+    FUSE_COLSCALE = 4,  // fp32 store of s_m * (x g W^T)[m, n] (lm_head logits)
+};
+
+struct Fuse {
+    int op;
+    int* tickets;
+    float* part;
+    const float* ssq_in;  // [n_ssq][M]
+    int n_ssq, H;
+    float eps;
+    // FUSE_QKV
+    int nq, nkv;
+    const float* gq;
+    const float* gk;
+    const float* rope_cos;
+    const float* rope_sin;
+    int max_positions;
+    PosIndex pos;
+    bf16* q_out;
+    int q_ld;
+    bf16* k_cache;
+    bf16* v_cache;
+    int max_seq;
+    uint32_t* status;
+    // FUSE_RESID
+    float* x;
+    const float* g_next;
+    bf16* xg_out;
+    float* ssq_out;
+    // FUSE_SWIGLU
+    bf16* h_out;
+};
+
+// Decode linear with a fused epilogue (k_gemm_tc.cu): A = bf16 [M, K] (M <= 64),
+// W [N, K]; out is the op's fp32 logits for FUSE_COLSCALE, unused otherwise.
+int launch_gemm_tc_fused(const bf16* A, int lda, const bf16* W, float* out, int M, int N, int K,
+                         int n_split, const Fuse& f, int num_sms, uint32_t* status, cudaStream_t s);
+// x = E[token] (embed) or the given x; xg = bf16(x * g); ssq[t][m] = sum over features
+// 128 t .. 128 t + 127 of x^2 (k_misc.cu).
+void launch_embed_gain(const void* E, int V, TokIndex tok, bool do_embed, float* x, const float* g,
+                       bf16* xg, float* ssq, int M, int H, uint32_t* status, cudaStream_t s);
 
 // Kernel selection (k_dispatch.cu).  linear: C = A W^T with epilogue `epi`; for
 // EPI_SWIGLU, N is the SwiGLU width I and W holds 2 I interleaved rows; `gu` is
