@@ -11,7 +11,7 @@ samples where causality lets a short prefix stand for the whole sequence.
 
 Workloads: rollout batch 16, prompt 512, 1024 teacher-forced decode steps;
 scoring batch 32 x 4096; the long-trajectory endpoint at batch 64 (prefill of
-8191 tokens per row, then one decode step at position 8191, cache 8192).
+8190 tokens per row, then decode steps at positions 8190 and 8191, cache 8192).
 """
 import gc
 
@@ -95,28 +95,36 @@ def test_score_b32_t4096(q8b):
 def test_long_trajectory_endpoint_b64_s8192(q8b):
     import torch
     s, W, dec = q8b
-    B, S = 64, 8192
+    B, S = 64, 8192  # positions 0 .. S-1 fill the cache (and the RoPE table) exactly
     seq = torch.tensor(synth.tokens((B, S + 1), s.vocab, stream=7), dtype=torch.int32,
                        device="cuda")
-    # path 1: scoring of all 8192 scored positions
-    lp_s = dec.score(seq).cpu().numpy()
+    # path 1: scoring of the S-token trajectory (positions 0 .. S-2 predict tokens 1 .. S-1)
+    lp_s = dec.score(seq[:, :S].contiguous()).cpu().numpy()
     assert dec.check_status() == 0
     dec._ws.clear()
     gc.collect()
     torch.cuda.empty_cache()
-    # path 2: prefill of 8191 tokens (scores position 8190), decode step at 8191 (scores 8191)
+    # path 2: prefill of S-2 tokens (scores position S-3), decode at S-2 (scores S-2),
+    # then decode at S-1, the last cache slot (target: token S of the stream)
     kv = dec.new_kv(B, S)
-    l1 = torch.empty(B, device="cuda")
-    a1 = torch.empty(B, dtype=torch.int32, device="cuda")
-    dec.prefill(kv, B, S, seq[:, :S - 1].contiguous(), 0, None, seq[:, S - 1].contiguous(), l1, a1)
-    l2 = torch.empty(B, device="cuda")
-    a2 = torch.empty(B, dtype=torch.int32, device="cuda")
-    pos = torch.full((B,), S - 1, dtype=torch.int32, device="cuda")
-    dec.decode_step(kv, B, S, seq[:, S - 1].contiguous(), pos, None, seq[:, S].contiguous(), l2, a2)
+    got = []
+    ams = []
+    l0 = torch.empty(B, device="cuda")
+    a0 = torch.empty(B, dtype=torch.int32, device="cuda")
+    dec.prefill(kv, B, S, seq[:, :S - 2].contiguous(), 0, None, seq[:, S - 2].contiguous(), l0, a0)
+    got.append(l0)
+    ams.append(a0)
+    for p in (S - 2, S - 1):
+        lp = torch.empty(B, device="cuda")
+        am = torch.empty(B, dtype=torch.int32, device="cuda")
+        pos = torch.full((B,), p, dtype=torch.int32, device="cuda")
+        dec.decode_step(kv, B, S, seq[:, p].contiguous(), pos, None, seq[:, p + 1].contiguous(), lp, am)
+        got.append(lp)
+        ams.append(am)
     assert dec.check_status() == 0
-    got = np.stack([l1.cpu().numpy(), l2.cpu().numpy()], axis=1)
-    _props(got, np.stack([a1.cpu().numpy(), a2.cpu().numpy()]), s.vocab)
-    diff = np.abs(got - lp_s[:, S - 2:S])
+    got = np.stack([t.cpu().numpy() for t in got], axis=1)
+    _props(got, np.stack([t.cpu().numpy() for t in ams]), s.vocab)
+    diff = np.abs(got[:, :2] - lp_s[:, S - 3:S - 1])
     assert diff.max() <= TWO_PATH_MAX and diff.mean() <= TWO_PATH_MEAN, (diff.max(), diff.mean())
     del kv
     dec._ws.clear()
