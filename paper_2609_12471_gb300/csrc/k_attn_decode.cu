@@ -34,6 +34,7 @@ namespace {
 constexpr int kD = 128;          // head_dim of this kernel
 constexpr int kTileKeys = 64;    // keys per stage
 constexpr int kStages = 3;
+constexpr int kMergeChunks = 4;  // chunk partials per load batch of the final merge
 constexpr int kHalfBytes = kTileKeys * 128;   // one 64-dim box: 64 rows x 128 B
 constexpr int kTileBytes = 2 * kHalfBytes;    // K (or V) tile: dims 0..63 then 64..127
 constexpr int kStageBytes = 2 * kTileBytes;   // K tile then V tile
@@ -254,32 +255,54 @@ __global__ void __launch_bounds__(128)
     if (n_split == 1) return;
     // The last CTA of this (row, kv head) to finish merges the chunks' partials:
     //   o = sum_s 2^(m_s - M) O_s / sum_s 2^(m_s - M) l_s,  M = max_s m_s,
-    // then resets the ticket for the next layer.
+    // then resets the ticket for the next layer.  The barrier orders every thread's
+    // partial stores before thread 0's release; its acquire orders the merge's reads
+    // after the other chunks' stores.
     __shared__ int last;
     __syncthreads();
-    if (threadIdx.x == 0) {
-        __threadfence();
-        const int n_valid = min(n_split, p / chunk + 1);
-        last = atomicAdd(&tickets[b * nkv + kvh], 1) == n_valid - 1;
-    }
+    const int n_valid = min(n_split, p / chunk + 1);
+    if (threadIdx.x == 0)
+        last = tc::atom_add_acq_rel_gpu(&tickets[b * nkv + kvh], 1) == n_valid - 1;
     __syncthreads();
     if (!last) return;
-    __threadfence();
-    const int n_valid = min(n_split, p / chunk + 1);
-    for (int gg = 0; gg < G; ++gg) {
-        const size_t head = (size_t)b * nq + kvh * G + gg;
-        const int d = threadIdx.x;
-        float M = -INFINITY;
-        for (int sp = 0; sp < n_valid; ++sp) M = fmaxf(M, __ldcg(&part_ml[head * n_split + sp]).x);
-        float acc = 0.f, L = 0.f;
-        for (int sp = 0; sp < n_valid; ++sp) {
-            const float2 ml = __ldcg(&part_ml[head * n_split + sp]);
-            const float f = ml.x == -INFINITY ? 0.f : exp2f(ml.x - M);
-            acc += f * __ldcg(&part_o[(head * n_split + sp) * kD + d]);
-            L += f * ml.y;
+    // Online merge over the chunks in order, kMergeChunks at a time: every load of a
+    // batch is issued before any is used, so a batch costs one L2 round trip.
+    const int d = threadIdx.x;
+    float Mh[8], Ah[8], Lh[8];
+#pragma unroll
+    for (int gg = 0; gg < 8; ++gg) Mh[gg] = -INFINITY, Ah[gg] = 0.f, Lh[gg] = 0.f;
+    for (int base = 0; base < n_valid; base += kMergeChunks) {
+        float ov[8][kMergeChunks];
+        float2 ml[8][kMergeChunks];
+#pragma unroll
+        for (int gg = 0; gg < 8; ++gg)
+#pragma unroll
+            for (int k = 0; k < kMergeChunks; ++k) {
+                const bool v = gg < G && base + k < n_valid;
+                const size_t i = ((size_t)b * nq + kvh * G + gg) * n_split + base + k;
+                ov[gg][k] = v ? __ldcg(&part_o[i * kD + d]) : 0.f;
+                ml[gg][k] = v ? __ldcg(&part_ml[i]) : make_float2(-INFINITY, 0.f);
+            }
+#pragma unroll
+        for (int gg = 0; gg < 8; ++gg) {
+            float Mn = Mh[gg];
+#pragma unroll
+            for (int k = 0; k < kMergeChunks; ++k) Mn = fmaxf(Mn, ml[gg][k].x);
+            if (Mn == -INFINITY) continue;  // padding head
+            const float sc = Mh[gg] == -INFINITY ? 0.f : exp2f(Mh[gg] - Mn);
+            float A = Ah[gg] * sc, L = Lh[gg] * sc;
+#pragma unroll
+            for (int k = 0; k < kMergeChunks; ++k) {
+                const float f = ml[gg][k].x == -INFINITY ? 0.f : exp2f(ml[gg][k].x - Mn);
+                A += f * ov[gg][k];
+                L += f * ml[gg][k].y;
+            }
+            Mh[gg] = Mn, Ah[gg] = A, Lh[gg] = L;
         }
-        out[head * kD + d] = __float2bfloat16_rn(acc / L);
     }
+#pragma unroll
+    for (int gg = 0; gg < 8; ++gg)
+        if (gg < G) out[((size_t)b * nq + kvh * G + gg) * kD + d] = __float2bfloat16_rn(Ah[gg] / Lh[gg]);
     if (threadIdx.x == 0) tickets[b * nkv + kvh] = 0;
 }
 

@@ -47,8 +47,9 @@ struct Cfg {
     static constexpr int B_BYTES = BN * 128;
     static constexpr int ACC_COLS = SWIGLU ? 2 * BN : BN;
     static constexpr int TMEM_COLS = pow2_at_least(2 * ACC_COLS);
-    // fused epilogue scratch (floats): s_row[64], p_row[64] (int), red[4][64], xch[128][BN], flag
-    static constexpr int FUSE_FLOATS = FUSED ? 64 + 64 + 4 * 64 + 128 * BN + 4 : 0;
+    // fused epilogue scratch (floats): s_row[64], p_row[64] (int), red[4][64], xch[BN][128],
+    // cos / sin [2][BN][64], flag
+    static constexpr int FUSE_FLOATS = FUSED ? 64 + 64 + 4 * 64 + 128 * BN + 128 * BN + 4 : 0;
     static constexpr int SMEM =
         STAGES * (A_BYTES + B_BYTES) + 1024 /*align*/ + 256 /*barriers*/ + FUSE_FLOATS * 4;
     static_assert(TMEM_COLS <= 512, "accumulators exceed TMEM");
@@ -58,6 +59,81 @@ struct Cfg {
 __device__ __forceinline__ float silu(float g) { return g / (1.f + __expf(-g)); }
 
 __device__ __forceinline__ void epi_bar() { asm volatile("bar.sync 1, 128;" ::: "memory"); }
+
+// One level of a reduce-scatter butterfly over the warp: C values per lane become
+// C / 2, each the sum of two lanes' values; lanes with `mask` set keep the upper half.
+template <int C>
+__device__ __forceinline__ void rs_level(float* v, int lane, int mask) {
+    const bool up = (lane & mask) != 0;
+#pragma unroll
+    for (int i = 0; i < C / 2; ++i) {
+        const float send = up ? v[i] : v[i + C / 2];
+        const float keep = up ? v[i + C / 2] : v[i];
+        v[i] = keep + __shfl_xor_sync(0xffffffffu, send, mask);
+    }
+}
+
+// out[i] = sum over the warp's 32 lanes of v[i], i < N (N = 16 or 32): log2 N
+// butterfly levels (N - 1 shuffles, then 5 - log2 N plain ones) instead of N
+// separate five-level reductions.  v is clobbered.
+template <int N>
+__device__ __forceinline__ void warp_col_sums(float (&v)[N], float* out, int lane) {
+    static_assert(N == 16 || N == 32, "16 or 32 values per lane");
+    rs_level<N>(v, lane, 16);
+    rs_level<N / 2>(v, lane, 8);
+    rs_level<N / 4>(v, lane, 4);
+    rs_level<N / 8>(v, lane, 2);
+    if constexpr (N == 32) rs_level<2>(v, lane, 1);
+    else v[0] += __shfl_xor_sync(0xffffffffu, v[0], 1);
+    // the value a lane holds: bits 4..1 (and 0 for N = 32) of the lane pick halves
+    int idx = ((lane >> 4) & 1) * (N / 2) + ((lane >> 3) & 1) * (N / 4) + ((lane >> 2) & 1) * (N / 8) +
+              ((lane >> 1) & 1) * (N / 16);
+    if constexpr (N == 32) idx += lane & 1;
+    if (N == 32 || (lane & 1) == 0) out[idx] = v[0];
+}
+
+// A CTA's work as a sequence of segments: tile (feat, tok) over k-blocks [kb0, kb1).
+//  * plain: unit t = blockIdx.x + i * gridDim.x of n_feat x n_tok x n_split, one
+//    segment per unit (split s covers k-blocks [s K / S, (s + 1) K / S));
+//  * FUSED (one token tile): the n_feat x kblocks k-block iterations are cut into
+//    gridDim.x equal ranges; CTA c takes [c I / C, (c + 1) I / C) and a segment is
+//    the part of its range inside one tile.  Every CTA streams the same weight
+//    bytes; a tile shared by several CTAs is finished by the last of them.
+struct Seg {
+    int feat, tok, split, kb0, kb1;
+    long long next;  // where the following segment starts
+};
+
+template <bool FUSED>
+__device__ __forceinline__ bool seg_at(Seg& sg, long long at, long long hi, int n_tok, int n_split,
+                                       int kblocks) {
+    if (at >= hi) return false;
+    if constexpr (FUSED) {
+        sg.feat = (int)(at / kblocks);
+        sg.tok = 0;
+        sg.split = 0;
+        sg.kb0 = (int)(at - (long long)sg.feat * kblocks);
+        const long long tile_end = (long long)(sg.feat + 1) * kblocks;
+        const long long end = hi < tile_end ? hi : tile_end;
+        sg.kb1 = sg.kb0 + (int)(end - at);
+        sg.next = end;
+    } else {
+        const int t = (int)at;
+        sg.split = t % n_split;
+        const int rest = t / n_split;
+        sg.feat = rest / n_tok;
+        sg.tok = rest % n_tok;
+        sg.kb0 = sg.split * kblocks / n_split;
+        sg.kb1 = (sg.split + 1) * kblocks / n_split;
+        sg.next = at + gridDim.x;
+    }
+    return true;
+}
+
+// CTA owning k-block iteration `it` of a FUSED launch (I iterations, C CTAs).
+__device__ __forceinline__ int it_owner(long long it, long long I, int C) {
+    return (int)(((it + 1) * C - 1) / I);
+}
 
 template <int BN, bool SWIGLU, int STAGES, bool FUSED>
 __global__ void __launch_bounds__(kThreads, 1)
@@ -81,10 +157,14 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int n_feat = N / 128;
     const int n_tok = (M + BN - 1) / BN;
-    // Work unit t = ((feat * n_tok) + tok) * n_split + split; a split covers k-blocks
-    // [split * kblocks / n_split, (split + 1) * kblocks / n_split).
+    // Plain work unit t = ((feat * n_tok) + tok) * n_split + split; a split covers k-blocks
+    // [split * kblocks / n_split, (split + 1) * kblocks / n_split).  FUSED: see seg_at.
     const int num_tiles = n_feat * n_tok * n_split;
     const int kblocks = K / kBK;
+    // segment iteration range: k-block iterations (FUSED) or unit indices (plain)
+    const long long n_iter = (long long)n_feat * kblocks;
+    const long long seg_lo = FUSED ? (long long)blockIdx.x * n_iter / gridDim.x : (long long)blockIdx.x;
+    const long long seg_hi = FUSED ? (long long)(blockIdx.x + 1) * n_iter / gridDim.x : (long long)num_tiles;
 
     if (threadIdx.x == 0) {
         for (int s = 0; s < STAGES; ++s) {
@@ -131,11 +211,11 @@ __global__ void __launch_bounds__(kThreads, 1)
                                     &full[pend_stage[i]]);
                 npend = 0;
             };
-            for (int t = blockIdx.x; ok && t < num_tiles; t += gridDim.x) {
-                const int split = t % n_split, rest = t / n_split;
-                const int feat = rest / n_tok, tok = rest % n_tok;
-                const int kb0 = split * kblocks / n_split, kb1 = (split + 1) * kblocks / n_split;
-                for (int kb = kb0; kb < kb1; ++kb) {
+            Seg sg;
+            for (bool have = seg_at<FUSED>(sg, seg_lo, seg_hi, n_tok, n_split, kblocks); ok && have;
+                 have = seg_at<FUSED>(sg, sg.next, seg_hi, n_tok, n_split, kblocks)) {
+                const int feat = sg.feat, tok = sg.tok;
+                for (int kb = sg.kb0; kb < sg.kb1; ++kb) {
                     if (!tc::mbar_wait(&empty[stage], phase ^ 1, abort_flag)) {
                         ok = false;
                         break;
@@ -175,9 +255,10 @@ __global__ void __launch_bounds__(kThreads, 1)
             int acc = 0;
             uint32_t acc_phase = 0;
             bool ok = true, issued = false;
-            for (int t = blockIdx.x; ok && t < num_tiles; t += gridDim.x) {
-                const int split = t % n_split;
-                const int kb0 = split * kblocks / n_split, kb1 = (split + 1) * kblocks / n_split;
+            Seg sg;
+            for (bool have = seg_at<FUSED>(sg, seg_lo, seg_hi, n_tok, n_split, kblocks); ok && have;
+                 have = seg_at<FUSED>(sg, sg.next, seg_hi, n_tok, n_split, kblocks)) {
+                const int kb0 = sg.kb0, kb1 = sg.kb1;
                 if (!tc::mbar_wait(&tempty[acc], acc_phase ^ 1, abort_flag)) {
                     ok = false;
                     break;
@@ -220,48 +301,86 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
     } else if constexpr (FUSED) {
         // ---------------------------------------------------- fused epilogue (warps 2..5)
-        // One token tile (M <= BN).  Each unit: TMEM -> registers, release the
-        // accumulator, write the fp32 partial, take the tile's ticket; the last unit
-        // of a tile sums the partials in split order and applies fz.op.
+        // One token tile (M <= BN).  Per segment: prefetch the op's inputs, TMEM ->
+        // registers, release the accumulator; a segment holding part of its tile's k
+        // range writes its fp32 partial and takes the tile's ticket, and the last one
+        // sums the tile's slots in k order; then the op.  Global loads on this path are
+        // issued in batches ahead of their use: under the weight stream of the next
+        // kernel's prefetch, one L2 round trip costs about a microsecond.
         const int q = warp & 3;
         const int e = threadIdx.x - 64;  // 0..127 across the epilogue warps
         const int row = q * 32 + lane;   // accumulator row (TMEM lane) = feature within the tile
-        // Per-token values used by every unit are computed once: the input-norm scale
-        // s_row and (QKV) the clamped cache position p_row.  Loops over the tile's
-        // tokens are predicated (no early exit) so their independent loads overlap.
-        float* s_row = fscr;                      // [64]
-        int* p_row = (int*)(fscr + 64);           // [64]
-        float* red = fscr + 128;                  // [4][64]
-        float* xch = fscr + 128 + 256;            // [128][BN]
-        volatile int* flag = (volatile int*)(fscr + 128 + 256 + 128 * BN);
-        if (fz.op == FUSE_QKV || fz.op == FUSE_SWIGLU || fz.op == FUSE_COLSCALE) {
-            for (int j = e; j < BN; j += 128) {
-                float t = 0.f;
-                if (j < M)
-                    for (int i = 0; i < fz.n_ssq; ++i) t += fz.ssq_in[(size_t)i * M + j];
-                s_row[j] = j < M ? rsqrtf(t / (float)fz.H + fz.eps) : 0.f;
-            }
-        }
-        if (fz.op == FUSE_QKV) {
-            const int lim = fz.max_seq < fz.max_positions ? fz.max_seq : fz.max_positions;
-            for (int j = e; j < BN; j += 128) {
+        float* s_row = fscr;                  // [64] input-norm scale per token
+        int* p_row = (int*)(fscr + 64);       // [64] clamped cache position per token (QKV)
+        float* red = fscr + 128;              // [4][64] per-warp sums
+        float* xch = fscr + 384;              // [BN][128]: QKV partner exchange, RESID x prefetch
+        float* rope_c = xch + 128 * BN;       // [BN][64] cos / sin at each token's position (QKV)
+        float* rope_s = rope_c + 64 * BN;
+        volatile int* flag = (volatile int*)(rope_s + 64 * BN);
+        {
+            // s_row[j] = rsqrt(sum_i ssq_in[i][j] / H + eps): 128 / BN threads per token
+            // each sum every (128 / BN)-th tile sum, then token j's thread adds them in order
+            constexpr int kParts = 128 / BN;
+            const bool need_s = fz.op == FUSE_QKV || fz.op == FUSE_SWIGLU || fz.op == FUSE_COLSCALE;
+            const int j = e % BN, part = e / BN;
+            float t = 0.f;
+            if (need_s && j < M)
+#pragma unroll 8
+                for (int i = part; i < fz.n_ssq; i += kParts) t += fz.ssq_in[(size_t)i * M + j];
+            xch[part * BN + j] = t;
+            if (fz.op == FUSE_QKV && e < BN) {
+                const int lim = fz.max_seq < fz.max_positions ? fz.max_seq : fz.max_positions;
                 int p = 0;
-                if (j < M) {
-                    p = fz.pos.pos_dev ? fz.pos.pos_dev[j] : fz.pos.start;
+                if (e < M) {
+                    p = fz.pos.pos_dev ? fz.pos.pos_dev[e] : fz.pos.start;
                     if (p < 0 || p >= lim) {
                         atomicOr(fz.status, QK_STATUS_BAD_POS);
                         p = p < 0 ? 0 : lim - 1;
                     }
                 }
-                p_row[j] = p;
+                p_row[e] = p;
             }
+            epi_bar();
+            if (e < BN) {
+                float tt = 0.f;
+                for (int pp = 0; pp < kParts; ++pp) tt += xch[pp * BN + e];
+                s_row[e] = e < M ? rsqrtf(tt / (float)fz.H + fz.eps) : 0.f;
+            }
+            if (fz.op == FUSE_QKV) {
+                for (int idx = e; idx < M * 64; idx += 128) {
+                    const int jj = idx >> 6, i = idx & 63;
+                    tc::cp_async4(&rope_c[idx], &fz.rope_cos[(size_t)p_row[jj] * 64 + i]);
+                    tc::cp_async4(&rope_s[idx], &fz.rope_sin[(size_t)p_row[jj] * 64 + i]);
+                }
+                tc::cp_async_commit();
+            }
+            epi_bar();  // s_row, p_row and xch settled
         }
-        epi_bar();
+        constexpr int PB = BN <= 16 ? 6 : (BN <= 32 ? 3 : 1);  // partial slots per load batch
         int acc = 0;
         uint32_t acc_phase = 0;
-        const size_t sstride = (size_t)M * N;
-        for (int t = blockIdx.x; t < num_tiles; t += gridDim.x) {
-            const int split = t % n_split, feat = t / n_split;
+        // Partials: slot (CTA + tile) holds one segment's [M][128] fp32 sums; the slots of
+        // tile f are owner(first k-block) + f .. owner(last k-block) + f, in k order.
+        const int n_cta = gridDim.x;
+        auto slot0 = [&](int ft) { return it_owner((long long)ft * kblocks, n_iter, n_cta) + ft; };
+        auto slot1 = [&](int ft) { return it_owner((long long)ft * kblocks + kblocks - 1, n_iter, n_cta) + ft; };
+        Seg sg;
+        for (bool have = seg_at<FUSED>(sg, seg_lo, seg_hi, n_tok, n_split, kblocks); have;
+             have = seg_at<FUSED>(sg, sg.next, seg_hi, n_tok, n_split, kblocks)) {
+            const int feat = sg.feat;
+            const int f = feat * 128 + row;
+            // ---- op inputs, loaded while the accumulator is still being produced
+            float gain = 0.f;
+            if (fz.op == FUSE_QKV) {
+                if (feat < fz.nq) gain = fz.gq[row];
+                else if (feat < fz.nq + fz.nkv) gain = fz.gk[row];
+            } else if (fz.op == FUSE_RESID) {
+                gain = fz.g_next[f];
+#pragma unroll
+                for (int j = 0; j < BN; ++j)
+                    if (j < M) tc::cp_async4(&xch[j * 128 + row], &fz.x[(size_t)j * N + f]);
+                tc::cp_async_commit();
+            }
             bool ok = tc::mbar_wait(&tfull[acc], acc_phase, abort_flag);
             ok = __all_sync(0xffffffffu, ok);
             if (!ok) break;
@@ -286,45 +405,49 @@ __global__ void __launch_bounds__(kThreads, 1)
             acc ^= 1;
             if (acc == 0) acc_phase ^= 1;
 
-            const int f = feat * 128 + row;
             const bool swiglu = fz.op == FUSE_SWIGLU;
-            const bool ticketed = swiglu || n_split > 1;
+            // a tile done whole by this CTA needs no partials (SwiGLU pairs two tiles: always)
+            const bool ticketed = swiglu || sg.kb0 != 0 || sg.kb1 != kblocks;
             const int key = swiglu ? feat >> 1 : feat;
+            const int my_slot = (int)blockIdx.x + feat;
             if (ticketed) {
 #pragma unroll
                 for (int j = 0; j < BN; ++j)
-                    if (j < M) fz.part[split * sstride + (size_t)j * N + f] = v[j];
+                    if (j < M) fz.part[((size_t)my_slot * M + j) * 128 + row] = v[j];
                 // The barrier orders every epilogue thread's stores before the ticket
-                // thread's fence, which publishes them at GPU scope before the atomic; the
-                // last unit's ticket thread fences again before its peers read (L2 loads).
+                // thread's release (cumulative over the barrier); its acquire orders the
+                // last segment's reads after every other segment's stores.
                 epi_bar();
                 if (e == 0) {
-                    const int need = swiglu ? 2 * n_split : n_split;
-                    __threadfence();
-                    const bool last = atomicAdd(&fz.tickets[key], 1) == need - 1;
-                    if (last) __threadfence();
-                    *flag = last;
+                    const int need = swiglu ? slot1(2 * key) - slot0(2 * key) + slot1(2 * key + 1) -
+                                                  slot0(2 * key + 1) + 2
+                                            : slot1(feat) - slot0(feat) + 1;
+                    *flag = tc::atom_add_acq_rel_gpu(&fz.tickets[key], 1) == need - 1;
                 }
                 epi_bar();
                 const bool last = *flag != 0;
                 if (!last) continue;  // uniform over the four warps
                 if (!swiglu) {
-                    // sum in split order; the loads of one split are independent, so each
-                    // split costs one L2 round trip (this unit's own split is in registers)
+                    // sum the tile's slots in k order (this CTA's own slot from registers)
                     float a[BN];
 #pragma unroll
                     for (int j = 0; j < BN; ++j) a[j] = 0.f;
-                    for (int sp = 0; sp < n_split; ++sp) {
-                        if (sp == split) {
+                    const int s0 = slot0(feat), s1 = slot1(feat);
+                    for (int base = s0; base <= s1; base += PB) {
+                        float ld[PB][BN];
 #pragma unroll
-                            for (int j = 0; j < BN; ++j) a[j] += v[j];
-                        } else {
-                            float ld[BN];
+                        for (int k = 0; k < PB; ++k) {
+                            const int sl = base + k;
+                            const bool rd = sl <= s1 && sl != my_slot;
 #pragma unroll
                             for (int j = 0; j < BN; ++j)
-                                ld[j] = j < M ? __ldcg(&fz.part[sp * sstride + (size_t)j * N + f]) : 0.f;
+                                ld[k][j] = rd && j < M ? __ldcg(&fz.part[((size_t)sl * M + j) * 128 + row]) : 0.f;
+                        }
 #pragma unroll
-                            for (int j = 0; j < BN; ++j) a[j] += ld[j];
+                        for (int k = 0; k < PB; ++k) {
+                            const bool mine = base + k == my_slot;
+#pragma unroll
+                            for (int j = 0; j < BN; ++j) a[j] += mine ? v[j] : ld[k][j];
                         }
                     }
 #pragma unroll
@@ -337,34 +460,30 @@ __global__ void __launch_bounds__(kThreads, 1)
                 for (int j = 0; j < BN; ++j) v[j] *= s_row[j];
                 if (hh < nq + nkv) {
                     // per-head RMSNorm over the 128 rows of the tile, per token
+                    constexpr int RW = BN < 32 ? BN : 32;
 #pragma unroll
-                    for (int j = 0; j < BN; ++j) {
-                        float sq = v[j] * v[j];
+                    for (int h = 0; h < BN; h += RW) {
+                        float sq[RW];
 #pragma unroll
-                        for (int o = 16; o > 0; o >>= 1) sq += __shfl_xor_sync(0xffffffffu, sq, o);
-                        if (lane == 0) red[q * 64 + j] = sq;
+                        for (int i = 0; i < RW; ++i) sq[i] = v[h + i] * v[h + i];
+                        warp_col_sums<RW>(sq, red + q * 64 + h, lane);
                     }
+                    tc::cp_async_wait_all();  // this thread's share of the cos / sin table
                     epi_bar();
-                    const float gain = hh < nq ? fz.gq[row] : fz.gk[row];
 #pragma unroll
                     for (int j = 0; j < BN; ++j) {
                         const float tot = red[j] + red[64 + j] + red[128 + j] + red[192 + j];
                         v[j] = v[j] * rsqrtf(tot / 128.f + fz.eps) * gain;
-                        xch[row * BN + j] = v[j];
+                        xch[j * 128 + row] = v[j];
                     }
                     epi_bar();
                     // rotate-half RoPE: row i < 64 pairs with row i + 64
                     const int i = row & 63;
-                    float c[BN], sn[BN];
 #pragma unroll
                     for (int j = 0; j < BN; ++j) {
-                        c[j] = fz.rope_cos[(size_t)p_row[j] * 64 + i];
-                        sn[j] = fz.rope_sin[(size_t)p_row[j] * 64 + i];
-                    }
-#pragma unroll
-                    for (int j = 0; j < BN; ++j) {
-                        const float partner = xch[(row ^ 64) * BN + j];
-                        const float o = row < 64 ? v[j] * c[j] - partner * sn[j] : v[j] * c[j] + partner * sn[j];
+                        const float c = rope_c[j * 64 + i], sn = rope_s[j * 64 + i];
+                        const float partner = xch[j * 128 + (row ^ 64)];
+                        const float o = row < 64 ? v[j] * c - partner * sn : v[j] * c + partner * sn;
                         if (j < M) {
                             if (hh < nq)
                                 fz.q_out[(size_t)j * fz.q_ld + (size_t)hh * 128 + row] = __float2bfloat16_rn(o);
@@ -381,43 +500,54 @@ __global__ void __launch_bounds__(kThreads, 1)
                                 __float2bfloat16_rn(v[j]);
                 }
             } else if (fz.op == FUSE_RESID) {
-                const float gn = fz.g_next[f];
-                float xo[BN];
-#pragma unroll
-                for (int j = 0; j < BN; ++j) xo[j] = j < M ? fz.x[(size_t)j * N + f] : 0.f;
+                tc::cp_async_wait_all();  // this thread's x values (prefetched at segment start)
 #pragma unroll
                 for (int j = 0; j < BN; ++j) {
-                    const float xn = xo[j] + v[j];
+                    const float xn = (j < M ? xch[j * 128 + row] : 0.f) + v[j];
                     if (j < M) {
                         fz.x[(size_t)j * N + f] = xn;
-                        fz.xg_out[(size_t)j * N + f] = __float2bfloat16_rn(xn * gn);
+                        fz.xg_out[(size_t)j * N + f] = __float2bfloat16_rn(xn * gain);
                     }
-                    float sq = j < M ? xn * xn : 0.f;
+                    v[j] = j < M ? xn : 0.f;
+                }
+                constexpr int RW = BN < 32 ? BN : 32;
 #pragma unroll
-                    for (int k = 16; k > 0; k >>= 1) sq += __shfl_xor_sync(0xffffffffu, sq, k);
-                    if (lane == 0) red[q * 64 + j] = sq;
+                for (int h = 0; h < BN; h += RW) {
+                    float sq[RW];
+#pragma unroll
+                    for (int i = 0; i < RW; ++i) sq[i] = v[h + i] * v[h + i];
+                    warp_col_sums<RW>(sq, red + q * 64 + h, lane);
                 }
                 epi_bar();
                 if (e < M) fz.ssq_out[(size_t)feat * M + e] = red[e] + red[64 + e] + red[128 + e] + red[192 + e];
             } else if (fz.op == FUSE_SWIGLU) {
-                // this unit completed the pair: gate tile 2 jb, up tile 2 jb + 1
+                // this segment completed the pair: gate tile 2 jb, up tile 2 jb + 1, each
+                // summed over its slots in k order; both tiles' loads go out in one batch
                 const int jb = feat >> 1, I = N / 2;
-                const int fg = (2 * jb) * 128 + row, fu = fg + 128;
+                constexpr int PS = PB > 1 ? PB / 2 : 1;
                 float gs[BN], us[BN];
 #pragma unroll
                 for (int j = 0; j < BN; ++j) gs[j] = us[j] = 0.f;
-                for (int sp = 0; sp < n_split; ++sp) {
-                    float lg[BN], lu[BN];
+                const int g0 = slot0(2 * jb), g1 = slot1(2 * jb), u0 = slot0(2 * jb + 1), u1 = slot1(2 * jb + 1);
+                const int nb = max(g1 - g0, u1 - u0) + 1;
+                for (int base = 0; base < nb; base += PS) {
+                    float lg[PS][BN], lu[PS][BN];
 #pragma unroll
-                    for (int j = 0; j < BN; ++j) {
-                        lg[j] = j < M ? __ldcg(&fz.part[sp * sstride + (size_t)j * N + fg]) : 0.f;
-                        lu[j] = j < M ? __ldcg(&fz.part[sp * sstride + (size_t)j * N + fu]) : 0.f;
+                    for (int k = 0; k < PS; ++k) {
+                        const int sg_ = g0 + base + k, su = u0 + base + k;
+#pragma unroll
+                        for (int j = 0; j < BN; ++j) {
+                            lg[k][j] = sg_ <= g1 && j < M ? __ldcg(&fz.part[((size_t)sg_ * M + j) * 128 + row]) : 0.f;
+                            lu[k][j] = su <= u1 && j < M ? __ldcg(&fz.part[((size_t)su * M + j) * 128 + row]) : 0.f;
+                        }
                     }
 #pragma unroll
-                    for (int j = 0; j < BN; ++j) {
-                        gs[j] += lg[j];
-                        us[j] += lu[j];
-                    }
+                    for (int k = 0; k < PS; ++k)
+#pragma unroll
+                        for (int j = 0; j < BN; ++j) {
+                            gs[j] += lg[k][j];
+                            us[j] += lu[k][j];
+                        }
                 }
 #pragma unroll
                 for (int j = 0; j < BN; ++j) {
@@ -432,8 +562,9 @@ __global__ void __launch_bounds__(kThreads, 1)
                     if (j < M) ((float*)C)[(size_t)j * ldc + f] = v[j] * s_row[j];
             }
             if (ticketed && e == 0) fz.tickets[key] = 0;
-            epi_bar();  // scratch (red, xch, flag) is reused by the next unit
+            epi_bar();  // scratch (red, xch, flag) is reused by the next segment
         }
+        tc::cp_async_wait_all();  // no copy into shared memory outlives the CTA
     } else {
         // ---------------------------------------------------- epilogue (warps 2..5)
         const int q = warp & 3;
@@ -543,8 +674,9 @@ int launch_cfg(const bf16* A, int lda, const bf16* W, void* C, int ldc, int M, i
     const int w_rows = SWIGLU ? 2 * N : N;
     if (!make_map(&tmW, W, K, w_rows, K, G::A_ROWS) || !make_map(&tmX, A, K, M, lda, BN))
         return QK_ECUDA;
-    const int tiles = (N / 128) * ((M + BN - 1) / BN) * n_split;
-    const int grid = tiles < num_sms ? tiles : num_sms;
+    const long long units = FUSED ? (long long)(N / 128) * (K / kBK)
+                                  : (long long)(N / 128) * ((M + BN - 1) / BN) * n_split;
+    const int grid = units < num_sms ? (int)units : num_sms;
     Fuse none{};
     launch_k(gemm_tc_kernel<BN, SWIGLU, STAGES, FUSED>, dim3(grid), dim3(kThreads), G::SMEM, s, tmW,
              tmX, C, ldc, M, N, K, epi, n_split, status, fz ? *fz : none);
@@ -576,39 +708,20 @@ int launch_gemm_tc(const bf16* A, int lda, const bf16* W, void* C, int ldc, int 
     return launch_cfg<256, false, 4>(A, lda, W, C, ldc, M, N, K, epi, 1, num_sms, status, s);
 }
 
-// Split count for a decode-sized GEMM (one token tile): the smallest S whose
-// N/128 * S work units fill the persistent grid to >= 80 % of its last round,
-// with at least 12 k-blocks per unit (each unit ends in a fused epilogue); the
-// best S found otherwise.
-int gemm_tc_split(int N, int K, int num_sms) {
-    const int n_feat = N / 128, kblocks = K / kBK;
-    int best = 1;
-    double best_eff = 0.0;
-    for (int S = 1; S <= 32 && kblocks / S >= 12; ++S) {
-        const int units = n_feat * S;
-        const int rounds = (units + num_sms - 1) / num_sms;
-        const double eff = (double)units / ((double)rounds * num_sms);
-        if (eff >= 0.8) return S;
-        if (eff > best_eff + 1e-9) {
-            best_eff = eff;
-            best = S;
-        }
-    }
-    return best;
-}
-
 // Decode linear with a fused epilogue (see Fuse); one token tile of M <= 64 rows.
 int launch_gemm_tc_fused(const bf16* A, int lda, const bf16* W, float* out, int M, int N, int K,
-                         int n_split, const Fuse& f, int num_sms, uint32_t* status, cudaStream_t s) {
+                         const Fuse& f, int num_sms, uint32_t* status, cudaStream_t s) {
     if (M <= 0) return QK_OK;
     if (M > 64) return QK_ESHAPE;
+    // every launch may split a tile over CTAs: partial slots and tickets are required
+    if (!f.part || !f.tickets || !f.status) return QK_EINVAL;
     if (M <= 16)
-        return launch_cfg<16, false, 8, true>(A, lda, W, out, N, M, N, K, EPI_PARTIAL_F32, n_split,
+        return launch_cfg<16, false, 8, true>(A, lda, W, out, N, M, N, K, EPI_PARTIAL_F32, 1,
                                               num_sms, status, s, &f);
     if (M <= 32)
-        return launch_cfg<32, false, 8, true>(A, lda, W, out, N, M, N, K, EPI_PARTIAL_F32, n_split,
+        return launch_cfg<32, false, 8, true>(A, lda, W, out, N, M, N, K, EPI_PARTIAL_F32, 1,
                                               num_sms, status, s, &f);
-    return launch_cfg<64, false, 7, true>(A, lda, W, out, N, M, N, K, EPI_PARTIAL_F32, n_split,
+    return launch_cfg<64, false, 6, true>(A, lda, W, out, N, M, N, K, EPI_PARTIAL_F32, 1,
                                           num_sms, status, s, &f);
 }
 

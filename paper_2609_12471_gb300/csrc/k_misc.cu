@@ -247,70 +247,122 @@ void launch_swiglu(const void* gu, void* h, int dtype, int M, int I, cudaStream_
 
 // ---------------------------------------------------------------- log-softmax / gather / argmax
 // One block per logits row: max and lowest arg-max, then logsumexp, then the target's log-prob.
-__global__ void logits_reduce_kernel(const float* __restrict__ logits, int V, OutIndex oi,
-                                     float* __restrict__ lp, int32_t* __restrict__ am,
-                                     uint32_t* status) {
-    __shared__ float red_v[32];
-    __shared__ int red_i[32];
-    __shared__ float red[32];
+// Online (max, arg-max, sum of exp) over a stream of logits: the running sum is kept
+// relative to the running max (rescaled when the max grows); ties keep the lowest index.
+struct MaxSum {
+    float m, s;
+    int i;
+};
+
+__device__ __forceinline__ void ms_push(MaxSum& a, float v, int i) {
+    if (v > a.m) {
+        a.s = (a.m == -INFINITY ? 0.f : a.s * expf(a.m - v)) + 1.f;
+        a.m = v;
+        a.i = i;
+    } else {
+        a.s += expf(v - a.m);
+    }
+}
+
+// a followed by b (b covers later indices, or is an unordered peer: ties take the lower index)
+__device__ __forceinline__ MaxSum ms_merge(MaxSum a, MaxSum b) {
+    MaxSum r;
+    r.m = fmaxf(a.m, b.m);
+    if (r.m == -INFINITY) return a;
+    r.s = (a.m == -INFINITY ? 0.f : a.s * expf(a.m - r.m)) + (b.m == -INFINITY ? 0.f : b.s * expf(b.m - r.m));
+    r.i = a.m > b.m ? a.i : (b.m > a.m ? b.i : min(a.i, b.i));
+    return r;
+}
+
+// One logits row per cluster of kLogitCtas CTAs: CTA k of the cluster reduces the
+// k-th slice of the row in one pass, then CTA 0 combines the slices' (max, arg-max,
+// sum of exp) in slice order through distributed shared memory and writes
+//   argmax, and log p(target) = z[target] - (max + log sum exp(z - max)).
+constexpr int kLogitCtas = 8;
+
+__global__ void __cluster_dims__(kLogitCtas, 1, 1) __launch_bounds__(256)
+    logits_reduce_kernel(const float* __restrict__ logits, int V, OutIndex oi,
+                         float* __restrict__ lp, int32_t* __restrict__ am, uint32_t* status) {
+    __shared__ MaxSum red[8];
+    __shared__ MaxSum part;
     pdl_wait();
     pdl_trigger();  // short kernel: let the next one launch and prefetch now
-    int r = blockIdx.x;
-    int g = oi.row0 + r;
-    int b = g / oi.T, t = g % oi.T;
-    if (t >= oi.out_lim) return;
+    const int r = blockIdx.y, k = blockIdx.x;
+    const int g = oi.row0 + r;
+    const int b = g / oi.T, t = g % oi.T;
+    const bool active = t < oi.out_lim;  // uniform over the cluster (one row per cluster)
     const float* z = logits + (size_t)r * V;
-    float best = -INFINITY;
-    int bi = 0x7fffffff;
-    for (int i = threadIdx.x * 4; i < V; i += blockDim.x * 4) {
-        float4 v = *reinterpret_cast<const float4*>(z + i);
-        if (v.x > best) { best = v.x; bi = i; }
-        if (v.y > best) { best = v.y; bi = i + 1; }
-        if (v.z > best) { best = v.z; bi = i + 2; }
-        if (v.w > best) { best = v.w; bi = i + 3; }
+    int tg = 0;
+    float z_tg = 0.f;
+    if (active && k == 0 && threadIdx.x == 0 && lp && oi.tgt) {  // fetched early, used last
+        tg = oi.tgt[(size_t)b * oi.tgt_ld + oi.tgt_off + t];
+        if (tg < 0 || tg >= V) {
+            atomicOr(status, QK_STATUS_BAD_TOKEN);
+            tg = 0;
+        }
+        z_tg = z[tg];
     }
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) {
-        float ov = __shfl_xor_sync(0xffffffffu, best, o);
-        int oidx = __shfl_xor_sync(0xffffffffu, bi, o);
-        if (ov > best || (ov == best && oidx < bi)) { best = ov; bi = oidx; }
-    }
-    int w = threadIdx.x >> 5, l = threadIdx.x & 31, nw = blockDim.x >> 5;
-    if (l == 0) { red_v[w] = best; red_i[w] = bi; }
-    __syncthreads();
-    best = l < nw ? red_v[l] : -INFINITY;
-    bi = l < nw ? red_i[l] : 0x7fffffff;
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) {
-        float ov = __shfl_xor_sync(0xffffffffu, best, o);
-        int oidx = __shfl_xor_sync(0xffffffffu, bi, o);
-        if (ov > best || (ov == best && oidx < bi)) { best = ov; bi = oidx; }
-    }
-    float se = 0.f;
-    for (int i = threadIdx.x * 4; i < V; i += blockDim.x * 4) {
-        float4 v = *reinterpret_cast<const float4*>(z + i);
-        se += expf(v.x - best) + expf(v.y - best) + expf(v.z - best) + expf(v.w - best);
-    }
-    se = block_sum(se, red);
-    if (threadIdx.x == 0) {
-        size_t o = (size_t)b * oi.out_ld + oi.out_off + t + (oi.dyn_off ? *oi.dyn_off : 0);
-        if (am) am[o] = bi;
-        if (lp && oi.tgt) {
-            int tg = oi.tgt[(size_t)b * oi.tgt_ld + oi.tgt_off + t];
-            if (tg < 0 || tg >= V) {
-                atomicOr(status, QK_STATUS_BAD_TOKEN);
-                tg = 0;
+    MaxSum a{-INFINITY, 0.f, 0x7fffffff};
+    if (active) {
+        // slice k: [lo, hi), a multiple of 4 wide except at the row's end
+        const int per = ((V + kLogitCtas - 1) / kLogitCtas + 3) & ~3;
+        const int lo = min(V, k * per), hi = min(V, lo + per);
+        if ((V & 3) == 0) {
+            for (int i = lo + threadIdx.x * 4; i < hi; i += blockDim.x * 4) {
+                const float4 v = *reinterpret_cast<const float4*>(z + i);
+                ms_push(a, v.x, i);
+                ms_push(a, v.y, i + 1);
+                ms_push(a, v.z, i + 2);
+                ms_push(a, v.w, i + 3);
             }
-            lp[o] = z[tg] - (best + logf(se));
+        } else {
+            for (int i = lo + threadIdx.x; i < hi; i += blockDim.x) ms_push(a, z[i], i);
         }
     }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+        MaxSum p;
+        p.m = __shfl_xor_sync(0xffffffffu, a.m, o);
+        p.s = __shfl_xor_sync(0xffffffffu, a.s, o);
+        p.i = __shfl_xor_sync(0xffffffffu, a.i, o);
+        a = ms_merge(a, p);
+    }
+    const int w = threadIdx.x >> 5, l = threadIdx.x & 31;
+    if (l == 0) red[w] = a;
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        MaxSum c = red[0];
+        for (int i = 1; i < (int)(blockDim.x >> 5); ++i) c = ms_merge(c, red[i]);
+        part = c;
+    }
+    // every slice's partial is in its CTA's shared memory before CTA 0 reads them
+    asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;" ::: "memory");
+    if (active && k == 0 && threadIdx.x == 0) {
+        MaxSum c{-INFINITY, 0.f, 0x7fffffff};
+        const uint32_t local = (uint32_t)__cvta_generic_to_shared(&part);
+        for (int q = 0; q < kLogitCtas; ++q) {
+            uint32_t remote;
+            asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(remote) : "r"(local), "r"(q));
+            MaxSum p;
+            asm volatile("ld.shared::cluster.f32 %0, [%1];" : "=f"(p.m) : "r"(remote));
+            asm volatile("ld.shared::cluster.f32 %0, [%1+4];" : "=f"(p.s) : "r"(remote));
+            asm volatile("ld.shared::cluster.s32 %0, [%1+8];" : "=r"(p.i) : "r"(remote));
+            c = ms_merge(c, p);
+        }
+        const size_t o = (size_t)b * oi.out_ld + oi.out_off + t + (oi.dyn_off ? *oi.dyn_off : 0);
+        if (am) am[o] = c.i;
+        if (lp && oi.tgt) lp[o] = z_tg - (c.m + logf(c.s));
+    }
+    // no CTA leaves while CTA 0 may still read its shared memory
+    asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;" ::: "memory");
 }
 
 void launch_logits_reduce(const float* logits, int M, int V, OutIndex oi, float* lp,
                           int32_t* argmax, uint32_t* status, cudaStream_t s) {
     note_launch();
     if (M <= 0) return;
-    launch_k(logits_reduce_kernel, dim3(M), dim3(512), 0, s, logits, V, oi, lp, argmax, status);
+    launch_k(logits_reduce_kernel, dim3(kLogitCtas, M), dim3(256), 0, s, logits, V, oi, lp, argmax,
+             status);
 }
 
 // ---------------------------------------------------------------- rollout cursor

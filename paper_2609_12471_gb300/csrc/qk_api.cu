@@ -126,45 +126,31 @@ static const int kScoreLogitRows = 4096;
 // output slot) in 256-byte-aligned slots after the prefill/decode workspace.
 static size_t rollout_cursor_bytes(int B) { return 5 * align256((size_t)(B > 1 ? B : 1) * 4); }
 
-// Decode batches of bf16 models with more than kGemvMaxRows and at most
-// kSplitMaxRows rows run their linear layers as split-K tcgen05 GEMMs whose fp32
-// partials are summed (in a fixed order) by the kernel that consumes them;
-// smaller batches stream the weights through the CUDA-core GEMV.
 static const int kSplitMaxRows = 64;
 
-struct Splits {
-    int qkv, o, gu, d;
-};
-
 // Decode steps of bf16 models with head_dim 128 and up to kSplitMaxRows rows run the
-// fused path: split-K tcgen05 linears whose last unit per tile applies QK-norm + RoPE,
-// the residual add (with the next norm's statistics) or SwiGLU in its epilogue.
-static const int kTicketSlots = 1024;
+// fused path: tcgen05 linears whose k-block iterations are split evenly over the
+// SMs; the last CTA of each tile sums its fp32 partials in k order and applies
+// QK-norm + RoPE, the residual add (with the next norm's statistics) or SwiGLU.
+static const int kTicketSlots = 4096;
 
 static bool use_splitk(const Model& m, int M) {
     const qk_config& c = m.cfg;
     return c.dtype == QK_DTYPE_BF16 && M >= 1 && M <= kSplitMaxRows && c.head_dim == 128 &&
-           c.hidden % 128 == 0 && (2 * c.intermediate) / 128 <= 2 * kTicketSlots &&
+           c.hidden % 128 == 0 && c.intermediate % 128 == 0 && c.vocab % 128 == 0 &&
+           c.vocab / 128 <= kTicketSlots && (2 * c.intermediate) / 128 <= kTicketSlots &&
            ((c.n_q_heads + 2 * c.n_kv_heads) * c.head_dim) / 128 <= kTicketSlots;
-}
-
-static Splits decode_splits(const Model& m) {
-    const qk_config& c = m.cfg;
-    const int nqkv = (c.n_q_heads + 2 * c.n_kv_heads) * c.head_dim;
-    return Splits{gemm_tc_split(nqkv, c.hidden, m.num_sms),
-                  gemm_tc_split(c.hidden, c.n_q_heads * c.head_dim, m.num_sms),
-                  gemm_tc_split(2 * c.intermediate, c.hidden, m.num_sms),
-                  gemm_tc_split(c.hidden, c.intermediate, m.num_sms)};
 }
 
 static size_t splitk_part_floats(const Model& m, int M) {
     const qk_config& c = m.cfg;
-    const Splits sp = decode_splits(m);
-    const size_t nqkv = (size_t)(c.n_q_heads + 2 * c.n_kv_heads) * c.head_dim;
-    size_t f = (size_t)sp.qkv * M * nqkv;
-    f = f > (size_t)sp.o * M * c.hidden ? f : (size_t)sp.o * M * c.hidden;
-    f = f > (size_t)sp.gu * M * 2 * c.intermediate ? f : (size_t)sp.gu * M * 2 * c.intermediate;
-    f = f > (size_t)sp.d * M * c.hidden ? f : (size_t)sp.d * M * c.hidden;
+    const int nqkv = (c.n_q_heads + 2 * c.n_kv_heads) * c.head_dim;
+    const int widths[5] = {nqkv, c.hidden, 2 * c.intermediate, c.hidden, c.vocab};
+    size_t f = 0;
+    for (int n : widths) {
+        const size_t g = gemm_fused_part_floats(M, n, m.num_sms);
+        f = g > f ? g : f;
+    }
     return f;
 }
 
@@ -261,7 +247,6 @@ static void run_layer_fused(Model& m, int l, const Workspace& w, int M, PosIndex
                             const KVView& kv, const float* g_next, cudaStream_t s) {
     const qk_config& c = m.cfg;
     const LayerW& L = m.layers[l];
-    const Splits sp = decode_splits(m);
     const int H = c.hidden, d = c.head_dim, nq = c.n_q_heads, nkv = c.n_kv_heads, I = c.intermediate;
     const int nqkv = (nq + 2 * nkv) * d;
     Fuse f{};
@@ -272,8 +257,8 @@ static void run_layer_fused(Model& m, int l, const Workspace& w, int M, PosIndex
     f.H = H;
     f.eps = (float)c.rms_eps;
     f.status = m.status;
-    auto gemm = [&](const void* A, int lda, const void* W, int N, int K, int S, const Fuse& fz) {
-        int rc = launch_gemm_tc_fused((const bf16*)A, lda, (const bf16*)W, nullptr, M, N, K, S, fz,
+    auto gemm = [&](const void* A, int lda, const void* W, int N, int K, const Fuse& fz) {
+        int rc = launch_gemm_tc_fused((const bf16*)A, lda, (const bf16*)W, nullptr, M, N, K, fz,
                                       m.num_sms, m.status, s);
         if (rc != QK_OK && !m.deferred_error) m.deferred_error = rc;
     };
@@ -294,7 +279,7 @@ static void run_layer_fused(Model& m, int l, const Workspace& w, int M, PosIndex
     fq.v_cache = (bf16*)kv.v(l);
     fq.max_seq = kv.max_seq;
     pr = prof_open(m, QK_PROF_QKV, s);
-    gemm(w.xg, H, L.w_qkv, nqkv, H, sp.qkv, fq);
+    gemm(w.xg, H, L.w_qkv, nqkv, H, fq);
     prof_close(m, pr, s);
     pr = prof_open(m, QK_PROF_ATTN, s);
     launch_attention(m, w.qkv, nqkv, kv.k(l), kv.v(l), M, kv.max_batch, kv.max_seq, pos, w.o,
@@ -307,18 +292,18 @@ static void run_layer_fused(Model& m, int l, const Workspace& w, int M, PosIndex
     fo.xg_out = w.xg;
     fo.ssq_out = w.ssq;
     pr = prof_open(m, QK_PROF_O, s);
-    gemm(w.o, nq * d, L.w_o, H, nq * d, sp.o, fo);
+    gemm(w.o, nq * d, L.w_o, H, nq * d, fo);
     prof_close(m, pr, s);
     Fuse fg = f;
     fg.op = FUSE_SWIGLU;
     fg.h_out = (bf16*)w.h;
     pr = prof_open(m, QK_PROF_GATE_UP, s);
-    gemm(w.xg, H, L.w_gu, 2 * I, H, sp.gu, fg);
+    gemm(w.xg, H, L.w_gu, 2 * I, H, fg);
     prof_close(m, pr, s);
     Fuse fd = fo;
     fd.g_next = g_next;
     pr = prof_open(m, QK_PROF_DOWN, s);
-    gemm(w.h, I, L.w_d, H, I, sp.d, fd);
+    gemm(w.h, I, L.w_d, H, I, fd);
     prof_close(m, pr, s);
 }
 
@@ -653,7 +638,6 @@ static int decode_impl(Model& m, void* kv, int max_batch, int max_seq, TokIndex 
     KVView view = cache_view(m, kv, max_batch, max_seq);
     QK_TRY(clear_attn_tickets(m, w, B, max_seq, s));
     m.in_decode = true;
-    launch_embed(m.embed, m.cfg.dtype, m.cfg.vocab, m.cfg.hidden, tok, B, w.x, m.status, s);
     if (w.part) {
         const qk_config& c = m.cfg;
         QK_TRY_CUDA(cudaMemsetAsync(w.tickets, 0, kTicketSlots * sizeof(int), s));
@@ -667,18 +651,22 @@ static int decode_impl(Model& m, void* kv, int max_batch, int max_seq, TokIndex 
             float* z = logits ? logits : w.logits;
             Fuse fl{};
             fl.op = FUSE_COLSCALE;
+            fl.tickets = w.tickets;
+            fl.part = w.part;
+            fl.status = m.status;
             fl.ssq_in = w.ssq;
             fl.n_ssq = c.hidden / 128;
             fl.H = c.hidden;
             fl.eps = (float)c.rms_eps;
             bool pr = prof_open(m, QK_PROF_LM_HEAD, s);
             int rc = launch_gemm_tc_fused(w.xg, c.hidden, (const bf16*)m.lm_head, z, B, c.vocab,
-                                          c.hidden, 1, fl, m.num_sms, m.status, s);
+                                          c.hidden, fl, m.num_sms, m.status, s);
             prof_close(m, pr, s);
             if (rc != QK_OK && !m.deferred_error) m.deferred_error = rc;
             if (lp || am) launch_logits_reduce(z, B, c.vocab, oi, lp, am, m.status, s);
         }
     } else {
+        launch_embed(m.embed, m.cfg.dtype, m.cfg.vocab, m.cfg.hidden, tok, B, w.x, m.status, s);
         for (int l = 0; l < m.cfg.n_layers; ++l) run_layer(m, l, w, B, pos, view, s);
         if (logits || lp || am) run_head(m, w, B, 1, 0, logits ? logits : w.logits, oi, lp, am, s);
     }

@@ -195,14 +195,14 @@ void launch_gemv_bf16(const bf16* A, int lda, const bf16* W, void* C, int ldc, i
 bool gemm_tc_supported(const void* A, int lda, int N, int K);
 int launch_gemm_tc(const bf16* A, int lda, const bf16* W, void* C, int ldc, int M, int N, int K,
                    int epi, int num_sms, uint32_t* status, cudaStream_t s);
-int gemm_tc_split(int N, int K, int num_sms);
 
-
-// Fused epilogue of a decode-sized split-K linear (one token tile, M <= 64 rows).
-// Every work unit writes its fp32 partial to part[split][M][N]; the last unit of a
-// tile (the last of a gate/up tile pair for FUSE_SWIGLU) takes the tile's ticket,
-// sums the partials in split order and applies `op`.  Tickets must be zero on
-// entry and are zero again on exit.  The linear's input is x * g (bf16, not yet
+// Fused epilogue of a decode-sized linear (one token tile, M <= 64 rows).  The
+// N/128 x K/64 k-block iterations are split evenly over the CTAs; a CTA that holds
+// only part of a tile's k range writes its fp32 partial [M][128] to slot (CTA +
+// tile) of `part` and takes the tile's ticket, and the last of them (the last of a
+// gate/up tile pair for FUSE_SWIGLU, whose halves always go through `part`) sums
+// the slots in k order and applies `op`.  `part` holds gemm_fused_part_floats()
+// floats, `tickets` N/128 ints (zero on entry, zero again on exit).  The linear's input is x * g (bf16, not yet
 // normalised); the RMSNorm scale s_m = rsqrt(sum_t ssq_in[t][m] / H + eps) of
 // token row m is applied after the product (W (x g s) = s W (x g)).
 enum FuseOp : int {
@@ -246,7 +246,10 @@ struct Fuse {
 // Decode linear with a fused epilogue (k_gemm_tc.cu): A = bf16 [M, K] (M <= 64),
 // W [N, K]; out is the op's fp32 logits for FUSE_COLSCALE, unused otherwise.
 int launch_gemm_tc_fused(const bf16* A, int lda, const bf16* W, float* out, int M, int N, int K,
-                         int n_split, const Fuse& f, int num_sms, uint32_t* status, cudaStream_t s);
+                         const Fuse& f, int num_sms, uint32_t* status, cudaStream_t s);
+inline size_t gemm_fused_part_floats(int M, int N, int num_sms) {
+    return ((size_t)num_sms + (size_t)(N / 128)) * (size_t)M * 128;
+}
 // x = E[token] (embed) or the given x; xg = bf16(x * g); ssq[t][m] = sum over features
 // 128 t .. 128 t + 127 of x^2 (k_misc.cu).
 void launch_embed_gain(const void* E, int V, TokIndex tok, bool do_embed, float* x, const float* g,
