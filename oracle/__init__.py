@@ -6,3 +6,4 @@ product path (``paper_2609_12471_gb300``) never imports it and shares no code
 with it; the two meet only in the seeded inputs of ``synth``.
 """
 from .qwen3 import *  # noqa: F401,F403
+from .grpo import group_advantages, grpo_loss_mean, grpo_token_loss, kl_k3  # noqa: F401

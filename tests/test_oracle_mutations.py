@@ -31,17 +31,40 @@ MUTATIONS = {
 }
 
 
-@pytest.mark.parametrize("name", sorted(MUTATIONS))
-def test_pins_catch_planted_mistake(name, tmp_path):
-    before, after = MUTATIONS[name]
+# Mistakes in the GRPO token-loss oracle, caught by test_oracle_grpo.py.
+GRPO_MUTATIONS = {
+    "advantage_variance_normalised": ("return (g - g.mean(axis=1, keepdims=True)).reshape(-1)",
+                                      "return ((g - g.mean(axis=1, keepdims=True)) / (g.std(axis=1, keepdims=True) + 1e-6)).reshape(-1)"),
+    "clip_bounds_swapped": ("np.clip(rho, 1.0 - eps_low, 1.0 + eps_high)", "np.clip(rho, 1.0 - eps_high, 1.0 + eps_low)"),
+    "max_instead_of_min": ("surrogate = np.minimum(", "surrogate = np.maximum("),
+    "ratio_inverted": ("rho = np.exp(lp - np.asarray(lp_old, dtype=np.float64))",
+                       "rho = np.exp(np.asarray(lp_old, dtype=np.float64) - lp)"),
+    "kl_sign": ("loss = loss + beta * kl_k3(lp, lp_ref)", "loss = loss - beta * kl_k3(lp, lp_ref)"),
+    "kl_k1_estimator": ("return np.exp(x) - x - 1.0", "return -x"),
+}
+
+
+def _run_mutated(tmp_path, module, before, after, name, pins):
     shutil.copytree(os.path.join(ROOT, "oracle"), tmp_path / "oracle",
                     ignore=shutil.ignore_patterns("__pycache__"))
-    p = tmp_path / "oracle" / "qwen3.py"
+    p = tmp_path / "oracle" / module
     src = p.read_text()
     assert src.count(before) >= 1, f"mutation anchor for {name} not found"
     p.write_text(src.replace(before, after))
     env = dict(os.environ, PYTHONPATH=os.pathsep.join([str(tmp_path), ROOT]))
     r = subprocess.run([sys.executable, "-m", "pytest", "-q", "-x", "-p", "no:cacheprovider",
-                        os.path.join(ROOT, "tests", "test_oracle_pins.py")],
+                        os.path.join(ROOT, "tests", pins)],
                        cwd=str(tmp_path), env=env, capture_output=True, text=True, timeout=600)
     assert r.returncode != 0, f"pins did not catch {name}:\n{r.stdout[-2000:]}"
+
+
+@pytest.mark.parametrize("name", sorted(MUTATIONS))
+def test_pins_catch_planted_mistake(name, tmp_path):
+    before, after = MUTATIONS[name]
+    _run_mutated(tmp_path, "qwen3.py", before, after, name, "test_oracle_pins.py")
+
+
+@pytest.mark.parametrize("name", sorted(GRPO_MUTATIONS))
+def test_grpo_pins_catch_planted_mistake(name, tmp_path):
+    before, after = GRPO_MUTATIONS[name]
+    _run_mutated(tmp_path, "grpo.py", before, after, name, "test_oracle_grpo.py")
