@@ -155,6 +155,37 @@ int qk_decode_layer(qk_model* m, int layer, void* kv, int max_batch, int max_seq
 int qk_score_logprobs(qk_model* m, const int32_t* tokens, int B, int T, float* logprobs,
                       int32_t* argmax, void* workspace, size_t ws_bytes, void* stream);
 
+/* ---- GRPO token loss (Sec. "GRPO Optimization", Eq. advantage and Eq. ppo) --
+ * Advantage of row b (Eq. advantage, no variance normalisation):
+ *   A_b = rewards[b] - mean(rewards[g0 .. g0 + group - 1]),  g0 = b - b % group.
+ * Per response token (Eq. ppo), rho = exp(lp - lp_old):
+ *   loss_tok = -min(rho A_b, clip(rho, 1 - eps_low, 1 + eps_high) A_b) + beta * k3,
+ *   k3 = exp(lp_ref - lp) - (lp_ref - lp) - 1  (the KL estimator is a reading:
+ *   the paper does not name one).
+ * loss_mean = sum(mask * loss_tok) / sum(mask) over the batch (0 for an empty
+ * mask).  Every [B, T] array is dev fp32, row-major with row stride ld >= T;
+ * mask dev uint8 (1 = response token) or NULL for all ones; lp_ref may be NULL
+ * only when beta == 0; rewards dev fp32 [B] with B % group == 0.  loss_tok
+ * receives all T entries of each row (masked ones included); loss_mean is dev
+ * fp32 [1] or NULL.  Sums run in a fixed order (deterministic).  workspace:
+ * qk_grpo_workspace_bytes(B) bytes of device scratch. */
+int qk_grpo_workspace_bytes(int B, size_t* bytes);
+int qk_grpo_token_loss(const float* lp, const float* lp_old, const float* lp_ref, int B, int T,
+                       int ld, const float* rewards, int group, const uint8_t* mask,
+                       float eps_low, float eps_high, float beta, float* loss_tok,
+                       float* loss_mean, void* workspace, size_t ws_bytes, void* stream);
+
+/* Scoring with the GRPO loss in its log-prob epilogue: as qk_score_logprobs for
+ * tokens [B, T] (logprobs dev fp32 [B, T-1]), and where each log-prob is formed
+ * its token loss as in qk_grpo_token_loss with ld = T-1 (lp_old, lp_ref, mask,
+ * loss_tok [B, T-1]).  workspace: qk_workspace_bytes(QK_CALL_SCORE, B, T, T)
+ * plus qk_grpo_workspace_bytes(B) bytes (the GRPO scratch follows the scoring
+ * scratch, 256-byte aligned). */
+int qk_score_grpo(qk_model* m, const int32_t* tokens, int B, int T, const float* lp_old,
+                  const float* lp_ref, const float* rewards, int group, const uint8_t* mask,
+                  float eps_low, float eps_high, float beta, float* logprobs, float* loss_tok,
+                  float* loss_mean, void* workspace, size_t ws_bytes, void* stream);
+
 /* Teacher-forced rollout: seq dev int32 [B, P+N+1] = prompt (P tokens) ++
  * c[0..N].  Prefill over the prompt scores c[0]; decode step j (0 <= j < N)
  * consumes c[j] at position P+j and scores c[j+1].  logprobs dev fp32 [B, N+1],

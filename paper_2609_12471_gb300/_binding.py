@@ -33,7 +33,7 @@ __all__ = [
     "qk_profile_end", "qk_launch_count", "qk_op_linear", "QK_PROF_QKV", "QK_PROF_O",
     "QK_PROF_GATE_UP", "QK_PROF_DOWN", "QK_PROF_ATTN", "QK_PROF_LM_HEAD", "QK_EPI_STORE",
     "QK_EPI_STORE_F32", "QK_EPI_RESID_F32", "QK_EPI_SWIGLU", "qk_op_linear_swiglu_static",
-    "QK_STATIC_SCRATCH_BYTES",
+    "QK_STATIC_SCRATCH_BYTES", "qk_grpo_workspace_bytes", "qk_grpo_token_loss", "qk_score_grpo",
 ]
 
 
@@ -59,7 +59,7 @@ def lib_path() -> str:
     return _LIB_FILE
 
 
-_P, _I, _SZ = ctypes.c_void_p, ctypes.c_int, ctypes.c_size_t
+_P, _I, _SZ, _F = ctypes.c_void_p, ctypes.c_int, ctypes.c_size_t, ctypes.c_float
 _SIGS = {
     "qk_config_preset": ([ctypes.c_char_p, ctypes.POINTER(qk_config)], _I),
     "qk_weight_count": ([ctypes.POINTER(qk_config), ctypes.POINTER(_I)], _I),
@@ -81,6 +81,9 @@ _SIGS = {
     "qk_launch_count": ([], ctypes.c_uint64),
     "qk_op_linear": ([_P, _P, _I, _P, _P, _I, _I, _I, _I, _I, _P, _SZ, _P], _I),
     "qk_op_linear_swiglu_static": ([_P, _P, _I, _P, _P, _I, _I, _I, _I, _P], _I),
+    "qk_grpo_workspace_bytes": ([_I, ctypes.POINTER(_SZ)], _I),
+    "qk_grpo_token_loss": ([_P, _P, _P, _I, _I, _I, _P, _I, _P, _F, _F, _F, _P, _P, _P, _SZ, _P], _I),
+    "qk_score_grpo": ([_P, _P, _I, _I, _P, _P, _P, _I, _P, _F, _F, _F, _P, _P, _P, _P, _SZ, _P], _I),
 }
 
 _lib = None
@@ -209,6 +212,28 @@ def qk_score_logprobs(m, tokens, B, T, logprobs, argmax=None, workspace=None, ws
     _check(_load().qk_score_logprobs(m, _ptr(tokens), B, T, _ptr(logprobs), _ptr(argmax),
                                      _ptr(workspace), _nbytes(workspace, ws_bytes),
                                      _stream(stream)))
+
+
+def qk_grpo_workspace_bytes(B) -> int:
+    v = ctypes.c_size_t()
+    _check(_load().qk_grpo_workspace_bytes(B, ctypes.byref(v)))
+    return v.value
+
+
+def qk_grpo_token_loss(lp, lp_old, lp_ref, B, T, ld, rewards, group, mask, eps_low, eps_high, beta,
+                       loss_tok, loss_mean=None, workspace=None, ws_bytes=None, stream=None):
+    _check(_load().qk_grpo_token_loss(_ptr(lp), _ptr(lp_old), _ptr(lp_ref), B, T, ld, _ptr(rewards),
+                                      group, _ptr(mask), eps_low, eps_high, beta, _ptr(loss_tok),
+                                      _ptr(loss_mean), _ptr(workspace), _nbytes(workspace, ws_bytes),
+                                      _stream(stream)))
+
+
+def qk_score_grpo(m, tokens, B, T, lp_old, lp_ref, rewards, group, mask, eps_low, eps_high, beta,
+                  logprobs, loss_tok, loss_mean=None, workspace=None, ws_bytes=None, stream=None):
+    _check(_load().qk_score_grpo(m, _ptr(tokens), B, T, _ptr(lp_old), _ptr(lp_ref), _ptr(rewards),
+                                 group, _ptr(mask), eps_low, eps_high, beta, _ptr(logprobs),
+                                 _ptr(loss_tok), _ptr(loss_mean), _ptr(workspace),
+                                 _nbytes(workspace, ws_bytes), _stream(stream)))
 
 
 def qk_rollout_teacher_forced(m, kv, max_batch, max_seq, seq, B, P, N, logprobs, argmax=None,

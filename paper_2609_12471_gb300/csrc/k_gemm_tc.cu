@@ -33,6 +33,14 @@ namespace {
 
 constexpr int kThreads = 192;
 constexpr int kBK = 64;  // bf16 elements per k-block: one 128-byte swizzle row
+// Decode (fused, 16-row) configuration.  Five ring stages (109 KB of shared
+// memory) and at most 168 registers a thread let a CTA of the next kernel become
+// resident beside one of this kernel, so its weight prefetch starts while this
+// kernel's last tiles finish (measured faster than an 8-stage ring that needs the
+// whole SM); partial slots are loaded two at a time to stay inside the registers.
+constexpr int kFused16Stages = 5;
+constexpr int kFusedCtasPerSm = 2;
+constexpr int kFused16PartialBatch = 2;
 
 __host__ __device__ constexpr int pow2_at_least(int v) {
     int p = 32;
@@ -136,7 +144,7 @@ __device__ __forceinline__ int it_owner(long long it, long long I, int C) {
 }
 
 template <int BN, bool SWIGLU, int STAGES, bool FUSED>
-__global__ void __launch_bounds__(kThreads, 1)
+__global__ void __launch_bounds__(kThreads, FUSED && BN == 16 ? kFusedCtasPerSm : 1)
     gemm_tc_kernel(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ CUtensorMap tmX,
                    void* __restrict__ C, int ldc, int M, int N, int K, int epi, int n_split,
                    uint32_t* __restrict__ status, const __grid_constant__ Fuse fz) {
@@ -356,7 +364,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             }
             epi_bar();  // s_row, p_row and xch settled
         }
-        constexpr int PB = BN <= 16 ? 6 : (BN <= 32 ? 3 : 1);  // partial slots per load batch
+        constexpr int PB = BN <= 16 ? kFused16PartialBatch : (BN <= 32 ? 3 : 1);  // partial slots per load batch
         int acc = 0;
         uint32_t acc_phase = 0;
         // Partials: slot (CTA + tile) holds one segment's [M][128] fp32 sums; the slots of
@@ -716,7 +724,7 @@ int launch_gemm_tc_fused(const bf16* A, int lda, const bf16* W, float* out, int 
     // every launch may split a tile over CTAs: partial slots and tickets are required
     if (!f.part || !f.tickets || !f.status) return QK_EINVAL;
     if (M <= 16)
-        return launch_cfg<16, false, 8, true>(A, lda, W, out, N, M, N, K, EPI_PARTIAL_F32, 1,
+        return launch_cfg<16, false, kFused16Stages, true>(A, lda, W, out, N, M, N, K, EPI_PARTIAL_F32, 1,
                                               num_sms, status, s, &f);
     if (M <= 32)
         return launch_cfg<32, false, 8, true>(A, lda, W, out, N, M, N, K, EPI_PARTIAL_F32, 1,

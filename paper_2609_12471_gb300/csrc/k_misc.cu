@@ -282,7 +282,8 @@ constexpr int kLogitCtas = 8;
 
 __global__ void __cluster_dims__(kLogitCtas, 1, 1) __launch_bounds__(256)
     logits_reduce_kernel(const float* __restrict__ logits, int V, OutIndex oi,
-                         float* __restrict__ lp, int32_t* __restrict__ am, uint32_t* status) {
+                         float* __restrict__ lp, int32_t* __restrict__ am, uint32_t* status,
+                         GrpoArgs grpo) {
     __shared__ MaxSum red[8];
     __shared__ MaxSum part;
     pdl_wait();
@@ -351,18 +352,29 @@ __global__ void __cluster_dims__(kLogitCtas, 1, 1) __launch_bounds__(256)
         }
         const size_t o = (size_t)b * oi.out_ld + oi.out_off + t + (oi.dyn_off ? *oi.dyn_off : 0);
         if (am) am[o] = c.i;
-        if (lp && oi.tgt) lp[o] = z_tg - (c.m + logf(c.s));
+        if (lp && oi.tgt) {
+            const float l = z_tg - (c.m + logf(c.s));
+            lp[o] = l;
+            if (grpo.loss_tok) {  // Eq. ppo for this token, where its log-prob is formed
+                const size_t go = (size_t)b * grpo.ld + t;
+                const float ref = grpo.lp_ref ? grpo.lp_ref[go] : l;
+                grpo.loss_tok[go] = grpo_token(l, grpo.lp_old[go], ref,
+                                               grpo_advantage(grpo.rewards, b, grpo.group), grpo);
+            }
+        }
     }
     // no CTA leaves while CTA 0 may still read its shared memory
     asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;" ::: "memory");
 }
 
 void launch_logits_reduce(const float* logits, int M, int V, OutIndex oi, float* lp,
-                          int32_t* argmax, uint32_t* status, cudaStream_t s) {
+                          int32_t* argmax, uint32_t* status, cudaStream_t s, const GrpoArgs* grpo) {
     note_launch();
     if (M <= 0) return;
+    GrpoArgs g{};
+    if (grpo) g = *grpo;
     launch_k(logits_reduce_kernel, dim3(kLogitCtas, M), dim3(256), 0, s, logits, V, oi, lp, argmax,
-             status);
+             status, g);
 }
 
 // ---------------------------------------------------------------- rollout cursor

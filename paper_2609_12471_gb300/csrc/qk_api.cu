@@ -714,16 +714,11 @@ int qk_decode_layer(qk_model* mh, int layer, void* kv, int max_batch, int max_se
     return check_launch(m, "decode layer");
 }
 
-int qk_score_logprobs(qk_model* mh, const int32_t* tokens, int B, int T, float* logprobs,
-                      int32_t* argmax, void* workspace, size_t ws_bytes, void* stream) {
-    if (!mh || !tokens || !logprobs) return set_error(QK_EINVAL, "null argument");
-    Model& m = *(Model*)mh;
-    if (B < 1 || T < 2) return set_error(QK_ESHAPE, "scoring needs B >= 1 and T >= 2 (got %d, %d)", B, T);
-    if (T > m.cfg.max_positions)
-        return set_error(QK_ESHAPE, "T %d exceeds the RoPE table (%d)", T, m.cfg.max_positions);
+static int score_impl(Model& m, const int32_t* tokens, int B, int T, float* logprobs,
+                      int32_t* argmax, void* workspace, size_t ws_bytes, cudaStream_t s,
+                      const GrpoArgs* grpo) {
     Workspace w;
     QK_TRY(get_ws(m, QK_CALL_SCORE, B, T, T, workspace, ws_bytes, &w));
-    cudaStream_t s = (cudaStream_t)stream;
     int M = B * T;
     // One layer's K and V live in scratch shaped like a cache of B rows x T positions;
     // every layer reuses it (layer stride 0).
@@ -741,9 +736,84 @@ int qk_score_logprobs(qk_model* mh, const int32_t* tokens, int B, int T, float* 
         linear(m, w.u, m.cfg.hidden, m.lm_head, w.logits, m.cfg.vocab, rows, m.cfg.vocab,
                m.cfg.hidden, EPI_STORE_F32, w.gu, s);
         OutIndex oi{T, T - 1, T - 1, 0, tokens, T, 1, r0};
-        launch_logits_reduce(w.logits, rows, m.cfg.vocab, oi, logprobs, argmax, m.status, s);
+        launch_logits_reduce(w.logits, rows, m.cfg.vocab, oi, logprobs, argmax, m.status, s, grpo);
     }
+    return QK_OK;
+}
+
+static int check_score_shape(const Model& m, int B, int T) {
+    if (B < 1 || T < 2) return set_error(QK_ESHAPE, "scoring needs B >= 1 and T >= 2 (got %d, %d)", B, T);
+    if (T > m.cfg.max_positions)
+        return set_error(QK_ESHAPE, "T %d exceeds the RoPE table (%d)", T, m.cfg.max_positions);
+    return QK_OK;
+}
+
+int qk_score_logprobs(qk_model* mh, const int32_t* tokens, int B, int T, float* logprobs,
+                      int32_t* argmax, void* workspace, size_t ws_bytes, void* stream) {
+    if (!mh || !tokens || !logprobs) return set_error(QK_EINVAL, "null argument");
+    Model& m = *(Model*)mh;
+    QK_TRY(check_score_shape(m, B, T));
+    QK_TRY(score_impl(m, tokens, B, T, logprobs, argmax, workspace, ws_bytes, (cudaStream_t)stream,
+                      nullptr));
     return check_launch(m, "score");
+}
+
+// ---------------------------------------------------------------- GRPO token loss
+int qk_grpo_workspace_bytes(int B, size_t* bytes) {
+    if (!bytes) return set_error(QK_EINVAL, "null argument");
+    if (B < 1) return set_error(QK_ESHAPE, "batch %d must be >= 1", B);
+    *bytes = grpo_scratch_bytes(B);
+    return QK_OK;
+}
+
+static int grpo_args(const float* lp_old, const float* lp_ref, int B, int T, int ld,
+                     const float* rewards, int group, const uint8_t* mask, float eps_low,
+                     float eps_high, float beta, float* loss_tok, GrpoArgs* g) {
+    if (!lp_old || !rewards || !loss_tok) return set_error(QK_EINVAL, "null argument");
+    if (beta != 0.f && !lp_ref) return set_error(QK_EINVAL, "beta != 0 needs lp_ref");
+    if (B < 1 || T < 1 || ld < T) return set_error(QK_ESHAPE, "need B >= 1, T >= 1, ld >= T");
+    if (group < 1 || B % group) return set_error(QK_ESHAPE, "batch %d is not a multiple of group %d", B, group);
+    if (!(eps_low >= 0.f && eps_low <= 1.f && eps_high >= 0.f))
+        return set_error(QK_EINVAL, "clip band needs 0 <= eps_low <= 1 and eps_high >= 0");
+    *g = GrpoArgs{lp_old, lp_ref, rewards, mask, loss_tok, group, ld, eps_low, eps_high, beta};
+    return QK_OK;
+}
+
+int qk_grpo_token_loss(const float* lp, const float* lp_old, const float* lp_ref, int B, int T,
+                       int ld, const float* rewards, int group, const uint8_t* mask,
+                       float eps_low, float eps_high, float beta, float* loss_tok,
+                       float* loss_mean, void* workspace, size_t ws_bytes, void* stream) {
+    if (!lp) return set_error(QK_EINVAL, "null argument");
+    GrpoArgs g;
+    QK_TRY(grpo_args(lp_old, lp_ref, B, T, ld, rewards, group, mask, eps_low, eps_high, beta,
+                     loss_tok, &g));
+    if (!workspace || ws_bytes < grpo_scratch_bytes(B))
+        return set_error(QK_ENOSPACE, "workspace has %zu bytes, needs %zu", ws_bytes,
+                         grpo_scratch_bytes(B));
+    launch_grpo_loss(lp, B, T, g, true, workspace, loss_mean, (cudaStream_t)stream);
+    return check_launch("grpo token loss");
+}
+
+int qk_score_grpo(qk_model* mh, const int32_t* tokens, int B, int T, const float* lp_old,
+                  const float* lp_ref, const float* rewards, int group, const uint8_t* mask,
+                  float eps_low, float eps_high, float beta, float* logprobs, float* loss_tok,
+                  float* loss_mean, void* workspace, size_t ws_bytes, void* stream) {
+    if (!mh || !tokens || !logprobs) return set_error(QK_EINVAL, "null argument");
+    Model& m = *(Model*)mh;
+    QK_TRY(check_score_shape(m, B, T));
+    GrpoArgs g;
+    QK_TRY(grpo_args(lp_old, lp_ref, B, T - 1, T - 1, rewards, group, mask, eps_low, eps_high,
+                     beta, loss_tok, &g));
+    size_t score_bytes;
+    QK_TRY(qk_workspace_bytes(mh, QK_CALL_SCORE, B, T, T, &score_bytes));
+    score_bytes = align256(score_bytes);
+    if (!workspace || ws_bytes < score_bytes + grpo_scratch_bytes(B))
+        return set_error(QK_ENOSPACE, "workspace has %zu bytes, needs %zu", ws_bytes,
+                         score_bytes + grpo_scratch_bytes(B));
+    cudaStream_t s = (cudaStream_t)stream;
+    QK_TRY(score_impl(m, tokens, B, T, logprobs, nullptr, workspace, score_bytes, s, &g));
+    launch_grpo_loss(logprobs, B, T - 1, g, false, (char*)workspace + score_bytes, loss_mean, s);
+    return check_launch(m, "score with GRPO loss");
 }
 
 int qk_rollout_teacher_forced(qk_model* mh, void* kv, int max_batch, int max_seq,

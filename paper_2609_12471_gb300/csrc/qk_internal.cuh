@@ -169,8 +169,49 @@ void launch_qk_norm_rope(void* qkv, int dtype, int M, int nq, int nkv, int d, co
                          int max_positions, PosIndex pos, void* k_cache, void* v_cache,
                          int max_seq, uint32_t* status, cudaStream_t s);
 void launch_swiglu(const void* gu, void* h, int dtype, int M, int I, cudaStream_t s);
+// GRPO token loss (Sec. "GRPO Optimization"): inputs and output of Eq. ppo for the
+// tokens whose log-prob a kernel forms; loss_tok == nullptr disables it.
+struct GrpoArgs {
+    const float* lp_old;
+    const float* lp_ref;   // may be null when beta == 0
+    const float* rewards;  // [B]
+    const uint8_t* mask;   // [B, ld] or null (all ones)
+    float* loss_tok;       // [B, ld]
+    int group, ld;
+    float eps_low, eps_high, beta;
+};
+
+// Eq. advantage: A_b = r_b - mean of r over b's group (summed in row order).
+__device__ __forceinline__ float grpo_advantage(const float* rewards, int b, int group) {
+    const int g0 = b - b % group;
+    float s = 0.f;
+    for (int i = 0; i < group; ++i) s += rewards[g0 + i];
+    return rewards[b] - s / (float)group;
+}
+
+// Eq. ppo for one token: -min(rho A, clip(rho, 1 - eps_low, 1 + eps_high) A) + beta k3,
+// rho = exp(lp - lp_old), k3 = e^x - x - 1 with x = lp_ref - lp (as expm1(x) - x).
+__device__ __forceinline__ float grpo_token(float lp, float lp_old, float lp_ref, float A,
+                                            const GrpoArgs& g) {
+    const float rho = expf(lp - lp_old);
+    const float clipped = fminf(fmaxf(rho, 1.f - g.eps_low), 1.f + g.eps_high);
+    float L = -fminf(rho * A, clipped * A);
+    if (g.beta != 0.f) {
+        const float x = lp_ref - lp;
+        L += g.beta * (expm1f(x) - x);
+    }
+    return L;
+}
+
 void launch_logits_reduce(const float* logits, int M, int V, OutIndex oi, float* lp,
-                          int32_t* argmax, uint32_t* status, cudaStream_t s);
+                          int32_t* argmax, uint32_t* status, cudaStream_t s,
+                          const GrpoArgs* grpo = nullptr);
+// GRPO reductions (k_grpo.cu).  With `compute`, loss_tok is formed from lp (else it
+// was formed by the scoring epilogue); then per-row sums of mask * loss and of the
+// mask go to `rows` ([B] float2) and loss_mean (if not null) = their ratio.
+size_t grpo_scratch_bytes(int B);
+void launch_grpo_loss(const float* lp, int B, int T, const GrpoArgs& g, bool compute,
+                      void* scratch, float* loss_mean, cudaStream_t s);
 // Rollout cursor: s = *step; pos[b] = P + s; tok[b] = seq[b, P + s]; tgt[b] = seq[b, P + s + 1];
 // *out_off = s + 1; *step = s + 1.
 void launch_rollout_prepare(const int32_t* seq, int L, int P, int B, int32_t* step, int32_t* pos,

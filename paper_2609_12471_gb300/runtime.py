@@ -101,6 +101,24 @@ class Decoder:
         B.qk_score_logprobs(self.handle, tokens, Bn, T, logprobs, argmax, ws)
         return logprobs
 
+    def score_grpo(self, tokens, lp_old, rewards, group, lp_ref=None, mask=None, eps_low=0.2,
+                   eps_high=0.28, beta=0.01):
+        """Scoring with the GRPO token loss formed in the log-prob epilogue.
+        Returns (logprobs [B, T-1], loss_tok [B, T-1], loss_mean [1])."""
+        Bn, T = tokens.shape
+        logprobs = torch.empty(Bn, T - 1, dtype=torch.float32, device=self.device)
+        loss_tok = torch.empty(Bn, T - 1, dtype=torch.float32, device=self.device)
+        loss_mean = torch.empty(1, dtype=torch.float32, device=self.device)
+        need = (B.qk_workspace_bytes(self.handle, B.QK_CALL_SCORE, Bn, T, T) + 255) // 256 * 256
+        need += B.qk_grpo_workspace_bytes(Bn)
+        ws = self._ws.get("score_grpo")
+        if ws is None or ws.numel() < need:
+            ws = torch.empty(need, dtype=torch.uint8, device=self.device)
+            self._ws["score_grpo"] = ws
+        B.qk_score_grpo(self.handle, tokens, Bn, T, lp_old, lp_ref, rewards, group, mask, eps_low,
+                        eps_high, beta, logprobs, loss_tok, loss_mean, ws)
+        return logprobs, loss_tok, loss_mean
+
     def rollout(self, kv, max_batch, max_seq, seq, P, logprobs=None, argmax=None):
         Bn, L = seq.shape
         N = L - P - 1
@@ -113,3 +131,16 @@ class Decoder:
 
     def check_status(self) -> int:
         return B.qk_check_status(self.handle)
+
+
+def grpo_token_loss(lp, lp_old, rewards, group, lp_ref=None, mask=None, eps_low=0.2, eps_high=0.28,
+                    beta=0.01, stream=None):
+    """GRPO token loss over precomputed log-probs [B, T] (contiguous rows): returns
+    (loss_tok [B, T], loss_mean [1]); every step runs in libqk's kernels."""
+    Bn, T = lp.shape
+    loss_tok = torch.empty_like(lp)
+    loss_mean = torch.empty(1, dtype=torch.float32, device=lp.device)
+    ws = torch.empty(B.qk_grpo_workspace_bytes(Bn), dtype=torch.uint8, device=lp.device)
+    B.qk_grpo_token_loss(lp, lp_old, lp_ref, Bn, T, T, rewards, group, mask, eps_low, eps_high, beta,
+                         loss_tok, loss_mean, ws, stream=stream)
+    return loss_tok, loss_mean
