@@ -7,3 +7,5 @@ with it; the two meet only in the seeded inputs of ``synth``.
 """
 from .qwen3 import *  # noqa: F401,F403
 from .grpo import group_advantages, grpo_loss_mean, grpo_token_loss, kl_k3  # noqa: F401
+from .sampling import (gumbel, mix64, rollout_sampled, sample_token, sample_uniforms,  # noqa: F401
+                       splitmix64_at)

@@ -44,6 +44,16 @@ GRPO_MUTATIONS = {
 }
 
 
+# Mistakes in the sampling oracle, caught by test_oracle_sampling.py.
+SAMPLING_MUTATIONS = {
+    "gumbel_sign": ("return -np.log(-np.log(u))", "return np.log(-np.log(u))"),
+    "temperature_multiplies": ("y = z / tau + gumbel(", "y = z * tau + gumbel("),
+    "mix_constant": ("_M1 = np.uint64(0xBF58476D1CE4E5B9)", "_M1 = np.uint64(0xBF58476D1CE4E5B8)"),
+    "counter_offset": ("(i + np.uint64(1)) * GAMMA", "i * GAMMA"),
+    "uniform_grid": ("+ 0.5) * 2.0 ** -24", "+ 0.0) * 2.0 ** -24"),
+}
+
+
 def _run_mutated(tmp_path, module, before, after, name, pins):
     shutil.copytree(os.path.join(ROOT, "oracle"), tmp_path / "oracle",
                     ignore=shutil.ignore_patterns("__pycache__"))
@@ -68,3 +78,9 @@ def test_pins_catch_planted_mistake(name, tmp_path):
 def test_grpo_pins_catch_planted_mistake(name, tmp_path):
     before, after = GRPO_MUTATIONS[name]
     _run_mutated(tmp_path, "grpo.py", before, after, name, "test_oracle_grpo.py")
+
+
+@pytest.mark.parametrize("name", sorted(SAMPLING_MUTATIONS))
+def test_sampling_pins_catch_planted_mistake(name, tmp_path):
+    before, after = SAMPLING_MUTATIONS[name]
+    _run_mutated(tmp_path, "sampling.py", before, after, name, "test_oracle_sampling.py")
