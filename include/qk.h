@@ -195,6 +195,19 @@ int qk_rollout_teacher_forced(qk_model* m, void* kv, int max_batch, int max_seq,
                               const int32_t* seq, int B, int P, int N, float* logprobs,
                               int32_t* argmax, void* workspace, size_t ws_bytes, void* stream);
 
+/* Sampled rollout at temperature tau > 0 (the paper samples at 1.0): prompt dev
+ * int32 [B, P].  The prefill's last logits draw c[0]; decode step j (0 <= j < N)
+ * consumes c[j] at position P+j and draws c[j+1].  A draw from softmax(z / tau)
+ * is the Gumbel-max rule c = argmax_v (z_v / tau - log(-log u_v)) (lowest index on
+ * ties), u_v the 24-bit uniform (floor(x / 2^40) + 1/2) / 2^24 of output
+ * i = b 2^40 + j 2^18 + v of the SplitMix64 stream seeded with `seed` (row b,
+ * step j, token v; needs B < 2^24, N < 2^22, vocab <= 2^18).  tokens dev int32
+ * [B, N+1] receives c[0..N]; logprobs dev fp32 [B, N+1] receives
+ * log softmax(z_j / tau)[c[j]].  Workspace and cache as qk_rollout_teacher_forced. */
+int qk_rollout_sampled(qk_model* m, void* kv, int max_batch, int max_seq, const int32_t* prompt,
+                       int B, int P, int N, float tau, uint64_t seed, int32_t* tokens,
+                       float* logprobs, void* workspace, size_t ws_bytes, void* stream);
+
 /* Synchronise `stream`, read the device status word into *flags (QK_STATUS_*
  * bits) and clear it.  Returns QK_EDEVICE if any bit was set, QK_OK otherwise. */
 int qk_check_status(qk_model* m, void* stream, uint32_t* flags);

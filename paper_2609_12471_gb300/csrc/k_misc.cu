@@ -252,6 +252,8 @@ void launch_swiglu(const void* gu, void* h, int dtype, int M, int I, cudaStream_
 struct MaxSum {
     float m, s;
     int i;
+    float ym;  // sampling: the largest perturbed score z / tau + G and its token
+    int yi;
 };
 
 __device__ __forceinline__ void ms_push(MaxSum& a, float v, int i) {
@@ -267,11 +269,32 @@ __device__ __forceinline__ void ms_push(MaxSum& a, float v, int i) {
 // a followed by b (b covers later indices, or is an unordered peer: ties take the lower index)
 __device__ __forceinline__ MaxSum ms_merge(MaxSum a, MaxSum b) {
     MaxSum r;
+    r.ym = fmaxf(a.ym, b.ym);
+    r.yi = a.ym > b.ym ? a.yi : (b.ym > a.ym ? b.yi : min(a.yi, b.yi));
     r.m = fmaxf(a.m, b.m);
-    if (r.m == -INFINITY) return a;
+    if (r.m == -INFINITY) {
+        a.ym = r.ym, a.yi = r.yi;
+        return a;
+    }
     r.s = (a.m == -INFINITY ? 0.f : a.s * expf(a.m - r.m)) + (b.m == -INFINITY ? 0.f : b.s * expf(b.m - r.m));
     r.i = a.m > b.m ? a.i : (b.m > a.m ? b.i : min(a.i, b.i));
     return r;
+}
+
+// Gumbel noise for (row b, sampling step j, token v): the uniform is output
+// i = b 2^40 + j 2^18 + v of the SplitMix64 stream seeded with `seed` (Steele, Lea,
+// Flood, OOPSLA 2014: state seed + (i + 1) gamma through the published finaliser),
+// on the 24-bit grid u = (x / 2^40 + 1/2) / 2^24 (exact in fp32, strictly inside
+// (0, 1)); G = -log(-log u).
+__device__ __forceinline__ float gumbel_noise(unsigned long long seed, int b, int j, int v) {
+    const unsigned long long i =
+        ((unsigned long long)b << 40) + ((unsigned long long)j << 18) + (unsigned long long)v;
+    unsigned long long z = seed + (i + 1ull) * 0x9E3779B97F4A7C15ull;
+    z = (z ^ (z >> 30)) * 0xBF58476D1CE4E5B9ull;
+    z = (z ^ (z >> 27)) * 0x94D049BB133111EBull;
+    z ^= z >> 31;
+    const float u = ((float)(z >> 40) + 0.5f) * 5.9604644775390625e-8f;  // 2^-24
+    return -logf(-logf(u));
 }
 
 // One logits row per cluster of kLogitCtas CTAs: CTA k of the cluster reduces the
@@ -283,7 +306,7 @@ constexpr int kLogitCtas = 8;
 __global__ void __cluster_dims__(kLogitCtas, 1, 1) __launch_bounds__(256)
     logits_reduce_kernel(const float* __restrict__ logits, int V, OutIndex oi,
                          float* __restrict__ lp, int32_t* __restrict__ am, uint32_t* status,
-                         GrpoArgs grpo) {
+                         GrpoArgs grpo, SampleArgs samp) {
     __shared__ MaxSum red[8];
     __shared__ MaxSum part;
     pdl_wait();
@@ -293,9 +316,13 @@ __global__ void __cluster_dims__(kLogitCtas, 1, 1) __launch_bounds__(256)
     const int b = g / oi.T, t = g % oi.T;
     const bool active = t < oi.out_lim;  // uniform over the cluster (one row per cluster)
     const float* z = logits + (size_t)r * V;
+    const bool sampling = samp.out_tokens != nullptr;
+    // the output column is the sampling step (prefill: 0; rollout decode step s: s + 1)
+    const int step = t + oi.out_off + (oi.dyn_off ? *oi.dyn_off : 0);
+    const float inv_tau = sampling ? samp.inv_tau : 1.f;
     int tg = 0;
     float z_tg = 0.f;
-    if (active && k == 0 && threadIdx.x == 0 && lp && oi.tgt) {  // fetched early, used last
+    if (active && !sampling && k == 0 && threadIdx.x == 0 && lp && oi.tgt) {  // fetched early, used last
         tg = oi.tgt[(size_t)b * oi.tgt_ld + oi.tgt_off + t];
         if (tg < 0 || tg >= V) {
             atomicOr(status, QK_STATUS_BAD_TOKEN);
@@ -303,7 +330,16 @@ __global__ void __cluster_dims__(kLogitCtas, 1, 1) __launch_bounds__(256)
         }
         z_tg = z[tg];
     }
-    MaxSum a{-INFINITY, 0.f, 0x7fffffff};
+    MaxSum a{-INFINITY, 0.f, 0x7fffffff, -INFINITY, 0x7fffffff};
+    // z / tau into the max / sum of exponentials; with sampling also z / tau + G into (ym, yi)
+    auto push = [&](float zv, int i) {
+        const float zz = zv * inv_tau;
+        ms_push(a, zz, i);
+        if (sampling) {
+            const float y = zz + gumbel_noise(samp.seed, b, step, i);
+            if (y > a.ym) a.ym = y, a.yi = i;
+        }
+    };
     if (active) {
         // slice k: [lo, hi), a multiple of 4 wide except at the row's end
         const int per = ((V + kLogitCtas - 1) / kLogitCtas + 3) & ~3;
@@ -311,13 +347,13 @@ __global__ void __cluster_dims__(kLogitCtas, 1, 1) __launch_bounds__(256)
         if ((V & 3) == 0) {
             for (int i = lo + threadIdx.x * 4; i < hi; i += blockDim.x * 4) {
                 const float4 v = *reinterpret_cast<const float4*>(z + i);
-                ms_push(a, v.x, i);
-                ms_push(a, v.y, i + 1);
-                ms_push(a, v.z, i + 2);
-                ms_push(a, v.w, i + 3);
+                push(v.x, i);
+                push(v.y, i + 1);
+                push(v.z, i + 2);
+                push(v.w, i + 3);
             }
         } else {
-            for (int i = lo + threadIdx.x; i < hi; i += blockDim.x) ms_push(a, z[i], i);
+            for (int i = lo + threadIdx.x; i < hi; i += blockDim.x) push(z[i], i);
         }
     }
 #pragma unroll
@@ -326,6 +362,8 @@ __global__ void __cluster_dims__(kLogitCtas, 1, 1) __launch_bounds__(256)
         p.m = __shfl_xor_sync(0xffffffffu, a.m, o);
         p.s = __shfl_xor_sync(0xffffffffu, a.s, o);
         p.i = __shfl_xor_sync(0xffffffffu, a.i, o);
+        p.ym = __shfl_xor_sync(0xffffffffu, a.ym, o);
+        p.yi = __shfl_xor_sync(0xffffffffu, a.yi, o);
         a = ms_merge(a, p);
     }
     const int w = threadIdx.x >> 5, l = threadIdx.x & 31;
@@ -339,7 +377,7 @@ __global__ void __cluster_dims__(kLogitCtas, 1, 1) __launch_bounds__(256)
     // every slice's partial is in its CTA's shared memory before CTA 0 reads them
     asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;" ::: "memory");
     if (active && k == 0 && threadIdx.x == 0) {
-        MaxSum c{-INFINITY, 0.f, 0x7fffffff};
+        MaxSum c{-INFINITY, 0.f, 0x7fffffff, -INFINITY, 0x7fffffff};
         const uint32_t local = (uint32_t)__cvta_generic_to_shared(&part);
         for (int q = 0; q < kLogitCtas; ++q) {
             uint32_t remote;
@@ -348,11 +386,21 @@ __global__ void __cluster_dims__(kLogitCtas, 1, 1) __launch_bounds__(256)
             asm volatile("ld.shared::cluster.f32 %0, [%1];" : "=f"(p.m) : "r"(remote));
             asm volatile("ld.shared::cluster.f32 %0, [%1+4];" : "=f"(p.s) : "r"(remote));
             asm volatile("ld.shared::cluster.s32 %0, [%1+8];" : "=r"(p.i) : "r"(remote));
+            asm volatile("ld.shared::cluster.f32 %0, [%1+12];" : "=f"(p.ym) : "r"(remote));
+            asm volatile("ld.shared::cluster.s32 %0, [%1+16];" : "=r"(p.yi) : "r"(remote));
             c = ms_merge(c, p);
         }
         const size_t o = (size_t)b * oi.out_ld + oi.out_off + t + (oi.dyn_off ? *oi.dyn_off : 0);
         if (am) am[o] = c.i;
-        if (lp && oi.tgt) {
+        if (sampling) {  // the drawn token and log softmax(z / tau) at it
+            int tok = c.yi;
+            if (tok < 0 || tok >= V) {  // only non-finite logits leave no maximum
+                atomicOr(status, QK_STATUS_BAD_TOKEN);
+                tok = 0;
+            }
+            samp.out_tokens[o] = tok;
+            if (lp) lp[o] = z[tok] * inv_tau - (c.m + logf(c.s));
+        } else if (lp && oi.tgt) {
             const float l = z_tg - (c.m + logf(c.s));
             lp[o] = l;
             if (grpo.loss_tok) {  // Eq. ppo for this token, where its log-prob is formed
@@ -368,13 +416,16 @@ __global__ void __cluster_dims__(kLogitCtas, 1, 1) __launch_bounds__(256)
 }
 
 void launch_logits_reduce(const float* logits, int M, int V, OutIndex oi, float* lp,
-                          int32_t* argmax, uint32_t* status, cudaStream_t s, const GrpoArgs* grpo) {
+                          int32_t* argmax, uint32_t* status, cudaStream_t s, const GrpoArgs* grpo,
+                          const SampleArgs* samp) {
     note_launch();
     if (M <= 0) return;
     GrpoArgs g{};
     if (grpo) g = *grpo;
+    SampleArgs sa{};
+    if (samp) sa = *samp;
     launch_k(logits_reduce_kernel, dim3(kLogitCtas, M), dim3(256), 0, s, logits, V, oi, lp, argmax,
-             status, g);
+             status, g, sa);
 }
 
 // ---------------------------------------------------------------- rollout cursor
@@ -401,6 +452,30 @@ void launch_rollout_prepare(const int32_t* seq, int L, int P, int B, int32_t* st
     note_launch();
     launch_k(rollout_prepare_kernel, dim3(1), dim3(256), 0, s, seq, L, P, B, step, pos, tok, tgt,
              out_off);
+}
+
+__global__ void rollout_prepare_sampled_kernel(const int32_t* __restrict__ sampled, int ld, int P,
+                                               int B, int32_t* step, int32_t* pos, int32_t* tok,
+                                               int32_t* out_off) {
+    pdl_wait();
+    pdl_trigger();
+    const int s = *step;
+    __syncthreads();  // every thread has read the step before it advances
+    for (int b = threadIdx.x; b < B; b += blockDim.x) {
+        pos[b] = P + s;
+        tok[b] = sampled[(size_t)b * ld + s];
+    }
+    if (threadIdx.x == 0) {
+        *out_off = s + 1;
+        *step = s + 1;
+    }
+}
+
+void launch_rollout_prepare_sampled(const int32_t* sampled, int ld, int P, int B, int32_t* step,
+                                    int32_t* pos, int32_t* tok, int32_t* out_off, cudaStream_t s) {
+    note_launch();
+    launch_k(rollout_prepare_sampled_kernel, dim3(1), dim3(256), 0, s, sampled, ld, P, B, step, pos,
+             tok, out_off);
 }
 
 // ---------------------------------------------------------------- load-time tables

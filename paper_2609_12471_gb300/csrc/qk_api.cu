@@ -320,7 +320,9 @@ static void run_head(Model& m, const Workspace& w, int M_out, int in_step, int i
     linear(m, w.u, c.hidden, m.lm_head, logits, c.vocab, M_out, c.vocab, c.hidden, EPI_STORE_F32,
            w.gu, s);
     prof_close(m, pr, s);
-    if (lp || am) launch_logits_reduce(logits, M_out, c.vocab, oi, lp, am, m.status, s);
+    if (lp || am)
+        launch_logits_reduce(logits, M_out, c.vocab, oi, lp, am, m.status, s, nullptr,
+                             m.sampling.out_tokens ? &m.sampling : nullptr);
 }
 
 // The split decode attention merges through tickets in its scratch that must be
@@ -663,7 +665,9 @@ static int decode_impl(Model& m, void* kv, int max_batch, int max_seq, TokIndex 
                                           c.hidden, fl, m.num_sms, m.status, s);
             prof_close(m, pr, s);
             if (rc != QK_OK && !m.deferred_error) m.deferred_error = rc;
-            if (lp || am) launch_logits_reduce(z, B, c.vocab, oi, lp, am, m.status, s);
+            if (lp || am)
+                launch_logits_reduce(z, B, c.vocab, oi, lp, am, m.status, s, nullptr,
+                                     m.sampling.out_tokens ? &m.sampling : nullptr);
         }
     } else {
         launch_embed(m.embed, m.cfg.dtype, m.cfg.vocab, m.cfg.hidden, tok, B, w.x, m.status, s);
@@ -816,11 +820,15 @@ int qk_score_grpo(qk_model* mh, const int32_t* tokens, int B, int T, const float
     return check_launch(m, "score with GRPO loss");
 }
 
-int qk_rollout_teacher_forced(qk_model* mh, void* kv, int max_batch, int max_seq,
-                              const int32_t* seq, int B, int P, int N, float* logprobs,
-                              int32_t* argmax, void* workspace, size_t ws_bytes, void* stream) {
-    if (!mh || !seq || !logprobs) return set_error(QK_EINVAL, "null argument");
-    Model& m = *(Model*)mh;
+// Rollout of B rows: prefill over the prompt, then N decode steps replayed from one
+// captured graph.  Teacher forcing (sampled == nullptr): seq [B, P+N+1] supplies
+// every input token and target.  Sampling: seq is the prompt [B, P]; the head of
+// each step draws the next token into sampled [B, N+1] (m.sampling), and the next
+// step reads it from there.
+static int rollout_impl(Model& m, qk_model* mh, void* kv, int max_batch, int max_seq,
+                        const int32_t* seq, int B, int P, int N, float* logprobs, int32_t* argmax,
+                        const SampleArgs* sampled, void* workspace, size_t ws_bytes,
+                        cudaStream_t s) {
     QK_TRY(check_cache(m, kv, max_batch, max_seq, B));
     if (P < 1 || N < 0 || (long)P + N > max_seq)
         return set_error(QK_ESHAPE, "prompt %d + steps %d exceed the cache of %d", P, N, max_seq);
@@ -828,9 +836,13 @@ int qk_rollout_teacher_forced(qk_model* mh, void* kv, int max_batch, int max_seq
     QK_TRY(qk_workspace_bytes(mh, QK_CALL_ROLLOUT, B, P, max_seq, &need));
     if (!workspace || ws_bytes < need)
         return set_error(QK_ENOSPACE, "workspace has %zu bytes, needs %zu", ws_bytes, need);
-    cudaStream_t s = (cudaStream_t)stream;
-    const int L = P + N + 1;
-    OutIndex oi{1, 1, N + 1, 0, seq, L, P, 0};
+    struct SamplingScope {  // m.sampling is set only for the duration of this call
+        Model& m;
+        SamplingScope(Model& mm, const SampleArgs* a) : m(mm) { m.sampling = a ? *a : SampleArgs{}; }
+        ~SamplingScope() { m.sampling = SampleArgs{}; }
+    } scope(m, sampled);
+    const int L = sampled ? P : P + N + 1;  // row length of seq
+    OutIndex oi{1, 1, N + 1, 0, sampled ? nullptr : seq, L, P, 0};
     QK_TRY(prefill_impl(m, kv, max_batch, max_seq, TokIndex{seq, P, L, 0}, B, P, 0, nullptr, oi,
                         logprobs, argmax, workspace, ws_bytes, s));
     if (N == 0) return QK_OK;
@@ -843,9 +855,15 @@ int qk_rollout_teacher_forced(qk_model* mh, void* kv, int max_batch, int max_seq
     int32_t* tgt = (int32_t*)(cur + 3 * slot);
     int32_t* off = (int32_t*)(cur + 4 * slot);
     QK_TRY_CUDA(cudaMemsetAsync(step, 0, sizeof(int32_t), s));
-    OutIndex od{1, 1, N + 1, 0, tgt, 1, 0, 0, off};
+    OutIndex od{1, 1, N + 1, 0, sampled ? nullptr : tgt, 1, 0, 0, off};
+    auto prepare = [&](cudaStream_t st) {
+        if (sampled)
+            launch_rollout_prepare_sampled(sampled->out_tokens, N + 1, P, B, step, pos, tok, off, st);
+        else
+            launch_rollout_prepare(seq, L, P, B, step, pos, tok, tgt, off, st);
+    };
     auto one_step = [&]() -> int {
-        launch_rollout_prepare(seq, L, P, B, step, pos, tok, tgt, off, s);
+        prepare(s);
         return decode_impl(m, kv, max_batch, max_seq, TokIndex{tok, 1, 1, 0}, PosIndex{pos, 0, 1},
                            B, nullptr, od, logprobs, argmax, workspace, ws_bytes, s);
     };
@@ -858,10 +876,15 @@ int qk_rollout_teacher_forced(qk_model* mh, void* kv, int max_batch, int max_seq
         for (int j = 1; j < N; ++j) QK_TRY(one_step());
         return QK_OK;
     }
+    uint32_t inv_tau_bits = 0;
+    if (sampled) memcpy(&inv_tau_bits, &sampled->inv_tau, 4);
     const uint64_t key[12] = {(uint64_t)(uintptr_t)kv, (uint64_t)max_batch, (uint64_t)max_seq,
                               (uint64_t)(uintptr_t)seq, (uint64_t)B, (uint64_t)P, (uint64_t)N,
                               (uint64_t)(uintptr_t)logprobs, (uint64_t)(uintptr_t)argmax,
-                              (uint64_t)(uintptr_t)workspace, (uint64_t)ws_bytes, 0};
+                              (uint64_t)(uintptr_t)workspace, (uint64_t)ws_bytes,
+                              sampled ? (uint64_t)(uintptr_t)sampled->out_tokens ^ sampled->seed ^
+                                            ((uint64_t)inv_tau_bits << 32) ^ 1ull
+                                      : 0ull};
     cudaGraphExec_t exec = nullptr;
     int kernels = 0;
     for (auto& g : m.graphs)
@@ -875,7 +898,7 @@ int qk_rollout_teacher_forced(qk_model* mh, void* kv, int max_batch, int max_seq
         cudaStream_t cs_stream = m.capture_stream;
         QK_TRY_CUDA(cudaStreamBeginCapture(cs_stream, cudaStreamCaptureModeThreadLocal));
         const uint64_t before = g_launches.load();
-        launch_rollout_prepare(seq, L, P, B, step, pos, tok, tgt, off, cs_stream);
+        prepare(cs_stream);
         int rc = decode_impl(m, kv, max_batch, max_seq, TokIndex{tok, 1, 1, 0}, PosIndex{pos, 0, 1},
                              B, nullptr, od, logprobs, argmax, workspace, ws_bytes, cs_stream);
         kernels = (int)(g_launches.load() - before);
@@ -905,6 +928,26 @@ int qk_rollout_teacher_forced(qk_model* mh, void* kv, int max_batch, int max_seq
         note_launch(kernels);
     }
     return QK_OK;
+}
+
+int qk_rollout_teacher_forced(qk_model* mh, void* kv, int max_batch, int max_seq,
+                              const int32_t* seq, int B, int P, int N, float* logprobs,
+                              int32_t* argmax, void* workspace, size_t ws_bytes, void* stream) {
+    if (!mh || !seq || !logprobs) return set_error(QK_EINVAL, "null argument");
+    return rollout_impl(*(Model*)mh, mh, kv, max_batch, max_seq, seq, B, P, N, logprobs, argmax,
+                        nullptr, workspace, ws_bytes, (cudaStream_t)stream);
+}
+
+int qk_rollout_sampled(qk_model* mh, void* kv, int max_batch, int max_seq, const int32_t* prompt,
+                       int B, int P, int N, float tau, uint64_t seed, int32_t* tokens,
+                       float* logprobs, void* workspace, size_t ws_bytes, void* stream) {
+    if (!mh || !prompt || !tokens || !logprobs) return set_error(QK_EINVAL, "null argument");
+    if (!(tau > 0.f) || !(1.f / tau < 3.0e38f)) return set_error(QK_EINVAL, "temperature must be > 0");
+    if (B >= (1 << 24) || N + 1 >= (1 << 22) || ((Model*)mh)->cfg.vocab > (1 << 18))
+        return set_error(QK_ESHAPE, "sampling counters need B < 2^24, N < 2^22, vocab <= 2^18");
+    const SampleArgs sa{(unsigned long long)seed, 1.f / tau, tokens};
+    return rollout_impl(*(Model*)mh, mh, kv, max_batch, max_seq, prompt, B, P, N, logprobs, nullptr,
+                        &sa, workspace, ws_bytes, (cudaStream_t)stream);
 }
 
 int qk_check_status(qk_model* mh, void* stream, uint32_t* flags) {

@@ -73,6 +73,15 @@ struct LayerW {
     void* w_d;    // [H, I]
 };
 
+// Temperature sampling of rollout tokens by the Gumbel-max rule: a kernel that forms
+// a row's logits z draws c = argmax_v (z_v / tau + G(seed, row, step, v)) and reports
+// log softmax(z / tau)[c]; out_tokens == nullptr disables it.
+struct SampleArgs {
+    unsigned long long seed;
+    float inv_tau;
+    int32_t* out_tokens;  // written at the same index as the log-prob
+};
+
 struct Model {
     qk_config cfg;
     int es;  // bytes per element of the model dtype
@@ -106,6 +115,7 @@ struct Model {
     // First host-side failure of a launch inside an orchestration (0 = none);
     // reported and cleared by the entry point that made the launches.
     int deferred_error = 0;
+    SampleArgs sampling{};  // set only while a sampled rollout runs
 };
 
 // Records the opening event of a bracketed launch; returns whether it did.
@@ -205,7 +215,7 @@ __device__ __forceinline__ float grpo_token(float lp, float lp_old, float lp_ref
 
 void launch_logits_reduce(const float* logits, int M, int V, OutIndex oi, float* lp,
                           int32_t* argmax, uint32_t* status, cudaStream_t s,
-                          const GrpoArgs* grpo = nullptr);
+                          const GrpoArgs* grpo = nullptr, const SampleArgs* samp = nullptr);
 // GRPO reductions (k_grpo.cu).  With `compute`, loss_tok is formed from lp (else it
 // was formed by the scoring epilogue); then per-row sums of mask * loss and of the
 // mask go to `rows` ([B] float2) and loss_mean (if not null) = their ratio.
@@ -216,6 +226,10 @@ void launch_grpo_loss(const float* lp, int B, int T, const GrpoArgs& g, bool com
 // *out_off = s + 1; *step = s + 1.
 void launch_rollout_prepare(const int32_t* seq, int L, int P, int B, int32_t* step, int32_t* pos,
                             int32_t* tok, int32_t* tgt, int32_t* out_off, cudaStream_t s);
+// Sampled rollout cursor: s = *step; pos[b] = P + s; tok[b] = sampled[b * ld + s];
+// *out_off = s + 1; *step = s + 1.
+void launch_rollout_prepare_sampled(const int32_t* sampled, int ld, int P, int B, int32_t* step,
+                                    int32_t* pos, int32_t* tok, int32_t* out_off, cudaStream_t s);
 void launch_rope_table(float* cos_t, float* sin_t, int max_positions, int d, double theta,
                        cudaStream_t s);
 void launch_widen_gain(const void* src, int dtype, float* dst, int n, cudaStream_t s);

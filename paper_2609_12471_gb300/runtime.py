@@ -119,6 +119,17 @@ class Decoder:
                         eps_high, beta, logprobs, loss_tok, loss_mean, ws)
         return logprobs, loss_tok, loss_mean
 
+    def rollout_sampled(self, kv, max_batch, max_seq, prompt, N, tau=1.0, seed=0):
+        """Sampled rollout (Gumbel-max at temperature tau): returns (tokens [B, N+1],
+        logprobs [B, N+1]) for the draws c[0..N] after the prompt [B, P]."""
+        Bn, P = prompt.shape
+        tokens = torch.empty(Bn, N + 1, dtype=torch.int32, device=self.device)
+        logprobs = torch.empty(Bn, N + 1, dtype=torch.float32, device=self.device)
+        ws = self.workspace(B.QK_CALL_ROLLOUT, Bn, P, max_seq)
+        B.qk_rollout_sampled(self.handle, kv, max_batch, max_seq, prompt, Bn, P, N, tau, seed, tokens,
+                             logprobs, ws)
+        return tokens, logprobs
+
     def rollout(self, kv, max_batch, max_seq, seq, P, logprobs=None, argmax=None):
         Bn, L = seq.shape
         N = L - P - 1
