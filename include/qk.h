@@ -148,6 +148,21 @@ int qk_decode_step(qk_model* m, void* kv, int max_batch, int max_seq, const int3
 int qk_decode_layer(qk_model* m, int layer, void* kv, int max_batch, int max_seq, float* x,
                     const int32_t* pos, int B, void* workspace, size_t ws_bytes, void* stream);
 
+/* Append a turn to rows that sit at different positions (multi-turn rollouts,
+ * Sec. "Multi-Turn On-Policy Reflection": feedback appended to each rollout).
+ * Row b appends tokens[b, 0 .. len[b]-1] (dev int32 [B, T], row stride T) at
+ * positions start[b] .. start[b] + len[b] - 1 (start, len dev int32 [B];
+ * len NULL = T; 1 <= len[b] <= T and start[b] + T <= max_seq are required: a
+ * position outside the cache sets QK_STATUS_BAD_POS and is clamped).  The
+ * entries t >= len[b] of a row are padding: they are computed and written at
+ * positions start[b] + len[b] .. start[b] + T - 1, which the row's next tokens
+ * overwrite and which no earlier position attends.  last_logits dev fp32 [B, V]
+ * or NULL: the logits after each row's last appended token.  Workspace:
+ * qk_workspace_bytes(QK_CALL_PREFILL, B, T, max_seq). */
+int qk_prefill_rows(qk_model* m, void* kv, int max_batch, int max_seq, const int32_t* tokens,
+                    int B, int T, const int32_t* start, const int32_t* len, float* last_logits,
+                    void* workspace, size_t ws_bytes, void* stream);
+
 /* Teacher-forced scoring (Eq. sft / Eq. ppo inputs): tokens dev int32 [B, T],
  * T >= 2.  logprobs dev fp32 [B, T-1]: logprobs[b, t] = log p(tokens[b, t+1] |
  * tokens[b, <= t]).  argmax dev int32 [B, T-1] or NULL.  Positions start at 0;

@@ -34,7 +34,7 @@ __all__ = [
     "QK_PROF_GATE_UP", "QK_PROF_DOWN", "QK_PROF_ATTN", "QK_PROF_LM_HEAD", "QK_EPI_STORE",
     "QK_EPI_STORE_F32", "QK_EPI_RESID_F32", "QK_EPI_SWIGLU", "qk_op_linear_swiglu_static",
     "QK_STATIC_SCRATCH_BYTES", "qk_grpo_workspace_bytes", "qk_grpo_token_loss", "qk_score_grpo",
-    "qk_rollout_sampled",
+    "qk_rollout_sampled", "qk_prefill_rows",
 ]
 
 
@@ -87,6 +87,7 @@ _SIGS = {
     "qk_score_grpo": ([_P, _P, _I, _I, _P, _P, _P, _I, _P, _F, _F, _F, _P, _P, _P, _P, _SZ, _P], _I),
     "qk_rollout_sampled": ([_P, _P, _I, _I, _P, _I, _I, _I, _F, ctypes.c_uint64, _P, _P, _P, _SZ, _P],
                            _I),
+    "qk_prefill_rows": ([_P, _P, _I, _I, _P, _I, _I, _P, _P, _P, _P, _SZ, _P], _I),
 }
 
 _lib = None
@@ -251,6 +252,13 @@ def qk_rollout_sampled(m, kv, max_batch, max_seq, prompt, B, P, N, tau, seed, to
     _check(_load().qk_rollout_sampled(m, _ptr(kv), max_batch, max_seq, _ptr(prompt), B, P, N, tau,
                                       seed, _ptr(tokens), _ptr(logprobs), _ptr(workspace),
                                       _nbytes(workspace, ws_bytes), _stream(stream)))
+
+
+def qk_prefill_rows(m, kv, max_batch, max_seq, tokens, B, T, start, length=None, last_logits=None,
+                    workspace=None, ws_bytes=None, stream=None):
+    _check(_load().qk_prefill_rows(m, _ptr(kv), max_batch, max_seq, _ptr(tokens), B, T, _ptr(start),
+                                   _ptr(length), _ptr(last_logits), _ptr(workspace),
+                                   _nbytes(workspace, ws_bytes), _stream(stream)))
 
 
 def qk_check_status(m, stream=None) -> int:

@@ -1,6 +1,7 @@
 // Causal GQA attention for prefill and teacher-forced scoring (bf16, d = 128).
 //
-// Row r = b * T + t is the query at position p = start + t; it attends cache
+// Row r = b * T + t is the query at position p = start_b + t (start_b = start, or
+// start_dev[b] when the rows start at different positions); it attends cache
 // positions 0 .. p of its sequence (keys written by this call's QK-norm/RoPE
 // kernel for positions >= start, by earlier calls below start).  One CTA per
 // (64-query tile, b, query head), 4 warps of 16 queries.  The CTA walks the key
@@ -43,8 +44,9 @@ using ms::pack_bf16;
 
 __global__ void __launch_bounds__(128)
     attn_prefill_kernel(const __grid_constant__ CUtensorMap tmKV, const bf16* __restrict__ q,
-                        int q_ld, int nq, int nkv, int max_batch, int max_seq, int start, int T,
-                        bf16* __restrict__ o, uint32_t* __restrict__ status) {
+                        int q_ld, int nq, int nkv, int max_batch, int max_seq, int start_all,
+                        const int32_t* __restrict__ start_dev, int T, bf16* __restrict__ o,
+                        uint32_t* __restrict__ status) {
     extern __shared__ uint8_t smem_raw[];
     uint8_t* smem = (uint8_t*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
     uint64_t* full = (uint64_t*)(smem + kStages * kStage);
@@ -58,6 +60,9 @@ __global__ void __launch_bounds__(128)
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int g = lane >> 2, tig = lane & 3;
     const int q0 = qt * kQT;
+    // this row's first position (clamped into the cache; the cache-write kernel flags it)
+    int start = start_dev ? start_dev[b] : start_all;
+    start = start < 0 ? 0 : (start > max_seq - T ? max_seq - T : start);
     const int kv_len = start + T;  // cache positions 0 .. kv_len-1 are written
     const int p_last = start + min(q0 + kQT - 1, T - 1);
     const int n_kt = p_last / kKT + 1;
@@ -240,7 +245,8 @@ typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t,
 bool attn_prefill_supported(int d, int nq, int nkv) { return d == kD && nq % nkv == 0; }
 
 int launch_attn_prefill(const bf16* q, int q_ld, const void* k_layer, int nq, int nkv,
-                        int max_batch, int max_seq, int B, int T, int start, bf16* o,
+                        int max_batch, int max_seq, int B, int T, int start,
+                        const int32_t* start_dev, bf16* o,
                         uint32_t* status, cudaStream_t s) {
     static bool attr_set = false;
     if (!attr_set) {
@@ -269,7 +275,7 @@ int launch_attn_prefill(const bf16* q, int q_ld, const void* k_layer, int nq, in
         return QK_ECUDA;
     dim3 grid((T + kQT - 1) / kQT, B * nq);
     launch_k(attn_prefill_kernel, grid, dim3(128), kSmem, s, map, q, q_ld, nq, nkv, max_batch,
-             max_seq, start, T, o, status);
+             max_seq, start, start_dev, T, o, status);
     note_launch();
     return QK_OK;
 }

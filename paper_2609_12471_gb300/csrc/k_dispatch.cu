@@ -41,13 +41,13 @@ void launch_attention(Model& m, const void* q, int q_ld, const void* k_cache, co
         if (rc != QK_OK && !m.deferred_error) m.deferred_error = rc;
         return;
     }
-    if (c.dtype == QK_DTYPE_BF16 && pos.T > 1 && !pos.pos_dev &&
+    if (c.dtype == QK_DTYPE_BF16 && pos.T > 1 &&
         attn_prefill_supported(c.head_dim, c.n_q_heads, c.n_kv_heads) &&
         (const char*)v_cache == (const char*)k_cache + (size_t)max_batch * c.n_kv_heads * max_seq *
                                                             c.head_dim * 2) {
         int rc = launch_attn_prefill((const bf16*)q, q_ld, k_cache, c.n_q_heads, c.n_kv_heads,
-                                     max_batch, max_seq, M / pos.T, pos.T, pos.start, (bf16*)o,
-                                     m.status, s);
+                                     max_batch, max_seq, M / pos.T, pos.T, pos.start, pos.pos_dev,
+                                     (bf16*)o, m.status, s);
         if (rc != QK_OK && !m.deferred_error) m.deferred_error = rc;
         return;
     }

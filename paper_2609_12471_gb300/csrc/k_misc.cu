@@ -97,13 +97,18 @@ void launch_embed_gain(const void* E, int V, TokIndex tok, bool do_embed, float*
 // ---------------------------------------------------------------- RMSNorm
 template <typename OutT>
 __global__ void rmsnorm_kernel(const float* __restrict__ x, int in_step, int in_off,
-                               const float* __restrict__ g, int H, float eps,
-                               OutT* __restrict__ out) {
+                               const int32_t* __restrict__ row_len, const float* __restrict__ g,
+                               int H, float eps, OutT* __restrict__ out) {
     __shared__ float red[32];
     pdl_wait();
     pdl_trigger();  // short kernel: let the next one launch and prefetch now
     int r = blockIdx.x;
-    const float* xr = x + ((size_t)r * in_step + in_off) * H;
+    int off = in_off;
+    if (row_len) {  // row r's last valid token: row_len[r] - 1, clamped into the row
+        off = row_len[r] - 1;
+        off = off < 0 ? 0 : (off >= in_step ? in_step - 1 : off);
+    }
+    const float* xr = x + ((size_t)r * in_step + off) * H;
     float ss = 0.f;
     for (int i = threadIdx.x * 4; i < H; i += blockDim.x * 4) {
         float4 v = *reinterpret_cast<const float4*>(xr + i);
@@ -123,16 +128,16 @@ __global__ void rmsnorm_kernel(const float* __restrict__ x, int in_step, int in_
 }
 
 void launch_rmsnorm(const float* x, int in_step, int in_off, const float* g, int H, float eps,
-                    void* out, int out_dtype, int M, cudaStream_t s) {
+                    void* out, int out_dtype, int M, cudaStream_t s, const int32_t* row_len) {
     note_launch();
     if (M <= 0) return;
     int threads = H >= 1024 ? 256 : 64;
     if (out_dtype == QK_DTYPE_BF16)
-        launch_k(rmsnorm_kernel<bf16>, dim3(M), dim3(threads), 0, s, x, in_step, in_off, g, H, eps,
-                 (bf16*)out);
+        launch_k(rmsnorm_kernel<bf16>, dim3(M), dim3(threads), 0, s, x, in_step, in_off, row_len, g,
+                 H, eps, (bf16*)out);
     else
-        launch_k(rmsnorm_kernel<float>, dim3(M), dim3(threads), 0, s, x, in_step, in_off, g, H, eps,
-                 (float*)out);
+        launch_k(rmsnorm_kernel<float>, dim3(M), dim3(threads), 0, s, x, in_step, in_off, row_len, g,
+                 H, eps, (float*)out);
 }
 
 // ---------------------------------------------------------------- QK-norm + RoPE + cache write

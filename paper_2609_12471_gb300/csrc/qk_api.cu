@@ -311,11 +311,11 @@ static void run_layer_fused(Model& m, int l, const Workspace& w, int M, PosIndex
 // lm_head into `logits`, then log-prob / argmax per row.
 static void run_head(Model& m, const Workspace& w, int M_out, int in_step, int in_off,
                      float* logits, OutIndex oi, float* lp, int32_t* am, cudaStream_t s,
-                     bool normed = false) {
+                     bool normed = false, const int32_t* row_len = nullptr) {
     const qk_config& c = m.cfg;
     if (!normed)
         launch_rmsnorm(w.x, in_step, in_off, m.final_norm, c.hidden, (float)c.rms_eps, w.u,
-                       c.dtype, M_out, s);
+                       c.dtype, M_out, s, row_len);
     bool pr = prof_open(m, QK_PROF_LM_HEAD, s);
     linear(m, w.u, c.hidden, m.lm_head, logits, c.vocab, M_out, c.vocab, c.hidden, EPI_STORE_F32,
            w.gu, s);
@@ -602,18 +602,22 @@ int qk_workspace_bytes(const qk_model* mh, int kind, int B, int T, int max_seq, 
     return QK_OK;
 }
 
+// start_dev (dev [B] or null): per-row first positions instead of start_pos; row_len
+// (dev [B] or null): the head reads row b's token row_len[b] - 1 instead of T - 1.
 static int prefill_impl(Model& m, void* kv, int max_batch, int max_seq, TokIndex tok, int B, int T,
                         int start_pos, float* last_logits, OutIndex oi, float* lp, int32_t* am,
-                        void* ws, size_t ws_bytes, cudaStream_t s) {
+                        void* ws, size_t ws_bytes, cudaStream_t s,
+                        const int32_t* start_dev = nullptr, const int32_t* row_len = nullptr) {
     Workspace w;
     QK_TRY(get_ws(m, QK_CALL_PREFILL, B, T, max_seq, ws, ws_bytes, &w));
     int M = B * T;
     KVView view = cache_view(m, kv, max_batch, max_seq);
     launch_embed(m.embed, m.cfg.dtype, m.cfg.vocab, m.cfg.hidden, tok, M, w.x, m.status, s);
-    PosIndex pos{nullptr, start_pos, T};
+    PosIndex pos{start_dev, start_pos, T};
     for (int l = 0; l < m.cfg.n_layers; ++l) run_layer(m, l, w, M, pos, view, s);
     if (last_logits || lp || am)
-        run_head(m, w, B, T, T - 1, last_logits ? last_logits : w.logits, oi, lp, am, s);
+        run_head(m, w, B, T, T - 1, last_logits ? last_logits : w.logits, oi, lp, am, s, false,
+                 row_len);
     return check_launch(m, "prefill");
 }
 
@@ -630,6 +634,18 @@ int qk_prefill(qk_model* mh, void* kv, int max_batch, int max_seq, const int32_t
     OutIndex oi{1, 1, 1, 0, targets, 1, 0, 0};
     return prefill_impl(m, kv, max_batch, max_seq, TokIndex{tokens, T, T, 0}, B, T, start_pos,
                         last_logits, oi, logprobs, argmax, workspace, ws_bytes, (cudaStream_t)stream);
+}
+
+int qk_prefill_rows(qk_model* mh, void* kv, int max_batch, int max_seq, const int32_t* tokens, int B,
+                    int T, const int32_t* start, const int32_t* len, float* last_logits,
+                    void* workspace, size_t ws_bytes, void* stream) {
+    if (!mh || !tokens || !start) return set_error(QK_EINVAL, "null argument");
+    Model& m = *(Model*)mh;
+    QK_TRY(check_cache(m, kv, max_batch, max_seq, B));
+    if (T < 1 || T > max_seq) return set_error(QK_ESHAPE, "T %d outside 1 .. max_seq %d", T, max_seq);
+    OutIndex oi{1, 1, 1, 0, nullptr, 1, 0, 0};
+    return prefill_impl(m, kv, max_batch, max_seq, TokIndex{tokens, T, T, 0}, B, T, 0, last_logits,
+                        oi, nullptr, nullptr, workspace, ws_bytes, (cudaStream_t)stream, start, len);
 }
 
 static int decode_impl(Model& m, void* kv, int max_batch, int max_seq, TokIndex tok, PosIndex pos,

@@ -171,8 +171,10 @@ struct OutIndex {
 void launch_embed(const void* E, int dtype, int V, int H, TokIndex tok, int M, float* x,
                   uint32_t* status, cudaStream_t s);
 // out[r] = x[r * in_step + in_off] * rsqrt(mean(x^2) + eps) * g, stored in out_dtype.
+// With row_len, row r reads x[r * in_step + row_len[r] - 1] instead (per-row last token).
 void launch_rmsnorm(const float* x, int in_step, int in_off, const float* g, int H, float eps,
-                    void* out, int out_dtype, int M, cudaStream_t s);
+                    void* out, int out_dtype, int M, cudaStream_t s,
+                    const int32_t* row_len = nullptr);
 // Per-head RMSNorm of q and k, RoPE of q and k, q written in place, k and v to the cache.
 void launch_qk_norm_rope(void* qkv, int dtype, int M, int nq, int nkv, int d, const float* gq,
                          const float* gk, float eps, const float* rope_cos, const float* rope_sin,
@@ -322,11 +324,12 @@ void launch_attention(Model& m, const void* q, int q_ld, const void* k_cache, co
                       int M, int max_batch, int max_seq, PosIndex pos, void* o, void* scratch,
                       cudaStream_t s);
 // Causal tensor-core attention for prefill / scoring (k_attn_prefill.cu): M = B x T
-// query rows at positions start .. start+T-1; head_dim 128.
+// query rows at positions start_b .. start_b+T-1, start_b = start_dev[b] when given,
+// else start; head_dim 128.
 bool attn_prefill_supported(int d, int nq, int nkv);
 int launch_attn_prefill(const bf16* q, int q_ld, const void* k_layer, int nq, int nkv,
-                        int max_batch, int max_seq, int B, int T, int start, bf16* o,
-                        uint32_t* status, cudaStream_t s);
+                        int max_batch, int max_seq, int B, int T, int start,
+                        const int32_t* start_dev, bf16* o, uint32_t* status, cudaStream_t s);
 // Split tensor-core decode attention (k_attn_decode.cu); head_dim 128, G <= 8.
 void attn_decode_split(int B, int nkv, int max_seq, int num_sms, int* chunk, int* n_split);
 size_t attn_decode_scratch_bytes(int B, int nq, int nkv, int max_seq, int num_sms);

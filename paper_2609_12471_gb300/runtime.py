@@ -119,6 +119,15 @@ class Decoder:
                         eps_high, beta, logprobs, loss_tok, loss_mean, ws)
         return logprobs, loss_tok, loss_mean
 
+    def prefill_rows(self, kv, max_batch, max_seq, tokens, start, length=None, last_logits=None):
+        """Append tokens[b, :length[b]] to row b at positions start[b] .. (rows at different
+        positions; entries past length[b] are padding)."""
+        Bn, T = tokens.shape
+        ws = self.workspace(B.QK_CALL_PREFILL, Bn, T, max_seq)
+        B.qk_prefill_rows(self.handle, kv, max_batch, max_seq, tokens, Bn, T, start, length,
+                          last_logits, ws)
+        return last_logits
+
     def rollout_sampled(self, kv, max_batch, max_seq, prompt, N, tau=1.0, seed=0):
         """Sampled rollout (Gumbel-max at temperature tau): returns (tokens [B, N+1],
         logprobs [B, N+1]) for the draws c[0..N] after the prompt [B, P]."""
