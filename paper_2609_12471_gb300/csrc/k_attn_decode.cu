@@ -1,10 +1,11 @@
 // GQA decode attention over the bf16 KV cache, split over the key sequence.
 //
 // One decode token per row b; query head h = kvh * G + g (G = n_q / n_kv <= 8)
-// attends cache positions 0 .. p(b).  The key range of each (b, kvh) is cut
-// into chunks; one CTA per (chunk, b, kvh) streams its chunk through a 3-stage
-// ring of 64-key K and V tiles loaded by TMA (128-byte swizzle, two 64-dim boxes
-// per tile, one mbarrier per stage).  Each of the 4 warps takes 16 keys of a
+// attends cache positions 0 .. p(b).  The key tiles 0 .. p/64 of each (b, kvh)
+// are cut evenly into n_split chunks at that row's position (n_split from a cost
+// model at the cache length); one CTA per (chunk, b, kvh) streams its chunk
+// through a 3-stage ring of 64-key K and V tiles loaded by TMA (128-byte swizzle,
+// two 64-dim boxes per tile, one mbarrier per stage).  Each of the 4 warps takes 16 keys of a
 // tile and runs, on the tensor cores (mma.sync m16n8k16, bf16 in, fp32 out):
 //   S[16 x 16] = Q_pad[16 x 128] * K^T   (rows 0..G-1 are the group's heads)
 //   online softmax in base 2 over its keys (running max m, running sum l)
@@ -76,9 +77,15 @@ __global__ void __launch_bounds__(128)
 
     int p = pos.pos_dev ? pos.pos_dev[b] : pos.start;
     if (p < 0 || p >= max_seq) p = p < 0 ? 0 : max_seq - 1;  // flagged by the cache-write kernel
-    const int k_begin = split * chunk;
-    if (k_begin > p) return;  // nothing to attend in this chunk; the combine kernel skips it
-    const int k_end = min(k_begin + chunk, p + 1);
+    // The row's key tiles 0 .. p/64 are cut into n_split equal runs at this row's own
+    // position (the grid is sized from the longest cache, the work from p); `chunk`
+    // caps a run at the cost model's length.
+    const int n_tiles_b = p / kTileKeys + 1;
+    const int per = min((n_tiles_b + n_split - 1) / n_split, chunk / kTileKeys);
+    const int n_valid = (n_tiles_b + per - 1) / per;  // splits that hold keys
+    const int k_begin = split * per * kTileKeys;
+    if (split >= n_valid) return;  // nothing to attend in this split; the merge skips it
+    const int k_end = min(k_begin + per * kTileKeys, p + 1);
     const int n_tiles = (k_end - k_begin + kTileKeys - 1) / kTileKeys;
     // Row of key 0 of (b, kvh) in the 2-D view of this layer's K (V follows after max_batch*nkv*max_seq rows).
     const int row0 = (b * nkv + kvh) * max_seq;
@@ -245,14 +252,14 @@ __global__ void __launch_bounds__(128)
             L += f * red_ml[(w * 8 + gg) * 2 + 1];
         }
         const size_t head = (size_t)b * nq + kvh * G + gg;
-        if (n_split == 1) {  // a single chunk is already the whole attention
+        if (n_valid == 1) {  // a single chunk is already the whole attention
             out[head * kD + d] = __float2bfloat16_rn(acc / L);
         } else {
             part_o[(head * n_split + split) * kD + d] = acc;
             if (d == 0) part_ml[head * n_split + split] = make_float2(M, L);
         }
     }
-    if (n_split == 1) return;
+    if (n_valid == 1) return;
     // The last CTA of this (row, kv head) to finish merges the chunks' partials:
     //   o = sum_s 2^(m_s - M) O_s / sum_s 2^(m_s - M) l_s,  M = max_s m_s,
     // then resets the ticket for the next layer.  The barrier orders every thread's
@@ -260,7 +267,6 @@ __global__ void __launch_bounds__(128)
     // after the other chunks' stores.
     __shared__ int last;
     __syncthreads();
-    const int n_valid = min(n_split, p / chunk + 1);
     if (threadIdx.x == 0)
         last = tc::atom_add_acq_rel_gpu(&tickets[b * nkv + kvh], 1) == n_valid - 1;
     __syncthreads();
