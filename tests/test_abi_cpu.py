@@ -80,3 +80,38 @@ def test_unknown_preset_and_null_arguments(lib):
     assert lib.qk_model_packed_bytes(None, None) == qk.QK_EINVAL
     lib.qk_workspace_bytes.argtypes = [ctypes.c_void_p] + [ctypes.c_int] * 4 + [ctypes.c_void_p]
     assert lib.qk_workspace_bytes(None, 0, 1, 1, 1, None) == qk.QK_EINVAL
+
+
+def test_grpo_and_turn_entry_points_validate_on_the_host(lib):
+    """Argument errors of the GRPO, sampling and multi-turn entry points come back
+    before any device work (fake non-null pointers are never dereferenced)."""
+    import paper_2609_12471_gb300 as qk
+    assert qk.qk_grpo_workspace_bytes(1) == 256
+    assert qk.qk_grpo_workspace_bytes(1000) == 8192
+    with pytest.raises(qk.QKError) as e:
+        qk.qk_grpo_workspace_bytes(0)
+    assert e.value.code == qk.QK_ESHAPE
+    P = 16  # a fake, aligned, never-dereferenced device address
+    args = dict(lp=P, lp_old=P, lp_ref=P, B=6, T=4, ld=4, rewards=P, group=3, mask=None,
+                eps_low=0.2, eps_high=0.28, beta=0.01, loss_tok=P)
+
+    def call(**over):
+        a = dict(args, **over)
+        with pytest.raises(qk.QKError) as e:
+            qk.qk_grpo_token_loss(a["lp"], a["lp_old"], a["lp_ref"], a["B"], a["T"], a["ld"],
+                                  a["rewards"], a["group"], a["mask"], a["eps_low"], a["eps_high"],
+                                  a["beta"], a["loss_tok"], None, None, 0, stream=0)
+        return e.value.code
+
+    assert call(lp=None) == qk.QK_EINVAL
+    assert call(lp_ref=None) == qk.QK_EINVAL          # beta != 0 needs a reference policy
+    assert call(group=4) == qk.QK_ESHAPE              # 6 rows are not whole groups of 4
+    assert call(ld=3) == qk.QK_ESHAPE                 # row stride below T
+    assert call(eps_low=1.5) == qk.QK_EINVAL
+    assert call() == qk.QK_ENOSPACE                   # valid arguments, no workspace
+    with pytest.raises(qk.QKError) as e:
+        qk.qk_rollout_sampled(None, P, 1, 8, P, 1, 4, 2, 1.0, 0, P, P, ws_bytes=0, stream=0)
+    assert e.value.code == qk.QK_EINVAL
+    with pytest.raises(qk.QKError) as e:
+        qk.qk_prefill_rows(None, P, 1, 8, P, 1, 4, P, ws_bytes=0, stream=0)
+    assert e.value.code == qk.QK_EINVAL
