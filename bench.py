@@ -318,7 +318,7 @@ def run_ours(args, world, rank, local):
     gu_bytes = 2 * c.intermediate * c.hidden * 2 + B * c.hidden * 2 + B * c.intermediate * 2
     avg_launch_s = (prof_ms / max(prof_n, 1)) / 1e3
     achieved = gu_bytes / avg_launch_s / 1e9
-    roofline = {"bound": "hbm", "kernel": "decode gate/up linear (tcgen05 split-K GEMM, 16 token rows)",
+    roofline = {"bound": "hbm", "kernel": "decode gate/up linear (tcgen05 stream-K GEMM, 16 token rows)",
                 "timed_launches": "the gate/up launches of each timed rollout's first decode step "
                                   "(later steps replay a captured CUDA graph without event nodes)",
                 "achieved": achieved, "peak": hbm_peak, "unit": "GB/s",
