@@ -587,9 +587,23 @@ __global__ void __launch_bounds__(kThreads, FUSED && BN == 16 ? kFusedCtasPerSm 
             tc::fence_after_sync();
             const int f = feat * 128 + q * 32 + lane;
             const uint32_t tbase = tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(acc * G::ACC_COLS);
+            // Residual add: the residual values of each 16-token chunk are loaded one
+            // chunk ahead, before the current chunk's stores, so the loads of a tile are
+            // pipelined instead of one read-modify-write round trip per token.
+            const bool resid = !SWIGLU && epi == EPI_RESID_F32;
+            float xo[16], xn[16];
+            auto load_x = [&](int tok0, float (&dst)[16]) {
+#pragma unroll
+                for (int j = 0; j < 16; ++j) {
+                    const int m = tok0 + j;
+                    dst[j] = m < M ? ((const float*)C)[(size_t)m * ldc + f] : 0.f;
+                }
+            };
+            if (resid) load_x(tok * BN, xo);
             for (int c0 = 0; c0 < BN; c0 += 16) {
                 const int tok0 = tok * BN + c0;
                 if (tok0 >= M) break;
+                if (resid && c0 + 16 < BN && tok0 + 16 < M) load_x(tok0 + 16, xn);
                 uint32_t r[16];
                 tc::tmem_ld16(tbase + c0, r);
                 uint32_t u[16];
@@ -610,8 +624,12 @@ __global__ void __launch_bounds__(kThreads, FUSED && BN == 16 ? kFusedCtasPerSm 
                     } else if (epi == EPI_STORE_F32) {
                         ((float*)C)[o] = v;
                     } else {
-                        ((float*)C)[o] += v;
+                        ((float*)C)[o] = xo[j] + v;
                     }
+                }
+                if (resid) {
+#pragma unroll
+                    for (int j = 0; j < 16; ++j) xo[j] = xn[j];
                 }
             }
             tc::fence_before_sync();
