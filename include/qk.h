@@ -60,7 +60,8 @@ extern "C" {
 #define QK_DTYPE_F32 1
 
 /* Bits of the device status word (qk_check_status). */
-#define QK_STATUS_BAD_TOKEN 1u    /* token id outside [0, vocab); id 0 was used   */
+#define QK_STATUS_BAD_TOKEN 1u    /* token id outside [0, vocab) (an input id, or no
+                                     drawable token: non-finite logits); 0 was used */
 #define QK_STATUS_BAD_POS 2u      /* position outside [0, max_seq); it was clamped */
 #define QK_STATUS_TIMEOUT 4u      /* a bounded device wait gave up                 */
 
