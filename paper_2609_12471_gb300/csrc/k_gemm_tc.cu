@@ -9,7 +9,8 @@
 // 32 consecutive features of one token row (coalesced), and the residual add,
 // SwiGLU and fp32 logits store happen on the accumulator without another pass.
 //
-// Per CTA (persistent, one per SM, 192 threads):
+// Per CTA (persistent, one per SM, 192 threads; the 16-row decode configuration
+// is small enough for a CTA of the next kernel to become resident beside it):
 //   warp 0, one lane : TMA producer over a STAGES-deep ring of (W, X) k-blocks;
 //   warp 1           : TMEM allocation; one lane issues tcgen05.mma + commits;
 //   warps 2..5       : epilogue, warp w reads TMEM lanes 32*(w%4) .. +31.
