@@ -1,6 +1,8 @@
 // Elementwise and row-wise kernels of the decoder forward pass: embedding
-// gather, RMSNorm, per-head QK-RMSNorm + RoPE + KV-cache write, SwiGLU,
-// vocabulary log-softmax / gather / argmax, and the load-time RoPE table.
+// gather, RMSNorm, per-head QK-RMSNorm + RoPE + KV-cache write, SwiGLU, the
+// vocabulary reduce (log-softmax / gather / arg-max, the Gumbel-max draw of a
+// sampled rollout and the GRPO token loss where a log-prob is formed), the
+// rollout cursors, and the load-time RoPE table.
 #include <math.h>
 
 #include "qk_internal.cuh"
