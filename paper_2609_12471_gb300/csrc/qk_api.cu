@@ -894,13 +894,13 @@ static int rollout_impl(Model& m, qk_model* mh, void* kv, int max_batch, int max
     }
     uint32_t inv_tau_bits = 0;
     if (sampled) memcpy(&inv_tau_bits, &sampled->inv_tau, 4);
-    const uint64_t key[12] = {(uint64_t)(uintptr_t)kv, (uint64_t)max_batch, (uint64_t)max_seq,
+    const uint64_t key[15] = {(uint64_t)(uintptr_t)kv, (uint64_t)max_batch, (uint64_t)max_seq,
                               (uint64_t)(uintptr_t)seq, (uint64_t)B, (uint64_t)P, (uint64_t)N,
                               (uint64_t)(uintptr_t)logprobs, (uint64_t)(uintptr_t)argmax,
                               (uint64_t)(uintptr_t)workspace, (uint64_t)ws_bytes,
-                              sampled ? (uint64_t)(uintptr_t)sampled->out_tokens ^ sampled->seed ^
-                                            ((uint64_t)inv_tau_bits << 32) ^ 1ull
-                                      : 0ull};
+                              sampled ? 1ull : 0ull,
+                              sampled ? (uint64_t)(uintptr_t)sampled->out_tokens : 0ull,
+                              sampled ? (uint64_t)sampled->seed : 0ull, (uint64_t)inv_tau_bits};
     cudaGraphExec_t exec = nullptr;
     int kernels = 0;
     for (auto& g : m.graphs)
