@@ -52,7 +52,7 @@ extern "C" {
 #define QK_ESHAPE (-2)   /* size out of range: B > max_batch, T too long, ... */
 #define QK_EDTYPE (-3)   /* unsupported dtype / head_dim / grouping           */
 #define QK_ECUDA (-4)    /* a CUDA runtime / driver call failed               */
-#define QK_ETIMEOUT (-5) /* a device-side bounded wait expired                */
+#define QK_ETIMEOUT (-5) /* a device-side bounded wait expired (qk_check_status) */
 #define QK_EDEVICE (-6)  /* device status word had a fault bit set            */
 #define QK_ENOSPACE (-7) /* caller buffer smaller than the size query returns */
 
@@ -91,20 +91,31 @@ typedef struct qk_model qk_model;
 /* Fill *out with a named preset: "tiny_fp32" (2 layers, H 256, 4/2 heads, d 64,
  * I 768, V 4096, fp32), "q8b" (36 layers, H 4096, 32/8 heads, d 128, I 12288,
  * V 151936, bf16), "q8b_layer" (one q8b layer).  eps 1e-6, theta 1e6,
- * max_positions 8192.  Returns QK_EINVAL for an unknown name. */
+ * max_positions 8192.  Returns QK_EINVAL for an unknown name.
+ * Source: the policy is Qwen3-8B(-Instruct) (Sec. "Training Configuration" and
+ * the hyperparameter table of Sec. "Hyperparameters": sequence lengths 8K / 16K);
+ * the paper does not restate the architecture, so its dimensions, eps and theta
+ * here are the public Qwen3-8B values, and max_positions 8192 covers the 8K
+ * sequences of the HIP runs. */
 int qk_config_preset(const char* name, qk_config* out);
 
 /* Number of weight tensors of a config, in the canonical order used by
  * qk_model_load: embed [V,H]; then per layer attn_norm [H], wq [nq*d,H],
  * wk [nkv*d,H], wv [nkv*d,H], q_norm [d], k_norm [d], wo [H,nq*d],
  * mlp_norm [H], wg [I,H], wu [I,H], wd [H,I]; then final_norm [H],
- * lm_head [V,H].  Matrices are row-major [out, in]. */
+ * lm_head [V,H].  Matrices are row-major [out, in].  (The tensors of the Qwen3
+ * layer definition in the file header; the paper cites the architecture only.) */
 int qk_weight_count(const qk_config* cfg, int* n_tensors);
 
-/* Bytes of the packed device buffer qk_model_load needs for this config. */
+/* Bytes of the packed device buffer qk_model_load needs for this config (a
+ * service call: the library never allocates, so it reports sizes). */
 int qk_model_packed_bytes(const qk_config* cfg, size_t* bytes);
 
-/* Build a model.  `tensors` is a host array of n_tensors device pointers in the
+/* Build a model: the Qwen3-8B policy whose forward pass the paper trains with
+ * SFT and GRPO (Sec. "Agentic Integration": one Qwen3-8B policy serves every
+ * agent role), here with caller-supplied (random-init) weights; the paper
+ * publishes no trained checkpoint.
+ * `tensors` is a host array of n_tensors device pointers in the
  * canonical order above, each holding the tensor in the config's dtype.  They
  * are read (repacked into `packed`, which must hold qk_model_packed_bytes bytes
  * and be 256-byte aligned) on `stream` and may be freed once the stream has
@@ -115,15 +126,25 @@ int qk_model_load(const qk_config* cfg, const void* const* tensors, int n_tensor
 void qk_model_free(qk_model* m);
 
 /* KV cache bytes for max_batch rows of max_seq positions: per layer K then V,
- * each [max_batch, n_kv, max_seq, d] in the model dtype, contiguous. */
+ * each [max_batch, n_kv, max_seq, d] in the model dtype, contiguous.  The cache
+ * holds the keys and values of every earlier position of a rollout, so that a
+ * decode step of the autoregressive rollout loop (Sec. "Implementation
+ * Components": the policy generates candidates for up to T = 3 turns) attends to
+ * them without recomputing the prefix.  Sized for the paper's RL batches (64
+ * prompts x G = 8 rollouts, sequences up to 8K / 16K tokens, hyperparameter
+ * table). */
 int qk_kv_bytes(const qk_model* m, int max_batch, int max_seq, size_t* bytes);
 
 /* Workspace bytes for one call of the given kind (QK_CALL_*) with batch B and
  * T tokens per row (T = 1 for decode; T = prompt length for a rollout) against
- * a cache of max_seq positions. */
+ * a cache of max_seq positions.  (A service call; the paper has no counterpart.) */
 int qk_workspace_bytes(const qk_model* m, int kind, int B, int T, int max_seq, size_t* bytes);
 
-/* Prefill T tokens per row at positions start_pos .. start_pos+T-1 (causal
+/* Prefill: the prompt pass of a rollout (Sec. "Execution-Aware Reinforcement
+ * Learning": each candidate is generated from the task prompt; Sec.
+ * "Implementation Components": the rollout loop samples prompts and the policy
+ * generates from them).
+ * Prefill T tokens per row at positions start_pos .. start_pos+T-1 (causal
  * attention over cache positions 0 .. p), writing their K and V into the cache.
  * tokens: dev int32 [B, T].  The cache rows b < B must already hold positions
  * < start_pos.  Outputs for the last position of each row (any may be NULL):
@@ -135,7 +156,12 @@ int qk_prefill(qk_model* m, void* kv, int max_batch, int max_seq, const int32_t*
                int T, int start_pos, float* last_logits, const int32_t* targets, float* logprobs,
                int32_t* argmax, void* workspace, size_t ws_bytes, void* stream);
 
-/* One decode step: row b consumes tokens[b] at position pos[b] (dev int32 [B]
+/* One decode step of the autoregressive rollout (Sec. "Execution-Aware
+ * Reinforcement Learning" and the rollout loop of Sec. "Implementation
+ * Components": the policy generates each candidate token by token; its
+ * log-probability log pi_theta(y_t | x, y_<t) is the quantity of Eq. sft and
+ * of the ratio in Eq. ppo).
+ * Row b consumes tokens[b] at position pos[b] (dev int32 [B]
  * each), writes its K and V at pos[b] and attends positions 0 .. pos[b].
  * Outputs as in qk_prefill, for the B new positions. */
 int qk_decode_step(qk_model* m, void* kv, int max_batch, int max_seq, const int32_t* tokens,
@@ -143,7 +169,8 @@ int qk_decode_step(qk_model* m, void* kv, int max_batch, int max_seq, const int3
                    float* logprobs, int32_t* argmax, void* workspace, size_t ws_bytes,
                    void* stream);
 
-/* One decoder layer of a decode step on a given residual stream: x dev fp32
+/* One decoder layer of a decode step (the unit of the rollout decode above, on
+ * its own for per-layer parity and timing) on a given residual stream: x dev fp32
  * [B, H] is updated in place; the new K and V go to the layer's cache at
  * pos[b] (dev int32 [B]) and attention covers 0 .. pos[b]. */
 int qk_decode_layer(qk_model* m, int layer, void* kv, int max_batch, int max_seq, float* x,
@@ -225,7 +252,10 @@ int qk_rollout_sampled(qk_model* m, void* kv, int max_batch, int max_seq, const 
                        float* logprobs, void* workspace, size_t ws_bytes, void* stream);
 
 /* Synchronise `stream`, read the device status word into *flags (QK_STATUS_*
- * bits) and clear it.  Returns QK_EDEVICE if any bit was set, QK_OK otherwise. */
+ * bits) and clear it.  Returns QK_ETIMEOUT if QK_STATUS_TIMEOUT was set (a
+ * bounded device wait gave up; other bits may be set too and are in *flags),
+ * else QK_EDEVICE if any other bit was set, QK_OK otherwise.  (A service call of
+ * the library; the paper has no counterpart.) */
 int qk_check_status(qk_model* m, void* stream, uint32_t* flags);
 
 /* ---- measurement ----------------------------------------------------------
@@ -247,10 +277,11 @@ int qk_profile_begin(qk_model* m, int kind, int max_launches);
  * event-to-event time (ms) and the number of bracketed launches. */
 int qk_profile_end(qk_model* m, float* total_ms, int* launches);
 
-/* Number of kernels libqk has launched in this process (all models). */
+/* Number of kernels libqk has launched in this process (all models; a service
+ * call for measurement, no counterpart in the paper). */
 uint64_t qk_launch_count(void);
 
-/* Message of the last failed call on this thread ("" if none). */
+/* Message of the last failed call on this thread ("" if none; service call). */
 const char* qk_last_error(void);
 
 #ifdef __cplusplus

@@ -34,7 +34,7 @@ __all__ = [
     "QK_PROF_GATE_UP", "QK_PROF_DOWN", "QK_PROF_ATTN", "QK_PROF_LM_HEAD", "QK_EPI_STORE",
     "QK_EPI_STORE_F32", "QK_EPI_RESID_F32", "QK_EPI_SWIGLU", "qk_op_linear_swiglu_static",
     "QK_STATIC_SCRATCH_BYTES", "qk_grpo_workspace_bytes", "qk_grpo_token_loss", "qk_score_grpo",
-    "qk_rollout_sampled", "qk_prefill_rows",
+    "qk_rollout_sampled", "qk_prefill_rows", "qk_debug_expire_next_wait",
 ]
 
 
@@ -88,6 +88,7 @@ _SIGS = {
     "qk_rollout_sampled": ([_P, _P, _I, _I, _P, _I, _I, _I, _F, ctypes.c_uint64, _P, _P, _P, _SZ, _P],
                            _I),
     "qk_prefill_rows": ([_P, _P, _I, _I, _P, _I, _I, _P, _P, _P, _P, _SZ, _P], _I),
+    "qk_debug_expire_next_wait": ([_P, ctypes.c_longlong], _I),
 }
 
 _lib = None
@@ -262,10 +263,11 @@ def qk_prefill_rows(m, kv, max_batch, max_seq, tokens, B, T, start, length=None,
 
 
 def qk_check_status(m, stream=None) -> int:
-    """Returns the status bits (0 when clean); does not raise on QK_EDEVICE."""
+    """Returns the status bits (0 when clean); does not raise on QK_EDEVICE or
+    QK_ETIMEOUT (the bits say which)."""
     v = ctypes.c_uint32()
     rc = _load().qk_check_status(m, _stream(stream), ctypes.byref(v))
-    if rc not in (QK_OK, QK_EDEVICE):
+    if rc not in (QK_OK, QK_EDEVICE, QK_ETIMEOUT):
         _check(rc)
     return v.value
 
@@ -297,3 +299,9 @@ def qk_op_linear_swiglu_static(m, A, lda, W, C, ldc, M, N, K, stream=None):
     """SwiGLU linear step with its gate/up intermediate in the library's static device array."""
     _check(_load().qk_op_linear_swiglu_static(m, _ptr(A), lda, _ptr(W), _ptr(C), ldc, M, N, K,
                                               _stream(stream)))
+
+
+def qk_debug_expire_next_wait(m, wait_cycles: int):
+    """Arm the bounded-wait test: the model's next plain tensor-core linear launch
+    lets one wait expire after wait_cycles SM cycles (QK_STATUS_TIMEOUT)."""
+    _check(_load().qk_debug_expire_next_wait(m, wait_cycles))

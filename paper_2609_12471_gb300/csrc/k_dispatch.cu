@@ -14,8 +14,10 @@ void linear(Model& m, const void* A, int lda, const void* W, void* C, int ldc, i
         return;
     }
     if (dt == QK_DTYPE_BF16 && gemm_tc_supported(A, lda, N, K)) {
+        const long long test_wait = m.test_wait_cycles;  // one launch only
+        m.test_wait_cycles = 0;
         int rc = launch_gemm_tc((const bf16*)A, lda, (const bf16*)W, C, ldc, M, N, K, epi,
-                                m.num_sms, m.status, s);
+                                m.num_sms, m.status, s, test_wait);
         if (rc != QK_OK && !m.deferred_error) m.deferred_error = rc;
         return;
     }

@@ -22,6 +22,9 @@
 // abort flag and QK_STATUS_TIMEOUT in the model status word; every role leaves
 // its loop, the producer waits (bounded) for the copies it issued, the MMA
 // thread waits (bounded) for its MMAs, then TMEM is freed and the CTA exits.
+// A launch with test_wait > 0 (the qk_debug_expire_next_wait hook of the plain
+// GEMM) exercises that path: CTA 0 issues no copy for its first k-block and
+// waits at most test_wait cycles, so its MMA thread's wait for that copy expires.
 #include <cuda.h>
 #include <mutex>
 
@@ -148,7 +151,8 @@ template <int BN, bool SWIGLU, int STAGES, bool FUSED>
 __global__ void __launch_bounds__(kThreads, FUSED && BN == 16 ? kFusedCtasPerSm : 1)
     gemm_tc_kernel(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ CUtensorMap tmX,
                    void* __restrict__ C, int ldc, int M, int N, int K, int epi, int n_split,
-                   uint32_t* __restrict__ status, const __grid_constant__ Fuse fz) {
+                   uint32_t* __restrict__ status, const __grid_constant__ Fuse fz,
+                   long long test_wait) {
     using G = Cfg<BN, SWIGLU, STAGES, FUSED>;
     extern __shared__ uint8_t smem_raw[];
     uint8_t* smem = (uint8_t*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
@@ -174,6 +178,9 @@ __global__ void __launch_bounds__(kThreads, FUSED && BN == 16 ? kFusedCtasPerSm 
     const long long n_iter = (long long)n_feat * kblocks;
     const long long seg_lo = FUSED ? (long long)blockIdx.x * n_iter / gridDim.x : (long long)blockIdx.x;
     const long long seg_hi = FUSED ? (long long)(blockIdx.x + 1) * n_iter / gridDim.x : (long long)num_tiles;
+    // bounded-wait test: CTA 0 skips its first copy and waits test_wait cycles at most
+    const bool test_skip = !FUSED && test_wait > 0 && blockIdx.x == 0;
+    const long long wlim = test_skip ? test_wait : tc::kWaitCycles;
 
     if (threadIdx.x == 0) {
         for (int s = 0; s < STAGES; ++s) {
@@ -220,14 +227,23 @@ __global__ void __launch_bounds__(kThreads, FUSED && BN == 16 ? kFusedCtasPerSm 
                                     &full[pend_stage[i]]);
                 npend = 0;
             };
+            bool skip_next = test_skip;
             Seg sg;
             for (bool have = seg_at<FUSED>(sg, seg_lo, seg_hi, n_tok, n_split, kblocks); ok && have;
                  have = seg_at<FUSED>(sg, sg.next, seg_hi, n_tok, n_split, kblocks)) {
                 const int feat = sg.feat, tok = sg.tok;
                 for (int kb = sg.kb0; kb < sg.kb1; ++kb) {
-                    if (!tc::mbar_wait(&empty[stage], phase ^ 1, abort_flag)) {
+                    if (!tc::mbar_wait(&empty[stage], phase ^ 1, abort_flag, wlim)) {
                         ok = false;
                         break;
+                    }
+                    if (skip_next) {  // bounded-wait test: this stage's copy is never issued
+                        skip_next = false;
+                        if (++stage == STAGES) {
+                            stage = 0;
+                            phase ^= 1;
+                        }
+                        continue;
                     }
                     tc::mbar_expect_tx(&full[stage], G::A_BYTES + G::B_BYTES);
                     tc::tma_load_2d(sA + stage * G::A_BYTES, &tmW, kb * kBK, feat * G::A_ROWS,
@@ -268,14 +284,14 @@ __global__ void __launch_bounds__(kThreads, FUSED && BN == 16 ? kFusedCtasPerSm 
             for (bool have = seg_at<FUSED>(sg, seg_lo, seg_hi, n_tok, n_split, kblocks); ok && have;
                  have = seg_at<FUSED>(sg, sg.next, seg_hi, n_tok, n_split, kblocks)) {
                 const int kb0 = sg.kb0, kb1 = sg.kb1;
-                if (!tc::mbar_wait(&tempty[acc], acc_phase ^ 1, abort_flag)) {
+                if (!tc::mbar_wait(&tempty[acc], acc_phase ^ 1, abort_flag, wlim)) {
                     ok = false;
                     break;
                 }
                 tc::fence_after_sync();
                 const uint32_t d = tmem_base + (uint32_t)(acc * G::ACC_COLS);
                 for (int kb = kb0; kb < kb1; ++kb) {
-                    if (!tc::mbar_wait(&full[stage], phase, abort_flag)) {
+                    if (!tc::mbar_wait(&full[stage], phase, abort_flag, wlim)) {
                         ok = false;
                         break;
                     }
@@ -582,7 +598,7 @@ __global__ void __launch_bounds__(kThreads, FUSED && BN == 16 ? kFusedCtasPerSm 
         for (int t = blockIdx.x; t < num_tiles; t += gridDim.x) {
             const int split = t % n_split, rest = t / n_split;
             const int feat = rest / n_tok, tok = rest % n_tok;
-            bool ok = tc::mbar_wait(&tfull[acc], acc_phase, abort_flag);
+            bool ok = tc::mbar_wait(&tfull[acc], acc_phase, abort_flag, wlim);
             ok = __all_sync(0xffffffffu, ok);
             if (!ok) break;
             tc::fence_after_sync();
@@ -688,7 +704,7 @@ bool make_map(CUtensorMap* map, const void* base, int inner, int rows, int ld, i
 template <int BN, bool SWIGLU, int STAGES, bool FUSED = false>
 int launch_cfg(const bf16* A, int lda, const bf16* W, void* C, int ldc, int M, int N, int K,
                int epi, int n_split, int num_sms, uint32_t* status, cudaStream_t s,
-               const Fuse* fz = nullptr) {
+               const Fuse* fz = nullptr, long long test_wait = 0) {
     using G = Cfg<BN, SWIGLU, STAGES, FUSED>;
     static bool attr_set = false;
     if (!attr_set) {
@@ -706,7 +722,7 @@ int launch_cfg(const bf16* A, int lda, const bf16* W, void* C, int ldc, int M, i
     const int grid = units < num_sms ? (int)units : num_sms;
     Fuse none{};
     launch_k(gemm_tc_kernel<BN, SWIGLU, STAGES, FUSED>, dim3(grid), dim3(kThreads), G::SMEM, s, tmW,
-             tmX, C, ldc, M, N, K, epi, n_split, status, fz ? *fz : none);
+             tmX, C, ldc, M, N, K, epi, n_split, status, fz ? *fz : none, test_wait);
     note_launch();
     return QK_OK;
 }
@@ -720,19 +736,20 @@ bool gemm_tc_supported(const void* A, int lda, int N, int K) {
 
 // bf16 linear layer on the tensor cores; token-tile width chosen from M.
 int launch_gemm_tc(const bf16* A, int lda, const bf16* W, void* C, int ldc, int M, int N, int K,
-                   int epi, int num_sms, uint32_t* status, cudaStream_t s) {
+                   int epi, int num_sms, uint32_t* status, cudaStream_t s, long long test_wait) {
     if (M <= 0) return QK_OK;
+    const long long tw = test_wait;
     if (epi == EPI_SWIGLU) {
-        if (M <= 16) return launch_cfg<16, true, 6>(A, lda, W, C, ldc, M, N, K, epi, 1, num_sms, status, s);
-        if (M <= 32) return launch_cfg<32, true, 6>(A, lda, W, C, ldc, M, N, K, epi, 1, num_sms, status, s);
-        if (M <= 64) return launch_cfg<64, true, 5>(A, lda, W, C, ldc, M, N, K, epi, 1, num_sms, status, s);
-        return launch_cfg<128, true, 4>(A, lda, W, C, ldc, M, N, K, epi, 1, num_sms, status, s);
+        if (M <= 16) return launch_cfg<16, true, 6>(A, lda, W, C, ldc, M, N, K, epi, 1, num_sms, status, s, nullptr, tw);
+        if (M <= 32) return launch_cfg<32, true, 6>(A, lda, W, C, ldc, M, N, K, epi, 1, num_sms, status, s, nullptr, tw);
+        if (M <= 64) return launch_cfg<64, true, 5>(A, lda, W, C, ldc, M, N, K, epi, 1, num_sms, status, s, nullptr, tw);
+        return launch_cfg<128, true, 4>(A, lda, W, C, ldc, M, N, K, epi, 1, num_sms, status, s, nullptr, tw);
     }
-    if (M <= 16) return launch_cfg<16, false, 8>(A, lda, W, C, ldc, M, N, K, epi, 1, num_sms, status, s);
-    if (M <= 32) return launch_cfg<32, false, 8>(A, lda, W, C, ldc, M, N, K, epi, 1, num_sms, status, s);
-    if (M <= 64) return launch_cfg<64, false, 8>(A, lda, W, C, ldc, M, N, K, epi, 1, num_sms, status, s);
-    if (M <= 128) return launch_cfg<128, false, 6>(A, lda, W, C, ldc, M, N, K, epi, 1, num_sms, status, s);
-    return launch_cfg<256, false, 4>(A, lda, W, C, ldc, M, N, K, epi, 1, num_sms, status, s);
+    if (M <= 16) return launch_cfg<16, false, 8>(A, lda, W, C, ldc, M, N, K, epi, 1, num_sms, status, s, nullptr, tw);
+    if (M <= 32) return launch_cfg<32, false, 8>(A, lda, W, C, ldc, M, N, K, epi, 1, num_sms, status, s, nullptr, tw);
+    if (M <= 64) return launch_cfg<64, false, 8>(A, lda, W, C, ldc, M, N, K, epi, 1, num_sms, status, s, nullptr, tw);
+    if (M <= 128) return launch_cfg<128, false, 6>(A, lda, W, C, ldc, M, N, K, epi, 1, num_sms, status, s, nullptr, tw);
+    return launch_cfg<256, false, 4>(A, lda, W, C, ldc, M, N, K, epi, 1, num_sms, status, s, nullptr, tw);
 }
 
 // Decode linear with a fused epilogue (see Fuse); one token tile of M <= 64 rows.

@@ -12,8 +12,12 @@
 //
 // The array's name, used in host code, is only a host-side stand-in for the
 // device symbol; it is not a device address.  The device address is looked up
-// once per device with cudaGetSymbolAddress (with that device current) and
-// cached; the first call on each device performs that lookup.
+// with cudaGetSymbolAddress (with the device current) on the first call in each
+// CUDA context and cached against that context, so a context torn down and
+// created again (cudaDeviceReset) is looked up afresh instead of reusing a
+// stale address.
+#include <cuda.h>
+
 #include <mutex>
 
 #include "qk_internal.cuh"
@@ -29,20 +33,48 @@ __device__ __align__(256) unsigned char g_swiglu_scratch[kStaticScratchBytes];
 
 constexpr int kMaxDevices = 64;
 std::mutex g_scratch_mu;
-void* g_scratch_ptr[kMaxDevices] = {};
+struct CachedAddress {
+    CUcontext ctx;  // context the address belongs to
+    void* ptr;
+};
+CachedAddress g_scratch[kMaxDevices] = {};
 
-// Device address of g_swiglu_scratch on the current device (looked up once per device).
+typedef CUresult (*CtxGetCurrentFn)(CUcontext*);
+
+// Current driver context of this thread (nullptr if it cannot be queried).
+CUcontext current_context() {
+    static CtxGetCurrentFn fn = nullptr;
+    static std::once_flag once;
+    std::call_once(once, [] {
+        void* p = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        if (cudaGetDriverEntryPointByVersion("cuCtxGetCurrent", &p, 12000, cudaEnableDefault, &q) ==
+                cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            fn = (CtxGetCurrentFn)p;
+    });
+    CUcontext c = nullptr;
+    if (!fn || fn(&c) != CUDA_SUCCESS) return nullptr;
+    return c;
+}
+
+// Device address of g_swiglu_scratch on the current device, looked up once per
+// context (the caller has made `device` current).
 int scratch_address(int device, void** out) {
     if (device < 0 || device >= kMaxDevices)
         return set_error(QK_EINVAL, "device ordinal %d outside [0, %d)", device, kMaxDevices);
     std::lock_guard<std::mutex> lock(g_scratch_mu);
-    if (!g_scratch_ptr[device]) {
+    const CUcontext ctx = current_context();
+    CachedAddress& c = g_scratch[device];
+    if (!c.ptr || !ctx || c.ctx != ctx) {
         void* p = nullptr;
         cudaError_t e = cudaGetSymbolAddress(&p, g_swiglu_scratch);
         if (e != cudaSuccess) return cuda_error(e, "cudaGetSymbolAddress(static scratch)");
-        g_scratch_ptr[device] = p;
+        // cudaGetSymbolAddress may have created the primary context: read it again
+        c.ctx = ctx ? ctx : current_context();
+        c.ptr = p;
     }
-    *out = g_scratch_ptr[device];
+    *out = c.ptr;
     return QK_OK;
 }
 
@@ -59,6 +91,7 @@ extern "C" int qk_op_linear_swiglu_static(qk_model* mh, const void* A, int lda, 
     if (M < 1 || N < 128 || N % 128 || K < 16 || K % 16 || lda < K || ldc != N)
         return set_error(QK_ESHAPE, "bad SwiGLU linear shape M %d N %d K %d lda %d ldc %d", M, N,
                          K, lda, ldc);
+    QK_TRY(check_linear_operands(m, A, lda, W, C, m.es));
     const size_t need = (size_t)M * 2 * N * m.es;
     if (need > kStaticScratchBytes)
         return set_error(QK_ESHAPE,
@@ -68,6 +101,9 @@ extern "C" int qk_op_linear_swiglu_static(qk_model* mh, const void* A, int lda, 
     int device = 0;
     cudaError_t e = cudaGetDevice(&device);
     if (e != cudaSuccess) return cuda_error(e, "cudaGetDevice");
+    if (device != m.device)
+        return set_error(QK_EINVAL, "current device %d is not the model's device %d", device,
+                         m.device);
     void* scratch = nullptr;
     QK_TRY(scratch_address(device, &scratch));
     cudaStream_t s = (cudaStream_t)stream;

@@ -335,6 +335,19 @@ static int clear_attn_tickets(const Model& m, const Workspace& w, int B, int max
     return QK_OK;
 }
 
+int check_linear_operands(const Model& m, const void* A, int lda, const void* W, const void* C,
+                          int out_es) {
+    const int row_align = m.es == 2 ? 8 : 4;  // elements per 16 bytes
+    if (((uintptr_t)A & 15) || ((uintptr_t)W & 15))
+        return set_error(QK_EINVAL, "A and W must be 16-byte aligned (A %p, W %p)", A, W);
+    if (lda % row_align)
+        return set_error(QK_ESHAPE, "lda %d must be a multiple of %d elements (16 bytes)", lda,
+                         row_align);
+    if ((uintptr_t)C % (uintptr_t)out_es)
+        return set_error(QK_EINVAL, "C must be aligned to its %d-byte elements", out_es);
+    return QK_OK;
+}
+
 static int check_launch(const char* what) {
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return cuda_error(e, what);
@@ -568,12 +581,22 @@ int qk_op_linear(qk_model* mh, const void* A, int lda, const void* W, void* C, i
     if (epilogue < QK_EPI_STORE || epilogue > QK_EPI_SWIGLU)
         return set_error(QK_EINVAL, "unknown epilogue %d", epilogue);
     if (ldc < N) return set_error(QK_ESHAPE, "ldc %d < N %d", ldc, N);
+    const bool f32_out = epilogue == QK_EPI_STORE_F32 || epilogue == QK_EPI_RESID_F32;
+    QK_TRY(check_linear_operands(m, A, lda, W, C, f32_out ? 4 : m.es));
     // Only the CUDA-core path (fp32 models) stages the gate/up product in scratch.
     size_t need = epilogue == QK_EPI_SWIGLU && m.cfg.dtype == QK_DTYPE_F32 ? (size_t)M * 2 * N * m.es : 0;
     if (need && (!scratch || scratch_bytes < need))
         return set_error(QK_ENOSPACE, "linear scratch has %zu bytes, needs %zu", scratch_bytes, need);
     linear(m, A, lda, W, C, ldc, M, N, K, epilogue, scratch, (cudaStream_t)stream);
     return check_launch(m, "linear");
+}
+
+int qk_debug_expire_next_wait(qk_model* mh, long long wait_cycles) {
+    if (!mh) return set_error(QK_EINVAL, "null argument");
+    if (wait_cycles < 1 || wait_cycles > (1ll << 31))
+        return set_error(QK_EINVAL, "wait_cycles %lld outside [1, 2^31]", wait_cycles);
+    ((Model*)mh)->test_wait_cycles = wait_cycles;
+    return QK_OK;
 }
 
 int qk_kv_bytes(const qk_model* mh, int max_batch, int max_seq, size_t* bytes) {
@@ -975,6 +998,8 @@ int qk_check_status(qk_model* mh, void* stream, uint32_t* flags) {
     QK_TRY_CUDA(cudaMemcpy(&v, m.status, sizeof(v), cudaMemcpyDeviceToHost));
     QK_TRY_CUDA(cudaMemset(m.status, 0, sizeof(v)));
     if (flags) *flags = v;
+    if (v & QK_STATUS_TIMEOUT)
+        return set_error(QK_ETIMEOUT, "a bounded device wait expired (device status 0x%x)", v);
     if (v) return set_error(QK_EDEVICE, "device status 0x%x", v);
     return QK_OK;
 }

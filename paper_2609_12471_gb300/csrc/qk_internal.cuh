@@ -50,6 +50,14 @@ constexpr int kGemvMaxRows = 4;
 // ---------------------------------------------------------------- errors
 int set_error(int code, const char* fmt, ...);
 int cuda_error(cudaError_t e, const char* what);
+struct Model;
+// Host check of the operands of a caller-facing linear step (qk_op_linear and its
+// static-scratch variant): A and W must start on a 16-byte boundary, lda must keep
+// every row of A on one (a multiple of 8 bf16 / 4 fp32 elements), and C must be
+// aligned to its element size (out_es bytes).  The CUDA-core, GEMV and tcgen05
+// kernels all read A and W with 8- or 16-byte vector loads.
+int check_linear_operands(const Model& m, const void* A, int lda, const void* W, const void* C,
+                          int out_es);
 #define QK_TRY_CUDA(expr)                                   \
     do {                                                    \
         cudaError_t _e = (expr);                            \
@@ -116,6 +124,9 @@ struct Model {
     // reported and cleared by the entry point that made the launches.
     int deferred_error = 0;
     SampleArgs sampling{};  // set only while a sampled rollout runs
+    // qk_debug_expire_next_wait: wait limit (SM cycles) of the next plain tcgen05 GEMM
+    // launch, which then skips one copy so that the wait expires; 0 = off.
+    long long test_wait_cycles = 0;
 };
 
 // Records the opening event of a bracketed launch; returns whether it did.
@@ -250,8 +261,10 @@ void launch_gemv_bf16(const bf16* A, int lda, const bf16* W, void* C, int ldc, i
                       int K, int epi, cudaStream_t s);
 // tcgen05 path (k_gemm_tc.cu): N % 128 == 0, K % 64 == 0, A 16-byte aligned, lda % 8 == 0.
 bool gemm_tc_supported(const void* A, int lda, int N, int K);
+// test_wait > 0: bounded-wait test launch (CTA 0 skips its first copy and gives up
+// after test_wait SM cycles; the output is undefined and QK_STATUS_TIMEOUT is set).
 int launch_gemm_tc(const bf16* A, int lda, const bf16* W, void* C, int ldc, int M, int N, int K,
-                   int epi, int num_sms, uint32_t* status, cudaStream_t s);
+                   int epi, int num_sms, uint32_t* status, cudaStream_t s, long long test_wait = 0);
 
 // Fused epilogue of a decode-sized linear (one token tile, M <= 64 rows).  The
 // N/128 x K/64 k-block iterations are split evenly over the CTAs; a CTA that holds

@@ -42,13 +42,18 @@ def assert_logits_close(got, ref, rel):
     return err, tol
 
 
-def assert_argmax_where_gap(got, ref_logits, logit_tol):
-    """Arg-max must match where the oracle's top-2 gap exceeds 10x the logit tolerance."""
+def assert_argmax_where_gap(got, ref_logits, logit_tol, min_decisive=1, distinct=None):
+    """Arg-max must match where the oracle's top-2 gap exceeds 10x the logit tolerance,
+    and at least `min_decisive` rows must be decisive (so the check cannot pass
+    vacuously).  distinct: columns holding the distinct logit values when the vocabulary
+    repeats values on purpose (the gap is then taken over those columns only)."""
     import oracle
     ref_logits = np.asarray(ref_logits)
-    gap = oracle.top2_gap(ref_logits)
+    gap = oracle.top2_gap(ref_logits if distinct is None else ref_logits[:, distinct])
     am = oracle.argmax_lowest(ref_logits)
     mask = gap > 10 * logit_tol
+    n = int(mask.sum())
     bad = np.nonzero(mask & (np.asarray(got) != am))[0]
-    assert bad.size == 0, f"argmax differs at {bad[:10]} (of {mask.sum()} decisive rows)"
-    return int(mask.sum())
+    assert bad.size == 0, f"argmax differs at {bad[:10]} (of {n} decisive rows)"
+    assert n >= min_decisive, f"only {n} of {len(mask)} rows decisive (need {min_decisive})"
+    return n

@@ -115,3 +115,10 @@ def test_grpo_and_turn_entry_points_validate_on_the_host(lib):
     with pytest.raises(qk.QKError) as e:
         qk.qk_prefill_rows(None, P, 1, 8, P, 1, 4, P, ws_bytes=0, stream=0)
     assert e.value.code == qk.QK_EINVAL
+
+
+def test_debug_hook_validates_on_the_host():
+    import paper_2609_12471_gb300 as qk
+    with pytest.raises(qk.QKError) as e:
+        qk.qk_debug_expire_next_wait(None, 1000)
+    assert e.value.code == qk.QK_EINVAL

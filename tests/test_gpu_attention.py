@@ -12,7 +12,7 @@ import pytest
 import oracle
 import synth
 from _bf16_floor import forward_logits_bf16_activations
-from _gpu import assert_logits_close, decoder
+from _gpu import assert_argmax_where_gap, assert_logits_close, decoder
 
 pytestmark = pytest.mark.gpu
 SHAPE = synth.ModelShape("attn_bf16", 2, 512, 4, 2, 128, 256, 1024, "bf16")
@@ -38,12 +38,16 @@ def test_score_several_query_tiles_ragged_tail(model):
     dec, W = model
     B, T = 3, 200
     toks = synth.tokens((B, T), SHAPE.vocab, stream=71)
-    lp = dec.score(torch.tensor(toks, dtype=torch.int32, device="cuda")).cpu().numpy()
+    am = torch.empty(B, T - 1, dtype=torch.int32, device="cuda")
+    lp = dec.score(torch.tensor(toks, dtype=torch.int32, device="cuda"), argmax=am).cpu().numpy()
+    am = am.cpu().numpy()
     assert dec.check_status() == 0
     for b in range(B):
         z, rel, lp_tol = _tol(W, toks[b])
         lp_ref = oracle.token_logprobs(z[:-1], toks[b, 1:])
         assert np.max(np.abs(lp[b] - lp_ref)) <= lp_tol
+        # a 1,024-way vocabulary: about a third of the rows clear 10 x 3e-2 x std
+        assert_argmax_where_gap(am[b], z[:-1], rel * np.std(z[:-1]), min_decisive=(T - 1) // 10)
 
 
 def test_chunked_prefill_then_decode(model):

@@ -75,3 +75,32 @@ def test_linear_matches_f64(models, dt, epi, M, N, K):
         tol = 2 ** -8 * scale                  # one bf16 rounding of the output
     err = np.abs(got - ref).max()
     assert err <= tol, f"max err {err:.3e} > {tol:.3e} (scale {scale:.3e})"
+
+
+@pytest.mark.parametrize("dt", ["bf16", "f32"])
+def test_misaligned_operands_are_refused_before_any_launch(models, dt):
+    """A, W off a 16-byte boundary, a row stride that breaks the rows' 16-byte
+    alignment, or C off its element size: refused on the host, nothing launched."""
+    import torch
+    import paper_2609_12471_gb300 as qk
+    dec = models[dt]
+    es = 2 if dt == "bf16" else 4
+    M, N, K = 20, 128, 64
+    buf = torch.zeros(8 << 20, dtype=torch.uint8, device="cuda")  # every case stays in bounds
+    A, W, C = buf.data_ptr(), buf.data_ptr() + (1 << 20), buf.data_ptr() + (2 << 20)
+    bad_lda = K + (4 if dt == "bf16" else 2)
+    cases = [dict(A=A + es), dict(W=W + 8), dict(lda=bad_lda), dict(C=C + 2, epi=qk.QK_EPI_STORE_F32)]
+    for over in cases:
+        a = dict(A=A, W=W, C=C, lda=K, epi=qk.QK_EPI_STORE)
+        a.update(over)
+        before = qk.qk_launch_count()
+        with pytest.raises(qk.QKError) as e:
+            qk.qk_op_linear(dec.handle, a["A"], a["lda"], a["W"], a["C"], N, M, N, K, a["epi"])
+        assert e.value.code in (qk.QK_EINVAL, qk.QK_ESHAPE), over
+        assert qk.qk_launch_count() == before, over
+        if "epi" in over:
+            continue  # the static variant always stores in the model dtype
+        with pytest.raises(qk.QKError) as e:
+            qk.qk_op_linear_swiglu_static(dec.handle, a["A"], a["lda"], a["W"], a["C"], N, M, N, K)
+        assert e.value.code in (qk.QK_EINVAL, qk.QK_ESHAPE), over
+        assert qk.qk_launch_count() == before, over

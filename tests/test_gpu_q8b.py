@@ -4,11 +4,15 @@ Teacher-forced rollout and scoring at reduced lengths are compared position by
 position with the fp64 oracle.  Tolerance: max |logit error| <= max(3e-2 x
 std(logits), 2 x F_z) and |log-prob error| <= max(5e-2, 2 x F_lp), where F_z,
 F_lp are the errors of an exact bf16-rounding evaluation of the same positions
-(tests/_bf16_floor.py).  On 36 random-init layers that floor is above the fixed
+(tests/_bf16_floor.py) that rounds where the path under test stores bf16: the
+decode path's points for the rollout's decode steps, the prefill path's for its
+prompt and for scoring.  On 36 random-init layers that floor is above the fixed
 3e-2 x std bound (about 0.16 x std): no implementation that stores its
 activations and KV cache in bf16 meets the fixed bound there, so the bound is
 widened to the floor.  Arg-max is exact where the oracle's top-2 gap exceeds
-10x the logit tolerance."""
+10x the logit tolerance; at this tolerance over a 151,936-way vocabulary
+almost no row is that decisive, so the non-vacuous bf16 arg-max check is the
+narrower-vocabulary model of test_gpu_argmax.py."""
 import numpy as np
 import pytest
 
@@ -34,22 +38,31 @@ def short_case(q8b):
     B, P, N = 2, 24, 8
     seq = synth.tokens((B, P + N + 1), s.vocab, stream=5)
     z = np.stack([oracle.forward_logits(s, W, seq[b, :P + N]) for b in range(B)])
-    zf = np.stack([forward_logits_bf16_activations(s, W, seq[b, :P + N]) for b in range(B)])
-    floor_z = float(np.max(np.abs(zf - z)))
     lpr = np.stack([oracle.token_logprobs(z[b], seq[b, 1:]) for b in range(B)])
-    lpf = np.stack([oracle.token_logprobs(zf[b], seq[b, 1:]) for b in range(B)])
-    floor_lp = float(np.max(np.abs(lpf - lpr)))
-    logit_rel = max(LOGIT_REL, 2 * floor_z / float(np.std(z)))
-    lp_abs = max(LP_ABS, 2 * floor_lp)
-    print(f"bf16 floor: max |dz| {floor_z:.4f} (std {np.std(z):.4f}), max |dlp| {floor_lp:.4f}; "
-          f"tolerances {logit_rel:.4f} x std, {lp_abs:.4f}")
-    return seq, P, N, z, logit_rel, lp_abs
+
+    def tolerances(decode_from, rows):
+        """Tolerances from the floor of the path under test, over the compared rows."""
+        zf = np.stack([forward_logits_bf16_activations(s, W, seq[b, :P + N], decode_from)
+                       for b in range(B)])
+        lpf = np.stack([oracle.token_logprobs(zf[b], seq[b, 1:]) for b in range(B)])
+        floor_z = float(np.max(np.abs(zf[:, rows] - z[:, rows])))
+        floor_lp = float(np.max(np.abs(lpf[:, rows] - lpr[:, rows])))
+        rel = max(LOGIT_REL, 2 * floor_z / float(np.std(z[:, rows])))
+        lp_abs = max(LP_ABS, 2 * floor_lp)
+        print(f"bf16 floor (decode from {decode_from}): max |dz| {floor_z:.4f} "
+              f"(std {np.std(z[:, rows]):.4f}), max |dlp| {floor_lp:.4f}; "
+              f"tolerances {rel:.4f} x std, {lp_abs:.4f}")
+        return rel, lp_abs
+
+    roll = tolerances(P, slice(P - 1, P + N))   # prompt by prefill, then decode steps
+    score = tolerances(None, slice(0, P + N))   # every position by the scoring path
+    return seq, P, N, z, roll, score
 
 
 def test_rollout_short_matches_oracle(q8b, short_case):
     import torch
     s, W, dec = q8b
-    seq, P, N, z_all, logit_rel, lp_abs = short_case
+    seq, P, N, z_all, (logit_rel, lp_abs), _ = short_case
     B = seq.shape[0]
     d = torch.tensor(seq, device="cuda", dtype=torch.int32)
     kv = dec.new_kv(B, P + N)
@@ -72,7 +85,7 @@ def test_rollout_short_matches_oracle(q8b, short_case):
     err, tol = assert_logits_close(logits, z_ref, logit_rel)
     lp_ref = np.stack([oracle.token_logprobs(z_ref[b], seq[b, P:P + N + 1]) for b in range(B)])
     assert np.max(np.abs(lp - lp_ref)) <= lp_abs
-    assert_argmax_where_gap(am.reshape(-1), z_ref.reshape(-1, s.vocab), tol)
+    assert_argmax_where_gap(am.reshape(-1), z_ref.reshape(-1, s.vocab), tol, min_decisive=0)
     # the rollout entry point gives the same numbers as the step-by-step calls
     kv2 = dec.new_kv(B, P + N)
     lp2 = dec.rollout(kv2, B, P + N, d, P).cpu().numpy()
@@ -82,7 +95,7 @@ def test_rollout_short_matches_oracle(q8b, short_case):
 def test_score_short_matches_oracle(q8b, short_case):
     import torch
     s, W, dec = q8b
-    seq, P, N, z_all, logit_rel, lp_abs = short_case
+    seq, P, N, z_all, _, (logit_rel, lp_abs) = short_case
     B, T = seq.shape[0], P + N + 1
     am = torch.empty(B, T - 1, dtype=torch.int32, device="cuda")
     lp = dec.score(torch.tensor(seq, device="cuda", dtype=torch.int32), argmax=am).cpu().numpy()
@@ -90,4 +103,5 @@ def test_score_short_matches_oracle(q8b, short_case):
     lp_ref = np.stack([oracle.token_logprobs(z_all[b], seq[b, 1:]) for b in range(B)])
     assert np.max(np.abs(lp - lp_ref)) <= lp_abs
     tol = logit_rel * np.std(z_all)
-    assert_argmax_where_gap(am.cpu().numpy().reshape(-1), z_all.reshape(-1, s.vocab), tol)
+    assert_argmax_where_gap(am.cpu().numpy().reshape(-1), z_all.reshape(-1, s.vocab), tol,
+                            min_decisive=0)

@@ -4,7 +4,10 @@ oracle follows the GPU's own draws, so every step compares the same prefix.
 Where the oracle's top-2 gap of the perturbed scores z / tau + G exceeds the
 logit tolerance the drawn token must be the oracle's; elsewhere it must be one
 of the near-maximal candidates.  Log-probs of the drawn tokens within the
-model's scoring tolerance; same seed, same tokens; another seed, other tokens."""
+model's teacher-forced log-prob tolerance divided by tau (the reported value is
+log softmax(z / tau)[c], whose error is the logits' error scaled by 1 / tau; the
+Gumbel noise enters only the choice of c, which both sides share); same seed,
+same tokens; another seed, other tokens."""
 import numpy as np
 import pytest
 
@@ -35,7 +38,8 @@ def _check_rollout(s, W, dec, B, P, N, tau, seed, gap_tol, lp_tol, min_decided):
             else:  # a near-tie: the GPU's token must be one of the near-maximal candidates
                 y = z[j] / tau + oracle.gumbel(oracle.sample_uniforms(seed, b, j, s.vocab))
                 assert y[toks[b, j]] >= y.max() - 2 * gap_tol
-        assert np.max(np.abs(lp[b] - lp_ref)) <= lp_tol, np.max(np.abs(lp[b] - lp_ref))
+        bar = lp_tol(lp_ref) / tau
+        assert np.all(np.abs(lp[b] - lp_ref) <= bar), np.max(np.abs(lp[b] - lp_ref) / bar)
     assert decided >= min_decided * B * (N + 1), decided
     return toks
 
@@ -50,9 +54,10 @@ def tiny():
 @pytest.mark.parametrize("tau", [1.0, 0.7])
 def test_sampled_rollout_tiny_matches_oracle(tiny, tau):
     s, W, dec = tiny
-    # fp32 model: logits within 1e-4 x std; Gumbel noise in fp32 within a few ulp
-    _check_rollout(s, W, dec, B=3, P=12, N=20, tau=tau, seed=1234, gap_tol=2e-3, lp_tol=2e-3,
-                   min_decided=0.9)
+    # fp32 model: logits within 1e-4 x std; Gumbel noise in fp32 within a few ulp; log-probs
+    # within the teacher-forced bar 1e-4 x max(1, |lp|), over tau
+    _check_rollout(s, W, dec, B=3, P=12, N=20, tau=tau, seed=1234, gap_tol=2e-3,
+                   lp_tol=lambda lp: 1e-4 * np.maximum(1.0, np.abs(lp)), min_decided=0.9)
 
 
 def test_same_seed_same_tokens_other_seed_other_tokens(tiny):
@@ -75,5 +80,7 @@ def test_sampled_rollout_bf16_matches_oracle():
     # hundredths, so near-ties are judged with a wider gap.  The top-2 gap of
     # Gumbel-perturbed scores is about Exp(1)-distributed, so ~78 % of the steps
     # clear 0.25; at least 60 % must.
-    _check_rollout(s, W, dec, B=6, P=20, N=12, tau=1.0, seed=77, gap_tol=0.25, lp_tol=0.15,
-                   min_decided=0.6)
+    # Log-probs within the bf16 teacher-forced bar 5e-2 (the floor of this 2-layer model
+    # is below it).
+    _check_rollout(s, W, dec, B=6, P=20, N=12, tau=1.0, seed=77, gap_tol=0.25,
+                   lp_tol=lambda lp: np.full_like(lp, 5e-2), min_decided=0.6)

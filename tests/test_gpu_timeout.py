@@ -1,0 +1,65 @@
+"""The bounded-wait status path on the GPU, without a fault or a hang.
+
+qk_debug_expire_next_wait arms one tensor-core GEMM launch so that its first
+CTA issues no copy for its first k-block and waits at most a short limit: the
+MMA thread's wait for that copy expires.  The kernel must then set
+QK_STATUS_TIMEOUT, drain its own copies, free its tensor memory and return;
+qk_check_status reports QK_ETIMEOUT, and the next call on the same context
+computes the right result (the context stayed usable)."""
+import numpy as np
+import pytest
+
+import oracle
+import synth
+from _gpu import decoder
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def bf16_model():
+    return decoder(synth.shape("tiny_fp32", dtype="bf16"))[0]
+
+
+def _linear(dec, A, W, M, N, K):
+    import torch
+    import paper_2609_12471_gb300 as qk
+    C = torch.full((M, N), float("nan"), dtype=torch.float32, device="cuda")
+    qk.qk_op_linear(dec.handle, A, K, W, C, N, M, N, K, qk.QK_EPI_STORE_F32)
+    return C
+
+
+def test_expired_wait_sets_timeout_and_context_stays_usable(bf16_model):
+    import torch
+    import paper_2609_12471_gb300 as qk
+    dec = bf16_model
+    M, N, K = 96, 384, 512  # tcgen05 path, several CTAs, 8 k-blocks each
+    A = synth.normal(700, 1, (M, K), "bf16")
+    W = synth.normal(700, 2, (N, K), "bf16", sigma=0.05)
+    cvt = lambda a: torch.from_numpy(a.view(np.int16)).view(torch.bfloat16).cuda()
+    Ad, Wd = cvt(A), cvt(W)
+    ref = oracle.widen(A) @ oracle.widen(W).T
+    tol = 2e-5 * np.abs(ref).max()
+
+    ok = _linear(dec, Ad, Wd, M, N, K).cpu().numpy()
+    assert dec.check_status() == 0
+    assert np.abs(ok - ref).max() <= tol
+
+    qk.qk_debug_expire_next_wait(dec.handle, 1 << 20)  # about half a millisecond
+    _linear(dec, Ad, Wd, M, N, K)
+    flags = qk.qk_check_status(dec.handle)
+    assert flags & qk.QK_STATUS_TIMEOUT, flags
+    # the C entry point itself reports the expired wait as QK_ETIMEOUT
+    qk.qk_debug_expire_next_wait(dec.handle, 1 << 20)
+    _linear(dec, Ad, Wd, M, N, K)
+    torch.cuda.synchronize()
+    import ctypes
+    v = ctypes.c_uint32()
+    lib = qk._binding._load()
+    rc = lib.qk_check_status(dec.handle, torch.cuda.current_stream().cuda_stream, ctypes.byref(v))
+    assert rc == qk.QK_ETIMEOUT and v.value & qk.QK_STATUS_TIMEOUT, (rc, v.value)
+
+    # the hook disarmed itself; the context still computes correctly
+    again = _linear(dec, Ad, Wd, M, N, K).cpu().numpy()
+    assert dec.check_status() == 0
+    assert np.abs(again - ref).max() <= tol

@@ -61,7 +61,9 @@ def test_prefill_and_decode_steps_match_oracle(tiny, rollout_ref):
     z, lp, am, _ = _run_steps(dec, seq, P, N)
     err, tol = assert_logits_close(z, z_ref, REL)
     assert np.all(np.abs(lp - lp_ref) <= REL * np.maximum(1.0, np.abs(lp_ref)))
-    assert_argmax_where_gap(am.reshape(-1), z_ref.reshape(-1, s.vocab), tol)
+    # at 1e-4 x std nearly every row of an fp32 model is decisive
+    assert_argmax_where_gap(am.reshape(-1), z_ref.reshape(-1, s.vocab), tol,
+                            min_decisive=int(0.9 * am.size))
 
 
 def test_rollout_entry_point_equals_step_by_step(tiny, rollout_ref):
@@ -105,7 +107,8 @@ def test_score_logprobs_matches_oracle(tiny):
             lp_ref, am_ref, gap = oracle.score_sequence(s, W, toks[b])
             assert np.all(np.abs(lp[b] - lp_ref) <= REL * np.maximum(1.0, np.abs(lp_ref)))
             z = oracle.forward_logits(s, W, toks[b])[:-1]
-            assert_argmax_where_gap(am[b].cpu().numpy(), z, REL * np.std(z))
+            assert_argmax_where_gap(am[b].cpu().numpy(), z, REL * np.std(z),
+                                    min_decisive=int(0.9 * (T - 1)))
 
 
 def test_ragged_positions_in_one_decode_step(tiny):
