@@ -2,11 +2,13 @@
 the Qwen3-8B layer width (H 4096, 32 / 8 heads, d 128, I 12288: the same GEMM
 tiles and split-K schedules as the full model) with a 1,024-way vocabulary.
 
-Over 1,024 logits the oracle's top-2 gap clears 10 x the 3e-2 x std logit
-tolerance on about a third of the positions, so the exact arg-max comparison of
-the bf16 decode path (fused split-K lm_head + cluster reduce) and of the
-scoring path (tcgen05 lm_head + reduce) has rows to bite on; each comparison
-requires a minimum number of decisive rows.
+The logit tolerance is max(3e-2, 2 x F) x std, F the largest error of the
+exact-bf16-rounding evaluation (about 0.03 x std here, most of it from the bf16
+lm_head input), so a row is decisive when its top-2 gap exceeds about 0.65 x
+std; over 512 distinct logits that holds on 8-13 % of the positions.  The exact
+arg-max comparison of the bf16 decode path (fused split-K lm_head + cluster
+reduce) and of the scoring path (tcgen05 lm_head + reduce) therefore has rows
+to bite on, and each comparison requires at least 4 % of its rows decisive.
 
 The lm_head repeats every even row in the odd row after it, so every logit
 appears twice and every maximum is an exact tie between indices 2i and 2i + 1
@@ -78,7 +80,7 @@ def test_oracle_ties_pairs_exactly(model):
 def test_decode_argmax_exact_where_decisive_and_ties_lowest(model):
     import torch
     dec, W = model
-    B, P, N = 4, 16, 12
+    B, P, N = 4, 16, 20
     seq = synth.tokens((B, P + N + 1), SHAPE.vocab, stream=91)
     kv = dec.new_kv(B, P + N)
     am = torch.empty(B, N + 1, dtype=torch.int32, device="cuda")
@@ -95,13 +97,13 @@ def test_decode_argmax_exact_where_decisive_and_ties_lowest(model):
         assert np.max(np.abs(lp[b] - lp_ref)) <= lp_tol
         decisive += assert_argmax_where_gap(am[b], zr, rel * np.std(zr), min_decisive=0,
                                             distinct=EVEN)
-    assert decisive >= B * (N + 1) // 10, decisive
+    assert decisive >= max(3, B * (N + 1) // 25), decisive
 
 
 def test_score_argmax_exact_where_decisive_and_ties_lowest(model):
     import torch
     dec, W = model
-    B, T = 3, 40
+    B, T = 3, 64
     toks = synth.tokens((B, T), SHAPE.vocab, stream=92)
     am = torch.empty(B, T - 1, dtype=torch.int32, device="cuda")
     lp = dec.score(torch.tensor(toks, dtype=torch.int32, device="cuda"), argmax=am).cpu().numpy()
@@ -115,4 +117,4 @@ def test_score_argmax_exact_where_decisive_and_ties_lowest(model):
         assert np.max(np.abs(lp[b] - lp_ref)) <= lp_tol
         decisive += assert_argmax_where_gap(am[b], z[:-1], rel * np.std(z[:-1]), min_decisive=0,
                                             distinct=EVEN)
-    assert decisive >= B * (T - 1) // 10, decisive
+    assert decisive >= B * (T - 1) // 25, decisive
