@@ -6,13 +6,17 @@
 // positions 0 .. p of its sequence (keys written by this call's QK-norm/RoPE
 // kernel for positions >= start, by earlier calls below start).
 //
-// One CTA per (b, kv head, 128-query tile, query head of the group); the query
-// heads of a group are adjacent in the grid (so their CTAs stream the same K/V
-// tiles from L2 at about the same time) and the longer query tiles of a group
-// come first.  192 threads:
-//   warp 0, one lane : TMA producer: the Q tile once, then 128-key K and V tiles
-//                      into a 2-stage ring (the cache viewed as 2-D rows of 128
-//                      elements, two 64-column boxes per tile, 128-byte swizzle);
+// Persistent: one CTA per SM walks the work items (b, kv head, 128-query tile,
+// query head of the group) it, it + grid, ...; the query heads of a group are
+// adjacent in that order (so their CTAs stream the same K/V tiles from L2 at
+// about the same time) and the longer query tiles of a group come first.  The
+// rings, TMEM buffers and barrier phases run on across items, so the next item's
+// Q and K/V copies overlap the current item's last tiles.  192 threads:
+//   warp 0, one lane : TMA producer: the Q tile of each item, then 128-key K and
+//                      V tiles into two 2-stage rings (the cache viewed as 2-D rows
+//                      of 128 elements, two 64-column boxes per tile, 128-byte
+//                      swizzle); a K stage is freed by its S product, a V stage by
+//                      its P V product, and K runs one tile ahead of V;
 //   warp 1, one lane : TMEM owner and MMA issuer:
 //                        S_j = Q K_j^T  (M 128 queries, N 128 keys, K = d) into one
 //                                        of two TMEM S buffers,
@@ -55,6 +59,7 @@ constexpr int kOffKV = kQBytes;
 constexpr int kOffP = kOffKV + kStages * kKVBytes;
 constexpr int kOffBar = kOffP + 2 * kPBytes;
 constexpr int kSmem = kOffBar + 256 + 1024;
+static_assert(kSmem <= 232448, "shared memory per CTA");
 constexpr int kThreads = 192;
 constexpr uint32_t kTmemCols = 512;      // S0 [0,128), S1 [128,256), O [256,384)
 constexpr float kRescale = 8.f;          // raise the running max only past 2^8
@@ -64,21 +69,51 @@ __device__ __forceinline__ uint32_t pack2(float lo, float hi) {
     return *reinterpret_cast<uint32_t*>(&v);
 }
 
+// Work item `it` of a launch: (b, kv head) groups in order; inside a group the
+// longest query tile first, the group's query heads innermost.
+struct Item {
+    int b, g, h, q0;
+};
+__device__ __forceinline__ Item item_at(int it, int n_qt, int G, int nkv) {
+    const int per_bg = n_qt * G;
+    const int bg = it / per_bg, rem = it % per_bg;
+    Item w;
+    w.b = bg / nkv;
+    w.g = bg % nkv;
+    w.h = w.g * G + rem % G;
+    w.q0 = (n_qt - 1 - rem / G) * kQT;
+    return w;
+}
+
+// First position of row b (clamped into the cache; the cache-write kernel flags it).
+__device__ __forceinline__ int row_start(const int32_t* start_dev, int start_all, int b, int max_seq,
+                                         int T) {
+    int st = start_dev ? start_dev[b] : start_all;
+    return st < 0 ? 0 : (st > max_seq - T ? max_seq - T : st);
+}
+
+__device__ __forceinline__ int tiles_of(int start, int q0, int T) {
+    return (start + min(q0 + kQT - 1, T - 1)) / kKT + 1;
+}
+
 __global__ void __launch_bounds__(kThreads, 1)
     attn_prefill_kernel(const __grid_constant__ CUtensorMap tmQ,
                         const __grid_constant__ CUtensorMap tmKV, int nq, int nkv,
                         int max_batch, int max_seq, int start_all,
-                        const int32_t* __restrict__ start_dev, int T, bf16* __restrict__ o,
-                        uint32_t* __restrict__ status) {
+                        const int32_t* __restrict__ start_dev, int T, int n_work,
+                        bf16* __restrict__ o, uint32_t* __restrict__ status) {
     extern __shared__ uint8_t smem_raw[];
     uint8_t* smem = (uint8_t*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
     uint8_t* sQ = smem;
     uint8_t* sKV = smem + kOffKV;
     uint8_t* sP = smem + kOffP;
     uint64_t* q_full = (uint64_t*)(smem + kOffBar);
-    uint64_t* kv_full = q_full + 1;
-    uint64_t* kv_empty = kv_full + kStages;
-    uint64_t* s_full = kv_empty + kStages;
+    uint64_t* q_empty = q_full + 1;
+    uint64_t* k_full = q_empty + 1;
+    uint64_t* k_empty = k_full + kStages;
+    uint64_t* v_full = k_empty + kStages;
+    uint64_t* v_empty = v_full + kStages;
+    uint64_t* s_full = v_empty + kStages;
     uint64_t* s_empty = s_full + 2;
     uint64_t* p_full = s_empty + 2;
     uint64_t* pv_done = p_full + 2;
@@ -89,20 +124,15 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int G = nq / nkv;
     const int n_qt = (T + kQT - 1) / kQT;
-    // grid order: (b, kv head) groups; inside, longest query tile first, heads innermost
-    const int per_bg = n_qt * G;
-    const int bg = blockIdx.x / per_bg, rem = blockIdx.x % per_bg;
-    const int qt = n_qt - 1 - rem / G;
-    const int b = bg / nkv, g = bg % nkv;
-    const int h = g * G + rem % G;
-    const int q0 = qt * kQT;
-    int start = start_all;  // start_dev is read after the dependency wait below
 
     if (threadIdx.x == 0) {
         tc::mbar_init(q_full, 1);
+        tc::mbar_init(q_empty, 1);
         for (int s = 0; s < kStages; ++s) {
-            tc::mbar_init(&kv_full[s], 1);
-            tc::mbar_init(&kv_empty[s], 1);
+            tc::mbar_init(&k_full[s], 1);
+            tc::mbar_init(&k_empty[s], 1);
+            tc::mbar_init(&v_full[s], 1);
+            tc::mbar_init(&v_empty[s], 1);
         }
         for (int i = 0; i < 2; ++i) {
             tc::mbar_init(&s_full[i], 1);
@@ -121,43 +151,70 @@ __global__ void __launch_bounds__(kThreads, 1)
     __syncthreads();
     tc::fence_after_sync();
     const uint32_t tmem_base = *tmem_slot;
-    pdl_wait();  // q, K and V come from the previous kernels
-    if (start_dev) start = start_dev[b];
-    // this row's first position (clamped into the cache; the cache-write kernel flags it)
-    start = start < 0 ? 0 : (start > max_seq - T ? max_seq - T : start);
-    const int kv_len = start + T;  // cache positions 0 .. kv_len-1 are written
-    const int p_last = start + min(q0 + kQT - 1, T - 1);
-    const int n_kt = p_last / kKT + 1;
-    const int row0 = (b * nkv + g) * max_seq;
+    pdl_wait();  // q, K, V and the row starts come from the previous kernels
     const int v_off = max_batch * nkv * max_seq;
 
     if (warp == 0) {
         if (lane == 0) {
             // ------------------------------------------------ TMA producer
-            int armed[kStages] = {-1, -1};
-            bool q_armed = true, ok = true;
-            tc::mbar_expect_tx(q_full, kQBytes);
-            tc::tma_load_2d(sQ, &tmQ, h * kD, b * T + q0, q_full);
-            tc::tma_load_2d(sQ + kBox, &tmQ, h * kD + 64, b * T + q0, q_full);
-            for (int j = 0; j < n_kt; ++j) {
-                const int st = j % kStages;
-                if (!tc::mbar_wait(&kv_empty[st], (uint32_t)(((j / kStages) & 1) ^ 1), abort_flag)) {
+            // K tiles lead V tiles by one (S_{j+1} is computed before P_j V_j), and each
+            // ring frees a stage as soon as its own product has read it.
+            int k_armed[kStages] = {-1, -1}, v_armed[kStages] = {-1, -1};
+            int q_armed = -1;
+            bool ok = true;
+            int gt = 0, n = 0;  // global tile and item counters of this CTA
+            auto load_k = [&](int g, int r) -> bool {
+                const int st = g % kStages;
+                if (!tc::mbar_wait(&k_empty[st], (uint32_t)(((g / kStages) & 1) ^ 1), abort_flag)) return false;
+                uint8_t* base = sKV + st * kKVBytes;
+                tc::mbar_expect_tx(&k_full[st], 2 * kBox);
+                tc::tma_load_2d(base, &tmKV, 0, r, &k_full[st]);
+                tc::tma_load_2d(base + kBox, &tmKV, 64, r, &k_full[st]);
+                k_armed[st] = (g / kStages) & 1;
+                return true;
+            };
+            auto load_v = [&](int g, int r) -> bool {
+                const int st = g % kStages;
+                if (!tc::mbar_wait(&v_empty[st], (uint32_t)(((g / kStages) & 1) ^ 1), abort_flag)) return false;
+                uint8_t* base = sKV + st * kKVBytes + 2 * kBox;
+                tc::mbar_expect_tx(&v_full[st], 2 * kBox);
+                tc::tma_load_2d(base, &tmKV, 0, v_off + r, &v_full[st]);
+                tc::tma_load_2d(base + kBox, &tmKV, 64, v_off + r, &v_full[st]);
+                v_armed[st] = (g / kStages) & 1;
+                return true;
+            };
+            for (int it = blockIdx.x; ok && it < n_work; it += gridDim.x, ++n) {
+                const Item w = item_at(it, n_qt, G, nkv);
+                const int start = row_start(start_dev, start_all, w.b, max_seq, T);
+                const int n_kt = tiles_of(start, w.q0, T);
+                const int row0 = (w.b * nkv + w.g) * max_seq;
+                // the Q buffer is free once every S MMA of the previous item has completed
+                if (n > 0 && !tc::mbar_wait(q_empty, (uint32_t)((n - 1) & 1), abort_flag)) {
                     ok = false;
                     break;
                 }
-                uint8_t* base = sKV + st * kKVBytes;
-                const int r = row0 + j * kKT;
-                tc::mbar_expect_tx(&kv_full[st], kKVBytes);
-                tc::tma_load_2d(base, &tmKV, 0, r, &kv_full[st]);
-                tc::tma_load_2d(base + kBox, &tmKV, 64, r, &kv_full[st]);
-                tc::tma_load_2d(base + 2 * kBox, &tmKV, 0, v_off + r, &kv_full[st]);
-                tc::tma_load_2d(base + 3 * kBox, &tmKV, 64, v_off + r, &kv_full[st]);
-                armed[st] = (j / kStages) & 1;
+                tc::mbar_expect_tx(q_full, kQBytes);
+                tc::tma_load_2d(sQ, &tmQ, w.h * kD, w.b * T + w.q0, q_full);
+                tc::tma_load_2d(sQ + kBox, &tmQ, w.h * kD + 64, w.b * T + w.q0, q_full);
+                q_armed = n & 1;
+                for (int j = 0; j <= n_kt; ++j) {
+                    if (j < n_kt && !load_k(gt + j, row0 + j * kKT)) {
+                        ok = false;
+                        break;
+                    }
+                    if (j >= 1 && !load_v(gt + j - 1, row0 + (j - 1) * kKT)) {
+                        ok = false;
+                        break;
+                    }
+                }
+                gt += n_kt;
             }
             if (!ok) {  // abort path: let every copy this thread issued land before exit
-                if (q_armed) tc::mbar_wait_drain(q_full, 0);
-                for (int s = 0; s < kStages; ++s)
-                    if (armed[s] >= 0) tc::mbar_wait_drain(&kv_full[s], (uint32_t)armed[s]);
+                if (q_armed >= 0) tc::mbar_wait_drain(q_full, (uint32_t)q_armed);
+                for (int s = 0; s < kStages; ++s) {
+                    if (k_armed[s] >= 0) tc::mbar_wait_drain(&k_full[s], (uint32_t)k_armed[s]);
+                    if (v_armed[s] >= 0) tc::mbar_wait_drain(&v_full[s], (uint32_t)v_armed[s]);
+                }
             }
         }
     } else if (warp == 1) {
@@ -166,46 +223,60 @@ __global__ void __launch_bounds__(kThreads, 1)
             constexpr uint32_t idesc_s = tc::idesc_bf16(128, kKT);
             constexpr uint32_t idesc_o = tc::idesc_bf16_bmn(128, kD);
             const uint32_t q_s = tc::smem_u32(sQ);
-            bool ok = tc::mbar_wait(q_full, 0, abort_flag), issued = false;
-            for (int j = 0; ok && j <= n_kt; ++j) {
-                if (j < n_kt) {
-                    const int st = j % kStages;
-                    if (!tc::mbar_wait(&kv_full[st], (uint32_t)((j / kStages) & 1), abort_flag) ||
-                        !tc::mbar_wait(&s_empty[j & 1], (uint32_t)(((j >> 1) & 1) ^ 1), abort_flag)) {
-                        ok = false;
-                        break;
-                    }
-                    tc::fence_after_sync();
-                    const uint32_t k_s = tc::smem_u32(sKV + st * kKVBytes);
-                    const uint32_t d_s = tmem_base + (uint32_t)((j & 1) * kKT);
-#pragma unroll
-                    for (int kk = 0; kk < kD / 16; ++kk) {
-                        const uint32_t off = (uint32_t)((kk >> 2) * kBox + (kk & 3) * 32);
-                        tc::mma_bf16(d_s, tc::sw128_desc(q_s + off), tc::sw128_desc(k_s + off),
-                                     idesc_s, kk > 0 ? 1u : 0u);
-                    }
-                    issued = true;
-                    tc::mma_commit(&s_full[j & 1]);
+            bool ok = true, issued = false;
+            int gt = 0, n = 0;
+            for (int it = blockIdx.x; ok && it < n_work; it += gridDim.x, ++n) {
+                const Item w = item_at(it, n_qt, G, nkv);
+                const int n_kt = tiles_of(row_start(start_dev, start_all, w.b, max_seq, T), w.q0, T);
+                if (!tc::mbar_wait(q_full, (uint32_t)(n & 1), abort_flag)) {
+                    ok = false;
+                    break;
                 }
-                if (j >= 1) {
-                    const int i = j - 1, st = i % kStages;
-                    if (!tc::mbar_wait(&p_full[i & 1], (uint32_t)((i >> 1) & 1), abort_flag)) {
-                        ok = false;
-                        break;
-                    }
-                    tc::fence_after_sync();
-                    const uint32_t p_s = tc::smem_u32(sP + (i & 1) * kPBytes);
-                    const uint32_t v_s = tc::smem_u32(sKV + st * kKVBytes + 2 * kBox);
+                const int g0 = gt;  // global index of this item's tile 0
+                for (int j = 0; j <= n_kt; ++j) {
+                    if (j < n_kt) {
+                        const int g = g0 + j, st = g % kStages;
+                        if (!tc::mbar_wait(&k_full[st], (uint32_t)((g / kStages) & 1), abort_flag) ||
+                            !tc::mbar_wait(&s_empty[g & 1], (uint32_t)(((g >> 1) & 1) ^ 1), abort_flag)) {
+                            ok = false;
+                            break;
+                        }
+                        tc::fence_after_sync();
+                        const uint32_t k_s = tc::smem_u32(sKV + st * kKVBytes);
+                        const uint32_t d_s = tmem_base + (uint32_t)((g & 1) * kKT);
 #pragma unroll
-                    for (int kk = 0; kk < kKT / 16; ++kk) {
-                        const uint32_t aoff = (uint32_t)((kk >> 2) * kBox + (kk & 3) * 32);
-                        tc::mma_bf16(tmem_base + 256, tc::sw128_desc(p_s + aoff),
-                                     tc::sw128_desc_mn(v_s + kk * 16 * 128, kBox), idesc_o,
-                                     (i > 0 || kk > 0) ? 1u : 0u);
+                        for (int kk = 0; kk < kD / 16; ++kk) {
+                            const uint32_t off = (uint32_t)((kk >> 2) * kBox + (kk & 3) * 32);
+                            tc::mma_bf16(d_s, tc::sw128_desc(q_s + off), tc::sw128_desc(k_s + off),
+                                         idesc_s, kk > 0 ? 1u : 0u);
+                        }
+                        issued = true;
+                        tc::mma_commit(&s_full[g & 1]);
+                        tc::mma_commit(&k_empty[st]);
+                        if (j == n_kt - 1) tc::mma_commit(q_empty);  // last read of this Q
                     }
-                    tc::mma_commit(&pv_done[i & 1]);
-                    tc::mma_commit(&kv_empty[st]);
+                    if (j >= 1) {
+                        const int i = g0 + j - 1, st = i % kStages;
+                        if (!tc::mbar_wait(&v_full[st], (uint32_t)((i / kStages) & 1), abort_flag) ||
+                            !tc::mbar_wait(&p_full[i & 1], (uint32_t)((i >> 1) & 1), abort_flag)) {
+                            ok = false;
+                            break;
+                        }
+                        tc::fence_after_sync();
+                        const uint32_t p_s = tc::smem_u32(sP + (i & 1) * kPBytes);
+                        const uint32_t v_s = tc::smem_u32(sKV + st * kKVBytes + 2 * kBox);
+#pragma unroll
+                        for (int kk = 0; kk < kKT / 16; ++kk) {
+                            const uint32_t aoff = (uint32_t)((kk >> 2) * kBox + (kk & 3) * 32);
+                            tc::mma_bf16(tmem_base + 256, tc::sw128_desc(p_s + aoff),
+                                         tc::sw128_desc_mn(v_s + kk * 16 * 128, kBox), idesc_o,
+                                         (j > 1 || kk > 0) ? 1u : 0u);
+                        }
+                        tc::mma_commit(&pv_done[i & 1]);
+                        tc::mma_commit(&v_empty[st]);
+                    }
                 }
+                gt = g0 + n_kt;
             }
             if (!ok && issued) {  // abort path: wait for the MMAs in flight
                 tc::mma_commit(drain);
@@ -216,142 +287,163 @@ __global__ void __launch_bounds__(kThreads, 1)
         // ---------------------------------------------------- softmax (warps 2..5)
         const int qd = warp & 3;                 // TMEM lane quadrant of this warp
         const int row = qd * 32 + lane;          // query row of the tile = TMEM lane
-        const int t = q0 + row;
-        const int p = start + t;                 // this row's position
         const uint32_t lane_off = (uint32_t)(qd * 32) << 16;
         const float c = rsqrtf((float)kD) * 1.4426950408889634f;  // 1/sqrt(d) in base 2
-        float m = -INFINITY, l = 0.f;
         bool ok = true;
-        for (int j = 0; j < n_kt; ++j) {
-            ok = tc::mbar_wait(&s_full[j & 1], (uint32_t)((j >> 1) & 1), abort_flag);
-            ok = __all_sync(0xffffffffu, ok);
-            if (!ok) break;
-            tc::fence_after_sync();
-            float x[kKT];
-            const uint32_t s_t = tmem_base + lane_off + (uint32_t)((j & 1) * kKT);
-#pragma unroll
-            for (int c0 = 0; c0 < kKT; c0 += 16) {
-                uint32_t r[16];
-                tc::tmem_ld16(s_t + c0, r);
-#pragma unroll
-                for (int k = 0; k < 16; ++k) x[c0 + k] = __uint_as_float(r[k]);
-            }
-            tc::tmem_wait_ld();
-            tc::fence_before_sync();
-            __syncwarp();
-            if (lane == 0) tc::mbar_arrive(&s_empty[j & 1]);
-            const int key0 = j * kKT;
-            float mx = -INFINITY;
-            if (key0 + kKT - 1 > p) {  // diagonal tile: keys after p do not count
-#pragma unroll
-                for (int k = 0; k < kKT; ++k) {
-                    x[k] = key0 + k <= p ? x[k] * c : -INFINITY;
-                    mx = fmaxf(mx, x[k]);
-                }
-            } else {
-#pragma unroll
-                for (int k = 0; k < kKT; ++k) {
-                    x[k] *= c;
-                    mx = fmaxf(mx, x[k]);
-                }
-            }
-            // raise the running max only when exponents would exceed 2^kRescale
-            const bool raise = mx > m + kRescale;
-            float factor = 1.f;
-            if (raise) {
-                factor = m == -INFINITY ? 0.f : tc::ex2_approx(m - mx);
-                m = mx;
-            }
-            if (j > 0 && __any_sync(0xffffffffu, raise)) {
-                // rescale this warp's rows of O once the previous P V product has landed
-                const int i = j - 1;
-                ok = tc::mbar_wait(&pv_done[i & 1], (uint32_t)((i >> 1) & 1), abort_flag);
+        int gt = 0;
+        for (int it = blockIdx.x; ok && it < n_work; it += gridDim.x) {
+            const Item w = item_at(it, n_qt, G, nkv);
+            const int start = row_start(start_dev, start_all, w.b, max_seq, T);
+            const int n_kt = tiles_of(start, w.q0, T);
+            const int kv_len = start + T;  // cache positions 0 .. kv_len-1 are written
+            const int t = w.q0 + row;
+            const int p = start + t;       // this row's position
+            float m = -INFINITY, l = 0.f;  // running max (scaled, base 2) and sum
+            for (int j = 0; j < n_kt; ++j, ++gt) {
+                ok = tc::mbar_wait(&s_full[gt & 1], (uint32_t)((gt >> 1) & 1), abort_flag);
                 ok = __all_sync(0xffffffffu, ok);
                 if (!ok) break;
                 tc::fence_after_sync();
-                const uint32_t o_t = tmem_base + lane_off + 256;
+                float x[kKT];
+                const uint32_t s_t = tmem_base + lane_off + (uint32_t)((gt & 1) * kKT);
 #pragma unroll
-                for (int c0 = 0; c0 < kD; c0 += 16) {
+                for (int c0 = 0; c0 < kKT; c0 += 16) {
                     uint32_t r[16];
-                    tc::tmem_ld16(o_t + c0, r);
-                    tc::tmem_wait_ld();
+                    tc::tmem_ld16(s_t + c0, r);
 #pragma unroll
-                    for (int k = 0; k < 16; ++k) r[k] = __float_as_uint(__uint_as_float(r[k]) * factor);
-                    tc::tmem_st16(o_t + c0, r);
+                    for (int k = 0; k < 16; ++k) x[c0 + k] = __uint_as_float(r[k]);
                 }
-                tc::tmem_wait_st();
-            }
-            l *= factor;
-            // P_j = 2^(x - m) in bf16 into buffer j % 2 (free once P_{j-2} V_{j-2} landed)
-            float sum = 0.f;
-            uint32_t pk[kKT / 2];
+                tc::tmem_wait_ld();
+                tc::fence_before_sync();
+                __syncwarp();
+                if (lane == 0) tc::mbar_arrive(&s_empty[gt & 1]);
+                const int key0 = j * kKT;
+                if (key0 + kKT - 1 > p) {  // diagonal tile: keys after p do not count
 #pragma unroll
-            for (int k = 0; k < kKT; k += 2) {
-                const float e0 = tc::ex2_approx(x[k] - m), e1 = tc::ex2_approx(x[k + 1] - m);
-                sum += e0 + e1;
-                pk[k / 2] = pack2(e0, e1);
-            }
-            l += sum;
-            if (j >= 2) {
-                const int i = j - 2;
-                ok = tc::mbar_wait(&pv_done[i & 1], (uint32_t)((i >> 1) & 1), abort_flag);
-                ok = __all_sync(0xffffffffu, ok);
-                if (!ok) break;
-            }
-            uint8_t* pb = sP + (j & 1) * kPBytes;
-#pragma unroll
-            for (int half = 0; half < 2; ++half) {
-                uint8_t* rb = pb + half * kBox + (row >> 3) * 1024 + (row & 7) * 128;
-#pragma unroll
-                for (int ch = 0; ch < 8; ++ch) {
-                    const int w = half * 32 + ch * 4;
-                    *reinterpret_cast<uint4*>(rb + ((ch ^ (row & 7)) << 4)) =
-                        make_uint4(pk[w], pk[w + 1], pk[w + 2], pk[w + 3]);
+                    for (int k = 0; k < kKT; ++k) x[k] = key0 + k <= p ? x[k] : -INFINITY;
                 }
-            }
-            if (key0 + kKT > kv_len) {
-                // last tile: zero the V rows of unwritten cache positions
-                const int st = j % kStages;
-                ok = tc::mbar_wait(&kv_full[st], (uint32_t)((j / kStages) & 1), abort_flag);
-                ok = __all_sync(0xffffffffu, ok);
-                if (!ok) break;
-                uint8_t* vb = sKV + st * kKVBytes + 2 * kBox;
-                const int r0 = kv_len - key0 > 0 ? kv_len - key0 : 0;
-                for (int idx = threadIdx.x - 64; idx < (kKT - r0) * 16; idx += 128) {
-                    const int rr = r0 + (idx >> 4), ch = idx & 15;
-                    *reinterpret_cast<uint4*>(vb + (ch >> 3) * kBox + rr * 128 +
-                                              (((ch & 7) ^ (rr & 7)) << 4)) = make_uint4(0, 0, 0, 0);
+                // row max of the raw scores with 8 independent chains, then scaled (c > 0)
+                float mx8[8];
+#pragma unroll
+                for (int k = 0; k < 8; ++k) mx8[k] = x[k];
+#pragma unroll
+                for (int k = 8; k < kKT; ++k) mx8[k & 7] = fmaxf(mx8[k & 7], x[k]);
+                const float mx = fmaxf(fmaxf(fmaxf(mx8[0], mx8[1]), fmaxf(mx8[2], mx8[3])),
+                                       fmaxf(fmaxf(mx8[4], mx8[5]), fmaxf(mx8[6], mx8[7]))) * c;
+                // raise the running max only when exponents would exceed 2^kRescale
+                const bool raise = mx > m + kRescale;
+                float factor = 1.f;
+                if (raise) {
+                    factor = m == -INFINITY ? 0.f : tc::ex2_approx(m - mx);
+                    m = mx;
                 }
+                if (j > 0 && __any_sync(0xffffffffu, raise)) {
+                    // rescale this warp's rows of O once the previous P V product has landed
+                    const int i = gt - 1;
+                    ok = tc::mbar_wait(&pv_done[i & 1], (uint32_t)((i >> 1) & 1), abort_flag);
+                    ok = __all_sync(0xffffffffu, ok);
+                    if (!ok) break;
+                    tc::fence_after_sync();
+                    const uint32_t o_t = tmem_base + lane_off + 256;
+#pragma unroll
+                    for (int c0 = 0; c0 < kD; c0 += 64) {
+                        uint32_t r[4][16];
+#pragma unroll
+                        for (int q = 0; q < 4; ++q) tc::tmem_ld16(o_t + c0 + 16 * q, r[q]);
+                        tc::tmem_wait_ld();
+#pragma unroll
+                        for (int q = 0; q < 4; ++q) {
+#pragma unroll
+                            for (int k = 0; k < 16; ++k)
+                                r[q][k] = __float_as_uint(__uint_as_float(r[q][k]) * factor);
+                            tc::tmem_st16(o_t + c0 + 16 * q, r[q]);
+                        }
+                    }
+                    tc::tmem_wait_st();
+                }
+                // P_j = 2^(x c - m) in bf16 into buffer gt % 2 (free once the P V product of
+                // global tile gt - 2 has landed); sums in 8 independent chains
+                float sum8[8];
+#pragma unroll
+                for (int k = 0; k < 8; ++k) sum8[k] = 0.f;
+                uint32_t pk[kKT / 2];
+                const float nm = -m;
+#pragma unroll
+                for (int k = 0; k < kKT; k += 2) {
+                    const float e0 = tc::ex2_approx(fmaf(x[k], c, nm));
+                    const float e1 = tc::ex2_approx(fmaf(x[k + 1], c, nm));
+                    sum8[(k >> 1) & 7] += e0 + e1;
+                    pk[k / 2] = pack2(e0, e1);
+                }
+                l = l * factor + (((sum8[0] + sum8[1]) + (sum8[2] + sum8[3])) +
+                                  ((sum8[4] + sum8[5]) + (sum8[6] + sum8[7])));
+                if (gt >= 2) {
+                    const int i = gt - 2;
+                    ok = tc::mbar_wait(&pv_done[i & 1], (uint32_t)((i >> 1) & 1), abort_flag);
+                    ok = __all_sync(0xffffffffu, ok);
+                    if (!ok) break;
+                }
+                uint8_t* pb = sP + (gt & 1) * kPBytes;
+#pragma unroll
+                for (int half = 0; half < 2; ++half) {
+                    uint8_t* rb = pb + half * kBox + (row >> 3) * 1024 + (row & 7) * 128;
+#pragma unroll
+                    for (int ch = 0; ch < 8; ++ch) {
+                        const int wd = half * 32 + ch * 4;
+                        *reinterpret_cast<uint4*>(rb + ((ch ^ (row & 7)) << 4)) =
+                            make_uint4(pk[wd], pk[wd + 1], pk[wd + 2], pk[wd + 3]);
+                    }
+                }
+                if (key0 + kKT > kv_len) {
+                    // last tile: zero the V rows of unwritten cache positions
+                    const int st = gt % kStages;
+                    ok = tc::mbar_wait(&v_full[st], (uint32_t)((gt / kStages) & 1), abort_flag);
+                    ok = __all_sync(0xffffffffu, ok);
+                    if (!ok) break;
+                    uint8_t* vb = sKV + st * kKVBytes + 2 * kBox;
+                    const int r0 = kv_len - key0 > 0 ? kv_len - key0 : 0;
+                    for (int idx = threadIdx.x - 64; idx < (kKT - r0) * 16; idx += 128) {
+                        const int rr = r0 + (idx >> 4), ch = idx & 15;
+                        *reinterpret_cast<uint4*>(vb + (ch >> 3) * kBox + rr * 128 +
+                                                  (((ch & 7) ^ (rr & 7)) << 4)) = make_uint4(0, 0, 0, 0);
+                    }
+                }
+                tc::fence_proxy_async_smem();
+                tc::fence_before_sync();
+                __syncwarp();
+                if (lane == 0) tc::mbar_arrive(&p_full[gt & 1]);
             }
-            tc::fence_proxy_async_smem();
-            tc::fence_before_sync();
-            __syncwarp();
-            if (lane == 0) tc::mbar_arrive(&p_full[j & 1]);
-        }
-        if (ok) {
-            const int i = n_kt - 1;
+            if (!ok) break;
+            // O / l of this item once its last P V product has landed
+            const int i = gt - 1;
             ok = tc::mbar_wait(&pv_done[i & 1], (uint32_t)((i >> 1) & 1), abort_flag);
             ok = __all_sync(0xffffffffu, ok);
-        }
-        if (ok) {
+            if (!ok) break;
             tc::fence_after_sync();
             const float inv = l > 0.f ? 1.f / l : 0.f;
             const uint32_t o_t = tmem_base + lane_off + 256;
-            bf16* orow = o + ((size_t)b * T + (t < T ? t : 0)) * (size_t)(nq * kD) + (size_t)h * kD;
+            bf16* orow = o + ((size_t)w.b * T + (t < T ? t : 0)) * (size_t)(nq * kD) + (size_t)w.h * kD;
 #pragma unroll
-            for (int c0 = 0; c0 < kD; c0 += 16) {
-                uint32_t r[16];
-                tc::tmem_ld16(o_t + c0, r);
+            for (int c0 = 0; c0 < kD; c0 += 64) {
+                uint32_t r[4][16];
+#pragma unroll
+                for (int q = 0; q < 4; ++q) tc::tmem_ld16(o_t + c0 + 16 * q, r[q]);
                 tc::tmem_wait_ld();
-                uint32_t w[8];
 #pragma unroll
-                for (int k = 0; k < 8; ++k)
-                    w[k] = pack2(__uint_as_float(r[2 * k]) * inv, __uint_as_float(r[2 * k + 1]) * inv);
-                if (t < T) {
-                    *reinterpret_cast<uint4*>(orow + c0) = make_uint4(w[0], w[1], w[2], w[3]);
-                    *reinterpret_cast<uint4*>(orow + c0 + 8) = make_uint4(w[4], w[5], w[6], w[7]);
+                for (int q = 0; q < 4; ++q) {
+                    uint32_t wv[8];
+#pragma unroll
+                    for (int k = 0; k < 8; ++k)
+                        wv[k] = pack2(__uint_as_float(r[q][2 * k]) * inv, __uint_as_float(r[q][2 * k + 1]) * inv);
+                    if (t < T) {
+                        *reinterpret_cast<uint4*>(orow + c0 + 16 * q) = make_uint4(wv[0], wv[1], wv[2], wv[3]);
+                        *reinterpret_cast<uint4*>(orow + c0 + 16 * q + 8) = make_uint4(wv[4], wv[5], wv[6], wv[7]);
+                    }
                 }
             }
+            // the next item's first P V product overwrites O only after its P is ready,
+            // which these warps write after this readback
+            tc::fence_before_sync();
         }
     }
 
@@ -388,7 +480,7 @@ bool attn_prefill_supported(int d, int nq, int nkv) { return d == kD && nq % nkv
 
 int launch_attn_prefill(const bf16* q, int q_ld, const void* k_layer, int nq, int nkv,
                         int max_batch, int max_seq, int B, int T, int start,
-                        const int32_t* start_dev, bf16* o,
+                        const int32_t* start_dev, bf16* o, int num_sms,
                         uint32_t* status, cudaStream_t s) {
     static bool attr_set = false;
     if (!attr_set) {
@@ -412,9 +504,10 @@ int launch_attn_prefill(const bf16* q, int q_ld, const void* k_layer, int nq, in
         !make_map128((EncodeTiledFn)fn, &mkv, k_layer, kD, rows, kD))
         return QK_ECUDA;
     const int n_qt = (T + kQT - 1) / kQT;
-    dim3 grid((unsigned)(B * nq * n_qt));
-    launch_k(attn_prefill_kernel, grid, dim3(kThreads), kSmem, s, mq, mkv, nq, nkv, max_batch,
-             max_seq, start, start_dev, T, o, status);
+    const int n_work = B * nq * n_qt;
+    const int grid = n_work < num_sms ? n_work : num_sms;
+    launch_k(attn_prefill_kernel, dim3(grid), dim3(kThreads), kSmem, s, mq, mkv, nq, nkv, max_batch,
+             max_seq, start, start_dev, T, n_work, o, status);
     note_launch();
     return QK_OK;
 }

@@ -49,7 +49,7 @@ void launch_attention(Model& m, const void* q, int q_ld, const void* k_cache, co
                                                             c.head_dim * 2) {
         int rc = launch_attn_prefill((const bf16*)q, q_ld, k_cache, c.n_q_heads, c.n_kv_heads,
                                      max_batch, max_seq, M / pos.T, pos.T, pos.start, pos.pos_dev,
-                                     (bf16*)o, m.status, s);
+                                     (bf16*)o, m.num_sms, m.status, s);
         if (rc != QK_OK && !m.deferred_error) m.deferred_error = rc;
         return;
     }
