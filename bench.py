@@ -240,7 +240,7 @@ def run_ours(args, world, rank, local):
 
     # ---- timed region: K whole rollouts, device-resident inputs
     n_layers = s.n_layers
-    qk.qk_profile_begin(dec.handle, qk.QK_PROF_GATE_UP, args.steps * N * n_layers)
+    qk.qk_profile_begin(dec.handle, qk.QK_PROF_STEP, args.steps * N)
     clocks = ClockSampler(local)
     barrier(world)
     torch.cuda.synchronize(dev)
@@ -261,13 +261,20 @@ def run_ours(args, world, rank, local):
         raise RuntimeError("device status flags set during the timed region")
     value = world * B * N / (ms_step / 1e3)
 
-    # ---- prefill alone (for the prefill tokens/s figure)
+    # ---- prefill alone (for the prefill tokens/s figure), warmed up first: its workspace
+    # kind differs from the rollout's
     pz = torch.empty(B, dtype=torch.float32, device=dev)
+
+    def prefill():
+        dec.prefill(kv, B, P + N, seq_d[:, :P].contiguous(), 0, None, seq_d[:, P].contiguous(), pz)
+
+    for _ in range(2):
+        prefill()
     torch.cuda.synchronize(dev)
     p0, p1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     p0.record(stream)
     for _ in range(args.steps):
-        dec.prefill(kv, B, P + N, seq_d[:, :P].contiguous(), 0, None, seq_d[:, P].contiguous(), pz)
+        prefill()
     p1.record(stream)
     torch.cuda.synchronize(dev)
     prefill_ms = p0.elapsed_time(p1) / args.steps
@@ -308,6 +315,9 @@ def run_ours(args, world, rank, local):
     if dec.check_status() != 0 or not torch.isfinite(score_lp).all():
         raise RuntimeError("scoring produced invalid output")
     del score_tok, score_lp
+    dec._ws.clear()
+    torch.cuda.empty_cache()
+    decode_configs = other_decode_configs(dec, dev, stream, rank)
 
     if rank != 0:
         return
@@ -315,18 +325,26 @@ def run_ours(args, world, rank, local):
     hbm_peak = peaks["hbm_gbs"] if peaks else 6800.0
     bf16_peak = peaks["bf16_tflops"] if peaks else 1900.0
     c = dec.cfg
-    gu_bytes = 2 * c.intermediate * c.hidden * 2 + B * c.hidden * 2 + B * c.intermediate * 2
-    avg_launch_s = (prof_ms / max(prof_n, 1)) / 1e3
-    achieved = gu_bytes / avg_launch_s / 1e9
-    roofline = {"bound": "hbm", "kernel": "decode gate/up linear (tcgen05 stream-K GEMM, 16 token rows)",
-                "timed_launches": "the gate/up launches of each timed rollout's first decode step "
-                                  "(later steps replay a captured CUDA graph without event nodes)",
+    if prof_n < 1:
+        raise RuntimeError("no decode-step launch was bracketed")
+    # the bracketed launch: decode step 0 of each timed rollout (position P, keys 0 .. P);
+    # weights of every layer and the lm_head, the K/V read, the K/V written, activations
+    step0_bytes = (STEP_WEIGHT_BYTES + B * (P + 1) * KV_BYTES_PER_TOKEN
+                   + c.n_layers * B * (3 * c.hidden * 4 + c.intermediate * 2 * 2)
+                   + B * c.vocab * 4)
+    avg_launch_s = (prof_ms / prof_n) / 1e3
+    achieved = step0_bytes / avg_launch_s / 1e9
+    roofline = {"bound": "hbm",
+                "kernel": "persistent decode-step kernel (36 layers + lm_head in one cooperative launch, "
+                          "16 token rows)",
+                "timed_launches": "decode step 0 of each timed rollout (later steps replay a captured "
+                                  "CUDA graph without event nodes)",
                 "achieved": achieved, "peak": hbm_peak, "unit": "GB/s",
                 "frac": achieved / hbm_peak,
                 "peak_source": "measured" if peaks else "fallback",
-                "algorithmic_bytes_per_launch": gu_bytes, "launches_timed": prof_n,
+                "algorithmic_bytes_per_launch": int(step0_bytes), "launches_timed": prof_n,
                 "avg_launch_us": avg_launch_s * 1e6,
-                "traffic": recorded_traffic("gate_up_decode_b16")}
+                "traffic": recorded_traffic("decode_step_b16")}
     step_bytes = 15136811008 + B * sum(P + j + 1 for j in range(N)) * 147456 / N
     line = {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": ms_step, "higher_is_better": True,
@@ -343,6 +361,7 @@ def run_ours(args, world, rank, local):
                                "frac": SCORE_FLOPS / score_s / 1e12 / bf16_peak,
                                "peak_source": "measured (burst)" if peaks else "fallback"},
             "decode_hbm_fraction_of_8tbs": (step_bytes * N / 1e9) / ((ms_step - prefill_ms) / 1e3) / 8000.0,
+            "decode_configs": decode_configs,
             "roofline": roofline, "clocks": clk, "gpu_launches": int(launches),
             "launches_before_timed": int(launches0),
             "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": int(seq.nbytes),
@@ -351,6 +370,112 @@ def run_ours(args, world, rank, local):
         v, dt, _ = oracle_sample(s, W, seq[0])
         line["cpu_baseline"] = cpu_baseline_entry(v, dt)
     print(json.dumps(line), flush=True)
+
+
+# --------------------------------------------------------------------------- other decode configs
+LAYER_WEIGHT_BYTES = 385875968        # one Qwen3-8B layer: qkv, o, gate/up, down (bf16)
+STEP_WEIGHT_BYTES = 15136811008       # 36 layers + lm_head + norms
+KV_BYTES_PER_TOKEN_LAYER = 4096       # K and V of 8 kv heads x 128 dims, bf16
+KV_BYTES_PER_TOKEN = 36 * KV_BYTES_PER_TOKEN_LAYER
+
+
+def _hbm_entry(bytes_per_step, step_s, hbm_peak, tokens_per_step):
+    gbs = bytes_per_step / step_s / 1e9
+    return {"tokens_per_s": tokens_per_step / step_s, "us_per_step": step_s * 1e6,
+            "bytes_per_step": int(bytes_per_step), "achieved_gbs": gbs,
+            "frac_of_measured_hbm": gbs / hbm_peak, "frac_of_8tbs": gbs / 8000.0}
+
+
+def _event_time(fn, reps, stream):
+    import torch
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(reps):
+        fn()
+    e1.record(stream)
+    torch.cuda.synchronize()
+    return e0.elapsed_time(e1) / 1e3 / reps
+
+
+def other_decode_configs(dec, dev, stream, rank):
+    """Decode throughput of the other decode workloads, each against its HBM roofline
+    (weight + KV bytes per step):
+      * batch-1 rollout decode of the 36-layer model (prompt 512, 256 teacher-forced steps);
+      * one 8B layer's decode step at batch 1 / 8 / 32 / 64 over a 2048-entry N(0, 1) cache
+        (new token at position 2048; layer 0 of the loaded model);
+      * the 36-layer model at batch 64 over a long cache (N(0, 1) entries), decode steps at
+        positions 4096, 6144 and 8191 (KV context 4097 .. 8192)."""
+    import torch
+    import synth
+    from paper_2609_12471_gb300 import _binding as qkb
+    peaks = measured_peaks()
+    hbm = peaks["hbm_gbs"] if peaks else 6800.0
+    gen = torch.Generator(device=dev)
+    gen.manual_seed(2)
+    out = {}
+    c = dec.cfg
+    # -- batch-1 rollout
+    P1, N1 = 512, 256
+    seq1 = torch.tensor(synth.tokens((1, P1 + N1 + 1), c.vocab, stream=300 + rank), dtype=torch.int32,
+                        device=dev)
+    kv1 = dec.new_kv(1, P1 + N1)
+    lp1 = torch.empty(1, N1 + 1, dtype=torch.float32, device=dev)
+    pz1 = torch.empty(1, dtype=torch.float32, device=dev)
+    roll = lambda: dec.rollout(kv1, 1, P1 + N1, seq1, P1, logprobs=lp1)
+    pre = lambda: dec.prefill(kv1, 1, P1 + N1, seq1[:, :P1].contiguous(), 0, None,
+                              seq1[:, P1].contiguous(), pz1)
+    for _ in range(2):
+        roll()
+        pre()
+    t_roll = _event_time(roll, 2, stream)
+    t_pre = _event_time(pre, 3, stream)
+    step_s = (t_roll - t_pre) / N1
+    kv_mean = sum(P1 + j + 1 for j in range(N1)) / N1 * KV_BYTES_PER_TOKEN
+    out["batch1_rollout"] = dict(_hbm_entry(STEP_WEIGHT_BYTES + kv_mean, step_s, hbm, 1),
+                                 workload="36 layers, batch 1, prompt 512, 256 teacher-forced steps")
+    del kv1
+    # -- one layer, KV 2048, batch 1 / 8 / 32 / 64
+    S = 2048
+    layer = {}
+    for Bn in (1, 8, 32, 64):
+        half = Bn * c.n_kv_heads * (S + 1) * c.head_dim
+        kvl = torch.empty(2 * half, dtype=torch.bfloat16, device=dev)
+        kvl.normal_(generator=gen)
+        x = torch.randn(Bn, c.hidden, generator=gen, device=dev)
+        pos = torch.full((Bn,), S, dtype=torch.int32, device=dev)
+        ws = dec.workspace(qkb.QK_CALL_DECODE, Bn, 1, S + 1)
+        f = lambda: qkb.qk_decode_layer(dec.handle, 0, kvl, Bn, S + 1, x, pos, Bn, ws)
+        for _ in range(5):
+            f()
+        t = _event_time(f, 50, stream)
+        layer[str(Bn)] = _hbm_entry(LAYER_WEIGHT_BYTES + Bn * S * KV_BYTES_PER_TOKEN_LAYER, t, hbm, Bn)
+        del kvl
+    out["one_layer_kv2048"] = layer
+    if dec.check_status() != 0:
+        raise RuntimeError("device status flags set in the one-layer decode configs")
+    # -- 36 layers, batch 64, long cache
+    Bn, Smax = 64, 8192
+    kvb = dec.new_kv(Bn, Smax)
+    kvb.view(torch.bfloat16).normal_(generator=gen)
+    tok = torch.tensor(synth.tokens((Bn,), c.vocab, stream=400 + rank), dtype=torch.int32, device=dev)
+    tgt = torch.tensor(synth.tokens((Bn,), c.vocab, stream=401 + rank), dtype=torch.int32, device=dev)
+    lpb = torch.empty(Bn, dtype=torch.float32, device=dev)
+    long = {}
+    for p in (4096, 6144, 8191):
+        pos = torch.full((Bn,), p, dtype=torch.int32, device=dev)
+        f = lambda: dec.decode_step(kvb, Bn, Smax, tok, pos, None, tgt, lpb)
+        for _ in range(2):
+            f()
+        t = _event_time(f, 5, stream)
+        long[str(p + 1)] = _hbm_entry(STEP_WEIGHT_BYTES + Bn * (p + 1) * KV_BYTES_PER_TOKEN, t, hbm, Bn)
+    out["batch64_long_context"] = {"workload": "36 layers, batch 64, KV context 4097 / 6145 / 8192",
+                                   "by_context": long}
+    if dec.check_status() != 0 or not torch.isfinite(lpb).all():
+        raise RuntimeError("the batch-64 long-context decode produced invalid output")
+    del kvb
+    dec._ws.clear()
+    torch.cuda.empty_cache()
+    return out
 
 
 def main():

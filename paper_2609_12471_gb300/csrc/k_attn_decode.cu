@@ -1,315 +1,40 @@
-// GQA decode attention over the bf16 KV cache, split over the key sequence.
-//
-// One decode token per row b; query head h = kvh * G + g (G = n_q / n_kv <= 8)
-// attends cache positions 0 .. p(b).  The key tiles 0 .. p/64 of each (b, kvh)
-// are cut evenly into n_split chunks at that row's position (n_split from a cost
-// model at the cache length); one CTA per (chunk, b, kvh) streams its chunk
-// through a 3-stage ring of 64-key K and V tiles loaded by TMA (128-byte swizzle,
-// two 64-dim boxes per tile, one mbarrier per stage).  Each of the 4 warps takes 16 keys of a
-// tile and runs, on the tensor cores (mma.sync m16n8k16, bf16 in, fp32 out):
-//   S[16 x 16] = Q_pad[16 x 128] * K^T   (rows 0..G-1 are the group's heads)
-//   online softmax in base 2 over its keys (running max m, running sum l)
-//   O[16 x 128] += P[16 x 16] * V[16 x 128]
-// The 4 warps are merged in shared memory and the CTA writes an unnormalised
-// partial (O, m, l) per head; the last CTA of a (row, kv head) to finish (an
-// atomic ticket) merges the chunks of its heads:
-//   o = sum_s 2^(m_s - M) O_s / sum_s 2^(m_s - M) l_s,  M = max_s m_s.
-//
-// Keys past p inside the last tile are masked to -inf in S, and their V rows
-// are zeroed in shared memory before P*V (cache memory beyond p is unwritten
-// and may hold NaN patterns; 0 * NaN would poison O).
-//
-// The mbarrier waits are bounded; on a timeout the CTA records
-// QK_STATUS_TIMEOUT, waits (bounded) for the copies it issued and exits
-// without writing its partial.
+// GQA decode attention over the bf16 KV cache, split over the key sequence: the
+// standalone kernel (one work item per CTA; the item itself is
+// attn::decode_item, attn_decode_core.cuh) and the host-side split model and
+// scratch layout it shares with the attention phase of the persistent
+// decode-step kernel.
 #include <cuda.h>
 
-#include "qk_internal.cuh"
-#include "mma_sync.cuh"
-#include "tc_ptx.cuh"
+#include "attn_decode_core.cuh"
 
 namespace qk {
 
 namespace {
 
-constexpr int kD = 128;          // head_dim of this kernel
-constexpr int kTileKeys = 64;    // keys per stage
-constexpr int kStages = 3;
-constexpr int kMergeChunks = 4;  // chunk partials per load batch of the final merge
-constexpr int kHalfBytes = kTileKeys * 128;   // one 64-dim box: 64 rows x 128 B
-constexpr int kTileBytes = 2 * kHalfBytes;    // K (or V) tile: dims 0..63 then 64..127
-constexpr int kStageBytes = 2 * kTileBytes;   // K tile then V tile
-// The warp-merge buffers ([4 warps][8 rows][128] O and [4][8][2] m, l) reuse the
-// stage buffers once every tile has been consumed.
-constexpr int kSmem = kStages * kStageBytes + 1024 + 256;
-static_assert(4 * 8 * kD * 4 + 4 * 8 * 2 * 4 <= kStages * kStageBytes, "merge buffers");
-
-using ms::ldsm_x4;
-using ms::ldsm_x4_t;
-using ms::mma16816;
-using ms::pack_bf16;
-
-// Address of (key row, 16-byte chunk c) in a 64-key K or V tile.
-__device__ __forceinline__ uint32_t tile_addr(uint32_t tile, int key, int c) {
-    return ms::sw_addr<kTileKeys>(tile, key, c);
-}
+using attn::kD;
+using attn::kTileKeys;
+constexpr int kSmem = attn::kRingBytes + 1024 + 256;
 
 __global__ void __launch_bounds__(128)
-    attn_decode_kernel(const __grid_constant__ CUtensorMap tmKV, const bf16* __restrict__ q,
-                       int q_ld, int nq, int nkv, int max_batch, int max_seq, PosIndex pos,
-                       int chunk, int n_split, float* __restrict__ part_o,
-                       float2* __restrict__ part_ml, int* __restrict__ tickets, bf16* __restrict__ out,
-                       uint32_t* __restrict__ status) {
+    attn_decode_kernel(const __grid_constant__ CUtensorMap tmKV, const __grid_constant__ attn::Args a) {
     extern __shared__ uint8_t smem_raw[];
     uint8_t* smem = (uint8_t*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
-    float* red = (float*)smem;           // [4 warps][8 rows][128], after the key loop
-    float* red_ml = red + 4 * 8 * kD;    // [4 warps][8 rows][2]
-    uint64_t* full = (uint64_t*)(smem + kStages * kStageBytes);
-    volatile int* abort_flag = (volatile int*)(full + kStages);
+    uint64_t* full = (uint64_t*)(smem + attn::kRingBytes);
+    volatile int* abort_flag = (volatile int*)(full + attn::kStages);
+    int* last_s = (int*)(full + attn::kStages) + 1;
 
     pdl_wait();
     pdl_trigger();  // the next kernel may launch once every CTA of this grid is resident
-    const int split = blockIdx.x;
-    const int b = blockIdx.y / nkv, kvh = blockIdx.y % nkv;
-    const int G = nq / nkv;
-    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int g = lane >> 2, tig = lane & 3;
-
-    int p = pos.pos_dev ? pos.pos_dev[b] : pos.start;
-    if (p < 0 || p >= max_seq) p = p < 0 ? 0 : max_seq - 1;  // flagged by the cache-write kernel
-    // The row's key tiles 0 .. p/64 are cut into n_split equal runs at this row's own
-    // position (the grid is sized from the longest cache, the work from p); `chunk`
-    // caps a run at the cost model's length.
-    const int n_tiles_b = p / kTileKeys + 1;
-    const int per = min((n_tiles_b + n_split - 1) / n_split, chunk / kTileKeys);
-    const int n_valid = (n_tiles_b + per - 1) / per;  // splits that hold keys
-    const int k_begin = split * per * kTileKeys;
-    if (split >= n_valid) return;  // nothing to attend in this split; the merge skips it
-    const int k_end = min(k_begin + per * kTileKeys, p + 1);
-    const int n_tiles = (k_end - k_begin + kTileKeys - 1) / kTileKeys;
-    // Row of key 0 of (b, kvh) in the 2-D view of this layer's K (V follows after max_batch*nkv*max_seq rows).
-    const int row0 = (b * nkv + kvh) * max_seq;
-    const int v_off = max_batch * nkv * max_seq;
-
     if (threadIdx.x == 0) {
-        for (int s = 0; s < kStages; ++s) tc::mbar_init(&full[s], 1);
+        for (int s = 0; s < attn::kStages; ++s) tc::mbar_init(&full[s], 1);
         *abort_flag = 0;
         tc::fence_mbar_init();
         tc::tma_prefetch_desc(&tmKV);
     }
     __syncthreads();
-    auto issue = [&](int t) {
-        const int st = t % kStages;
-        uint8_t* base = smem + st * kStageBytes;
-        const int r = row0 + k_begin + t * kTileKeys;
-        tc::mbar_expect_tx(&full[st], kStageBytes);
-        tc::tma_load_2d(base, &tmKV, 0, r, &full[st]);
-        tc::tma_load_2d(base + kHalfBytes, &tmKV, 64, r, &full[st]);
-        tc::tma_load_2d(base + kTileBytes, &tmKV, 0, v_off + r, &full[st]);
-        tc::tma_load_2d(base + kTileBytes + kHalfBytes, &tmKV, 64, v_off + r, &full[st]);
-    };
-    int n_issued = 0;  // meaningful in thread 0 only
-    if (threadIdx.x == 0)
-        for (; n_issued < kStages && n_issued < n_tiles; ++n_issued) issue(n_issued);
-
-    // Q fragments (A operand, rows = heads of the group, padded to 16): a0a1 / a4a5
-    // hold row g, dims 16ks + 2tig (+8); rows 8..15 are zero.
-    uint32_t qa[8][2];
-    {
-        const bool valid = g < G;
-        const bf16* qrow = q + (size_t)b * q_ld + (size_t)(kvh * G + (valid ? g : 0)) * kD;
-#pragma unroll
-        for (int ks = 0; ks < 8; ++ks) {
-            uint32_t lo = *reinterpret_cast<const uint32_t*>(qrow + 16 * ks + 2 * tig);
-            uint32_t hi = *reinterpret_cast<const uint32_t*>(qrow + 16 * ks + 8 + 2 * tig);
-            qa[ks][0] = valid ? lo : 0u;
-            qa[ks][1] = valid ? hi : 0u;
-        }
-    }
-    const float scale = rsqrtf((float)kD) * 1.4426950408889634f;  // 1/sqrt(d) * log2(e)
-    float m_run = -INFINITY, l_run = 0.f;
-    float o[16][4];
-#pragma unroll
-    for (int j = 0; j < 16; ++j) o[j][0] = o[j][1] = o[j][2] = o[j][3] = 0.f;
-
-    bool ok = true;
-    int t_fail = n_tiles;
-    for (int t = 0; t < n_tiles; ++t) {
-        const int st = t % kStages;
-        const uint32_t phase = (uint32_t)((t / kStages) & 1);
-        bool got = tc::mbar_wait(&full[st], phase, abort_flag);
-        if (!__syncthreads_and(got)) {
-            ok = false;
-            t_fail = t;
-            break;
-        }
-        uint8_t* base = smem + st * kStageBytes;
-        const int key0 = k_begin + t * kTileKeys;  // absolute position of the tile's first key
-        if (key0 + kTileKeys - 1 > p) {
-            // zero the V rows past p (16-byte stores over both boxes)
-            for (int i = threadIdx.x; i < kTileKeys * 16; i += blockDim.x) {
-                const int key = i >> 4, c = i & 15;
-                if (key0 + key > p)
-                    *reinterpret_cast<uint4*>(base + kTileBytes + (c >> 3) * kHalfBytes + key * 128 +
-                                              (((c & 7) ^ (key & 7)) << 4)) = make_uint4(0, 0, 0, 0);
-            }
-            __syncthreads();
-        }
-        const uint32_t kt = tc::smem_u32(base), vt = tc::smem_u32(base + kTileBytes);
-        const int kw = warp * 16;  // this warp's 16 keys within the tile
-        // ---- S = Q K^T for keys kw .. kw+15 (two n8 tiles)
-        float s0[4] = {0.f, 0.f, 0.f, 0.f}, s1[4] = {0.f, 0.f, 0.f, 0.f};
-#pragma unroll
-        for (int ks = 0; ks < 8; ++ks) {
-            // matrices: (keys 0-7, dims lo), (keys 0-7, dims hi), (keys 8-15, lo), (keys 8-15, hi)
-            const int mi = lane >> 3, r = lane & 7;
-            const int key = kw + (mi >> 1) * 8 + r, c = 2 * ks + (mi & 1);
-            uint32_t b00, b01, b10, b11;
-            ldsm_x4(tile_addr(kt, key, c), b00, b01, b10, b11);
-            const uint32_t a[4] = {qa[ks][0], 0u, qa[ks][1], 0u};
-            mma16816(s0, a, b00, b01);
-            mma16816(s1, a, b10, b11);
-        }
-        // ---- online softmax (row g; rows 8..15 are padding)
-        float sv[4] = {s0[0] * scale, s0[1] * scale, s1[0] * scale, s1[1] * scale};
-        const int kk[4] = {kw + 2 * tig, kw + 2 * tig + 1, kw + 8 + 2 * tig, kw + 9 + 2 * tig};
-#pragma unroll
-        for (int i = 0; i < 4; ++i)
-            if (key0 + kk[i] > p) sv[i] = -INFINITY;
-        float mx = fmaxf(fmaxf(sv[0], sv[1]), fmaxf(sv[2], sv[3]));
-        mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 1));
-        mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 2));
-        const float m_new = fmaxf(m_run, mx);
-        float pv[4], ps = 0.f;
-        if (m_new == -INFINITY) {  // every key so far masked (cannot happen for key 0 <= p)
-            pv[0] = pv[1] = pv[2] = pv[3] = 0.f;
-        } else {
-#pragma unroll
-            for (int i = 0; i < 4; ++i) {
-                pv[i] = exp2f(sv[i] - m_new);
-                ps += pv[i];
-            }
-        }
-        ps += __shfl_xor_sync(0xffffffffu, ps, 1);
-        ps += __shfl_xor_sync(0xffffffffu, ps, 2);
-        const float corr = m_run == -INFINITY ? 0.f : exp2f(m_run - m_new);
-        l_run = l_run * corr + ps;
-        m_run = m_new;
-#pragma unroll
-        for (int j = 0; j < 16; ++j) {
-            o[j][0] *= corr;
-            o[j][1] *= corr;
-        }
-        // ---- O += P V: P as the A operand (rows 8..15 zero), V^T fragments via ldmatrix.trans
-        const uint32_t pa[4] = {pack_bf16(pv[0], pv[1]), 0u, pack_bf16(pv[2], pv[3]), 0u};
-#pragma unroll
-        for (int jj = 0; jj < 8; ++jj) {
-            // matrices: (keys 0-7, dims 16jj..+7), (keys 8-15, same), (keys 0-7, dims 16jj+8..), (keys 8-15, ...)
-            const int mi = lane >> 3, r = lane & 7;
-            const int key = kw + (mi & 1) * 8 + r, c = 2 * jj + (mi >> 1);
-            uint32_t v0, v1, v2, v3;
-            ldsm_x4_t(tile_addr(vt, key, c), v0, v1, v2, v3);
-            mma16816(o[2 * jj], pa, v0, v1);
-            mma16816(o[2 * jj + 1], pa, v2, v3);
-        }
-        __syncthreads();  // every warp is done with this stage
-        if (threadIdx.x == 0 && n_issued < n_tiles) issue(n_issued++);
-    }
-
-    if (!ok) {
-        if (threadIdx.x == 0) {
-            atomicOr(status, QK_STATUS_TIMEOUT);
-            // let the copies issued for tiles not yet consumed land before exiting
-            for (int t = t_fail; t < n_issued; ++t)
-                tc::mbar_wait_drain(&full[t % kStages], (uint32_t)((t / kStages) & 1));
-        }
-        return;
-    }
-
-    // ---- merge the 4 warps: row g (< 8) of each warp's O (dims 8j + 2tig, +1)
-    if (g < 8) {
-#pragma unroll
-        for (int j = 0; j < 16; ++j) {
-            red[(warp * 8 + g) * kD + 8 * j + 2 * tig] = o[j][0];
-            red[(warp * 8 + g) * kD + 8 * j + 2 * tig + 1] = o[j][1];
-        }
-        if (tig == 0) {
-            red_ml[(warp * 8 + g) * 2] = m_run;
-            red_ml[(warp * 8 + g) * 2 + 1] = l_run;
-        }
-    }
-    __syncthreads();
-    // thread -> (row gg, dim d): 128 threads cover one row's 128 dims; loop over the G rows
-    for (int gg = 0; gg < G; ++gg) {
-        const int d = threadIdx.x;
-        float M = -INFINITY;
-        for (int w = 0; w < 4; ++w) M = fmaxf(M, red_ml[(w * 8 + gg) * 2]);
-        float acc = 0.f, L = 0.f;
-        for (int w = 0; w < 4; ++w) {
-            const float mw = red_ml[(w * 8 + gg) * 2];
-            const float f = mw == -INFINITY ? 0.f : exp2f(mw - M);
-            acc += f * red[(w * 8 + gg) * kD + d];
-            L += f * red_ml[(w * 8 + gg) * 2 + 1];
-        }
-        const size_t head = (size_t)b * nq + kvh * G + gg;
-        if (n_valid == 1) {  // a single chunk is already the whole attention
-            out[head * kD + d] = __float2bfloat16_rn(acc / L);
-        } else {
-            part_o[(head * n_split + split) * kD + d] = acc;
-            if (d == 0) part_ml[head * n_split + split] = make_float2(M, L);
-        }
-    }
-    if (n_valid == 1) return;
-    // The last CTA of this (row, kv head) to finish merges the chunks' partials:
-    //   o = sum_s 2^(m_s - M) O_s / sum_s 2^(m_s - M) l_s,  M = max_s m_s,
-    // then resets the ticket for the next layer.  The barrier orders every thread's
-    // partial stores before thread 0's release; its acquire orders the merge's reads
-    // after the other chunks' stores.
-    __shared__ int last;
-    __syncthreads();
-    if (threadIdx.x == 0)
-        last = tc::atom_add_acq_rel_gpu(&tickets[b * nkv + kvh], 1) == n_valid - 1;
-    __syncthreads();
-    if (!last) return;
-    // Online merge over the chunks in order, kMergeChunks at a time: every load of a
-    // batch is issued before any is used, so a batch costs one L2 round trip.
-    const int d = threadIdx.x;
-    float Mh[8], Ah[8], Lh[8];
-#pragma unroll
-    for (int gg = 0; gg < 8; ++gg) Mh[gg] = -INFINITY, Ah[gg] = 0.f, Lh[gg] = 0.f;
-    for (int base = 0; base < n_valid; base += kMergeChunks) {
-        float ov[8][kMergeChunks];
-        float2 ml[8][kMergeChunks];
-#pragma unroll
-        for (int gg = 0; gg < 8; ++gg)
-#pragma unroll
-            for (int k = 0; k < kMergeChunks; ++k) {
-                const bool v = gg < G && base + k < n_valid;
-                const size_t i = ((size_t)b * nq + kvh * G + gg) * n_split + base + k;
-                ov[gg][k] = v ? __ldcg(&part_o[i * kD + d]) : 0.f;
-                ml[gg][k] = v ? __ldcg(&part_ml[i]) : make_float2(-INFINITY, 0.f);
-            }
-#pragma unroll
-        for (int gg = 0; gg < 8; ++gg) {
-            float Mn = Mh[gg];
-#pragma unroll
-            for (int k = 0; k < kMergeChunks; ++k) Mn = fmaxf(Mn, ml[gg][k].x);
-            if (Mn == -INFINITY) continue;  // padding head
-            const float sc = Mh[gg] == -INFINITY ? 0.f : exp2f(Mh[gg] - Mn);
-            float A = Ah[gg] * sc, L = Lh[gg] * sc;
-#pragma unroll
-            for (int k = 0; k < kMergeChunks; ++k) {
-                const float f = ml[gg][k].x == -INFINITY ? 0.f : exp2f(ml[gg][k].x - Mn);
-                A += f * ov[gg][k];
-                L += f * ml[gg][k].y;
-            }
-            Mh[gg] = Mn, Ah[gg] = A, Lh[gg] = L;
-        }
-    }
-#pragma unroll
-    for (int gg = 0; gg < 8; ++gg)
-        if (gg < G) out[((size_t)b * nq + kvh * G + gg) * kD + d] = __float2bfloat16_rn(Ah[gg] / Lh[gg]);
-    if (threadIdx.x == 0) tickets[b * nkv + kvh] = 0;
+    int tiles = 0;
+    attn::decode_item(a, &tmKV, 0, blockIdx.x, blockIdx.y / a.nkv, blockIdx.y % a.nkv, smem, full,
+                      tiles, abort_flag, last_s, threadIdx.x);
 }
 
 typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*,
@@ -343,20 +68,68 @@ void attn_decode_split(int B, int nkv, int max_seq, int num_sms, int* chunk, int
     *n_split = (n_tiles + best_c - 1) / best_c;
 }
 
+// Split of the persistent decode-step kernel's attention phase: one item slot per
+// SM (its epilogue warps), so waves x (tiles per item + 1.5) with num_sms slots.
+void attn_decode_split_persist(int B, int nkv, int max_seq, int num_sms, int* chunk, int* n_split) {
+    attn_decode_split(B, nkv, max_seq, num_sms / 2 > 0 ? num_sms / 2 : 1, chunk, n_split);
+}
+
+static int max_split(int B, int nkv, int max_seq, int num_sms) {
+    int c, n1, n2;
+    attn_decode_split(B, nkv, max_seq, num_sms, &c, &n1);
+    attn_decode_split_persist(B, nkv, max_seq, num_sms, &c, &n2);
+    return n1 > n2 ? n1 : n2;
+}
+
 // Partials [B nq][n_split][128] fp32, (m, l) [B nq][n_split], then the merge tickets
 // [B nkv] (int, must be zero before the first layer of a step: attn_decode_tickets).
+// The regions are sized for the larger split of the two attention schedules; each
+// schedule indexes them with its own split count.
 size_t attn_decode_scratch_bytes(int B, int nq, int nkv, int max_seq, int num_sms) {
-    int chunk, n_split;
-    attn_decode_split(B, nkv, max_seq, num_sms, &chunk, &n_split);
     const size_t heads = (size_t)B * nq;
-    return heads * n_split * (kD * sizeof(float) + sizeof(float2)) + (size_t)B * nkv * 4 + 256;
+    return heads * max_split(B, nkv, max_seq, num_sms) * (kD * sizeof(float) + sizeof(float2)) +
+           (size_t)B * nkv * 4 + 256;
 }
 
 int* attn_decode_tickets(void* scratch, int B, int nq, int nkv, int max_seq, int num_sms) {
-    int chunk, n_split;
-    attn_decode_split(B, nkv, max_seq, num_sms, &chunk, &n_split);
     const size_t heads = (size_t)B * nq;
-    return (int*)((char*)scratch + heads * n_split * (kD * sizeof(float) + sizeof(float2)));
+    return (int*)((char*)scratch +
+                  heads * max_split(B, nkv, max_seq, num_sms) * (kD * sizeof(float) + sizeof(float2)));
+}
+
+void attn_scratch_parts(void* scratch, int B, int nq, int nkv, int max_seq, int num_sms, int n_split,
+                        float** part_o, float2** part_ml, int** tickets) {
+    const size_t heads = (size_t)B * nq;
+    const int ms = max_split(B, nkv, max_seq, num_sms);
+    *part_o = (float*)scratch;
+    *part_ml = (float2*)((char*)scratch + heads * ms * kD * sizeof(float));
+    *tickets = attn_decode_tickets(scratch, B, nq, nkv, max_seq, num_sms);
+    (void)n_split;
+}
+
+// 3-D map over the K / V caches of `layers` layers (layer stride layer_bytes): rows of
+// 128 bf16 elements, K rows of a layer first, then its V rows; 64 x 64-row boxes,
+// 128-byte swizzle.
+bool make_kv_map(CUtensorMap* map, const void* k_layer0, int max_batch, int nkv, int max_seq,
+                 int layers, size_t layer_bytes) {
+    void* fn = nullptr;
+    cudaDriverEntryPointQueryResult qr;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000, cudaEnableDefault,
+                                         &qr) != cudaSuccess ||
+        qr != cudaDriverEntryPointSuccess)
+        return false;
+    const size_t rows = 2 * (size_t)max_batch * nkv * max_seq;
+    if (rows >= ((size_t)1 << 31)) return false;
+    if (layers < 1) return false;
+    if (layers == 1) layer_bytes = rows * kD * 2;
+    cuuint64_t dims[3] = {(cuuint64_t)kD, (cuuint64_t)rows, (cuuint64_t)layers};
+    cuuint64_t strides[2] = {(cuuint64_t)kD * 2, (cuuint64_t)layer_bytes};
+    cuuint32_t box[3] = {64, (cuuint32_t)kTileKeys, 1};
+    cuuint32_t estr[3] = {1, 1, 1};
+    return ((EncodeTiledFn)fn)(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(k_layer0),
+                               dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
+                               CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                               CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
 bool attn_decode_supported(int d, int nq, int nkv) { return d == kD && nq / nkv <= 8; }
@@ -371,33 +144,23 @@ int launch_attn_decode(const bf16* q, int q_ld, const void* k_layer, int nq, int
             return QK_ECUDA;
         attr_set = true;
     }
-    void* fn = nullptr;
-    cudaDriverEntryPointQueryResult qr;
-    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000, cudaEnableDefault,
-                                         &qr) != cudaSuccess ||
-        qr != cudaDriverEntryPointSuccess)
-        return QK_ECUDA;
-    // This layer's K and V as one 2-D array of 128-element rows: K rows first, then V rows.
-    const size_t rows = 2 * (size_t)max_batch * nkv * max_seq;
-    if (rows >= ((size_t)1 << 31)) return QK_ESHAPE;
     CUtensorMap map;
-    cuuint64_t dims[2] = {(cuuint64_t)kD, (cuuint64_t)rows};
-    cuuint64_t strides[1] = {(cuuint64_t)kD * 2};
-    cuuint32_t box[2] = {64, (cuuint32_t)kTileKeys};
-    cuuint32_t estr[2] = {1, 1};
-    if (((EncodeTiledFn)fn)(&map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(k_layer),
-                            dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
-                            CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
-                            CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
-        return QK_ECUDA;
-    int chunk, n_split;
-    attn_decode_split(B, nkv, max_seq, num_sms, &chunk, &n_split);
-    float* part_o = (float*)scratch;
-    float2* part_ml = (float2*)((char*)scratch + (size_t)B * nq * n_split * kD * sizeof(float));
-    int* tickets = attn_decode_tickets(scratch, B, nq, nkv, max_seq, num_sms);
-    dim3 grid(n_split, B * nkv);
-    launch_k(attn_decode_kernel, grid, dim3(128), kSmem, s, map, q, q_ld, nq, nkv, max_batch,
-             max_seq, pos, chunk, n_split, part_o, part_ml, tickets, o, status);
+    if (!make_kv_map(&map, k_layer, max_batch, nkv, max_seq, 1, 0)) return QK_ECUDA;
+    attn::Args a;
+    a.q = q;
+    a.q_ld = q_ld;
+    a.nq = nq;
+    a.nkv = nkv;
+    a.max_batch = max_batch;
+    a.max_seq = max_seq;
+    a.pos = pos;
+    attn_decode_split(B, nkv, max_seq, num_sms, &a.chunk, &a.n_split);
+    attn_scratch_parts(scratch, B, nq, nkv, max_seq, num_sms, a.n_split, &a.part_o, &a.part_ml,
+                       &a.tickets);
+    a.out = o;
+    a.status = status;
+    dim3 grid(a.n_split, B * nkv);
+    launch_k(attn_decode_kernel, grid, dim3(128), kSmem, s, map, a);
     note_launch(1);
     return QK_OK;
 }
