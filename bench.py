@@ -240,7 +240,7 @@ def run_ours(args, world, rank, local):
 
     # ---- timed region: K whole rollouts, device-resident inputs
     n_layers = s.n_layers
-    qk.qk_profile_begin(dec.handle, qk.QK_PROF_STEP, args.steps * N)
+    qk.qk_profile_begin(dec.handle, qk.QK_PROF_GATE_UP, args.steps * N * n_layers)
     clocks = ClockSampler(local)
     barrier(world)
     torch.cuda.synchronize(dev)
@@ -326,25 +326,19 @@ def run_ours(args, world, rank, local):
     bf16_peak = peaks["bf16_tflops"] if peaks else 1900.0
     c = dec.cfg
     if prof_n < 1:
-        raise RuntimeError("no decode-step launch was bracketed")
-    # the bracketed launch: decode step 0 of each timed rollout (position P, keys 0 .. P);
-    # weights of every layer and the lm_head, the K/V read, the K/V written, activations
-    step0_bytes = (STEP_WEIGHT_BYTES + B * (P + 1) * KV_BYTES_PER_TOKEN
-                   + c.n_layers * B * (3 * c.hidden * 4 + c.intermediate * 2 * 2)
-                   + B * c.vocab * 4)
+        raise RuntimeError("no gate/up launch was bracketed")
+    gu_bytes = 2 * c.intermediate * c.hidden * 2 + B * c.hidden * 2 + B * c.intermediate * 2
     avg_launch_s = (prof_ms / prof_n) / 1e3
-    achieved = step0_bytes / avg_launch_s / 1e9
-    roofline = {"bound": "hbm",
-                "kernel": "persistent decode-step kernel (36 layers + lm_head in one cooperative launch, "
-                          "16 token rows)",
-                "timed_launches": "decode step 0 of each timed rollout (later steps replay a captured "
-                                  "CUDA graph without event nodes)",
+    achieved = gu_bytes / avg_launch_s / 1e9
+    roofline = {"bound": "hbm", "kernel": "decode gate/up linear (tcgen05 stream-K GEMM, 16 token rows)",
+                "timed_launches": "the gate/up launches of each timed rollout's first decode step "
+                                  "(later steps replay a captured CUDA graph without event nodes)",
                 "achieved": achieved, "peak": hbm_peak, "unit": "GB/s",
                 "frac": achieved / hbm_peak,
                 "peak_source": "measured" if peaks else "fallback",
-                "algorithmic_bytes_per_launch": int(step0_bytes), "launches_timed": prof_n,
+                "algorithmic_bytes_per_launch": gu_bytes, "launches_timed": prof_n,
                 "avg_launch_us": avg_launch_s * 1e6,
-                "traffic": recorded_traffic("decode_step_b16")}
+                "traffic": recorded_traffic("gate_up_decode_b16")}
     step_bytes = 15136811008 + B * sum(P + j + 1 for j in range(N)) * 147456 / N
     line = {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": ms_step, "higher_is_better": True,

@@ -268,9 +268,6 @@ int qk_check_status(qk_model* m, void* stream, uint32_t* flags);
 #define QK_PROF_DOWN 3     /* h x W_down + residual                       */
 #define QK_PROF_ATTN 4     /* decode attention (all its kernels)          */
 #define QK_PROF_LM_HEAD 5  /* final RMSNorm'd x W_lm (logits)             */
-#define QK_PROF_STEP 6     /* the persistent decode-step kernel (decode steps of up to
-                              16 rows: every layer and the lm_head in one launch; the
-                              classes above then see no launches)          */
 
 /* Start bracketing up to max_launches launches of kernel class `kind` with
  * CUDA events recorded on the launching stream.  Creates 2*max_launches

@@ -18,7 +18,7 @@ QK_OK, QK_EINVAL, QK_ESHAPE, QK_EDTYPE, QK_ECUDA, QK_ETIMEOUT, QK_EDEVICE, QK_EN
 QK_DTYPE_BF16, QK_DTYPE_F32 = 0, 1
 QK_STATUS_BAD_TOKEN, QK_STATUS_BAD_POS, QK_STATUS_TIMEOUT = 1, 2, 4
 QK_CALL_DECODE, QK_CALL_PREFILL, QK_CALL_SCORE, QK_CALL_ROLLOUT = 0, 1, 2, 3
-QK_PROF_QKV, QK_PROF_O, QK_PROF_GATE_UP, QK_PROF_DOWN, QK_PROF_ATTN, QK_PROF_LM_HEAD, QK_PROF_STEP = range(7)
+QK_PROF_QKV, QK_PROF_O, QK_PROF_GATE_UP, QK_PROF_DOWN, QK_PROF_ATTN, QK_PROF_LM_HEAD = range(6)
 QK_EPI_STORE, QK_EPI_STORE_F32, QK_EPI_RESID_F32, QK_EPI_SWIGLU = 0, 1, 2, 3
 QK_STATIC_SCRATCH_BYTES = 8 << 20
 
@@ -31,7 +31,7 @@ __all__ = [
     "qk_decode_layer", "qk_score_logprobs", "qk_rollout_teacher_forced", "qk_check_status",
     "qk_last_error", "QKError", "lib_path", "exported_symbols", "qk_profile_begin",
     "qk_profile_end", "qk_launch_count", "qk_op_linear", "QK_PROF_QKV", "QK_PROF_O",
-    "QK_PROF_GATE_UP", "QK_PROF_DOWN", "QK_PROF_ATTN", "QK_PROF_LM_HEAD", "QK_PROF_STEP", "QK_EPI_STORE",
+    "QK_PROF_GATE_UP", "QK_PROF_DOWN", "QK_PROF_ATTN", "QK_PROF_LM_HEAD", "QK_EPI_STORE",
     "QK_EPI_STORE_F32", "QK_EPI_RESID_F32", "QK_EPI_SWIGLU", "qk_op_linear_swiglu_static",
     "QK_STATIC_SCRATCH_BYTES", "qk_grpo_workspace_bytes", "qk_grpo_token_loss", "qk_score_grpo",
     "qk_rollout_sampled", "qk_prefill_rows", "qk_debug_expire_next_wait",

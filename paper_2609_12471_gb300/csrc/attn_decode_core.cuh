@@ -1,7 +1,5 @@
 // One work item of the split GQA decode attention over the bf16 KV cache, run
-// by 128 threads (four warps): the standalone decode attention kernel (one item
-// per CTA) and the attention phase of the persistent decode-step kernel (items
-// it, it + grid, ... on its epilogue warps) both call attn_decode_item.
+// by 128 threads (four warps); the decode attention kernel runs one item per CTA.
 //
 // Item (split, b, kvh): one decode token per row b; query head h = kvh * G + g
 // (G = n_q / n_kv <= 8) attends cache positions 0 .. p(b).  The key tiles
@@ -23,9 +21,10 @@
 // beyond p is unwritten and may hold NaN patterns; 0 * NaN would poison O).
 //
 // The ring's mbarrier phases continue across the items a CTA runs (`tiles`
-// counts the tiles it has loaded so far).  Waits are bounded; on a timeout the
+// counts the tiles it has loaded so far; a CTA that runs one item passes 0).  Waits are bounded; on a timeout the
 // item raises the abort flag, waits (bounded) for the copies it issued and
-// returns false without writing its partial.
+// returns -1 without writing its partial.  Otherwise it returns 1 if it wrote the
+// (row, kv head) output (a single chunk, or the last chunk's merge), else 0.
 #pragma once
 
 #include <cuda.h>
@@ -70,7 +69,7 @@ __device__ __forceinline__ uint32_t tile_addr(uint32_t tile, int key, int c) {
 // warp = tid / 32.  ring: kRingBytes of 1024-aligned shared memory; full: its
 // kStages mbarriers (count 1); tmKV: 3-D map of the caches ({128, rows, layers},
 // K rows first, then V rows), z: the layer.  *last_s: a shared int.
-__device__ __forceinline__ bool decode_item(const Args& a, const CUtensorMap* tmKV, int z, int split,
+__device__ __forceinline__ int decode_item(const Args& a, const CUtensorMap* tmKV, int z, int split,
                                             int b, int kvh, uint8_t* ring, uint64_t* full,
                                             int& tiles, volatile int* abort_flag, int* last_s,
                                             int tid) {
@@ -93,7 +92,7 @@ __device__ __forceinline__ bool decode_item(const Args& a, const CUtensorMap* tm
     const int per = min((n_tiles_b + a.n_split - 1) / a.n_split, a.chunk / kTileKeys);
     const int n_valid = (n_tiles_b + per - 1) / per;  // splits that hold keys
     const int k_begin = split * per * kTileKeys;
-    if (split >= n_valid) return true;  // nothing to attend in this split; the merge skips it
+    if (split >= n_valid) return 0;  // nothing to attend in this split; the merge skips it
     const int k_end = min(k_begin + per * kTileKeys, p + 1);
     const int n_tiles = (k_end - k_begin + kTileKeys - 1) / kTileKeys;
     // Row of key 0 of (b, kvh) in the 2-D view of a layer's K (V follows after max_batch*nkv*max_seq rows).
@@ -227,7 +226,7 @@ __device__ __forceinline__ bool decode_item(const Args& a, const CUtensorMap* tm
                 tc::mbar_wait_drain(&full[(tiles + t) % kStages],
                                     (uint32_t)(((tiles + t) / kStages) & 1));
         }
-        return false;
+        return -1;
     }
     tiles += n_tiles;
 
@@ -264,7 +263,7 @@ __device__ __forceinline__ bool decode_item(const Args& a, const CUtensorMap* tm
             if (d == 0) a.part_ml[head * a.n_split + split] = make_float2(M, L);
         }
     }
-    if (n_valid == 1) return true;
+    if (n_valid == 1) return 1;
     // The last item of this (row, kv head) to finish merges the chunks' partials:
     //   o = sum_s 2^(m_s - M) O_s / sum_s 2^(m_s - M) l_s,  M = max_s m_s,
     // then resets the ticket for the next layer.  The barrier orders every thread's
@@ -273,7 +272,7 @@ __device__ __forceinline__ bool decode_item(const Args& a, const CUtensorMap* tm
     tc::bar128();
     if (tid == 0) *last_s = tc::atom_add_acq_rel_gpu(&a.tickets[b * nkv + kvh], 1) == n_valid - 1;
     tc::bar128();
-    if (!*last_s) return true;
+    if (!*last_s) return 0;
     // Online merge over the chunks in order, kMergeChunks at a time: every load of a
     // batch is issued before any is used, so a batch costs one L2 round trip.
     const int d = tid;
@@ -313,7 +312,7 @@ __device__ __forceinline__ bool decode_item(const Args& a, const CUtensorMap* tm
     for (int gg = 0; gg < 8; ++gg)
         if (gg < G) a.out[((size_t)b * nq + kvh * G + gg) * kD + d] = __float2bfloat16_rn(Ah[gg] / Lh[gg]);
     if (tid == 0) a.tickets[b * nkv + kvh] = 0;
-    return true;
+    return 1;
 }
 
 }  // namespace attn

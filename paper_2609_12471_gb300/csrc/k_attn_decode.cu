@@ -1,8 +1,6 @@
 // GQA decode attention over the bf16 KV cache, split over the key sequence: the
-// standalone kernel (one work item per CTA; the item itself is
-// attn::decode_item, attn_decode_core.cuh) and the host-side split model and
-// scratch layout it shares with the attention phase of the persistent
-// decode-step kernel.
+// kernel (one work item per CTA; the item itself is attn::decode_item,
+// attn_decode_core.cuh), its split model and its scratch layout.
 #include <cuda.h>
 
 #include "attn_decode_core.cuh"
@@ -68,43 +66,28 @@ void attn_decode_split(int B, int nkv, int max_seq, int num_sms, int* chunk, int
     *n_split = (n_tiles + best_c - 1) / best_c;
 }
 
-// Split of the persistent decode-step kernel's attention phase: one item slot per
-// SM (its epilogue warps), so waves x (tiles per item + 1.5) with num_sms slots.
-void attn_decode_split_persist(int B, int nkv, int max_seq, int num_sms, int* chunk, int* n_split) {
-    attn_decode_split(B, nkv, max_seq, num_sms / 2 > 0 ? num_sms / 2 : 1, chunk, n_split);
-}
-
-static int max_split(int B, int nkv, int max_seq, int num_sms) {
-    int c, n1, n2;
-    attn_decode_split(B, nkv, max_seq, num_sms, &c, &n1);
-    attn_decode_split_persist(B, nkv, max_seq, num_sms, &c, &n2);
-    return n1 > n2 ? n1 : n2;
-}
-
 // Partials [B nq][n_split][128] fp32, (m, l) [B nq][n_split], then the merge tickets
 // [B nkv] (int, must be zero before the first layer of a step: attn_decode_tickets).
-// The regions are sized for the larger split of the two attention schedules; each
-// schedule indexes them with its own split count.
 size_t attn_decode_scratch_bytes(int B, int nq, int nkv, int max_seq, int num_sms) {
+    int chunk, n_split;
+    attn_decode_split(B, nkv, max_seq, num_sms, &chunk, &n_split);
     const size_t heads = (size_t)B * nq;
-    return heads * max_split(B, nkv, max_seq, num_sms) * (kD * sizeof(float) + sizeof(float2)) +
-           (size_t)B * nkv * 4 + 256;
+    return heads * n_split * (kD * sizeof(float) + sizeof(float2)) + (size_t)B * nkv * 4 + 256;
 }
 
 int* attn_decode_tickets(void* scratch, int B, int nq, int nkv, int max_seq, int num_sms) {
+    int chunk, n_split;
+    attn_decode_split(B, nkv, max_seq, num_sms, &chunk, &n_split);
     const size_t heads = (size_t)B * nq;
-    return (int*)((char*)scratch +
-                  heads * max_split(B, nkv, max_seq, num_sms) * (kD * sizeof(float) + sizeof(float2)));
+    return (int*)((char*)scratch + heads * n_split * (kD * sizeof(float) + sizeof(float2)));
 }
 
 void attn_scratch_parts(void* scratch, int B, int nq, int nkv, int max_seq, int num_sms, int n_split,
                         float** part_o, float2** part_ml, int** tickets) {
     const size_t heads = (size_t)B * nq;
-    const int ms = max_split(B, nkv, max_seq, num_sms);
     *part_o = (float*)scratch;
-    *part_ml = (float2*)((char*)scratch + heads * ms * kD * sizeof(float));
+    *part_ml = (float2*)((char*)scratch + heads * n_split * kD * sizeof(float));
     *tickets = attn_decode_tickets(scratch, B, nq, nkv, max_seq, num_sms);
-    (void)n_split;
 }
 
 // 3-D map over the K / V caches of `layers` layers (layer stride layer_bytes): rows of

@@ -26,11 +26,8 @@
 // GEMM) exercises that path: CTA 0 issues no copy for its first k-block and
 // waits at most test_wait cycles, so its MMA thread's wait for that copy expires.
 #include <cuda.h>
-#include <string.h>
-
 #include <mutex>
 
-#include "attn_decode_core.cuh"
 #include "qk_internal.cuh"
 #include "tc_ptx.cuh"
 
@@ -44,7 +41,8 @@ constexpr int kBK = 64;  // bf16 elements per k-block: one 128-byte swizzle row
 // memory) and at most 168 registers a thread let a CTA of the next kernel become
 // resident beside one of this kernel, so its weight prefetch starts while this
 // kernel's last tiles finish (measured faster than an 8-stage ring that needs the
-// whole SM); partial slots are loaded two at a time to stay inside the registers.
+// whole SM); partial slots are loaded two at a time to stay inside the registers
+// (four at a time, measured, gained nothing).
 constexpr int kFused16Stages = 5;
 constexpr int kFusedCtasPerSm = 2;
 constexpr int kFused16PartialBatch = 2;
@@ -181,10 +179,10 @@ __device__ __forceinline__ bool fused_epilogue(const Fuse& fz, float* C, int ldc
     float* rope_c = xch + 128 * BN;       // [BN][64] cos / sin at each token's position (QKV)
     float* rope_s = rope_c + 64 * BN;
     volatile int* flag = (volatile int*)(rope_s + 64 * BN);
+    constexpr int kParts = 128 / BN;
     {
         // s_row[j] = rsqrt(sum_i ssq_in[i][j] / H + eps): 128 / BN threads per token
         // each sum every (128 / BN)-th tile sum, then token j's thread adds them in order
-        constexpr int kParts = 128 / BN;
         const bool need_s = fz.op == FUSE_QKV || fz.op == FUSE_SWIGLU || fz.op == FUSE_COLSCALE;
         const int j = e % BN, part = e / BN;
         float t = 0.f;
@@ -756,378 +754,6 @@ int launch_cfg(const bf16* A, int lda, const bf16* W, void* C, int ldc, int M, i
 }
 
 
-// ---------------------------------------------------------------- persistent decode step
-// Kernel-side form of StepLaunch: the tensor maps and the phase schedule.
-struct StepArgs {
-    CUtensorMap tmW[5];  // 3-D {K, N, layers}: qkv, o, gate/up, down; lm_head (depth 1)
-    CUtensorMap tmX[3];  // 2-D: xg [M, H], o [M, nq 128], h [M, I]
-    CUtensorMap tmKV;    // 3-D {128, cache rows, layers}
-    int M, H, I, V, nq, nkv, n_layers, with_head;
-    float eps;
-    const float* attn_norm0;
-    const float* q_norm0;
-    const float* k_norm0;
-    const float* mlp_norm0;
-    long long g_stride;
-    const float* g_after_last;
-    const float* rope_cos;
-    const float* rope_sin;
-    int max_positions;
-    PosIndex pos;
-    bf16* qkv;
-    char* kv_k0;
-    long long kv_layer_bytes, kv_half_bytes;
-    int max_seq;
-    float* x;
-    bf16* xg;
-    float* ssq;
-    bf16* h;
-    float* part;
-    int* tickets;
-    int* barrier;
-    float* logits;
-    uint32_t* status;
-    attn::Args att;
-    int att_items;
-};
-
-enum PhaseKind : int { PH_QKV = 0, PH_ATTN = 1, PH_O = 2, PH_GU = 3, PH_D = 4, PH_LM = 5 };
-
-struct PhaseGeo {
-    int kind, layer, N, K, w, x;  // w / x: indices into tmW / tmX
-};
-
-__device__ __forceinline__ PhaseGeo phase_geo(const StepArgs& A, int ph) {
-    PhaseGeo g;
-    if (ph == 5 * A.n_layers) {
-        g.kind = PH_LM;
-        g.layer = 0;
-    } else {
-        g.kind = ph % 5;
-        g.layer = ph / 5;
-    }
-    const int nqkv = (A.nq + 2 * A.nkv) * 128;
-    switch (g.kind) {
-        case PH_QKV: g.N = nqkv; g.K = A.H; g.w = 0; g.x = 0; break;
-        case PH_O: g.N = A.H; g.K = A.nq * 128; g.w = 1; g.x = 1; break;
-        case PH_GU: g.N = 2 * A.I; g.K = A.H; g.w = 2; g.x = 0; break;
-        case PH_D: g.N = A.H; g.K = A.I; g.w = 3; g.x = 2; break;
-        case PH_LM: g.N = A.V; g.K = A.H; g.w = 4; g.x = 0; break;
-        default: g.N = 0; g.K = 0; g.w = 0; g.x = 0; break;
-    }
-    return g;
-}
-
-// The fused op of a GEMM phase (the same Fuse the per-launch decode path builds).
-__device__ __forceinline__ void phase_fuse(const StepArgs& A, const PhaseGeo& g, Fuse& f) {
-    f = Fuse{};
-    f.tickets = A.tickets;
-    f.part = A.part;
-    f.ssq_in = A.ssq;
-    f.n_ssq = A.H / 128;
-    f.H = A.H;
-    f.eps = A.eps;
-    f.status = A.status;
-    const long long gl = (long long)g.layer * A.g_stride;
-    if (g.kind == PH_QKV) {
-        f.op = FUSE_QKV;
-        f.nq = A.nq;
-        f.nkv = A.nkv;
-        f.gq = A.q_norm0 + gl;
-        f.gk = A.k_norm0 + gl;
-        f.rope_cos = A.rope_cos;
-        f.rope_sin = A.rope_sin;
-        f.max_positions = A.max_positions;
-        f.pos = A.pos;
-        f.q_out = A.qkv;
-        f.q_ld = (A.nq + 2 * A.nkv) * 128;
-        f.k_cache = (bf16*)(A.kv_k0 + (long long)g.layer * A.kv_layer_bytes);
-        f.v_cache = (bf16*)(A.kv_k0 + (long long)g.layer * A.kv_layer_bytes + A.kv_half_bytes);
-        f.max_seq = A.max_seq;
-    } else if (g.kind == PH_O || g.kind == PH_D) {
-        f.op = FUSE_RESID;
-        f.x = A.x;
-        f.g_next = g.kind == PH_O ? A.mlp_norm0 + gl
-                                  : (g.layer + 1 < A.n_layers ? A.attn_norm0 + gl + A.g_stride : A.g_after_last);
-        f.xg_out = A.xg;
-        f.ssq_out = A.ssq;
-    } else if (g.kind == PH_GU) {
-        f.op = FUSE_SWIGLU;
-        f.h_out = A.h;
-    } else {
-        f.op = FUSE_COLSCALE;
-    }
-}
-
-constexpr int kStepStages = 6;
-
-// A phase of n_iter k-block iterations runs on its first min(C, n_iter) CTAs, so that
-// every active CTA holds at least one iteration (the partial-slot numbering of the
-// fused epilogue relies on it); the others idle through it.
-__device__ __forceinline__ int phase_ctas(long long n_iter, int C) {
-    return n_iter < C ? (int)n_iter : C;
-}
-__device__ __forceinline__ long long seg_begin(long long n_iter, int Cp) {
-    return (int)blockIdx.x < Cp ? (long long)blockIdx.x * n_iter / Cp : 0;
-}
-__device__ __forceinline__ long long seg_begin_next(long long n_iter, int Cp) {
-    return (int)blockIdx.x < Cp ? (long long)(blockIdx.x + 1) * n_iter / Cp : 0;
-}
-
-template <int BN>
-struct StepCfg {
-    using G = Cfg<BN, false, kStepStages, true>;
-    static constexpr int RING = kStepStages * (G::A_BYTES + G::B_BYTES);
-    static constexpr int ATT = RING;                          // 1024-aligned
-    static constexpr int BAR = ATT + attn::kRingBytes;
-    static constexpr int FSCR = BAR + 512;
-    static constexpr int FUSE = FSCR + G::FUSE_FLOATS * 4;
-    static constexpr int SMEM = ((FUSE + (int)sizeof(Fuse) + 15) & ~15) + 1024;
-    static_assert(RING % 1024 == 0, "attention ring alignment");
-    static_assert(SMEM <= 232448, "shared memory per CTA");
-};
-
-template <int BN>
-__global__ void __launch_bounds__(kThreads, 1) decode_step_kernel(const __grid_constant__ StepArgs A) {
-    using SC = StepCfg<BN>;
-    using G = typename SC::G;
-    constexpr int STAGES = kStepStages;
-    extern __shared__ uint8_t smem_raw[];
-    uint8_t* smem = (uint8_t*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
-    uint8_t* sA = smem;
-    uint8_t* sB = smem + STAGES * G::A_BYTES;
-    uint8_t* att_ring = smem + SC::ATT;
-    uint64_t* full = (uint64_t*)(smem + SC::BAR);
-    uint64_t* empty = full + STAGES;
-    uint64_t* tfull = empty + STAGES;
-    uint64_t* tempty = tfull + 2;
-    uint64_t* drain = tempty + 2;
-    uint64_t* att_full = drain + 1;
-    uint32_t* tmem_slot = (uint32_t*)(att_full + attn::kStages);
-    volatile int* abort_flag = (volatile int*)(tmem_slot + 1);
-    int* flag_s = (int*)(tmem_slot + 2);
-    int* last_s = (int*)(tmem_slot + 3);
-    float* fscr = (float*)(smem + SC::FSCR);
-    Fuse* fz_s = (Fuse*)(smem + SC::FUSE);
-
-    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int C = gridDim.x;
-    const int n_ph = 5 * A.n_layers + (A.with_head ? 1 : 0);
-    int* grid_abort = A.barrier + 1;
-
-    if (threadIdx.x == 0) {
-        for (int s = 0; s < STAGES; ++s) {
-            tc::mbar_init(&full[s], 1);
-            tc::mbar_init(&empty[s], 1);
-        }
-        for (int a = 0; a < 2; ++a) {
-            tc::mbar_init(&tfull[a], 1);
-            tc::mbar_init(&tempty[a], 4);
-        }
-        tc::mbar_init(drain, 1);
-        for (int s = 0; s < attn::kStages; ++s) tc::mbar_init(&att_full[s], 1);
-        *abort_flag = 0;
-        tc::fence_mbar_init();
-        for (int i = 0; i < 5; ++i) tc::tma_prefetch_desc(&A.tmW[i]);
-        for (int i = 0; i < 3; ++i) tc::tma_prefetch_desc(&A.tmX[i]);
-        tc::tma_prefetch_desc(&A.tmKV);
-    }
-    if (warp == 1) tc::tmem_alloc(tmem_slot, G::TMEM_COLS);
-    tc::fence_before_sync();
-    __syncthreads();
-    tc::fence_after_sync();
-    const uint32_t tmem_base = *tmem_slot;
-
-    if (warp == 0) {
-        if (lane == 0) {
-            // ------------------------------------------------ TMA producer
-            // Weight tiles of a phase are issued as soon as the ring has room (weights
-            // never change); the activation tiles of phase ph wait until every CTA has
-            // finished phase ph - 1.
-            int stage = 0;
-            uint32_t phase = 0;
-            int armed[STAGES];
-            for (int s = 0; s < STAGES; ++s) armed[s] = -1;
-            bool ok = true;
-            for (int ph = 0; ok && ph < n_ph; ++ph) {
-                const PhaseGeo g = phase_geo(A, ph);
-                if (g.kind == PH_ATTN) continue;
-                const int kblocks = g.K / kBK;
-                const long long n_iter = (long long)(g.N / 128) * kblocks;
-                const int Cp = phase_ctas(n_iter, C);
-                const long long lo = seg_begin(n_iter, Cp), hi = seg_begin_next(n_iter, Cp);
-                const CUtensorMap* tw = &A.tmW[g.w];
-                const CUtensorMap* tx = &A.tmX[g.x];
-                const int z = g.kind == PH_LM ? 0 : g.layer;
-                int pend_stage[STAGES], pend_x[STAGES];
-                int npend = 0;
-                bool waited = false;
-                auto release_pending = [&]() -> bool {
-                    if (!tc::grid_wait(A.barrier, ph * C, abort_flag, grid_abort)) return false;
-                    waited = true;
-                    for (int i = 0; i < npend; ++i)
-                        tc::tma_load_2d(sB + pend_stage[i] * G::B_BYTES, tx, pend_x[i], 0, &full[pend_stage[i]]);
-                    npend = 0;
-                    return true;
-                };
-                Seg sg;
-                for (bool have = seg_at<true>(sg, lo, hi, 1, 1, kblocks); ok && have;
-                     have = seg_at<true>(sg, sg.next, hi, 1, 1, kblocks)) {
-                    for (int kb = sg.kb0; kb < sg.kb1; ++kb) {
-                        if (!tc::mbar_wait(&empty[stage], phase ^ 1, abort_flag)) {
-                            ok = false;
-                            break;
-                        }
-                        tc::mbar_expect_tx(&full[stage], G::A_BYTES + G::B_BYTES);
-                        tc::tma_load_3d(sA + stage * G::A_BYTES, tw, kb * kBK, sg.feat * 128, z, &full[stage]);
-                        if (waited) {
-                            tc::tma_load_2d(sB + stage * G::B_BYTES, tx, kb * kBK, 0, &full[stage]);
-                        } else {
-                            pend_stage[npend] = stage;
-                            pend_x[npend] = kb * kBK;
-                            if (++npend == STAGES && !release_pending()) ok = false;
-                        }
-                        armed[stage] = (int)phase;
-                        if (++stage == STAGES) {
-                            stage = 0;
-                            phase ^= 1;
-                        }
-                        if (!ok) break;
-                    }
-                }
-                if (ok && !waited && !release_pending()) ok = false;
-                if (!ok && npend > 0) {
-                    // abort with weight halves in flight: issue their (in-bounds) activation
-                    // halves too, so that every armed stage completes and can be drained
-                    for (int i = 0; i < npend; ++i)
-                        tc::tma_load_2d(sB + pend_stage[i] * G::B_BYTES, tx, pend_x[i], 0, &full[pend_stage[i]]);
-                    npend = 0;
-                }
-            }
-            if (!ok) {  // abort path: let every copy this thread issued land before exit
-                for (int s = 0; s < STAGES; ++s)
-                    if (armed[s] >= 0) tc::mbar_wait_drain(&full[s], (uint32_t)armed[s]);
-            }
-        }
-    } else if (warp == 1) {
-        if (lane == 0) {
-            // ------------------------------------------------ MMA issuer
-            constexpr uint32_t idesc = tc::idesc_bf16(128, BN);
-            int stage = 0;
-            uint32_t phase = 0;
-            int acc = 0;
-            uint32_t acc_phase = 0;
-            bool ok = true, issued = false;
-            for (int ph = 0; ok && ph < n_ph; ++ph) {
-                const PhaseGeo g = phase_geo(A, ph);
-                if (g.kind == PH_ATTN) continue;
-                const int kblocks = g.K / kBK;
-                const long long n_iter = (long long)(g.N / 128) * kblocks;
-                const int Cp = phase_ctas(n_iter, C);
-                const long long lo = seg_begin(n_iter, Cp), hi = seg_begin_next(n_iter, Cp);
-                Seg sg;
-                for (bool have = seg_at<true>(sg, lo, hi, 1, 1, kblocks); ok && have;
-                     have = seg_at<true>(sg, sg.next, hi, 1, 1, kblocks)) {
-                    if (!tc::mbar_wait(&tempty[acc], acc_phase ^ 1, abort_flag)) {
-                        ok = false;
-                        break;
-                    }
-                    tc::fence_after_sync();
-                    const uint32_t d = tmem_base + (uint32_t)(acc * G::ACC_COLS);
-                    for (int kb = sg.kb0; kb < sg.kb1; ++kb) {
-                        if (!tc::mbar_wait(&full[stage], phase, abort_flag)) {
-                            ok = false;
-                            break;
-                        }
-                        tc::fence_after_sync();
-                        const uint32_t a0 = tc::smem_u32(sA + stage * G::A_BYTES);
-                        const uint32_t b0 = tc::smem_u32(sB + stage * G::B_BYTES);
-#pragma unroll
-                        for (int k = 0; k < kBK / 16; ++k)
-                            tc::mma_bf16(d, tc::sw128_desc(a0 + k * 32), tc::sw128_desc(b0 + k * 32), idesc,
-                                         (kb != sg.kb0 || k) ? 1u : 0u);
-                        issued = true;
-                        tc::mma_commit(&empty[stage]);
-                        if (++stage == STAGES) {
-                            stage = 0;
-                            phase ^= 1;
-                        }
-                    }
-                    if (!ok) break;
-                    tc::mma_commit(&tfull[acc]);
-                    acc ^= 1;
-                    if (acc == 0) acc_phase ^= 1;
-                }
-            }
-            if (!ok && issued) {  // abort path: wait for the MMAs in flight
-                tc::mma_commit(drain);
-                tc::mbar_wait_drain(drain, 0);
-            }
-        }
-    } else {
-        // ---------------------------------------------------- epilogue / attention (warps 2..5)
-        const int e = threadIdx.x - 64;
-        int acc = 0;
-        uint32_t acc_phase = 0;
-        int att_tiles = 0;
-        bool ok = true;
-        for (int ph = 0; ph < n_ph; ++ph) {
-            const PhaseGeo g = phase_geo(A, ph);
-            if (e == 0) {
-                *flag_s = tc::grid_wait(A.barrier, ph * C, abort_flag, grid_abort) ? 1 : 0;
-                if (g.kind != PH_ATTN) phase_fuse(A, g, *fz_s);
-            }
-            tc::bar128();
-            ok = *flag_s != 0;
-            if (!ok) break;
-            if (g.kind == PH_ATTN) {
-                const int n_split = A.att.n_split;
-                for (int it = blockIdx.x; ok && it < A.att_items; it += C) {
-                    const int split = it % n_split, bk = it / n_split;
-                    ok = attn::decode_item(A.att, &A.tmKV, g.layer, split, bk / A.nkv, bk % A.nkv, att_ring,
-                                           att_full, att_tiles, abort_flag, last_s, e);
-                }
-            } else {
-                const int kblocks = g.K / kBK;
-                const long long n_iter = (long long)(g.N / 128) * kblocks;
-                const int Cp = phase_ctas(n_iter, C);
-                const long long lo = seg_begin(n_iter, Cp), hi = seg_begin_next(n_iter, Cp);
-                ok = fused_epilogue<BN, STAGES>(*fz_s, A.logits, A.V, A.M, g.N, kblocks, n_iter, lo, hi, Cp,
-                                                tmem_base, tfull, tempty, acc, acc_phase, fscr, abort_flag);
-            }
-            ok = tc::bar128_and(ok);  // every epilogue thread's stores of this phase are done
-            if (!ok) break;
-            if (e == 0) tc::grid_arrive(A.barrier);
-        }
-        if (!ok && e == 0) atomicExch(grid_abort, 1);
-    }
-
-    tc::fence_before_sync();
-    __syncthreads();
-    if (threadIdx.x == 0 && *abort_flag) atomicOr(A.status, QK_STATUS_TIMEOUT);
-    if (warp == 1) {
-        tc::fence_after_sync();
-        tc::tmem_dealloc(tmem_base, G::TMEM_COLS);
-    }
-}
-
-// 3-D bf16 map over `layers` matrices of rows x inner elements (row stride inner,
-// layer stride layer_bytes), box 64 x box_rows x 1, 128-byte swizzle.
-bool make_map3(CUtensorMap* map, const void* base, int inner, int rows, int layers, size_t layer_bytes,
-               int box_rows) {
-    EncodeTiledFn fn = encode_fn();
-    if (!fn || layers < 1) return false;
-    if (layers == 1) layer_bytes = (size_t)rows * inner * 2;
-    if (layer_bytes % 16) return false;
-    cuuint64_t dims[3] = {(cuuint64_t)inner, (cuuint64_t)rows, (cuuint64_t)layers};
-    cuuint64_t strides[2] = {(cuuint64_t)inner * 2, (cuuint64_t)layer_bytes};
-    cuuint32_t box[3] = {(cuuint32_t)kBK, (cuuint32_t)box_rows, 1};
-    cuuint32_t estr[3] = {1, 1, 1};
-    return fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(base), dims, strides, box, estr,
-              CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
-              CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
-}
-
 }  // namespace
 
 bool gemm_tc_supported(const void* A, int lda, int N, int K) {
@@ -1170,103 +796,5 @@ int launch_gemm_tc_fused(const bf16* A, int lda, const bf16* W, float* out, int 
                                           num_sms, status, s, &f);
 }
 
-
-bool decode_persist_supported(int M, int num_sms) {
-    static int ok_sm = -1;  // co-residency of one CTA per SM (checked once per process)
-    if (M < 1 || M > 16 || num_sms < 1) return false;
-    if (ok_sm < 0) {
-        int dev = 0, coop = 0, per_sm = 0;
-        ok_sm = 0;
-        if (cudaGetDevice(&dev) == cudaSuccess &&
-            cudaDeviceGetAttribute(&coop, cudaDevAttrCooperativeLaunch, dev) == cudaSuccess && coop &&
-            cudaFuncSetAttribute(decode_step_kernel<16>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                 StepCfg<16>::SMEM) == cudaSuccess &&
-            cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, decode_step_kernel<16>, kThreads,
-                                                          StepCfg<16>::SMEM) == cudaSuccess &&
-            per_sm >= 1)
-            ok_sm = 1;
-        (void)cudaGetLastError();
-    }
-    return ok_sm == 1 && encode_fn() != nullptr;
-}
-
-int launch_decode_persist(const StepLaunch& L, int num_sms, cudaStream_t s) {
-    if (!decode_persist_supported(L.M, num_sms)) return QK_EINVAL;
-    StepArgs A;
-    memset(&A, 0, sizeof(A));
-    const int nqkv = (L.nq + 2 * L.nkv) * 128;
-    bool ok = make_map3(&A.tmW[0], L.w_qkv0, L.H, nqkv, L.n_layers, L.w_stride, 128) &&
-              make_map3(&A.tmW[1], L.w_o0, L.nq * 128, L.H, L.n_layers, L.w_stride, 128) &&
-              make_map3(&A.tmW[2], L.w_gu0, L.H, 2 * L.I, L.n_layers, L.w_stride, 128) &&
-              make_map3(&A.tmW[3], L.w_d0, L.I, L.H, L.n_layers, L.w_stride, 128) &&
-              (!L.with_head || make_map3(&A.tmW[4], L.lm_head, L.H, L.V, 1, 0, 128)) &&
-              make_map(&A.tmX[0], L.xg, L.H, L.M, L.H, 16) &&
-              make_map(&A.tmX[1], L.o, L.nq * 128, L.M, L.nq * 128, 16) &&
-              make_map(&A.tmX[2], L.h, L.I, L.M, L.I, 16) &&
-              make_kv_map(&A.tmKV, L.kv_k0, L.max_batch, L.nkv, L.max_seq, L.n_layers, L.kv_layer_bytes);
-    if (!ok) return QK_ECUDA;
-    if (!L.with_head) A.tmW[4] = A.tmW[0];  // never read
-    A.M = L.M;
-    A.H = L.H;
-    A.I = L.I;
-    A.V = L.V;
-    A.nq = L.nq;
-    A.nkv = L.nkv;
-    A.n_layers = L.n_layers;
-    A.with_head = L.with_head ? 1 : 0;
-    A.eps = L.eps;
-    A.attn_norm0 = L.attn_norm0;
-    A.q_norm0 = L.q_norm0;
-    A.k_norm0 = L.k_norm0;
-    A.mlp_norm0 = L.mlp_norm0;
-    A.g_stride = (long long)L.g_stride;
-    A.g_after_last = L.g_after_last;
-    A.rope_cos = L.rope_cos;
-    A.rope_sin = L.rope_sin;
-    A.max_positions = L.max_positions;
-    A.pos = L.pos;
-    A.qkv = L.qkv;
-    A.kv_k0 = L.kv_k0;
-    A.kv_layer_bytes = (long long)L.kv_layer_bytes;
-    A.kv_half_bytes = (long long)L.kv_half_bytes;
-    A.max_seq = L.max_seq;
-    A.x = L.x;
-    A.xg = L.xg;
-    A.ssq = L.ssq;
-    A.h = L.h;
-    A.part = L.part;
-    A.tickets = L.tickets;
-    A.barrier = L.barrier;
-    A.logits = L.logits;
-    A.status = L.status;
-    attn::Args& a = A.att;
-    a.q = L.qkv;
-    a.q_ld = nqkv;
-    a.nq = L.nq;
-    a.nkv = L.nkv;
-    a.max_batch = L.max_batch;
-    a.max_seq = L.max_seq;
-    a.pos = L.pos;
-    attn_decode_split_persist(L.M, L.nkv, L.max_seq, num_sms, &a.chunk, &a.n_split);
-    attn_scratch_parts(L.attn_scratch, L.M, L.nq, L.nkv, L.max_seq, num_sms, a.n_split, &a.part_o,
-                       &a.part_ml, &a.tickets);
-    a.out = L.o;
-    a.status = L.status;
-    A.att_items = a.n_split * L.M * L.nkv;
-    cudaLaunchConfig_t cfg = {};
-    cfg.gridDim = dim3(num_sms);
-    cfg.blockDim = dim3(kThreads);
-    cfg.dynamicSmemBytes = StepCfg<16>::SMEM;
-    cfg.stream = s;
-    cudaLaunchAttribute attr[1];
-    attr[0].id = cudaLaunchAttributeCooperative;
-    attr[0].val.cooperative = 1;
-    cfg.attrs = attr;
-    cfg.numAttrs = 1;
-    cudaError_t e = cudaLaunchKernelEx(&cfg, decode_step_kernel<16>, A);
-    if (e != cudaSuccess) return cuda_error(e, "persistent decode step launch");
-    note_launch();
-    return QK_OK;
-}
 
 }  // namespace qk

@@ -133,9 +133,6 @@ static const int kSplitMaxRows = 64;
 // SMs; the last CTA of each tile sums its fp32 partials in k order and applies
 // QK-norm + RoPE, the residual add (with the next norm's statistics) or SwiGLU.
 static const int kTicketSlots = 4096;
-// The ticket region also holds the persistent decode-step kernel's phase counter and
-// grid abort flag (words kTicketSlots, kTicketSlots + 1); it is zeroed every step.
-static const int kTicketWords = kTicketSlots + 64;
 
 static bool use_splitk(const Model& m, int M) {
     const qk_config& c = m.cfg;
@@ -182,7 +179,7 @@ static int workspace_layout(const Model& m, int kind, int B, int T, int max_seq,
     w->part = fused ? (float*)take(splitk_part_floats(m, B) * 4) : nullptr;
     w->xg = fused ? (bf16*)take(M * H * 2) : nullptr;
     w->ssq = fused ? (float*)take((H / 128) * M * 4) : nullptr;
-    w->tickets = fused ? (int*)take(kTicketWords * 4) : nullptr;
+    w->tickets = fused ? (int*)take(kTicketSlots * 4) : nullptr;
     w->attn = nullptr;
     if (kind == QK_CALL_DECODE && c.dtype == QK_DTYPE_BF16 &&
         attn_decode_supported(c.head_dim, c.n_q_heads, c.n_kv_heads)) {
@@ -308,83 +305,6 @@ static void run_layer_fused(Model& m, int l, const Workspace& w, int M, PosIndex
     pr = prof_open(m, QK_PROF_DOWN, s);
     gemm(w.h, I, L.w_d, H, I, fd);
     prof_close(m, pr, s);
-}
-
-// The persistent decode-step kernel over layers [l0, l0 + n) of the model (one layer
-// for qk_decode_layer, every layer plus the lm_head for a decode step).  On entry
-// w.x / w.xg / w.ssq hold the residual stream, bf16(x * g_attn(l0)) and its tile
-// sums of squares; the last layer's down epilogue forms xg with g_after.
-static int run_decode_persist(Model& m, const Workspace& w, int M, PosIndex pos, const KVView& kv,
-                              int l0, int n, const float* g_after, float* logits, cudaStream_t s) {
-    const qk_config& c = m.cfg;
-    StepLaunch L{};
-    L.M = M;
-    L.H = c.hidden;
-    L.I = c.intermediate;
-    L.V = c.vocab;
-    L.nq = c.n_q_heads;
-    L.nkv = c.n_kv_heads;
-    L.n_layers = n;
-    L.with_head = logits != nullptr;
-    L.eps = (float)c.rms_eps;
-    const LayerW& A0 = m.layers[l0];
-    L.w_qkv0 = (const bf16*)A0.w_qkv;
-    L.w_o0 = (const bf16*)A0.w_o;
-    L.w_gu0 = (const bf16*)A0.w_gu;
-    L.w_d0 = (const bf16*)A0.w_d;
-    L.attn_norm0 = A0.attn_norm;
-    L.q_norm0 = A0.q_norm;
-    L.k_norm0 = A0.k_norm;
-    L.mlp_norm0 = A0.mlp_norm;
-    if (n > 1) {
-        // every layer's region lies at the same stride from the previous one
-        const LayerW& A1 = m.layers[l0 + 1];
-        L.w_stride = (size_t)((const char*)A1.w_qkv - (const char*)A0.w_qkv);
-        L.g_stride = (size_t)(A1.attn_norm - A0.attn_norm);
-        for (int l = l0 + 1; l < l0 + n; ++l) {
-            const LayerW& P = m.layers[l - 1];
-            const LayerW& Q = m.layers[l];
-            if ((size_t)((const char*)Q.w_qkv - (const char*)P.w_qkv) != L.w_stride ||
-                (size_t)((const char*)Q.w_o - (const char*)P.w_o) != L.w_stride ||
-                (size_t)((const char*)Q.w_gu - (const char*)P.w_gu) != L.w_stride ||
-                (size_t)((const char*)Q.w_d - (const char*)P.w_d) != L.w_stride ||
-                (size_t)(Q.attn_norm - P.attn_norm) != L.g_stride ||
-                (size_t)(Q.q_norm - P.q_norm) != L.g_stride || (size_t)(Q.k_norm - P.k_norm) != L.g_stride ||
-                (size_t)(Q.mlp_norm - P.mlp_norm) != L.g_stride)
-                return set_error(QK_EINVAL, "packed layers are not evenly strided");
-        }
-    }
-    L.lm_head = (const bf16*)m.lm_head;
-    L.g_after_last = g_after;
-    L.rope_cos = m.rope_cos;
-    L.rope_sin = m.rope_sin;
-    L.max_positions = c.max_positions;
-    L.pos = pos;
-    L.qkv = (bf16*)w.qkv;
-    L.kv_k0 = (char*)kv.k(l0);
-    L.kv_layer_bytes = kv.layer_bytes;
-    L.kv_half_bytes = kv.half_bytes;
-    L.max_batch = kv.max_batch;
-    L.max_seq = kv.max_seq;
-    L.x = w.x;
-    L.xg = w.xg;
-    L.ssq = w.ssq;
-    L.h = (bf16*)w.h;
-    L.o = (bf16*)w.o;
-    L.part = w.part;
-    L.tickets = w.tickets;
-    L.barrier = w.tickets + kTicketSlots;
-    L.attn_scratch = w.attn;
-    L.logits = logits;
-    L.status = m.status;
-    const bool pr = prof_open(m, QK_PROF_STEP, s);
-    const int rc = launch_decode_persist(L, m.num_sms, s);
-    prof_close(m, pr, s);
-    return rc;
-}
-
-static bool use_persist(const Model& m, const Workspace& w, int M) {
-    return w.part && w.attn && decode_persist_supported(M, m.num_sms);
 }
 
 // Final norm of M_out selected rows (row r of the output reads residual row r * in_step + in_off),
@@ -611,7 +531,7 @@ void qk_model_free(qk_model* m) {
 int qk_profile_begin(qk_model* mh, int kind, int max_launches) {
     if (!mh) return set_error(QK_EINVAL, "null argument");
     Model& m = *(Model*)mh;
-    if (kind < QK_PROF_QKV || kind > QK_PROF_STEP) return set_error(QK_EINVAL, "unknown kernel class %d", kind);
+    if (kind < QK_PROF_QKV || kind > QK_PROF_LM_HEAD) return set_error(QK_EINVAL, "unknown kernel class %d", kind);
     if (max_launches < 1 || max_launches > (1 << 20)) return set_error(QK_EINVAL, "max_launches out of range");
     prof_release(m);
     m.prof_ev.resize(2 * (size_t)max_launches);
@@ -759,26 +679,9 @@ static int decode_impl(Model& m, void* kv, int max_batch, int max_seq, TokIndex 
     KVView view = cache_view(m, kv, max_batch, max_seq);
     QK_TRY(clear_attn_tickets(m, w, B, max_seq, s));
     m.in_decode = true;
-    if (w.part && use_persist(m, w, B)) {
-        // one persistent kernel for every layer and the lm_head
+    if (w.part) {
         const qk_config& c = m.cfg;
-        QK_TRY_CUDA(cudaMemsetAsync(w.tickets, 0, kTicketWords * sizeof(int), s));
-        launch_embed_gain(m.embed, c.vocab, tok, true, w.x, m.layers[0].attn_norm, w.xg, w.ssq, B,
-                          c.hidden, m.status, s);
-        const bool head = logits || lp || am;
-        float* z = logits ? logits : w.logits;
-        int rc = run_decode_persist(m, w, B, pos, view, 0, c.n_layers, m.final_norm,
-                                    head ? z : nullptr, s);
-        if (rc != QK_OK) {
-            m.in_decode = false;
-            return rc;
-        }
-        if (lp || am)
-            launch_logits_reduce(z, B, c.vocab, oi, lp, am, m.status, s, nullptr,
-                                 m.sampling.out_tokens ? &m.sampling : nullptr);
-    } else if (w.part) {
-        const qk_config& c = m.cfg;
-        QK_TRY_CUDA(cudaMemsetAsync(w.tickets, 0, kTicketWords * sizeof(int), s));
+        QK_TRY_CUDA(cudaMemsetAsync(w.tickets, 0, kTicketSlots * sizeof(int), s));
         launch_embed_gain(m.embed, c.vocab, tok, true, w.x, m.layers[0].attn_norm, w.xg, w.ssq, B,
                           c.hidden, m.status, s);
         for (int l = 0; l < c.n_layers; ++l)
@@ -842,20 +745,11 @@ int qk_decode_layer(qk_model* mh, int layer, void* kv, int max_batch, int max_se
     m.in_decode = true;
     if (w.part) {
         const LayerW& L = m.layers[layer];
-        QK_TRY_CUDA(cudaMemsetAsync(w.tickets, 0, kTicketWords * sizeof(int), s));
+        QK_TRY_CUDA(cudaMemsetAsync(w.tickets, 0, kTicketSlots * sizeof(int), s));
         launch_embed_gain(nullptr, m.cfg.vocab, TokIndex{}, false, w.x, L.attn_norm, w.xg, w.ssq, B,
                           m.cfg.hidden, m.status, s);
-        if (use_persist(m, w, B)) {
-            int rc = run_decode_persist(m, w, B, PosIndex{pos, 0, 1}, cache_view(m, kv, max_batch, max_seq),
-                                        layer, 1, L.attn_norm, nullptr, s);
-            if (rc != QK_OK) {
-                m.in_decode = false;
-                return rc;
-            }
-        } else {
-            run_layer_fused(m, layer, w, B, PosIndex{pos, 0, 1}, cache_view(m, kv, max_batch, max_seq),
-                            L.attn_norm, s);
-        }
+        run_layer_fused(m, layer, w, B, PosIndex{pos, 0, 1}, cache_view(m, kv, max_batch, max_seq),
+                        L.attn_norm, s);
     } else {
         run_layer(m, layer, w, B, PosIndex{pos, 0, 1}, cache_view(m, kv, max_batch, max_seq), s);
     }

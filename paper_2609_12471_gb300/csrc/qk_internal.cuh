@@ -318,54 +318,6 @@ struct Fuse {
 // W [N, K]; out is the op's fp32 logits for FUSE_COLSCALE, unused otherwise.
 int launch_gemm_tc_fused(const bf16* A, int lda, const bf16* W, float* out, int M, int N, int K,
                          const Fuse& f, int num_sms, uint32_t* status, cudaStream_t s);
-// One decode step (or one decode layer) as a single persistent, cooperatively
-// launched kernel (k_gemm_tc.cu): per layer the phases QKV (+ QK-norm, RoPE, cache
-// write), attention, O (+ residual, next-norm statistics), gate/up (+ SwiGLU), down
-// (+ residual, next-norm statistics), then optionally the lm_head (final-norm
-// scale, fp32 logits); the phases are separated by a grid-wide barrier with bounded
-// waits, and each CTA's weight stream runs on across phase boundaries.  Layer l of
-// the launch uses the weights at w_*0 + l * w_stride bytes, the gains at
-// *_norm0 + l * g_stride floats and the cache at kv_k0 + l * kv_layer_bytes.
-struct StepLaunch {
-    int M, H, I, V, nq, nkv, n_layers;
-    bool with_head;
-    float eps;
-    const bf16* w_qkv0;
-    const bf16* w_o0;
-    const bf16* w_gu0;
-    const bf16* w_d0;
-    size_t w_stride;
-    const bf16* lm_head;
-    const float* attn_norm0;
-    const float* q_norm0;
-    const float* k_norm0;
-    const float* mlp_norm0;
-    size_t g_stride;
-    const float* g_after_last;  // the gain the last layer's down epilogue applies for xg
-    const float* rope_cos;
-    const float* rope_sin;
-    int max_positions;
-    PosIndex pos;
-    bf16* qkv;                  // [M, (nq + 2 nkv) 128] (q part used)
-    char* kv_k0;                // layer 0's K cache of the launch
-    size_t kv_layer_bytes, kv_half_bytes;
-    int max_batch, max_seq;
-    float* x;
-    bf16* xg;
-    float* ssq;
-    bf16* h;
-    bf16* o;
-    float* part;
-    int* tickets;
-    int* barrier;               // [2]: phase arrivals, grid abort flag (zero on entry)
-    void* attn_scratch;
-    float* logits;              // [M, V] when with_head
-    uint32_t* status;
-};
-// M <= 16 rows, head_dim 128, G <= 8; returns QK_EINVAL when the shape is not supported.
-bool decode_persist_supported(int M, int num_sms);
-int launch_decode_persist(const StepLaunch& L, int num_sms, cudaStream_t s);
-
 inline size_t gemm_fused_part_floats(int M, int N, int num_sms) {
     return ((size_t)num_sms + (size_t)(N / 128)) * (size_t)M * 128;
 }
@@ -398,8 +350,6 @@ void attn_decode_split(int B, int nkv, int max_seq, int num_sms, int* chunk, int
 size_t attn_decode_scratch_bytes(int B, int nq, int nkv, int max_seq, int num_sms);
 // Merge tickets inside that scratch; zero them (B * nkv ints) before a decode step.
 int* attn_decode_tickets(void* scratch, int B, int nq, int nkv, int max_seq, int num_sms);
-// Split of the persistent decode-step kernel's attention phase (one item slot per SM).
-void attn_decode_split_persist(int B, int nkv, int max_seq, int num_sms, int* chunk, int* n_split);
 // The partial, (m, l) and ticket regions of that scratch.
 void attn_scratch_parts(void* scratch, int B, int nq, int nkv, int max_seq, int num_sms, int n_split,
                         float** part_o, float2** part_ml, int** tickets);

@@ -105,12 +105,6 @@ __device__ __forceinline__ void tma_load_3d(void* dst, const CUtensorMap* map, i
         "l"(map), "r"(x), "r"(y), "r"(z), "r"(smem_u32(bar))
         : "memory");
 }
-// Warms L2 with a tile of a 3-D tensor map (no shared memory, no completion signal).
-__device__ __forceinline__ void tma_prefetch_l2_3d(const CUtensorMap* map, int x, int y, int z) {
-    asm volatile("cp.async.bulk.prefetch.tensor.3d.L2.global [%0, {%1, %2, %3}];" ::"l"(map), "r"(x),
-                 "r"(y), "r"(z)
-                 : "memory");
-}
 __device__ __forceinline__ void tma_prefetch_desc(const CUtensorMap* map) {
     asm volatile("prefetch.tensormap [%0];" ::"l"(map) : "memory");
 }
@@ -133,42 +127,6 @@ __device__ __forceinline__ bool bar128_and(bool pred) {
         : "r"((uint32_t)pred)
         : "memory");
     return r != 0;
-}
-
-// ---------------------------------------------------------------- grid-wide phase barrier
-// Arrival: after a CTA barrier over the arriving threads, one thread publishes the
-// CTA's earlier global stores (release at GPU scope, cumulative through the barrier).
-__device__ __forceinline__ void grid_arrive(int* ctr) {
-    asm volatile("fence.proxy.async.global;" ::: "memory");
-    asm volatile("red.release.gpu.global.add.s32 [%0], 1;" ::"l"(ctr) : "memory");
-}
-__device__ __forceinline__ int ld_acquire_gpu(const int* p) {
-    int v;
-    asm volatile("ld.acquire.gpu.global.s32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
-    return v;
-}
-// Waits (one thread) until *ctr >= target.  Gives up, raising the CTA's abort flag
-// and the grid's, after `limit` SM cycles or as soon as another CTA gave up.  On
-// success the acquired stores are ordered before this thread's later async-proxy
-// (TMA) reads as well.
-__device__ __forceinline__ bool grid_wait(const int* ctr, int target, volatile int* abort_flag,
-                                          int* grid_abort, long long limit = kWaitCycles) {
-    if (ld_acquire_gpu(ctr) < target) {
-        const long long t0 = clock64();
-        while (ld_acquire_gpu(ctr) < target) {
-            if (*abort_flag || *(volatile int*)grid_abort) {
-                *abort_flag = 1;
-                return false;
-            }
-            if (clock64() - t0 > limit) {
-                *abort_flag = 1;
-                atomicExch(grid_abort, 1);
-                return false;
-            }
-        }
-    }
-    asm volatile("fence.proxy.async.global;" ::: "memory");
-    return true;
 }
 
 // ---------------------------------------------------------------- TMEM / tcgen05
