@@ -62,7 +62,9 @@ struct Cfg {
     static constexpr int TMEM_COLS = pow2_at_least(2 * ACC_COLS);
     // fused epilogue scratch (floats): s_row[64], p_row[64] (int), red[4][64], xch[BN][128],
     // cos / sin [2][BN][64], flag
-    static constexpr int FUSE_FLOATS = FUSED ? 64 + 64 + 4 * 64 + 128 * BN + 128 * BN + 4 : 0;
+    // plain GEMM: the EPI_LSE transpose buffer [16 tokens][128 features] and the tile's targets
+    static constexpr int FUSE_FLOATS = FUSED ? 64 + 64 + 4 * 64 + 128 * BN + 128 * BN + 4
+                                             : 16 * 128 + (BN > 16 ? BN : 16);
     static constexpr int SMEM =
         STAGES * (A_BYTES + B_BYTES) + 1024 /*align*/ + 256 /*barriers*/ + FUSE_FLOATS * 4;
     static_assert(TMEM_COLS <= 512, "accumulators exceed TMEM");
@@ -621,11 +623,31 @@ __global__ void __launch_bounds__(kThreads, FUSED && BN == 16 ? kFusedCtasPerSm 
         const int q = warp & 3;
         int acc = 0;
         uint32_t acc_phase = 0;
+        const int e = threadIdx.x - 64;
+        float* tr = fscr;                        // EPI_LSE: [16][128] logits of a token chunk
+        int* tgt_s = (int*)(fscr + 16 * 128);    // EPI_LSE: the tile's targets
+        const bool lse = !SWIGLU && epi == EPI_LSE;
+        const int n_vt = N / 128;
         for (int t = blockIdx.x; t < num_tiles; t += gridDim.x) {
             const int split = t % n_split, rest = t / n_split;
             const int feat = rest / n_tok, tok = rest % n_tok;
+            if (lse) {
+                // targets of the tile's tokens (rows past M and last positions: none)
+                for (int j = e; j < BN; j += 128) {
+                    const int m = tok * BN + j;
+                    int tg = -1;
+                    if (m < M) {
+                        const int g = fz.lse_row0 + m;
+                        if (g % fz.lse_T < fz.lse_T - 1) {
+                            tg = fz.lse_tok[g + 1];
+                            if (tg < 0 || tg >= N) tg = 0;  // flagged by the combine
+                        }
+                    }
+                    tgt_s[j] = tg;
+                }
+            }
             bool ok = tc::mbar_wait(&tfull[acc], acc_phase, abort_flag, wlim);
-            ok = __all_sync(0xffffffffu, ok);
+            ok = lse ? tc::bar128_and(ok) : __all_sync(0xffffffffu, ok);
             if (!ok) break;
             tc::fence_after_sync();
             const int f = feat * 128 + q * 32 + lane;
@@ -652,6 +674,45 @@ __global__ void __launch_bounds__(kThreads, FUSED && BN == 16 ? kFusedCtasPerSm 
                 uint32_t u[16];
                 if (SWIGLU) tc::tmem_ld16(tbase + BN + c0, u);
                 tc::tmem_wait_ld();
+                if (lse) {
+                    // 16 tokens x 128 features through shared memory, then 8 threads per
+                    // token: max / lowest arg-max / sum exp over 16 features each, merged
+                    // over the 8 lanes in a fixed order
+#pragma unroll
+                    for (int j = 0; j < 16; ++j) {
+                        const float v = __uint_as_float(r[j]);
+                        tr[j * 128 + q * 32 + lane] = v;
+                        if (tgt_s[c0 + j] == f && tok0 + j < M) fz.lse_zt[tok0 + j] = v;
+                    }
+                    tc::bar128();
+                    const int col = e >> 3, part = e & 7;
+                    const float* zc = tr + col * 128 + part * 16;
+                    float mv = zc[0];
+                    int mi = part * 16;
+#pragma unroll
+                    for (int k = 1; k < 16; ++k)
+                        if (zc[k] > mv) mv = zc[k], mi = part * 16 + k;
+                    float sv = 0.f;
+#pragma unroll
+                    for (int k = 0; k < 16; ++k) sv += expf(zc[k] - mv);
+#pragma unroll
+                    for (int o = 1; o < 8; o <<= 1) {
+                        const float m2 = __shfl_xor_sync(0xffffffffu, mv, o);
+                        const float s2 = __shfl_xor_sync(0xffffffffu, sv, o);
+                        const int i2 = __shfl_xor_sync(0xffffffffu, mi, o);
+                        const float mx = fmaxf(mv, m2);
+                        sv = sv * expf(mv - mx) + s2 * expf(m2 - mx);
+                        mi = mv > m2 ? mi : (m2 > mv ? i2 : min(mi, i2));
+                        mv = mx;
+                    }
+                    const int m = tok0 + col;
+                    if (part == 0 && m < M) {
+                        fz.lse_ms[(size_t)m * n_vt + feat] = make_float2(mv, sv);
+                        fz.lse_idx[(size_t)m * n_vt + feat] = feat * 128 + mi;
+                    }
+                    tc::bar128();  // the buffer is rewritten by the next chunk
+                    continue;
+                }
 #pragma unroll
                 for (int j = 0; j < 16; ++j) {
                     const int m = tok0 + j;
@@ -763,8 +824,17 @@ bool gemm_tc_supported(const void* A, int lda, int N, int K) {
 
 // bf16 linear layer on the tensor cores; token-tile width chosen from M.
 int launch_gemm_tc(const bf16* A, int lda, const bf16* W, void* C, int ldc, int M, int N, int K,
-                   int epi, int num_sms, uint32_t* status, cudaStream_t s, long long test_wait) {
+                   int epi, int num_sms, uint32_t* status, cudaStream_t s, long long test_wait,
+                   const Fuse* lse) {
     if (M <= 0) return QK_OK;
+    if (epi == EPI_LSE) {
+        if (!lse || N % 128) return QK_EINVAL;
+        if (M <= 16) return launch_cfg<16, false, 8>(A, lda, W, C, ldc, M, N, K, epi, 1, num_sms, status, s, lse, test_wait);
+        if (M <= 32) return launch_cfg<32, false, 8>(A, lda, W, C, ldc, M, N, K, epi, 1, num_sms, status, s, lse, test_wait);
+        if (M <= 64) return launch_cfg<64, false, 8>(A, lda, W, C, ldc, M, N, K, epi, 1, num_sms, status, s, lse, test_wait);
+        if (M <= 128) return launch_cfg<128, false, 6>(A, lda, W, C, ldc, M, N, K, epi, 1, num_sms, status, s, lse, test_wait);
+        return launch_cfg<256, false, 4>(A, lda, W, C, ldc, M, N, K, epi, 1, num_sms, status, s, lse, test_wait);
+    }
     const long long tw = test_wait;
     if (epi == EPI_SWIGLU) {
         if (M <= 16) return launch_cfg<16, true, 6>(A, lda, W, C, ldc, M, N, K, epi, 1, num_sms, status, s, nullptr, tw);

@@ -435,6 +435,82 @@ void launch_logits_reduce(const float* logits, int M, int V, OutIndex oi, float*
              status, g, sa);
 }
 
+// ---------------------------------------------------------------- vocabulary-tile combine
+// One block of 128 threads per logits row: merges the row's per-tile (max, sum of
+// exponentials, lowest arg-max) in a fixed order (thread i takes tiles i, i + 128, ...
+// ascending, then a fixed tree; equal maxima keep the lower index), then
+//   log p(target) = z[target] - (max + log sum exp(z - max)),
+// the arg-max and, with grpo, the GRPO token loss, with the output indexing of
+// logits_reduce_kernel.
+__device__ __forceinline__ void tile_merge(float& m, float& s, int& i, float m2, float s2, int i2) {
+    const float mx = fmaxf(m, m2);
+    if (mx == -INFINITY) return;
+    s = (m == -INFINITY ? 0.f : s * expf(m - mx)) + (m2 == -INFINITY ? 0.f : s2 * expf(m2 - mx));
+    i = m > m2 ? i : (m2 > m ? i2 : min(i, i2));
+    m = mx;
+}
+
+__global__ void __launch_bounds__(128)
+    lse_combine_kernel(const float2* __restrict__ ms, const int* __restrict__ idx,
+                       const float* __restrict__ zt, int n_vt, int V, OutIndex oi,
+                       float* __restrict__ lp, int32_t* __restrict__ am, uint32_t* status,
+                       GrpoArgs grpo) {
+    __shared__ float sm[4], ss[4];
+    __shared__ int si[4];
+    pdl_wait();
+    pdl_trigger();
+    const int r = blockIdx.x;
+    const int g = oi.row0 + r;
+    const int b = g / oi.T, t = g % oi.T;
+    if (t >= oi.out_lim) return;  // uniform over the block
+    float m = -INFINITY, sum = 0.f;
+    int i = 0x7fffffff;
+    const float2* row = ms + (size_t)r * n_vt;
+    const int* rowi = idx + (size_t)r * n_vt;
+    for (int v = threadIdx.x; v < n_vt; v += 128) {
+        const float2 p = row[v];
+        tile_merge(m, sum, i, p.x, p.y, rowi[v]);
+    }
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+        const float m2 = __shfl_xor_sync(0xffffffffu, m, o);
+        const float s2 = __shfl_xor_sync(0xffffffffu, sum, o);
+        const int i2 = __shfl_xor_sync(0xffffffffu, i, o);
+        tile_merge(m, sum, i, m2, s2, i2);
+    }
+    const int w = threadIdx.x >> 5;
+    if ((threadIdx.x & 31) == 0) sm[w] = m, ss[w] = sum, si[w] = i;
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        for (int k = 1; k < 4; ++k) tile_merge(m, sum, i, sm[k], ss[k], si[k]);
+        const size_t o = (size_t)b * oi.out_ld + oi.out_off + t + (oi.dyn_off ? *oi.dyn_off : 0);
+        if (am) am[o] = i;
+        if (lp && oi.tgt) {
+            const int tg = oi.tgt[(size_t)b * oi.tgt_ld + oi.tgt_off + t];
+            if (tg < 0 || tg >= V) atomicOr(status, QK_STATUS_BAD_TOKEN);  // token 0 was used
+            const float l = zt[r] - (m + logf(sum));
+            lp[o] = l;
+            if (grpo.loss_tok) {  // Eq. ppo for this token, where its log-prob is formed
+                const size_t go = (size_t)b * grpo.ld + t;
+                const float ref = grpo.lp_ref ? grpo.lp_ref[go] : l;
+                grpo.loss_tok[go] = grpo_token(l, grpo.lp_old[go], ref,
+                                               grpo_advantage(grpo.rewards, b, grpo.group), grpo);
+            }
+        }
+    }
+}
+
+void launch_lse_combine(const float2* ms, const int* idx, const float* zt, int n_vt, int V, int M,
+                        OutIndex oi, float* lp, int32_t* argmax, uint32_t* status, cudaStream_t s,
+                        const GrpoArgs* grpo) {
+    note_launch();
+    if (M <= 0) return;
+    GrpoArgs g{};
+    if (grpo) g = *grpo;
+    launch_k(lse_combine_kernel, dim3(M), dim3(128), 0, s, ms, idx, zt, n_vt, V, oi, lp, argmax,
+             status, g);
+}
+
 // ---------------------------------------------------------------- rollout cursor
 __global__ void rollout_prepare_kernel(const int32_t* __restrict__ seq, int L, int P, int B,
                                        int32_t* step, int32_t* pos, int32_t* tok, int32_t* tgt,

@@ -117,6 +117,11 @@ struct Workspace {
     int* tickets;   // decode: last-unit tickets of the fused linears
     float* logits;  // [logit_rows, V]
     int logit_rows;
+    // scoring of bf16 models: per (row, 128-entry vocabulary tile) softmax statistics
+    // formed in the lm_head epilogue instead of logits (null: logits + reduce)
+    float2* lse_ms;  // [logit_rows, V / 128]
+    int* lse_idx;    // [logit_rows, V / 128]
+    float* lse_zt;   // [logit_rows]
     size_t total;
 };
 
@@ -140,6 +145,13 @@ static bool use_splitk(const Model& m, int M) {
            c.hidden % 128 == 0 && c.intermediate % 128 == 0 && c.vocab % 128 == 0 &&
            c.vocab / 128 <= kTicketSlots && (2 * c.intermediate) / 128 <= kTicketSlots &&
            ((c.n_q_heads + 2 * c.n_kv_heads) * c.head_dim) / 128 <= kTicketSlots;
+}
+
+// Scoring of bf16 models forms the log-softmax statistics per vocabulary tile in the
+// tcgen05 lm_head epilogue; the fp32 model (CUDA-core GEMM) materialises its logits.
+static bool use_lse_head(const Model& m) {
+    const qk_config& c = m.cfg;
+    return c.dtype == QK_DTYPE_BF16 && c.vocab % 128 == 0 && c.hidden % 64 == 0;
 }
 
 static size_t splitk_part_floats(const Model& m, int M) {
@@ -188,7 +200,18 @@ static int workspace_layout(const Model& m, int kind, int B, int T, int max_seq,
     }
     size_t rows = kind == QK_CALL_SCORE ? (M < (size_t)kScoreLogitRows ? M : kScoreLogitRows) : B;
     w->logit_rows = (int)rows;
-    w->logits = (float*)take(rows * (size_t)c.vocab * 4);
+    w->lse_ms = nullptr;
+    w->lse_idx = nullptr;
+    w->lse_zt = nullptr;
+    if (kind == QK_CALL_SCORE && use_lse_head(m)) {
+        const size_t nvt = (size_t)c.vocab / 128;
+        w->logits = nullptr;
+        w->lse_ms = (float2*)take(rows * nvt * 8);
+        w->lse_idx = (int*)take(rows * nvt * 4);
+        w->lse_zt = (float*)take(rows * 4);
+    } else {
+        w->logits = (float*)take(rows * (size_t)c.vocab * 4);
+    }
     w->total = off;
     return QK_OK;
 }
@@ -776,10 +799,27 @@ static int score_impl(Model& m, const int32_t* tokens, int B, int T, float* logp
         int rows = M - r0 < w.logit_rows ? M - r0 : w.logit_rows;
         launch_rmsnorm(w.x + (size_t)r0 * m.cfg.hidden, 1, 0, m.final_norm, m.cfg.hidden,
                        (float)m.cfg.rms_eps, w.u, m.cfg.dtype, rows, s);
-        linear(m, w.u, m.cfg.hidden, m.lm_head, w.logits, m.cfg.vocab, rows, m.cfg.vocab,
-               m.cfg.hidden, EPI_STORE_F32, w.gu, s);
         OutIndex oi{T, T - 1, T - 1, 0, tokens, T, 1, r0};
-        launch_logits_reduce(w.logits, rows, m.cfg.vocab, oi, logprobs, argmax, m.status, s, grpo);
+        if (w.lse_ms) {
+            // the softmax statistics per vocabulary tile come out of the lm_head epilogue
+            Fuse lf{};
+            lf.lse_ms = w.lse_ms;
+            lf.lse_idx = w.lse_idx;
+            lf.lse_zt = w.lse_zt;
+            lf.lse_tok = tokens;
+            lf.lse_T = T;
+            lf.lse_row0 = r0;
+            int rc = launch_gemm_tc((const bf16*)w.u, m.cfg.hidden, (const bf16*)m.lm_head, nullptr,
+                                    m.cfg.vocab, rows, m.cfg.vocab, m.cfg.hidden, EPI_LSE, m.num_sms,
+                                    m.status, s, 0, &lf);
+            if (rc != QK_OK) return set_error(rc, "lm_head statistics launch");
+            launch_lse_combine(w.lse_ms, w.lse_idx, w.lse_zt, m.cfg.vocab / 128, m.cfg.vocab, rows, oi,
+                               logprobs, argmax, m.status, s, grpo);
+        } else {
+            linear(m, w.u, m.cfg.hidden, m.lm_head, w.logits, m.cfg.vocab, rows, m.cfg.vocab,
+                   m.cfg.hidden, EPI_STORE_F32, w.gu, s);
+            launch_logits_reduce(w.logits, rows, m.cfg.vocab, oi, logprobs, argmax, m.status, s, grpo);
+        }
     }
     return QK_OK;
 }

@@ -154,6 +154,9 @@ enum Epi : int {
     EPI_RESID_F32 = 2,   // C (fp32, ldc) += acc
     EPI_SWIGLU = 3,      // W holds gate/up blocks of 128 rows; C[m, j] = silu(gate) * up, N = I
     EPI_PARTIAL_F32 = 4, // split-K unit s writes its fp32 partial to C[s][m][n] (ldc = N)
+    EPI_LSE = 5,         // lm_head: per (token row, 128-entry vocabulary tile) the max, sum of
+                         // exponentials and lowest arg-max of the logits, and the target's logit
+                         // (Fuse::lse_*); no logits are stored
 };
 
 // Token id of flattened row r: tokens[(r / T) * ld + off + r % T].
@@ -262,10 +265,18 @@ void launch_gemv_bf16(const bf16* A, int lda, const bf16* W, void* C, int ldc, i
                       int K, int epi, cudaStream_t s);
 // tcgen05 path (k_gemm_tc.cu): N % 128 == 0, K % 64 == 0, A 16-byte aligned, lda % 8 == 0.
 bool gemm_tc_supported(const void* A, int lda, int N, int K);
+struct Fuse;
 // test_wait > 0: bounded-wait test launch (CTA 0 skips its first copy and gives up
 // after test_wait SM cycles; the output is undefined and QK_STATUS_TIMEOUT is set).
 int launch_gemm_tc(const bf16* A, int lda, const bf16* W, void* C, int ldc, int M, int N, int K,
-                   int epi, int num_sms, uint32_t* status, cudaStream_t s, long long test_wait = 0);
+                   int epi, int num_sms, uint32_t* status, cudaStream_t s, long long test_wait = 0,
+                   const Fuse* lse = nullptr);
+// Combines the EPI_LSE partials of M logits rows over n_vt vocabulary tiles into the
+// log-prob of each row's target, its arg-max and (grpo) its GRPO token loss, with the
+// output indexing of launch_logits_reduce (k_misc.cu).
+void launch_lse_combine(const float2* ms, const int* idx, const float* zt, int n_vt, int V, int M,
+                        OutIndex oi, float* lp, int32_t* argmax, uint32_t* status, cudaStream_t s,
+                        const GrpoArgs* grpo = nullptr);
 
 // Fused epilogue of a decode-sized linear (one token tile, M <= 64 rows).  The
 // N/128 x K/64 k-block iterations are split evenly over the CTAs; a CTA that holds
@@ -312,6 +323,16 @@ struct Fuse {
     float* ssq_out;
     // FUSE_SWIGLU
     bf16* h_out;
+    // EPI_LSE (plain tcgen05 GEMM over the lm_head): token row m of the launch is
+    // global row g = lse_row0 + m of tokens [., lse_T]; its target is tokens[g + 1]
+    // when g % lse_T < lse_T - 1 (an id outside [0, V) counts as 0).  Outputs per
+    // (row, vocabulary tile v): lse_ms[m * n_vt + v] = (max, sum exp(z - max)),
+    // lse_idx[...] = lowest index of the max; lse_zt[m] = the target's logit.
+    float2* lse_ms;
+    int* lse_idx;
+    float* lse_zt;
+    const int32_t* lse_tok;
+    int lse_T, lse_row0;
 };
 
 // Decode linear with a fused epilogue (k_gemm_tc.cu): A = bf16 [M, K] (M <= 64),
