@@ -56,6 +56,39 @@ def grpo_token_loss(lp, lp_old, lp_ref, adv_rows, eps_low: float, eps_high: floa
     return loss
 
 
+def grpo_token_grad(lp, lp_old, lp_ref, adv_rows, eps_low: float, eps_high: float,
+                    beta: float) -> np.ndarray:
+    """d L_t / d lp_t of Eq. ppo per token (same arguments as grpo_token_loss).
+
+    d rho / d lp = rho.  The min picks the unclipped term rho A where rho A <=
+    clip(rho) A; there its derivative is rho A.  Elsewhere the clipped term is
+    smaller, which happens only with rho outside [1 - eps_low, 1 + eps_high],
+    where clip(rho) is constant: derivative 0.  d k3 / d lp = 1 - e^x,
+    x = lp_ref - lp.
+    """
+    lp = np.asarray(lp, dtype=np.float64)
+    rho = np.exp(lp - np.asarray(lp_old, dtype=np.float64))
+    a = np.asarray(adv_rows, dtype=np.float64)[:, None]
+    unclipped = rho * a <= np.clip(rho, 1.0 - eps_low, 1.0 + eps_high) * a
+    g = -np.where(unclipped, rho * a, 0.0)
+    if beta != 0.0:
+        g = g + beta * (1.0 - np.exp(np.asarray(lp_ref, dtype=np.float64) - lp))
+    return g
+
+
+def grpo_coef(lp, lp_old, lp_ref, adv_rows, eps_low: float, eps_high: float, beta: float,
+              mask=None) -> np.ndarray:
+    """Per-token weights c with d(grpo_loss_mean)/d theta = d/d theta sum c (-lp).
+
+    The batch loss is sum(mask L) / sum(mask), so c_t = -mask_t (dL_t/dlp_t) / sum(mask)
+    (all zero for an empty mask).
+    """
+    g = grpo_token_grad(lp, lp_old, lp_ref, adv_rows, eps_low, eps_high, beta)
+    m = np.ones_like(g) if mask is None else np.asarray(mask, dtype=np.float64)
+    n = m.sum()
+    return -m * g / n if n > 0 else np.zeros_like(g)
+
+
 def grpo_loss_mean(loss_tok, mask=None) -> float:
     """Token mean over the response tokens (mask 1) of the whole batch."""
     loss_tok = np.asarray(loss_tok, dtype=np.float64)

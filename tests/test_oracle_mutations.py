@@ -54,6 +54,33 @@ SAMPLING_MUTATIONS = {
 }
 
 
+# Mistakes in the backward oracle and the GRPO derivative, caught by test_oracle_backward.py.
+BACKWARD_MUTATIONS = {
+    "rms_dx_dropped_projection": ("dx = r * a - (r ** 3 / n) * x * np.sum(a * x, axis=-1, keepdims=True)",
+                                  "dx = r * a"),
+    "rms_gain_grad_unscaled": ("dg = np.sum((dy * x * r).reshape(-1, n), axis=0)",
+                               "dg = np.sum((dy * x).reshape(-1, n), axis=0)"),
+    "rope_backward_forward_rotation": ("d1 * c + d2 * s, -d1 * s + d2 * c", "d1 * c - d2 * s, d1 * s + d2 * c"),
+    "softmax_backward_no_rowsum": ("dS = P * (dP - np.sum(dP * P, axis=-1, keepdims=True))", "dS = P * dP"),
+    "gqa_dv_overwritten": ("dv[:, g] += P.T @ do[:, h]", "dv[:, g] = P.T @ do[:, h]"),
+    "dk_missing_scale": ("dkr[:, g] += dS.T @ c[\"qr\"][:, h] / np.sqrt(d)", "dkr[:, g] += dS.T @ c[\"qr\"][:, h]"),
+    "silu_derivative": ("sg * (1.0 + c[\"g\"] * (1.0 - sg))", "sg"),
+    "mlp_residual_gradient_dropped": ("dx = dx + dxm", "dx = dxm"),
+    "embedding_duplicates_lost": ("np.add.at(grads[\"embed\"], np.asarray(tok), dx)",
+                                  "grads[\"embed\"][np.asarray(tok)] += dx"),
+    "onehot_sign": ("dz[np.arange(T), tgt] -= 1.0", "dz[np.arange(T), tgt] += 1.0"),
+    "target_not_shifted": ("tgt[:T - 1] = np.asarray(tok)[1:]", "tgt[:T - 1] = np.asarray(tok)[:-1]"),
+    "du1_missing_value_path": ("du1 = dq @ Lw[\"wq\"] + dk @ Lw[\"wk\"] + dv @ Lw[\"wv\"]",
+                               "du1 = dq @ Lw[\"wq\"] + dk @ Lw[\"wk\"]"),
+}
+
+GRPO_GRAD_MUTATIONS = {
+    "clipped_branch_passes_gradient": ("g = -np.where(unclipped, rho * a, 0.0)", "g = -rho * a"),
+    "kl_grad_sign": ("g = g + beta * (1.0 - np.exp(", "g = g - beta * (1.0 - np.exp("),
+    "coef_not_normalised": ("return -m * g / n if n > 0 else np.zeros_like(g)", "return -m * g"),
+}
+
+
 def _run_mutated(tmp_path, module, before, after, name, pins):
     shutil.copytree(os.path.join(ROOT, "oracle"), tmp_path / "oracle",
                     ignore=shutil.ignore_patterns("__pycache__"))
@@ -84,3 +111,15 @@ def test_grpo_pins_catch_planted_mistake(name, tmp_path):
 def test_sampling_pins_catch_planted_mistake(name, tmp_path):
     before, after = SAMPLING_MUTATIONS[name]
     _run_mutated(tmp_path, "sampling.py", before, after, name, "test_oracle_sampling.py")
+
+
+@pytest.mark.parametrize("name", sorted(BACKWARD_MUTATIONS))
+def test_backward_pins_catch_planted_mistake(name, tmp_path):
+    before, after = BACKWARD_MUTATIONS[name]
+    _run_mutated(tmp_path, "backward.py", before, after, name, "test_oracle_backward.py")
+
+
+@pytest.mark.parametrize("name", sorted(GRPO_GRAD_MUTATIONS))
+def test_grpo_grad_pins_catch_planted_mistake(name, tmp_path):
+    before, after = GRPO_GRAD_MUTATIONS[name]
+    _run_mutated(tmp_path, "grpo.py", before, after, name, "test_oracle_backward.py")
