@@ -70,6 +70,7 @@ extern "C" {
 #define QK_CALL_PREFILL 1  /* qk_prefill: B x T tokens                             */
 #define QK_CALL_SCORE 2    /* qk_score_logprobs: B x T tokens, no KV cache         */
 #define QK_CALL_ROLLOUT 3  /* qk_rollout_teacher_forced: prefill B x T then decode */
+#define QK_CALL_BACKWARD 4 /* qk_backward_logprob: B x T tokens (max_seq ignored)     */
 
 typedef struct qk_config {
     int32_t n_layers;      /* decoder layers                                  */
@@ -228,6 +229,48 @@ int qk_score_grpo(qk_model* m, const int32_t* tokens, int B, int T, const float*
                   const float* lp_ref, const float* rewards, int group, const uint8_t* mask,
                   float eps_low, float eps_high, float beta, float* logprobs, float* loss_tok,
                   float* loss_mean, void* workspace, size_t ws_bytes, void* stream);
+
+/* Per-token coefficients of the GRPO gradient (Sec. "GRPO Optimization", Eq. ppo):
+ * with loss_mean = sum(mask * loss_tok) / sum(mask) as in qk_grpo_token_loss,
+ *   coef[b, t] = -mask[b, t] * (d loss_tok[b, t] / d lp[b, t]) / sum(mask),
+ * so that qk_backward_logprob with these coefficients returns d loss_mean / d theta
+ * (the chain rule through the log-probs; lp_old, lp_ref and the advantages are
+ * constants).  d loss_tok / d lp = -rho A where rho A <= clip(rho) A (the unclipped
+ * term is the minimum), 0 elsewhere (the clipped term is constant there), plus
+ * beta (1 - exp(lp_ref - lp)).  Arguments and workspace as qk_grpo_token_loss
+ * (loss_tok and loss_mean are written too); coef dev fp32 [B, ld], entries t < T.
+ * All zero for an empty mask. */
+int qk_grpo_coef(const float* lp, const float* lp_old, const float* lp_ref, int B, int T, int ld,
+                 const float* rewards, int group, const uint8_t* mask, float eps_low, float eps_high,
+                 float beta, float* coef, float* loss_tok, float* loss_mean, void* workspace,
+                 size_t ws_bytes, void* stream);
+
+/* ---- Backward pass (gradient of the token log-likelihood) -------------------
+ * The SFT objective (Sec. "Task Serialization and SFT Objective", Eq. sft)
+ * maximises log pi_theta(y* | x) over the target tokens; the GRPO objective
+ * (Eq. ppo) depends on theta only through the same per-token log-probs.  Both
+ * gradients are therefore the gradient of
+ *   loss = sum_{b, t < T-1} coef[b, t] * (-log p(tokens[b, t+1] | tokens[b, <= t]))
+ * for per-token coefficients coef (SFT: mask / number of target tokens; GRPO:
+ * qk_grpo_coef).  tokens dev int32 [B, T], T >= 2, positions 0 .. T-1; coef dev
+ * fp32 [B, T-1].  grads: host array of n_grads = qk_weight_count() device fp32
+ * pointers, one per weight tensor in the canonical order and shape of
+ * qk_model_load (row-major [out, in]), each 16-byte aligned; each receives
+ * d loss / d tensor (accumulate == 0: overwritten; else added to).  loss dev fp32
+ * [1] or NULL receives the loss.  workspace: qk_workspace_bytes(QK_CALL_BACKWARD,
+ * B, T, 0), 256-byte aligned (it holds each layer's fp32 input residual, the
+ * attention probabilities of one layer and a [min(B T, 4096), V] block of logit
+ * gradients).  bf16 models need T % 128 == 0, head_dim 128 and vocab % 64 == 0
+ * (QK_ESHAPE otherwise); fp32 models take any shape.  Activations are rounded to
+ * the model dtype where the forward pass rounds them (and the logit and attention
+ * gradients, which are tensor-core operands, likewise); accumulation, norms,
+ * softmax statistics, the residual gradient and every weight gradient are fp32.
+ * Gain gradients sum in a fixed order; embedding rows that share a token are
+ * added with fp32 atomics (order-dependent rounding only).  A token id outside
+ * [0, V) sets QK_STATUS_BAD_TOKEN and counts as 0. */
+int qk_backward_logprob(qk_model* m, const int32_t* tokens, int B, int T, const float* coef,
+                        float* const* grads, int n_grads, int accumulate, float* loss,
+                        void* workspace, size_t ws_bytes, void* stream);
 
 /* Teacher-forced rollout: seq dev int32 [B, P+N+1] = prompt (P tokens) ++
  * c[0..N].  Prefill over the prompt scores c[0]; decode step j (0 <= j < N)

@@ -17,7 +17,7 @@ QK_OK, QK_EINVAL, QK_ESHAPE, QK_EDTYPE, QK_ECUDA, QK_ETIMEOUT, QK_EDEVICE, QK_EN
     0, -1, -2, -3, -4, -5, -6, -7)
 QK_DTYPE_BF16, QK_DTYPE_F32 = 0, 1
 QK_STATUS_BAD_TOKEN, QK_STATUS_BAD_POS, QK_STATUS_TIMEOUT = 1, 2, 4
-QK_CALL_DECODE, QK_CALL_PREFILL, QK_CALL_SCORE, QK_CALL_ROLLOUT = 0, 1, 2, 3
+QK_CALL_DECODE, QK_CALL_PREFILL, QK_CALL_SCORE, QK_CALL_ROLLOUT, QK_CALL_BACKWARD = 0, 1, 2, 3, 4
 QK_PROF_QKV, QK_PROF_O, QK_PROF_GATE_UP, QK_PROF_DOWN, QK_PROF_ATTN, QK_PROF_LM_HEAD = range(6)
 QK_EPI_STORE, QK_EPI_STORE_F32, QK_EPI_RESID_F32, QK_EPI_SWIGLU = 0, 1, 2, 3
 QK_STATIC_SCRATCH_BYTES = 8 << 20
@@ -34,7 +34,8 @@ __all__ = [
     "QK_PROF_GATE_UP", "QK_PROF_DOWN", "QK_PROF_ATTN", "QK_PROF_LM_HEAD", "QK_EPI_STORE",
     "QK_EPI_STORE_F32", "QK_EPI_RESID_F32", "QK_EPI_SWIGLU", "qk_op_linear_swiglu_static",
     "QK_STATIC_SCRATCH_BYTES", "qk_grpo_workspace_bytes", "qk_grpo_token_loss", "qk_score_grpo",
-    "qk_rollout_sampled", "qk_prefill_rows", "qk_debug_expire_next_wait",
+    "qk_rollout_sampled", "qk_prefill_rows", "qk_debug_expire_next_wait", "QK_CALL_BACKWARD",
+    "qk_grpo_coef", "qk_backward_logprob",
 ]
 
 
@@ -89,6 +90,8 @@ _SIGS = {
                            _I),
     "qk_prefill_rows": ([_P, _P, _I, _I, _P, _I, _I, _P, _P, _P, _P, _SZ, _P], _I),
     "qk_debug_expire_next_wait": ([_P, ctypes.c_longlong], _I),
+    "qk_grpo_coef": ([_P, _P, _P, _I, _I, _I, _P, _I, _P, _F, _F, _F, _P, _P, _P, _P, _SZ, _P], _I),
+    "qk_backward_logprob": ([_P, _P, _I, _I, _P, ctypes.POINTER(_P), _I, _I, _P, _P, _SZ, _P], _I),
 }
 
 _lib = None
@@ -231,6 +234,23 @@ def qk_grpo_token_loss(lp, lp_old, lp_ref, B, T, ld, rewards, group, mask, eps_l
                                       group, _ptr(mask), eps_low, eps_high, beta, _ptr(loss_tok),
                                       _ptr(loss_mean), _ptr(workspace), _nbytes(workspace, ws_bytes),
                                       _stream(stream)))
+
+
+def qk_grpo_coef(lp, lp_old, lp_ref, B, T, ld, rewards, group, mask, eps_low, eps_high, beta, coef,
+                 loss_tok, loss_mean=None, workspace=None, ws_bytes=None, stream=None):
+    _check(_load().qk_grpo_coef(_ptr(lp), _ptr(lp_old), _ptr(lp_ref), B, T, ld, _ptr(rewards), group,
+                                _ptr(mask), eps_low, eps_high, beta, _ptr(coef), _ptr(loss_tok),
+                                _ptr(loss_mean), _ptr(workspace), _nbytes(workspace, ws_bytes),
+                                _stream(stream)))
+
+
+def qk_backward_logprob(m, tokens, B, T, coef, grads, accumulate=0, loss=None, workspace=None,
+                        ws_bytes=None, stream=None):
+    """grads: a sequence of device fp32 buffers (tensors or addresses), canonical tensor order."""
+    arr = (ctypes.c_void_p * len(grads))(*[_ptr(g) for g in grads])
+    _check(_load().qk_backward_logprob(m, _ptr(tokens), B, T, _ptr(coef), arr, len(grads), accumulate,
+                                       _ptr(loss), _ptr(workspace), _nbytes(workspace, ws_bytes),
+                                       _stream(stream)))
 
 
 def qk_score_grpo(m, tokens, B, T, lp_old, lp_ref, rewards, group, mask, eps_low, eps_high, beta,

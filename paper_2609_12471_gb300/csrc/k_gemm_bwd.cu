@@ -1,0 +1,402 @@
+// The batched GEMM of the backward pass (bwd_common.cuh): a tcgen05 / TMEM / TMA
+// kernel for bf16 models and a CUDA-core kernel for fp32 models, both over the
+// same operand descriptors, tile schedule and epilogue.
+//
+// tcgen05 kernel, one persistent CTA per SM, 192 threads:
+//   warp 0, one lane : TMA producer over a STAGES-deep ring of (A, B) k-blocks of 64;
+//   warp 1           : TMEM allocation; one lane issues tcgen05.mma (M 128, N BN, K 16)
+//                      and the commits;
+//   warps 2..5       : epilogue; warp w reads TMEM lanes 32 (w % 4) .. + 31, one output
+//                      row per thread, 16 columns per tcgen05.ld.
+// A K-major operand tile is one 128-byte-swizzled box (64 k x 128 or BN rows); an
+// MN-major one is boxes of 64 m/n x 64 k (8 KB each), whose descriptor steps 64
+// m/n elements by the leading byte offset (8 KB) and 8 k rows by the stride byte
+// offset (1 KB).  Two TMEM accumulators alternate so the epilogue of one tile
+// overlaps the main loop of the next.  Every mbarrier wait is bounded; on a timeout
+// the CTA raises QK_STATUS_TIMEOUT, drains its copies and MMAs and exits.
+#include <cuda.h>
+#include <math.h>
+
+#include "bwd_common.cuh"
+#include "tc_ptx.cuh"
+
+namespace qk {
+namespace bwd {
+
+namespace {
+
+// ------------------------------------------------------------------ CUDA-core kernel
+constexpr int kSimtTile = 64, kSimtBK = 16, kSimtThreads = 256;
+
+template <typename T>
+__device__ __forceinline__ float op_load(const Op& o, int z, int i, int k) {
+    int x, y;
+    op_xy(o, z, i, k, x, y);
+    return ld_act((const T*)o.ptr + (size_t)y * o.ld + x);
+}
+
+// One 64 x 64 output tile per CTA; thread t owns row t / 4, columns 16 (t % 4) .. + 15.
+template <typename T>
+__global__ void __launch_bounds__(kSimtThreads) gemm_bwd_simt_kernel(Gemm g, long long per) {
+    __shared__ float As[kSimtBK][kSimtTile + 1], Bs[kSimtBK][kSimtTile + 1];
+    pdl_wait();
+    const Sched& sc = g.sc;
+    int z, mt, nt;
+    tile_at(sc, kSimtTile, kSimtTile, per, (long long)blockIdx.x, z, mt, nt);
+    const int m0 = mt * kSimtTile, n0 = nt * kSimtTile;
+    const int tid = threadIdx.x, r = tid >> 2, cg = tid & 3;
+    float acc[16];
+#pragma unroll
+    for (int c = 0; c < 16; ++c) acc[c] = 0.f;
+    const int nkb = kblocks(sc, kSimtTile, kSimtBK, m0);
+    for (int j = 0; j < nkb; ++j) {
+        int k0, kend;
+        kblock_at(sc, kSimtTile, kSimtBK, m0, j, k0, kend);
+        for (int e = tid; e < kSimtTile * kSimtBK; e += kSimtThreads) {
+            const int i = e % kSimtTile, kq = e / kSimtTile, k = k0 + kq;
+            const bool kv = k < kend;
+            As[kq][i] = (kv && m0 + i < sc.M) ? op_load<T>(g.A, z, m0 + i, k) : 0.f;
+            Bs[kq][i] = (kv && n0 + i < sc.N) ? op_load<T>(g.B, z, n0 + i, k) : 0.f;
+        }
+        __syncthreads();
+#pragma unroll
+        for (int kq = 0; kq < kSimtBK; ++kq) {
+            const float a = As[kq][r];
+#pragma unroll
+            for (int c = 0; c < 16; ++c) acc[c] = fmaf(a, Bs[kq][cg * 16 + c], acc[c]);
+        }
+        __syncthreads();
+    }
+    const int m = m0 + r, n = n0 + cg * 16;
+    int nv = sc.N - n;
+    nv = nv < 0 ? 0 : (nv > 16 ? 16 : nv);
+    RowStat st{-INFINITY, 0.f};
+    if (m < sc.M && nv > 0) epi16<T, false>(g.epi, g.out, z, m, n, nv, acc, st);
+    if (g.epi.mode == E_STATS) {  // merge the row's four 16-column parts
+#pragma unroll
+        for (int o = 1; o < 4; o <<= 1) {
+            const float m2 = __shfl_xor_sync(0xffffffffu, st.mx, o);
+            const float s2 = __shfl_xor_sync(0xffffffffu, st.sm, o);
+            stat_merge(st, m2, s2);
+        }
+        if (cg == 0 && m < sc.M)
+            g.epi.stats[(size_t)(z * g.epi.rows_per_z + m) * g.epi.n_ct + nt] = make_float2(st.mx, st.sm);
+    }
+}
+
+// ------------------------------------------------------------------ tcgen05 kernel
+constexpr int kThreads = 192;
+constexpr int kBK = 64;
+constexpr int kBox = 64 * 128;  // one 64 x 64 bf16 box (8 KB)
+
+template <int BN>
+struct TcCfg {
+    static constexpr int STAGES = BN == 256 ? 4 : 6;
+    static constexpr int A_BYTES = 128 * 128;
+    static constexpr int B_BYTES = BN * 128;
+    static constexpr int TMEM_COLS = 2 * BN;
+    static constexpr int SMEM = STAGES * (A_BYTES + B_BYTES) + 1024 + 256;
+    static_assert(TMEM_COLS <= 512, "accumulators exceed TMEM");
+};
+
+template <int BN, bool AMN, bool BMN>
+__global__ void __launch_bounds__(kThreads, 1)
+    gemm_bwd_tc_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant__ CUtensorMap mapB,
+                       const __grid_constant__ Gemm g, long long per, long long total,
+                       uint32_t* __restrict__ status) {
+    using G = TcCfg<BN>;
+    constexpr int STAGES = G::STAGES;
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t* smem = (uint8_t*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
+    uint8_t* sA = smem;
+    uint8_t* sB = smem + STAGES * G::A_BYTES;
+    uint64_t* full = (uint64_t*)(sB + STAGES * G::B_BYTES);
+    uint64_t* empty = full + STAGES;
+    uint64_t* tfull = empty + STAGES;
+    uint64_t* tempty = tfull + 2;
+    uint64_t* drain = tempty + 2;
+    uint32_t* tmem_slot = (uint32_t*)(drain + 1);
+    volatile int* abort_flag = (volatile int*)(tmem_slot + 1);
+
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const Sched& sc = g.sc;
+
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < STAGES; ++s) {
+            tc::mbar_init(&full[s], 1);
+            tc::mbar_init(&empty[s], 1);
+        }
+        for (int a = 0; a < 2; ++a) {
+            tc::mbar_init(&tfull[a], 1);
+            tc::mbar_init(&tempty[a], 4);
+        }
+        tc::mbar_init(drain, 1);
+        *abort_flag = 0;
+        tc::fence_mbar_init();
+        tc::tma_prefetch_desc(&mapA);
+        tc::tma_prefetch_desc(&mapB);
+    }
+    if (warp == 1) tc::tmem_alloc(tmem_slot, G::TMEM_COLS);
+    tc::fence_before_sync();
+    __syncthreads();
+    tc::fence_after_sync();
+    const uint32_t tmem_base = *tmem_slot;
+    pdl_wait();
+
+    if (warp == 0) {
+        if (lane == 0) {
+            // ------------------------------------------------ TMA producer
+            int stage = 0;
+            uint32_t phase = 0;
+            int armed[STAGES];
+            for (int s = 0; s < STAGES; ++s) armed[s] = -1;
+            bool ok = true;
+            for (long long t = blockIdx.x; ok && t < total; t += gridDim.x) {
+                int z, mt, nt;
+                tile_at(sc, 128, BN, per, t, z, mt, nt);
+                const int m0 = mt * 128, n0 = nt * BN;
+                const int nkb = kblocks(sc, 128, kBK, m0);
+                for (int j = 0; j < nkb; ++j) {
+                    int k0, kend;
+                    kblock_at(sc, 128, kBK, m0, j, k0, kend);
+                    if (!tc::mbar_wait(&empty[stage], phase ^ 1, abort_flag)) {
+                        ok = false;
+                        break;
+                    }
+                    tc::mbar_expect_tx(&full[stage], G::A_BYTES + G::B_BYTES);
+                    uint8_t* a_s = sA + stage * G::A_BYTES;
+                    uint8_t* b_s = sB + stage * G::B_BYTES;
+                    int x, y;
+                    if (AMN) {
+#pragma unroll
+                        for (int c = 0; c < 2; ++c) {
+                            op_xy(g.A, z, m0 + 64 * c, k0, x, y);
+                            tc::tma_load_2d(a_s + c * kBox, &mapA, x, y, &full[stage]);
+                        }
+                    } else {
+                        op_xy(g.A, z, m0, k0, x, y);
+                        tc::tma_load_2d(a_s, &mapA, x, y, &full[stage]);
+                    }
+                    if (BMN) {
+#pragma unroll
+                        for (int c = 0; c < BN / 64; ++c) {
+                            op_xy(g.B, z, n0 + 64 * c, k0, x, y);
+                            tc::tma_load_2d(b_s + c * kBox, &mapB, x, y, &full[stage]);
+                        }
+                    } else {
+                        op_xy(g.B, z, n0, k0, x, y);
+                        tc::tma_load_2d(b_s, &mapB, x, y, &full[stage]);
+                    }
+                    armed[stage] = (int)phase;
+                    if (++stage == STAGES) {
+                        stage = 0;
+                        phase ^= 1;
+                    }
+                }
+            }
+            pdl_trigger();
+            if (!ok) {
+                for (int s = 0; s < STAGES; ++s)
+                    if (armed[s] >= 0) tc::mbar_wait_drain(&full[s], (uint32_t)armed[s]);
+            }
+        }
+    } else if (warp == 1) {
+        if (lane == 0) {
+            // ------------------------------------------------ MMA issuer
+            constexpr uint32_t idesc =
+                tc::idesc_bf16(128, BN) | (AMN ? (1u << 15) : 0u) | (BMN ? (1u << 16) : 0u);
+            int stage = 0;
+            uint32_t phase = 0;
+            int acc = 0;
+            uint32_t acc_phase = 0;
+            bool ok = true, issued = false;
+            for (long long t = blockIdx.x; ok && t < total; t += gridDim.x) {
+                int z, mt, nt;
+                tile_at(sc, 128, BN, per, t, z, mt, nt);
+                const int nkb = kblocks(sc, 128, kBK, mt * 128);
+                if (!tc::mbar_wait(&tempty[acc], acc_phase ^ 1, abort_flag)) {
+                    ok = false;
+                    break;
+                }
+                tc::fence_after_sync();
+                const uint32_t d = tmem_base + (uint32_t)(acc * BN);
+                for (int j = 0; j < nkb; ++j) {
+                    if (!tc::mbar_wait(&full[stage], phase, abort_flag)) {
+                        ok = false;
+                        break;
+                    }
+                    tc::fence_after_sync();
+                    const uint32_t a0 = tc::smem_u32(sA + stage * G::A_BYTES);
+                    const uint32_t b0 = tc::smem_u32(sB + stage * G::B_BYTES);
+#pragma unroll
+                    for (int k = 0; k < kBK / 16; ++k) {
+                        const uint64_t ad = AMN ? tc::sw128_desc_mn(a0 + k * 2048, kBox)
+                                                : tc::sw128_desc(a0 + k * 32);
+                        const uint64_t bd = BMN ? tc::sw128_desc_mn(b0 + k * 2048, kBox)
+                                                : tc::sw128_desc(b0 + k * 32);
+                        tc::mma_bf16(d, ad, bd, idesc, (j || k) ? 1u : 0u);
+                    }
+                    issued = true;
+                    tc::mma_commit(&empty[stage]);
+                    if (++stage == STAGES) {
+                        stage = 0;
+                        phase ^= 1;
+                    }
+                }
+                if (!ok) break;
+                tc::mma_commit(&tfull[acc]);
+                acc ^= 1;
+                if (acc == 0) acc_phase ^= 1;
+            }
+            if (!ok && issued) {
+                tc::mma_commit(drain);
+                tc::mbar_wait_drain(drain, 0);
+            }
+        }
+    } else {
+        // ---------------------------------------------------- epilogue (warps 2..5)
+        const int q = warp & 3;
+        int acc = 0;
+        uint32_t acc_phase = 0;
+        for (long long t = blockIdx.x; t < total; t += gridDim.x) {
+            int z, mt, nt;
+            tile_at(sc, 128, BN, per, t, z, mt, nt);
+            const int m0 = mt * 128, n0 = nt * BN;
+            bool ok = tc::mbar_wait(&tfull[acc], acc_phase, abort_flag);
+            ok = __all_sync(0xffffffffu, ok);
+            if (!ok) break;
+            tc::fence_after_sync();
+            const int m = m0 + q * 32 + lane;
+            const uint32_t tbase = tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(acc * BN);
+            RowStat st{-INFINITY, 0.f};
+            for (int c0 = 0; c0 < BN; c0 += 16) {
+                const int n = n0 + c0;
+                if (n >= sc.N) break;  // uniform over the warp
+                uint32_t r[16];
+                tc::tmem_ld16(tbase + c0, r);
+                tc::tmem_wait_ld();
+                float v[16];
+#pragma unroll
+                for (int j = 0; j < 16; ++j) v[j] = __uint_as_float(r[j]);
+                if (m < sc.M) epi16<bf16, true>(g.epi, g.out, z, m, n, 16, v, st);
+            }
+            if (g.epi.mode == E_STATS && m < sc.M)
+                g.epi.stats[(size_t)(z * g.epi.rows_per_z + m) * g.epi.n_ct + nt] = make_float2(st.mx, st.sm);
+            tc::fence_before_sync();
+            __syncwarp();
+            if (lane == 0) tc::mbar_arrive(&tempty[acc]);
+            acc ^= 1;
+            if (acc == 0) acc_phase ^= 1;
+        }
+    }
+
+    tc::fence_before_sync();
+    __syncthreads();
+    if (threadIdx.x == 0 && *abort_flag) atomicOr(status, QK_STATUS_TIMEOUT);
+    if (warp == 1) {
+        tc::fence_after_sync();
+        tc::tmem_dealloc(tmem_base, G::TMEM_COLS);
+    }
+}
+
+typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*,
+                                  const cuuint64_t*, const cuuint64_t*, const cuuint32_t*,
+                                  const cuuint32_t*, CUtensorMapInterleave, CUtensorMapSwizzle,
+                                  CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+EncodeTiledFn encode_fn() {
+    static EncodeTiledFn fn = nullptr;
+    static bool tried = false;
+    if (!tried) {
+        tried = true;
+        void* p = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault,
+                                             &q) == cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            fn = (EncodeTiledFn)p;
+    }
+    return fn;
+}
+
+// bf16 map over the whole operand buffer, box 64 columns x box_rows rows, 128-byte swizzle.
+bool make_op_map(CUtensorMap* map, const Op& o, int box_rows) {
+    EncodeTiledFn fn = encode_fn();
+    if (!fn) return false;
+    cuuint64_t dims[2] = {(cuuint64_t)o.cols, (cuuint64_t)o.rows};
+    cuuint64_t strides[1] = {(cuuint64_t)o.ld * 2};
+    cuuint32_t box[2] = {64, (cuuint32_t)box_rows};
+    cuuint32_t estr[2] = {1, 1};
+    return fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(o.ptr), dims, strides, box,
+              estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+              CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+template <int BN, bool AMN, bool BMN>
+int launch_tc(Model& m, const Gemm& g, cudaStream_t s) {
+    using G = TcCfg<BN>;
+    static bool attr_set = false;
+    if (!attr_set) {
+        if (cudaFuncSetAttribute(gemm_bwd_tc_kernel<BN, AMN, BMN>,
+                                 cudaFuncAttributeMaxDynamicSharedMemorySize, G::SMEM) != cudaSuccess)
+            return set_error(QK_ECUDA, "backward GEMM: shared-memory attribute");
+        attr_set = true;
+    }
+    CUtensorMap ma, mb;
+    if (!make_op_map(&ma, g.A, AMN ? 64 : 128) || !make_op_map(&mb, g.B, BMN ? 64 : BN))
+        return set_error(QK_ECUDA, "backward GEMM: tensor map encoding failed");
+    const long long per = tiles_per_z(g.sc, 128, BN);
+    const long long total = per * g.sc.Z;
+    const int grid = total < m.num_sms ? (int)total : m.num_sms;
+    launch_k(gemm_bwd_tc_kernel<BN, AMN, BMN>, dim3(grid), dim3(kThreads), G::SMEM, s, ma, mb, g,
+             per, total, m.status);
+    note_launch();
+    return QK_OK;
+}
+
+bool aligned16(const void* p) { return ((uintptr_t)p & 15) == 0; }
+
+}  // namespace
+
+int gemm_tile_n(const Model& m, int N, int tri) {
+    if (m.cfg.dtype != QK_DTYPE_BF16) return kSimtTile;
+    return (tri || N <= 128) ? 128 : 256;
+}
+
+int run_gemm(Model& m, const Gemm& g, cudaStream_t s) {
+    const Sched& sc = g.sc;
+    if (sc.Z <= 0 || sc.M <= 0 || sc.N <= 0) return QK_OK;
+    if (m.cfg.dtype != QK_DTYPE_BF16) {
+        const long long per = tiles_per_z(sc, kSimtTile, kSimtTile);
+        const long long total = per * sc.Z;
+        if (total >= (1ll << 31)) return set_error(QK_ESHAPE, "backward GEMM: too many tiles");
+        launch_k(gemm_bwd_simt_kernel<float>, dim3((unsigned)total), dim3(kSimtThreads), 0, s, g, per);
+        note_launch();
+        return QK_OK;
+    }
+    const int BN = gemm_tile_n(m, sc.N, sc.tri);
+    // Every k-block is whole, every TMA box starts on a 16-byte boundary and every
+    // epilogue access of 16 outputs is 16-byte aligned.
+    bool ok = sc.K % kBK == 0 && aligned16(g.A.ptr) && aligned16(g.B.ptr) && g.A.ld % 8 == 0 &&
+              g.B.ld % 8 == 0 && sc.N % 16 == 0 && aligned16(g.out.C) && g.out.zcol % 16 == 0;
+    ok = ok && (g.epi.mode == E_F32 ? g.out.ldc % 4 == 0 : g.out.ldc % 8 == 0);
+    ok = ok && (!g.out.addend || aligned16(g.out.addend)) && (!g.epi.P || aligned16(g.epi.P));
+    ok = ok && (sc.red != RED_SUFFIX || (sc.seg % kBK == 0 && sc.seg > 0 && sc.K % sc.seg == 0));
+    ok = ok && (!g.A.kwrap || g.A.kwrap % kBK == 0) && (!g.B.kwrap || g.B.kwrap % kBK == 0);
+    ok = ok && g.B.pitch == 128 && g.A.pitch % 64 == 0 && (!sc.tri || (BN == 128 && sc.M == sc.N));
+    if (!ok) return set_error(QK_ESHAPE, "backward GEMM: shape or alignment outside the tcgen05 path");
+    const bool amn = g.A.mn != 0, bmn = g.B.mn != 0;
+    if (BN == 256) {
+        if (!amn && !bmn) return launch_tc<256, false, false>(m, g, s);
+        if (!amn && bmn) return launch_tc<256, false, true>(m, g, s);
+        if (amn && bmn) return launch_tc<256, true, true>(m, g, s);
+    } else {
+        if (!amn && !bmn) return launch_tc<128, false, false>(m, g, s);
+        if (!amn && bmn) return launch_tc<128, false, true>(m, g, s);
+        if (amn && bmn) return launch_tc<128, true, true>(m, g, s);
+    }
+    return set_error(QK_EINVAL, "backward GEMM: MN-major A with K-major B is not instantiated");
+}
+
+}  // namespace bwd
+}  // namespace qk

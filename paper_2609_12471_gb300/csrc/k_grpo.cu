@@ -64,7 +64,44 @@ __global__ void __launch_bounds__(kThreads)
     if (threadIdx.x == 0) *loss_mean = tot.y > 0.f ? tot.x / tot.y : 0.f;
 }
 
+// d L_t / d lp_t of Eq. ppo: rho A where the unclipped term is the minimum (its
+// derivative; rho = exp(lp - lp_old) has d rho / d lp = rho), 0 where the clipped term
+// is smaller (clip(rho) is then constant), plus beta (1 - e^x), x = lp_ref - lp, the
+// derivative of k3.  coef = -mask * dL / n with n the batch's mask count (so that the
+// gradient of sum coef * (-lp) is the gradient of the masked token mean).
+__global__ void __launch_bounds__(kThreads)
+    grpo_coef_kernel(const float* __restrict__ lp, int T, GrpoArgs g, const float2* __restrict__ rows,
+                     int B, float* __restrict__ coef) {
+    __shared__ float2 red[kThreads / 32];
+    __shared__ float n_sh;
+    pdl_wait();
+    float2 acc = make_float2(0.f, 0.f);
+    for (int b = threadIdx.x; b < B; b += blockDim.x) acc.y += rows[b].y;
+    const float2 tot = block_sum2(acc, red);
+    if (threadIdx.x == 0) n_sh = tot.y;
+    __syncthreads();
+    const float n = n_sh;
+    const int b = blockIdx.x;
+    const size_t r0 = (size_t)b * g.ld;
+    const float A = grpo_advantage(g.rewards, b, g.group);
+    for (int t = threadIdx.x; t < T; t += blockDim.x) {
+        const float l = lp[r0 + t];
+        const float rho = expf(l - g.lp_old[r0 + t]);
+        const float clipped = fminf(fmaxf(rho, 1.f - g.eps_low), 1.f + g.eps_high);
+        float dL = rho * A <= clipped * A ? -rho * A : 0.f;
+        if (g.beta != 0.f) dL += g.beta * (1.f - expf(g.lp_ref[r0 + t] - l));
+        const float m = g.mask ? (float)g.mask[r0 + t] : 1.f;
+        coef[r0 + t] = n > 0.f ? -m * dL / n : 0.f;
+    }
+}
+
 }  // namespace
+
+void launch_grpo_coef(const float* lp, int B, int T, const GrpoArgs& g, const void* scratch, float* coef,
+                      cudaStream_t s) {
+    launch_k(grpo_coef_kernel, dim3(B), dim3(kThreads), 0, s, lp, T, g, (const float2*)scratch, B, coef);
+    note_launch();
+}
 
 size_t grpo_scratch_bytes(int B) { return (((size_t)B * sizeof(float2)) + 255) & ~(size_t)255; }
 

@@ -641,6 +641,7 @@ int qk_workspace_bytes(const qk_model* mh, int kind, int B, int T, int max_seq, 
         *bytes = (w.total > w2.total ? w.total : w2.total) + rollout_cursor_bytes(B);
         return QK_OK;
     }
+    if (kind == QK_CALL_BACKWARD) return backward_workspace_bytes(m, B, T, bytes);
     if (kind != QK_CALL_DECODE && kind != QK_CALL_PREFILL && kind != QK_CALL_SCORE)
         return set_error(QK_EINVAL, "unknown call kind %d", kind);
     QK_TRY(workspace_layout(m, kind, B, T, max_seq, &w, nullptr));
@@ -875,6 +876,23 @@ int qk_grpo_token_loss(const float* lp, const float* lp_old, const float* lp_ref
                          grpo_scratch_bytes(B));
     launch_grpo_loss(lp, B, T, g, true, workspace, loss_mean, (cudaStream_t)stream);
     return check_launch("grpo token loss");
+}
+
+int qk_grpo_coef(const float* lp, const float* lp_old, const float* lp_ref, int B, int T, int ld,
+                 const float* rewards, int group, const uint8_t* mask, float eps_low, float eps_high,
+                 float beta, float* coef, float* loss_tok, float* loss_mean, void* workspace,
+                 size_t ws_bytes, void* stream) {
+    if (!lp || !coef) return set_error(QK_EINVAL, "null argument");
+    GrpoArgs g;
+    QK_TRY(grpo_args(lp_old, lp_ref, B, T, ld, rewards, group, mask, eps_low, eps_high, beta,
+                     loss_tok, &g));
+    if (!workspace || ws_bytes < grpo_scratch_bytes(B))
+        return set_error(QK_ENOSPACE, "workspace has %zu bytes, needs %zu", ws_bytes,
+                         grpo_scratch_bytes(B));
+    cudaStream_t s = (cudaStream_t)stream;
+    launch_grpo_loss(lp, B, T, g, true, workspace, loss_mean, s);
+    launch_grpo_coef(lp, B, T, g, workspace, coef, s);
+    return check_launch("grpo coefficients");
 }
 
 int qk_score_grpo(qk_model* mh, const int32_t* tokens, int B, int T, const float* lp_old,

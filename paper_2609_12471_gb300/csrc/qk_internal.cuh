@@ -239,6 +239,12 @@ void launch_logits_reduce(const float* logits, int M, int V, OutIndex oi, float*
 size_t grpo_scratch_bytes(int B);
 void launch_grpo_loss(const float* lp, int B, int T, const GrpoArgs& g, bool compute,
                       void* scratch, float* loss_mean, cudaStream_t s);
+// Per-token coefficients of the GRPO gradient (after launch_grpo_loss filled `scratch`):
+// coef = -mask * (d loss_tok / d lp) / sum(mask), same indexing as lp.
+void launch_grpo_coef(const float* lp, int B, int T, const GrpoArgs& g, const void* scratch, float* coef,
+                      cudaStream_t s);
+// Workspace of qk_backward_logprob (qk_backward.cu).
+int backward_workspace_bytes(const Model& m, int B, int T, size_t* bytes);
 // Rollout cursor: s = *step; pos[b] = P + s; tok[b] = seq[b, P + s]; tgt[b] = seq[b, P + s + 1];
 // *out_off = s + 1; *step = s + 1.
 void launch_rollout_prepare(const int32_t* seq, int L, int P, int B, int32_t* step, int32_t* pos,

@@ -119,6 +119,28 @@ class Decoder:
                         eps_high, beta, logprobs, loss_tok, loss_mean, ws)
         return logprobs, loss_tok, loss_mean
 
+    def weight_shapes(self):
+        """Shapes of the weight tensors in the canonical order of qk_model_load."""
+        c = self.cfg
+        H, d, nq, nkv, I, V = c.hidden, c.head_dim, c.n_q_heads, c.n_kv_heads, c.intermediate, c.vocab
+        layer = [(H,), (nq * d, H), (nkv * d, H), (nkv * d, H), (d,), (d,), (H, nq * d), (H,), (I, H),
+                 (I, H), (H, I)]
+        return [(V, H)] + layer * c.n_layers + [(H,), (V, H)]
+
+    def new_grads(self):
+        """fp32 gradient buffers, one per weight tensor (canonical order)."""
+        return [torch.empty(shp, dtype=torch.float32, device=self.device) for shp in self.weight_shapes()]
+
+    def backward(self, tokens, coef, grads, accumulate=False, loss=None):
+        """d/d theta of sum coef[b, t] * (-log p(tokens[b, t+1] | tokens[b, <= t])) into grads
+        (qk_backward_logprob); returns loss [1]."""
+        Bn, T = tokens.shape
+        if loss is None:
+            loss = torch.empty(1, dtype=torch.float32, device=self.device)
+        ws = self.workspace(B.QK_CALL_BACKWARD, Bn, T)
+        B.qk_backward_logprob(self.handle, tokens, Bn, T, coef, grads, int(bool(accumulate)), loss, ws)
+        return loss
+
     def prefill_rows(self, kv, max_batch, max_seq, tokens, start, length=None, last_logits=None):
         """Append tokens[b, :length[b]] to row b at positions start[b] .. (rows at different
         positions; entries past length[b] are padding)."""

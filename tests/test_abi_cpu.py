@@ -117,6 +117,25 @@ def test_grpo_and_turn_entry_points_validate_on_the_host(lib):
     assert e.value.code == qk.QK_EINVAL
 
 
+def test_backward_entry_points_validate_on_the_host(lib):
+    """qk_grpo_coef and qk_backward_logprob reject bad arguments before any device work."""
+    import paper_2609_12471_gb300 as qk
+    P = 16
+    with pytest.raises(qk.QKError) as e:
+        qk.qk_grpo_coef(None, P, P, 6, 4, 4, P, 3, None, 0.2, 0.28, 0.01, P, P, None, None, 0, stream=0)
+    assert e.value.code == qk.QK_EINVAL
+    with pytest.raises(qk.QKError) as e:  # 6 rows are not whole groups of 4
+        qk.qk_grpo_coef(P, P, P, 6, 4, 4, P, 4, None, 0.2, 0.28, 0.01, P, P, None, None, 0, stream=0)
+    assert e.value.code == qk.QK_ESHAPE
+    with pytest.raises(qk.QKError) as e:  # valid arguments, no workspace
+        qk.qk_grpo_coef(P, P, P, 6, 4, 4, P, 3, None, 0.2, 0.28, 0.01, P, P, None, None, 0, stream=0)
+    assert e.value.code == qk.QK_ENOSPACE
+    with pytest.raises(qk.QKError) as e:
+        qk.qk_backward_logprob(None, P, 1, 4, P, [P] * 25, ws_bytes=0, stream=0)
+    assert e.value.code == qk.QK_EINVAL
+    assert qk.QK_CALL_BACKWARD == 4
+
+
 def test_debug_hook_validates_on_the_host():
     import paper_2609_12471_gb300 as qk
     with pytest.raises(qk.QKError) as e:
