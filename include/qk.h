@@ -258,9 +258,9 @@ int qk_grpo_coef(const float* lp, const float* lp_old, const float* lp_ref, int 
  * qk_model_load (row-major [out, in]), each 16-byte aligned; each receives
  * d loss / d tensor (accumulate == 0: overwritten; else added to).  loss dev fp32
  * [1] or NULL receives the loss.  workspace: qk_workspace_bytes(QK_CALL_BACKWARD,
- * B, T, 0), 256-byte aligned (it holds each layer's fp32 input residual, the
- * attention probabilities of one layer and a [min(B T, 4096), V] block of logit
- * gradients).  bf16 models need T % 128 == 0, head_dim 128 and vocab % 64 == 0
+ * B, T, 0), 256-byte aligned (it keeps every layer's forward activations, about
+ * 1.1 GB per layer per 8192 tokens at Qwen3-8B size, the attention probabilities of
+ * one layer and a [min(B T, 4096), V] block of logit gradients).  bf16 models need T % 128 == 0, head_dim 128 and vocab % 64 == 0
  * (QK_ESHAPE otherwise); fp32 models take any shape.  Activations are rounded to
  * the model dtype where the forward pass rounds them (and the logit and attention
  * gradients, which are tensor-core operands, likewise); accumulation, norms,

@@ -35,10 +35,12 @@ struct Op {
     int pitch;
 };
 
-// Output element (z, m, n) is C[(z / zq) * zrow + m, (z % zq) * zcol + n] (row stride ldc).
+// Output element (z, m, n) is C[(z / zq) * zrow + m, (z % zq) * zcol + n] of the buffer
+// C [rows, cols] (row stride ldc).
 struct Out {
     void* C;
     long long ldc;
+    int rows, cols;
     int zq, zrow, zcol;
     const float* addend;  // E_F32: C = addend + acc, addend indexed like C (may be C itself)
 };
@@ -99,7 +101,7 @@ __device__ __forceinline__ void tile_at(const Sched& s, int BM, int BN, long lon
     long long r = t - (long long)z * per;
     const int nm = cdiv(s.M, BM), nn = cdiv(s.N, BN);
     if (s.tri) {  // row i holds i + 1 tiles (nn == nm)
-        int i = (int)((sqrt(8.0 * (double)r + 1.0) - 1.0) * 0.5);
+        int i = (int)((sqrtf(8.f * (float)r + 1.f) - 1.f) * 0.5f);
         while ((long long)(i + 1) * (i + 2) / 2 <= r) ++i;
         while ((long long)i * (i + 1) / 2 > r) --i;
         mt = i;
@@ -161,6 +163,20 @@ __device__ __forceinline__ float ld_act(const bf16* p) { return __bfloat162float
 __device__ __forceinline__ void st_act(float* p, float v) { *p = v; }
 __device__ __forceinline__ void st_act(bf16* p, float v) { *p = __float2bfloat16_rn(v); }
 
+// Element offset of output (z, m, n) in C.
+__device__ __forceinline__ size_t out_offset(const Out& o, int z, int m, int n) {
+    const size_t row = (size_t)(z / o.zq) * o.zrow + m;
+    return row * (size_t)o.ldc + (size_t)(z % o.zq) * o.zcol + n;
+}
+
+constexpr float kLog2e = 1.4426950408889634f;
+// 2^x on the special-function unit (relative error about 2^-22; 2^-inf = 0).
+__device__ __forceinline__ float exp2f_fast(float x) {
+    float y;
+    asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+    return y;
+}
+
 struct RowStat {
     float mx, sm;
 };
@@ -177,11 +193,12 @@ __device__ __forceinline__ void stat_merge(RowStat& a, float m2, float s2) {
     a.mx = mx;
 }
 
-// The epilogue of nv <= 16 consecutive outputs (z, m, n .. n + nv - 1) with values v.
-// VEC: nv == 16 and every address 16-byte aligned (vector loads and stores).
+// Epilogue values of nv <= 16 consecutive outputs (z, m, n .. n + nv - 1) from the
+// accumulators v: E_STATS updates st and returns false (nothing to store); the other
+// modes fill y and return true.  VEC: nv == 16 and every address 16-byte aligned.
 template <typename act_t, bool VEC>
-__device__ __forceinline__ void epi16(const Epi& e, const Out& o, int z, int m, int n, int nv,
-                                      const float (&v)[16], RowStat& st) {
+__device__ __forceinline__ bool epi_values(const Epi& e, const Out& o, int z, int m, int n, int nv,
+                                           const float (&v)[16], RowStat& st, float (&y)[16]) {
     const int r = z * e.rows_per_z + m;
     if (e.mode == E_STATS) {
         float t[16];
@@ -194,16 +211,16 @@ __device__ __forceinline__ void epi16(const Epi& e, const Out& o, int z, int m, 
             cmax = fmaxf(cmax, t[j]);
             if (ok && n + j == tg) e.zt[r] = t[j];
         }
-        if (cmax == -INFINITY) return;
+        if (cmax == -INFINITY) return false;
+        // e^(t - cmax) = 2^((t - cmax) log2 e); masked entries give 2^-inf = 0
+        const float c2 = cmax * kLog2e;
         float cs = 0.f;
 #pragma unroll
-        for (int j = 0; j < 16; ++j) cs += expf(t[j] - cmax);  // exp(-inf) = 0 for masked entries
+        for (int j = 0; j < 16; ++j) cs += exp2f_fast(fmaf(t[j], kLog2e, -c2));
         stat_merge(st, cmax, cs);
-        return;
+        return false;
     }
-    const size_t row = (size_t)(z / o.zq) * o.zrow + m;
-    const size_t off = row * (size_t)o.ldc + (size_t)(z % o.zq) * o.zcol + n;
-    float y[16];
+    const size_t off = out_offset(o, z, m, n);
     if (e.mode == E_F32 || e.mode == E_ACT) {
 #pragma unroll
         for (int j = 0; j < 16; ++j) y[j] = v[j];
@@ -220,13 +237,14 @@ __device__ __forceinline__ void epi16(const Epi& e, const Out& o, int z, int m, 
             }
         }
     } else if (e.mode == E_SOFTMAX) {
-        const float l = e.lse[r];
+        // e^(scale acc - lse) = 2^(acc scale log2 e - lse log2 e)
+        const float l2 = e.lse[r] * kLog2e, c = e.scale * kLog2e;
         const float w = e.w ? e.w[r] : 1.f;
         const int tg = e.tgt ? e.tgt[r] : -1;
 #pragma unroll
         for (int j = 0; j < 16; ++j) {
             const bool masked = e.causal && n + j > m;
-            const float p = masked ? 0.f : expf(v[j] * e.scale - l);
+            const float p = masked ? 0.f : exp2f_fast(fmaf(v[j], c, -l2));
             y[j] = (p - (n + j == tg ? 1.f : 0.f)) * w;
         }
     } else {  // E_DS
@@ -246,27 +264,22 @@ __device__ __forceinline__ void epi16(const Epi& e, const Out& o, int z, int m, 
 #pragma unroll
         for (int j = 0; j < 16; ++j) y[j] = p[j] * (v[j] - d) * e.scale;
     }
+    return true;
+}
+
+// The epilogue of nv <= 16 consecutive outputs with plain stores (CUDA-core path).
+template <typename act_t>
+__device__ __forceinline__ void epi16(const Epi& e, const Out& o, int z, int m, int n, int nv,
+                                      const float (&v)[16], RowStat& st) {
+    float y[16];
+    if (!epi_values<act_t, false>(e, o, z, m, n, nv, v, st, y)) return;
+    const size_t off = out_offset(o, z, m, n);
     if (e.mode == E_F32) {
         float* c = (float*)o.C + off;
-        if constexpr (VEC) {
-#pragma unroll
-            for (int j = 0; j < 16; j += 4) *(float4*)(c + j) = make_float4(y[j], y[j + 1], y[j + 2], y[j + 3]);
-        } else {
-            for (int j = 0; j < nv; ++j) c[j] = y[j];
-        }
+        for (int j = 0; j < nv; ++j) c[j] = y[j];
     } else {
         act_t* c = (act_t*)o.C + off;
-        if constexpr (VEC && sizeof(act_t) == 2) {
-            uint4 q0, q1;
-            bf16* b0 = (bf16*)&q0;
-            bf16* b1 = (bf16*)&q1;
-#pragma unroll
-            for (int j = 0; j < 8; ++j) b0[j] = __float2bfloat16_rn(y[j]), b1[j] = __float2bfloat16_rn(y[j + 8]);
-            *(uint4*)c = q0;
-            *(uint4*)(c + 8) = q1;
-        } else {
-            for (int j = 0; j < nv; ++j) st_act(c + j, y[j]);
-        }
+        for (int j = 0; j < nv; ++j) st_act(c + j, y[j]);
     }
 }
 
@@ -280,17 +293,19 @@ struct Gemm {
 
 // Runs g on the model's path: tcgen05 for bf16 models, CUDA cores for fp32 models.
 int run_gemm(Model& m, const Gemm& g, cudaStream_t s);
-// Column-tile width of the kernel run_gemm picks for N columns (E_STATS partials per row).
+// Column width of the E_STATS partials of the kernel run_gemm picks for N columns
+// (half its N tile on the tensor-core path, its tile on the CUDA-core path).
 int gemm_tile_n(const Model& m, int N, int tri);
 
 // ---------------------------------------------------------------- row / elementwise kernels
 // tgt[r] = tokens[b, t + 1] and w[r] = coef[b, t] for r = b T + t, t < T - 1; -1 and 0 for t = T - 1.
 void launch_rows_prep(const int32_t* tokens, int B, int T, const float* coef, int V, int* tgt, float* w,
                       uint32_t* status, cudaStream_t s);
-// qr [M, nq d] / kr [M, nkv d] = RoPE(RMSNorm(raw head) g) of the q / k heads of qkv
-// (row stride ld), position r % Tlen.
+// From the raw projections qkv [M, (nq + 2 nkv) d] (row stride ld) of M = B Tlen rows at
+// positions r % Tlen: qr [M, nq d] = RoPE(RMSNorm(q head) g_q) (token major); kvh =
+// [2][B][nkv][Tlen][d], K = RoPE(RMSNorm(k head) g_k) then V = the raw v heads (head major).
 void launch_qk_fwd(const void* qkv, int ld, int M, int Tlen, int nq, int nkv, int d, const float* gq,
-                   const float* gk, float eps, const float* rc, const float* rs, void* qr, void* kr,
+                   const float* gk, float eps, const float* rc, const float* rs, void* qr, void* kvh,
                    int dtype, cudaStream_t s);
 // lse[r] from the E_STATS partials st [R][n_ct] (column tiles of ct_w; causal: only the
 // tiles at or left of the diagonal of row r % rows_per_z); loss_rows (may be null).

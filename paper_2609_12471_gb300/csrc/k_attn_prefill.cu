@@ -101,7 +101,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                         const __grid_constant__ CUtensorMap tmKV, int nq, int nkv,
                         int max_batch, int max_seq, int start_all,
                         const int32_t* __restrict__ start_dev, int T, int n_work,
-                        bf16* __restrict__ o, uint32_t* __restrict__ status) {
+                        bf16* __restrict__ o, float* __restrict__ lse, uint32_t* __restrict__ status) {
     extern __shared__ uint8_t smem_raw[];
     uint8_t* smem = (uint8_t*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
     uint8_t* sQ = smem;
@@ -421,6 +421,8 @@ __global__ void __launch_bounds__(kThreads, 1)
             if (!ok) break;
             tc::fence_after_sync();
             const float inv = l > 0.f ? 1.f / l : 0.f;
+            // log-sum-exp of the row's scaled scores: sum_k e^(s_k / sqrt(d)) = l 2^m
+            if (lse && t < T) lse[((size_t)w.b * nq + w.h) * T + t] = (m + log2f(l)) * 0.6931471805599453f;
             const uint32_t o_t = tmem_base + lane_off + 256;
             bf16* orow = o + ((size_t)w.b * T + (t < T ? t : 0)) * (size_t)(nq * kD) + (size_t)w.h * kD;
 #pragma unroll
@@ -481,7 +483,7 @@ bool attn_prefill_supported(int d, int nq, int nkv) { return d == kD && nq % nkv
 int launch_attn_prefill(const bf16* q, int q_ld, const void* k_layer, int nq, int nkv,
                         int max_batch, int max_seq, int B, int T, int start,
                         const int32_t* start_dev, bf16* o, int num_sms,
-                        uint32_t* status, cudaStream_t s) {
+                        uint32_t* status, cudaStream_t s, float* lse) {
     static bool attr_set = false;
     if (!attr_set) {
         if (cudaFuncSetAttribute(attn_prefill_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
@@ -507,7 +509,7 @@ int launch_attn_prefill(const bf16* q, int q_ld, const void* k_layer, int nq, in
     const int n_work = B * nq * n_qt;
     const int grid = n_work < num_sms ? n_work : num_sms;
     launch_k(attn_prefill_kernel, dim3(grid), dim3(kThreads), kSmem, s, mq, mkv, nq, nkv, max_batch,
-             max_seq, start, start_dev, T, n_work, o, status);
+             max_seq, start, start_dev, T, n_work, o, lse, status);
     note_launch();
     return QK_OK;
 }

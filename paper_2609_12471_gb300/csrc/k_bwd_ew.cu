@@ -65,21 +65,31 @@ __global__ void rows_prep_kernel(const int32_t* __restrict__ tokens, int B, int 
     }
 }
 
-// One warp per (token row, q or k head): qr / kr = RoPE(RMSNorm(raw) g) at position r % T.
+// One warp per (token row r = b T + t, head of qkv): q heads -> qr [M, nq D] (token
+// major) = RoPE(RMSNorm(raw) g_q); k heads -> kvh rows (b nkv + g) T + t = RoPE(RMSNorm(raw) g_k);
+// v heads copied to kvh rows M nkv + (b nkv + g) T + t (K then V, head major, the layout
+// of a KV cache holding B rows of T positions).
 template <typename T, int D>
 __global__ void qk_fwd_kernel(const T* __restrict__ qkv, int ld, int M, int Tlen, int nq, int nkv,
                               const float* __restrict__ gq, const float* __restrict__ gk, float eps,
                               const float* __restrict__ rc, const float* __restrict__ rs,
-                              T* __restrict__ qr, T* __restrict__ kr) {
+                              T* __restrict__ qr, T* __restrict__ kvh) {
     constexpr int E = D / 32, HALF = D / 2;
     pdl_wait();
     const int lane = threadIdx.x & 31;
     const long long item = (long long)blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
-    const int nh = nq + nkv;
+    const int nh = nq + 2 * nkv;
     if (item >= (long long)M * nh) return;
     const int r = (int)(item / nh), hh = (int)(item % nh);
-    const int p = r % Tlen;
+    const int b = r / Tlen, p = r % Tlen;
     const T* src = qkv + (size_t)r * ld + (size_t)hh * D;
+    if (hh >= nq + nkv) {
+        const int g = hh - nq - nkv;
+        T* dst = kvh + ((size_t)M * nkv + ((size_t)b * nkv + g) * Tlen + p) * D;
+#pragma unroll
+        for (int i = 0; i < E; ++i) dst[lane + 32 * i] = src[lane + 32 * i];
+        return;
+    }
     float e[E];
 #pragma unroll
     for (int i = 0; i < E; ++i) e[i] = ld_act(src + lane + 32 * i);
@@ -94,12 +104,12 @@ __global__ void qk_fwd_kernel(const T* __restrict__ qkv, int ld, int M, int Tlen
     for (int i = 0; i < E / 2; ++i) {
         const int j = lane + 32 * i;
         const float c = rc[(size_t)p * HALF + j], sn = rs[(size_t)p * HALF + j];
-        const float a = e[i], b = e[i + E / 2];
-        e[i] = a * c - b * sn;
-        e[i + E / 2] = b * c + a * sn;
+        const float a = e[i], bb = e[i + E / 2];
+        e[i] = a * c - bb * sn;
+        e[i + E / 2] = bb * c + a * sn;
     }
     T* dst = hh < nq ? qr + (size_t)r * nq * D + (size_t)hh * D
-                     : kr + (size_t)r * nkv * D + (size_t)(hh - nq) * D;
+                     : kvh + (((size_t)b * nkv + (hh - nq)) * Tlen + p) * D;
 #pragma unroll
     for (int i = 0; i < E; ++i) st_act(dst + lane + 32 * i, e[i]);
 }
@@ -338,18 +348,18 @@ void launch_rows_prep(const int32_t* tokens, int B, int T, const float* coef, in
 }
 
 void launch_qk_fwd(const void* qkv, int ld, int M, int Tlen, int nq, int nkv, int d, const float* gq,
-                   const float* gk, float eps, const float* rc, const float* rs, void* qr, void* kr,
+                   const float* gk, float eps, const float* rc, const float* rs, void* qr, void* kvh,
                    int dtype, cudaStream_t s) {
-    const long long items = (long long)M * (nq + nkv);
+    const long long items = (long long)M * (nq + 2 * nkv);
     const dim3 grid((unsigned)((items + 7) / 8));
     launch_act(dtype, [&](auto* tp) {
         using A = std::remove_pointer_t<decltype(tp)>;
         if (d == 128)
             launch_k(qk_fwd_kernel<A, 128>, grid, dim3(256), 0, s, (const A*)qkv, ld, M, Tlen, nq, nkv, gq,
-                     gk, eps, rc, rs, (A*)qr, (A*)kr);
+                     gk, eps, rc, rs, (A*)qr, (A*)kvh);
         else
             launch_k(qk_fwd_kernel<A, 64>, grid, dim3(256), 0, s, (const A*)qkv, ld, M, Tlen, nq, nkv, gq,
-                     gk, eps, rc, rs, (A*)qr, (A*)kr);
+                     gk, eps, rc, rs, (A*)qr, (A*)kvh);
     });
     note_launch();
 }

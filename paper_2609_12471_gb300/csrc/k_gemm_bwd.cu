@@ -2,12 +2,13 @@
 // kernel for bf16 models and a CUDA-core kernel for fp32 models, both over the
 // same operand descriptors, tile schedule and epilogue.
 //
-// tcgen05 kernel, one persistent CTA per SM, 192 threads:
+// tcgen05 kernel, one persistent CTA per SM, 320 threads:
 //   warp 0, one lane : TMA producer over a STAGES-deep ring of (A, B) k-blocks of 64;
 //   warp 1           : TMEM allocation; one lane issues tcgen05.mma (M 128, N BN, K 16)
 //                      and the commits;
-//   warps 2..5       : epilogue; warp w reads TMEM lanes 32 (w % 4) .. + 31, one output
-//                      row per thread, 16 columns per tcgen05.ld.
+//   warps 2..9       : epilogue; warp w reads TMEM lanes 32 (w % 4) .. + 31 (one output
+//                      row per thread) and half (w - 2) / 4 of the tile's columns, 16
+//                      columns per tcgen05.ld, four loads per wait.
 // A K-major operand tile is one 128-byte-swizzled box (64 k x 128 or BN rows); an
 // MN-major one is boxes of 64 m/n x 64 k (8 KB each), whose descriptor steps 64
 // m/n elements by the leading byte offset (8 KB) and 8 k rows by the stride byte
@@ -16,6 +17,7 @@
 // the CTA raises QK_STATUS_TIMEOUT, drains its copies and MMAs and exits.
 #include <cuda.h>
 #include <math.h>
+#include <string.h>
 
 #include "bwd_common.cuh"
 #include "tc_ptx.cuh"
@@ -71,7 +73,7 @@ __global__ void __launch_bounds__(kSimtThreads) gemm_bwd_simt_kernel(Gemm g, lon
     int nv = sc.N - n;
     nv = nv < 0 ? 0 : (nv > 16 ? 16 : nv);
     RowStat st{-INFINITY, 0.f};
-    if (m < sc.M && nv > 0) epi16<T, false>(g.epi, g.out, z, m, n, nv, acc, st);
+    if (m < sc.M && nv > 0) epi16<T>(g.epi, g.out, z, m, n, nv, acc, st);
     if (g.epi.mode == E_STATS) {  // merge the row's four 16-column parts
 #pragma unroll
         for (int o = 1; o < 4; o <<= 1) {
@@ -85,7 +87,8 @@ __global__ void __launch_bounds__(kSimtThreads) gemm_bwd_simt_kernel(Gemm g, lon
 }
 
 // ------------------------------------------------------------------ tcgen05 kernel
-constexpr int kThreads = 192;
+constexpr int kEpiWarps = 8;  // two per TMEM lane quadrant, each owning half of the tile's columns
+constexpr int kThreads = 64 + 32 * kEpiWarps;
 constexpr int kBK = 64;
 constexpr int kBox = 64 * 128;  // one 64 x 64 bf16 box (8 KB)
 
@@ -95,22 +98,24 @@ struct TcCfg {
     static constexpr int A_BYTES = 128 * 128;
     static constexpr int B_BYTES = BN * 128;
     static constexpr int TMEM_COLS = 2 * BN;
-    static constexpr int SMEM = STAGES * (A_BYTES + B_BYTES) + 1024 + 256;
+    static constexpr int STAGE_OUT = kEpiWarps * 2 * 32 * 16 * 4;  // per epilogue warp: two 32 x 16 fp32 blocks
+    static constexpr int SMEM = STAGES * (A_BYTES + B_BYTES) + STAGE_OUT + 1024 + 256;
     static_assert(TMEM_COLS <= 512, "accumulators exceed TMEM");
 };
 
 template <int BN, bool AMN, bool BMN>
 __global__ void __launch_bounds__(kThreads, 1)
     gemm_bwd_tc_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant__ CUtensorMap mapB,
-                       const __grid_constant__ Gemm g, long long per, long long total,
-                       uint32_t* __restrict__ status) {
+                       const __grid_constant__ CUtensorMap mapC, const __grid_constant__ Gemm g,
+                       long long per, long long total, int a3, int b3, uint32_t* __restrict__ status) {
     using G = TcCfg<BN>;
     constexpr int STAGES = G::STAGES;
     extern __shared__ uint8_t smem_raw[];
     uint8_t* smem = (uint8_t*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
     uint8_t* sA = smem;
     uint8_t* sB = smem + STAGES * G::A_BYTES;
-    uint64_t* full = (uint64_t*)(sB + STAGES * G::B_BYTES);
+    uint8_t* sOut = sB + STAGES * G::B_BYTES;
+    uint64_t* full = (uint64_t*)(sOut + G::STAGE_OUT);
     uint64_t* empty = full + STAGES;
     uint64_t* tfull = empty + STAGES;
     uint64_t* tempty = tfull + 2;
@@ -128,7 +133,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         for (int a = 0; a < 2; ++a) {
             tc::mbar_init(&tfull[a], 1);
-            tc::mbar_init(&tempty[a], 4);
+            tc::mbar_init(&tempty[a], kEpiWarps);
         }
         tc::mbar_init(drain, 1);
         *abort_flag = 0;
@@ -167,21 +172,31 @@ __global__ void __launch_bounds__(kThreads, 1)
                     uint8_t* a_s = sA + stage * G::A_BYTES;
                     uint8_t* b_s = sB + stage * G::B_BYTES;
                     int x, y;
-                    if (AMN) {
+                    if (AMN) {  // MN chunks of 64: one 3-D box (chunk index as the third axis) or one box each
+                        if (a3) {
+                            op_xy(g.A, z, m0, k0, x, y);
+                            tc::tma_load_3d(a_s, &mapA, 0, y, x >> 6, &full[stage]);
+                        } else {
 #pragma unroll
-                        for (int c = 0; c < 2; ++c) {
-                            op_xy(g.A, z, m0 + 64 * c, k0, x, y);
-                            tc::tma_load_2d(a_s + c * kBox, &mapA, x, y, &full[stage]);
+                            for (int c = 0; c < 2; ++c) {
+                                op_xy(g.A, z, m0 + 64 * c, k0, x, y);
+                                tc::tma_load_2d(a_s + c * kBox, &mapA, x, y, &full[stage]);
+                            }
                         }
                     } else {
                         op_xy(g.A, z, m0, k0, x, y);
                         tc::tma_load_2d(a_s, &mapA, x, y, &full[stage]);
                     }
                     if (BMN) {
+                        if (b3) {
+                            op_xy(g.B, z, n0, k0, x, y);
+                            tc::tma_load_3d(b_s, &mapB, 0, y, x >> 6, &full[stage]);
+                        } else {
 #pragma unroll
-                        for (int c = 0; c < BN / 64; ++c) {
-                            op_xy(g.B, z, n0 + 64 * c, k0, x, y);
-                            tc::tma_load_2d(b_s + c * kBox, &mapB, x, y, &full[stage]);
+                            for (int c = 0; c < BN / 64; ++c) {
+                                op_xy(g.B, z, n0 + 64 * c, k0, x, y);
+                                tc::tma_load_2d(b_s + c * kBox, &mapB, x, y, &full[stage]);
+                            }
                         }
                     } else {
                         op_xy(g.B, z, n0, k0, x, y);
@@ -254,9 +269,16 @@ __global__ void __launch_bounds__(kThreads, 1)
             }
         }
     } else {
-        // ---------------------------------------------------- epilogue (warps 2..5)
-        const int q = warp & 3;
-        int acc = 0;
+        // ---------------------------------------------------- epilogue (warps 2..9)
+        // Warp w reads TMEM lanes 32 (w % 4) .. + 31 (its rows) and the columns of half
+        // (w - 2) / 4 of the tile, four 16-column blocks per TMEM wait.  Each 32-row x
+        // 16-column block of outputs goes through the warp's staging buffer (two
+        // alternating halves) and out with one TMA store.
+        const int q = warp & 3, half = (warp - 2) >> 2;
+        constexpr int HC = BN / 2;
+        const bool f32 = g.epi.mode == E_F32;
+        uint8_t* stg = sOut + (warp - 2) * (2 * 32 * 16 * 4);
+        int acc = 0, blk = 0;
         uint32_t acc_phase = 0;
         for (long long t = blockIdx.x; t < total; t += gridDim.x) {
             int z, mt, nt;
@@ -268,26 +290,62 @@ __global__ void __launch_bounds__(kThreads, 1)
             tc::fence_after_sync();
             const int m = m0 + q * 32 + lane;
             const uint32_t tbase = tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(acc * BN);
+            const int orow = (z / g.out.zq) * g.out.zrow + m0 + q * 32;
+            const int ocol = (z % g.out.zq) * g.out.zcol;
             RowStat st{-INFINITY, 0.f};
-            for (int c0 = 0; c0 < BN; c0 += 16) {
-                const int n = n0 + c0;
-                if (n >= sc.N) break;  // uniform over the warp
-                uint32_t r[16];
-                tc::tmem_ld16(tbase + c0, r);
-                tc::tmem_wait_ld();
-                float v[16];
+            for (int c4 = half * HC; c4 < (half + 1) * HC; c4 += 64) {
+                if (n0 + c4 >= sc.N) break;  // uniform over the warp
+                uint32_t r[4][16];
 #pragma unroll
-                for (int j = 0; j < 16; ++j) v[j] = __uint_as_float(r[j]);
-                if (m < sc.M) epi16<bf16, true>(g.epi, g.out, z, m, n, 16, v, st);
+                for (int u = 0; u < 4; ++u)
+                    if (n0 + c4 + 16 * u < sc.N) tc::tmem_ld16(tbase + c4 + 16 * u, r[u]);
+                tc::tmem_wait_ld();
+#pragma unroll
+                for (int u = 0; u < 4; ++u) {
+                    const int n = n0 + c4 + 16 * u;
+                    if (n >= sc.N) break;
+                    float v[16], y[16];
+#pragma unroll
+                    for (int j = 0; j < 16; ++j) v[j] = __uint_as_float(r[u][j]);
+                    const bool store = m < sc.M && epi_values<bf16, true>(g.epi, g.out, z, m, n, 16, v, st, y);
+                    if (g.epi.mode == E_STATS) continue;
+                    uint8_t* buf = stg + (blk & 1) * (32 * 16 * 4);
+                    if (lane == 0) tc::bulk_wait_read<1>();  // the store issued from this half two blocks ago
+                    __syncwarp();
+                    if (f32) {
+                        float4* d = (float4*)(buf + lane * 64);
+#pragma unroll
+                        for (int j = 0; j < 4; ++j)
+                            d[j] = store ? make_float4(y[4 * j], y[4 * j + 1], y[4 * j + 2], y[4 * j + 3])
+                                         : make_float4(0.f, 0.f, 0.f, 0.f);
+                    } else {
+                        uint4 w[2];
+                        bf16* b = (bf16*)w;
+#pragma unroll
+                        for (int j = 0; j < 16; ++j) b[j] = __float2bfloat16_rn(store ? y[j] : 0.f);
+                        uint4* d = (uint4*)(buf + lane * 32);
+                        d[0] = w[0];
+                        d[1] = w[1];
+                    }
+                    tc::fence_proxy_async_smem();
+                    __syncwarp();
+                    if (lane == 0) {
+                        tc::tma_store_2d(&mapC, ocol + n, orow, buf);
+                        tc::bulk_commit();
+                    }
+                    ++blk;
+                }
             }
-            if (g.epi.mode == E_STATS && m < sc.M)
-                g.epi.stats[(size_t)(z * g.epi.rows_per_z + m) * g.epi.n_ct + nt] = make_float2(st.mx, st.sm);
+            const int ct = nt * 2 + half;  // statistics column tile of HC columns
+            if (g.epi.mode == E_STATS && m < sc.M && ct < g.epi.n_ct)
+                g.epi.stats[(size_t)(z * g.epi.rows_per_z + m) * g.epi.n_ct + ct] = make_float2(st.mx, st.sm);
             tc::fence_before_sync();
             __syncwarp();
             if (lane == 0) tc::mbar_arrive(&tempty[acc]);
             acc ^= 1;
             if (acc == 0) acc_phase ^= 1;
         }
+        if (lane == 0) tc::bulk_wait<0>();  // every store of this warp has completed
     }
 
     tc::fence_before_sync();
@@ -332,6 +390,35 @@ bool make_op_map(CUtensorMap* map, const Op& o, int box_rows) {
               CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+// MN-major operand as a 3-D map: (element within a 64-column chunk, row, chunk), box
+// 64 x 64 rows x nch chunks, so that one copy lands the nch chunks of a k-block one
+// after another (8 KB apart), the layout the MMA descriptors expect.
+bool make_op_map3(CUtensorMap* map, const Op& o, int nch) {
+    EncodeTiledFn fn = encode_fn();
+    if (!fn || o.cols % 64) return false;
+    cuuint64_t dims[3] = {64, (cuuint64_t)o.rows, (cuuint64_t)(o.cols / 64)};
+    cuuint64_t strides[2] = {(cuuint64_t)o.ld * 2, 128};
+    cuuint32_t box[3] = {64, 64, (cuuint32_t)nch};
+    cuuint32_t estr[3] = {1, 1, 1};
+    return fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(o.ptr), dims, strides, box,
+              estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+              CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+// Output map: fp32 or bf16 over C [rows, cols], box 16 columns x 32 rows, no swizzle.
+bool make_out_map(CUtensorMap* map, const Out& o, bool f32) {
+    EncodeTiledFn fn = encode_fn();
+    if (!fn) return false;
+    const size_t es = f32 ? 4 : 2;
+    cuuint64_t dims[2] = {(cuuint64_t)o.cols, (cuuint64_t)o.rows};
+    cuuint64_t strides[1] = {(cuuint64_t)o.ldc * es};
+    cuuint32_t box[2] = {16, 32};
+    cuuint32_t estr[2] = {1, 1};
+    return fn(map, f32 ? CU_TENSOR_MAP_DATA_TYPE_FLOAT32 : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, o.C, dims,
+              strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE,
+              CU_TENSOR_MAP_L2_PROMOTION_NONE, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
 template <int BN, bool AMN, bool BMN>
 int launch_tc(Model& m, const Gemm& g, cudaStream_t s) {
     using G = TcCfg<BN>;
@@ -342,14 +429,20 @@ int launch_tc(Model& m, const Gemm& g, cudaStream_t s) {
             return set_error(QK_ECUDA, "backward GEMM: shared-memory attribute");
         attr_set = true;
     }
-    CUtensorMap ma, mb;
-    if (!make_op_map(&ma, g.A, AMN ? 64 : 128) || !make_op_map(&mb, g.B, BMN ? 64 : BN))
+    CUtensorMap ma, mb, mc;
+    int a3 = 0, b3 = 0;
+    if (AMN) a3 = make_op_map3(&ma, g.A, 2) ? 1 : 0;
+    if (BMN) b3 = make_op_map3(&mb, g.B, BN / 64) ? 1 : 0;
+    if ((!a3 && !make_op_map(&ma, g.A, AMN ? 64 : 128)) || (!b3 && !make_op_map(&mb, g.B, BMN ? 64 : BN)))
         return set_error(QK_ECUDA, "backward GEMM: tensor map encoding failed");
+    memset(&mc, 0, sizeof(mc));
+    if (g.epi.mode != E_STATS && !make_out_map(&mc, g.out, g.epi.mode == E_F32))
+        return set_error(QK_ECUDA, "backward GEMM: output tensor map encoding failed");
     const long long per = tiles_per_z(g.sc, 128, BN);
     const long long total = per * g.sc.Z;
     const int grid = total < m.num_sms ? (int)total : m.num_sms;
-    launch_k(gemm_bwd_tc_kernel<BN, AMN, BMN>, dim3(grid), dim3(kThreads), G::SMEM, s, ma, mb, g,
-             per, total, m.status);
+    launch_k(gemm_bwd_tc_kernel<BN, AMN, BMN>, dim3(grid), dim3(kThreads), G::SMEM, s, ma, mb, mc, g,
+             per, total, a3, b3, m.status);
     note_launch();
     return QK_OK;
 }
@@ -358,9 +451,14 @@ bool aligned16(const void* p) { return ((uintptr_t)p & 15) == 0; }
 
 }  // namespace
 
-int gemm_tile_n(const Model& m, int N, int tri) {
+// Width of the column tiles of the N tile chosen for N columns (tri: causal, square tiles).
+static int tile_bn(const Model& m, int N, int tri) {
     if (m.cfg.dtype != QK_DTYPE_BF16) return kSimtTile;
     return (tri || N <= 128) ? 128 : 256;
+}
+
+int gemm_tile_n(const Model& m, int N, int tri) {
+    return m.cfg.dtype != QK_DTYPE_BF16 ? kSimtTile : tile_bn(m, N, tri) / 2;
 }
 
 int run_gemm(Model& m, const Gemm& g, cudaStream_t s) {
@@ -374,7 +472,7 @@ int run_gemm(Model& m, const Gemm& g, cudaStream_t s) {
         note_launch();
         return QK_OK;
     }
-    const int BN = gemm_tile_n(m, sc.N, sc.tri);
+    const int BN = tile_bn(m, sc.N, sc.tri);
     // Every k-block is whole, every TMA box starts on a 16-byte boundary and every
     // epilogue access of 16 outputs is 16-byte aligned.
     bool ok = sc.K % kBK == 0 && aligned16(g.A.ptr) && aligned16(g.B.ptr) && g.A.ld % 8 == 0 &&
@@ -384,6 +482,8 @@ int run_gemm(Model& m, const Gemm& g, cudaStream_t s) {
     ok = ok && (sc.red != RED_SUFFIX || (sc.seg % kBK == 0 && sc.seg > 0 && sc.K % sc.seg == 0));
     ok = ok && (!g.A.kwrap || g.A.kwrap % kBK == 0) && (!g.B.kwrap || g.B.kwrap % kBK == 0);
     ok = ok && g.B.pitch == 128 && g.A.pitch % 64 == 0 && (!sc.tri || (BN == 128 && sc.M == sc.N));
+    // output tiles are whole 128-row blocks of a batch entry, or clipped at the buffer's last row
+    ok = ok && (sc.M % 128 == 0 || (sc.Z == 1 && g.out.rows == sc.M)) && g.out.rows > 0 && g.out.cols > 0;
     if (!ok) return set_error(QK_ESHAPE, "backward GEMM: shape or alignment outside the tcgen05 path");
     const bool amn = g.A.mn != 0, bmn = g.B.mn != 0;
     if (BN == 256) {

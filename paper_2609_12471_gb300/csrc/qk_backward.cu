@@ -7,16 +7,18 @@
 // coef = -d L / d lp (qk_grpo_coef).
 //
 // Schedule (one call, one stream):
-//   1. forward over all layers, keeping only each layer's input residual x_l (fp32);
+//   1. forward over all layers, keeping each layer's activations (input residual x_l
+//      and x_mid in fp32; norms, projections, rotated q / k, v, attention output and
+//      log-sum-exp, SwiGLU inputs and output in the activation type);
 //   2. head, in chunks of rows: lm_head logits -> per-row log-sum-exp (tile
 //      statistics + combine), then dz = coef (softmax - onehot) in the activation
 //      type from a second pass over the logits, dW_lm (+)= dz^T hn, d hn = dz W_lm;
 //      final-norm backward;
-//   3. per layer, last to first: recompute the layer forward from x_l (attention
-//      probabilities P materialised per head, causal tiles only), then the backward
-//      of the MLP, of W_o, of the attention (dS = P (dP - D), dQ = dS K, dK and dV
-//      summed over each GQA group), of QK-norm and RoPE, of W_qkv and of the input
-//      norm, adding into the running residual gradient;
+//   3. per layer, last to first: the backward of the MLP and of W_o, then the
+//      attention probabilities P of the layer again from its log-sum-exp (causal tiles
+//      only, one [T, T] block per (row, head)), dS = P (dP - D), dQ = dS K, dK and dV
+//      summed over each GQA group, then QK-norm and RoPE, W_qkv and the input norm,
+//      adding into the running residual gradient;
 //   4. embedding gradient (scatter-add of the residual gradient).
 // Every product is a bwd::Gemm (k_gemm_bwd.cu): tcgen05 for bf16 models, CUDA cores
 // for fp32 models.  Gain gradients are reduced in a fixed order; the embedding
@@ -35,8 +37,18 @@ constexpr int kHeadRows = 4096;  // lm_head rows per chunk (the dz buffer is [ro
 
 size_t align256(size_t v) { return (v + 255) & ~(size_t)255; }
 
+// A buffer with one copy per layer.
+struct PerLayer {
+    char* base;
+    size_t stride;
+    void* at(int l) const { return base ? base + (size_t)l * stride : nullptr; }
+};
+
 struct BwdLayout {
     float* xs;  // (L + 1) x [M, H]: x_0 (embedding) .. x_L
+    // kept from the forward pass, per layer
+    PerLayer u1, qkv, qr, kvh, lse_a, O, x_mid, u2, gu, h;
+    // one copy
     int* tgt;
     float* w;
     float* loss_rows;
@@ -47,18 +59,8 @@ struct BwdLayout {
     float* lse_h;
     float* zt;
     void* dz;
-    void* u1;
-    void* qkv;
-    void* qr;
-    void* kr;
     float2* st_a;
-    float* lse_a;
     void* P;
-    void* O;
-    float* x_mid;
-    void* u2;
-    void* gu;
-    void* h;
     float* dh;
     void* dgu;
     float* du;
@@ -76,7 +78,7 @@ int bwd_layout(const Model& m, int B, int T, char* base, BwdLayout* L) {
     const qk_config& c = m.cfg;
     const size_t es = m.es, M = (size_t)B * T, H = c.hidden, d = c.head_dim, nq = c.n_q_heads,
                  nkv = c.n_kv_heads, I = c.intermediate, V = c.vocab, nqkv = (nq + 2 * nkv) * d,
-                 Z = (size_t)B * nq;
+                 Z = (size_t)B * nq, nl = c.n_layers;
     const size_t Mc = M < (size_t)kHeadRows ? M : (size_t)kHeadRows;
     const size_t nct_v = cdiv(c.vocab, gemm_tile_n(m, c.vocab, 0));
     const size_t nct_a = cdiv(T, gemm_tile_n(m, T, 1));
@@ -86,7 +88,23 @@ int bwd_layout(const Model& m, int B, int T, char* base, BwdLayout* L) {
         off = align256(off + bytes);
         return p;
     };
-    L->xs = (float*)take((size_t)(c.n_layers + 1) * M * H * 4);
+    auto per_layer = [&](size_t bytes) {
+        PerLayer q;
+        q.stride = align256(bytes);
+        q.base = (char*)take(q.stride * nl);
+        return q;
+    };
+    L->xs = (float*)take((nl + 1) * M * H * 4);
+    L->u1 = per_layer(M * H * es);
+    L->qkv = per_layer(M * nqkv * es);
+    L->qr = per_layer(M * nq * d * es);
+    L->kvh = per_layer(2 * M * nkv * d * es);
+    L->lse_a = per_layer(Z * T * 4);
+    L->O = per_layer(M * nq * d * es);
+    L->x_mid = per_layer(M * H * 4);
+    L->u2 = per_layer(M * H * es);
+    L->gu = per_layer(M * 2 * I * es);
+    L->h = per_layer(M * I * es);
     L->tgt = (int*)take(M * 4);
     L->w = (float*)take(M * 4);
     L->loss_rows = (float*)take(M * 4);
@@ -97,18 +115,8 @@ int bwd_layout(const Model& m, int B, int T, char* base, BwdLayout* L) {
     L->lse_h = (float*)take(Mc * 4);
     L->zt = (float*)take(Mc * 4);
     L->dz = take(Mc * V * es);
-    L->u1 = take(M * H * es);
-    L->qkv = take(M * nqkv * es);
-    L->qr = take(M * nq * d * es);
-    L->kr = take(M * nkv * d * es);
     L->st_a = (float2*)take(Z * T * nct_a * 8);
-    L->lse_a = (float*)take(Z * T * 4);
     L->P = take(Z * T * T * es);
-    L->O = take(M * nq * d * es);
-    L->x_mid = (float*)take(M * H * 4);
-    L->u2 = take(M * H * es);
-    L->gu = take(M * 2 * I * es);
-    L->h = take(M * I * es);
     L->dh = (float*)take(M * I * 4);
     L->dgu = take(M * 2 * I * es);
     L->du = (float*)take(M * H * 4);
@@ -141,10 +149,12 @@ Op opm(const void* p, long long ld, int rows, int cols) {
     o.mn = 1;
     return o;
 }
-Out out2(void* C, long long ldc, const float* addend = nullptr) {
+Out out2(void* C, long long ldc, int rows, int cols, const float* addend = nullptr) {
     Out o{};
     o.C = C;
     o.ldc = ldc;
+    o.rows = rows;
+    o.cols = cols;
     o.zq = 1;
     o.addend = addend;
     return o;
@@ -180,7 +190,7 @@ int lin_fwd(const Ctx& x, const void* X, int K, const void* W, int N, void* C, i
     Gemm g{};
     g.A = opk(X, K, x.M, K);
     g.B = opk(W, K, N, K);
-    g.out = out2(C, N, addend);
+    g.out = out2(C, N, x.M, N, addend);
     g.epi = epi_mode(mode);
     g.sc = sch(1, x.M, N, K);
     return run_gemm(x.m, g, x.s);
@@ -192,7 +202,7 @@ int lin_dx(const Ctx& x, const void* dY, long long ldy, const void* W, int Nout,
     Gemm g{};
     g.A = opk(dY, ldy, M, Nout);
     g.B = opm(W, Kin, Nout, Kin);
-    g.out = out2(C, Kin);
+    g.out = out2(C, Kin, M, Kin);
     g.epi = epi_mode(mode);
     g.sc = sch(1, M, Kin, Nout);
     return run_gemm(x.m, g, x.s);
@@ -207,78 +217,113 @@ int lin_dw(const Ctx& x, const void* dY, long long ldy, int cols_dy, int xb, int
     g.A.xb = xb;
     g.A.pitch = pitch;
     g.B = opm(X, ldx, M, Kin);
-    g.out = out2(G, Kin, add ? G : nullptr);
+    g.out = out2(G, Kin, Mo, Kin, add ? G : nullptr);
     g.epi = epi_mode(E_F32);
     g.sc = sch(1, Mo, Kin, M);
     return run_gemm(x.m, g, x.s);
 }
 
-// Attention operands over token-major buffers: batch entry z = b nq + h (query head) or
-// b nkv + g (kv head) selects rows b T .. and the head's d columns.
-Op head_op(const void* p, int ld, int M, int heads, int d, int T, int zdiv, bool mn, int xb = 0) {
+// Attention operands.  Token-major buffers [M, heads * d]: batch entry z = b nq + h (or
+// b nkv + g) selects rows b T .. and the head's d columns.  Head-major K / V ([2][B][nkv][T][d],
+// K then V): the kv head of query head z is plane z / (nq / nkv).
+Op head_op(const void* p, int ld, int M, int heads, int d, int T, bool mn) {
     Op o = mn ? opm(p, ld, M, ld) : opk(p, ld, M, ld);
-    o.xb = xb;
-    o.zdiv = zdiv;
     o.zq = heads;
     o.zx = d;
     o.zy = T;
     return o;
 }
+Op kv_op(const void* kvh, int M, int nkv, int d, int T, int grp, bool mn, bool v) {
+    const int rows = M * nkv;
+    Op o = mn ? opm(kvh, d, 2 * rows, d) : opk(kvh, d, 2 * rows, d);
+    o.yb = v ? rows : 0;
+    o.zdiv = grp;
+    o.zy = T;
+    return o;
+}
+
+// S = q k^T / sqrt(d) over the causal tiles of every (row, query head), epilogue e.
+Gemm scores_gemm(const Ctx& x, int l, const bwd::Epi& e) {
+    const qk_config& c = x.m.cfg;
+    const int d = c.head_dim, nq = c.n_q_heads, nkv = c.n_kv_heads, T = x.T, M = x.M;
+    Gemm g{};
+    g.A = head_op(x.L.qr.at(l), nq * d, M, nq, d, T, false);
+    g.B = kv_op(x.L.kvh.at(l), M, nkv, d, T, nq / nkv, false, false);
+    g.sc = sch(x.B * nq, T, T, d);
+    g.sc.tri = 1;
+    g.epi = e;
+    g.epi.scale = 1.f / sqrtf((float)d);
+    g.epi.causal = 1;
+    g.epi.rows_per_z = T;
+    g.out = out2(x.L.P, T, x.B * nq * T, T);
+    g.out.zrow = T;
+    return g;
+}
+
+// P = softmax of the causal scores of layer l from its stored log-sum-exp.
+int probs(const Ctx& x, int l) {
+    bwd::Epi e = epi_mode(E_SOFTMAX);
+    e.lse = (const float*)x.L.lse_a.at(l);
+    return run_gemm(x.m, scores_gemm(x, l, e), x.s);
+}
+
+// Causal attention of layer l: O and the per-row log-sum-exp.  bf16 models with
+// head_dim 128: the tcgen05 flash kernel (k_attn_prefill.cu); otherwise scores ->
+// statistics -> P -> P V through the batched GEMM.
+int attn_fwd(const Ctx& x, int l) {
+    Model& m = x.m;
+    const qk_config& c = m.cfg;
+    const int d = c.head_dim, nq = c.n_q_heads, nkv = c.n_kv_heads, T = x.T, M = x.M, Z = x.B * nq;
+    const BwdLayout& L = x.L;
+    float* lse = (float*)L.lse_a.at(l);
+    if (c.dtype == QK_DTYPE_BF16 && attn_prefill_supported(d, nq, nkv))
+        return launch_attn_prefill((const bf16*)L.qr.at(l), nq * d, L.kvh.at(l), nq, nkv, x.B, T, x.B, T, 0,
+                                   nullptr, (bf16*)L.O.at(l), m.num_sms, m.status, x.s, lse);
+    const int tn = gemm_tile_n(m, T, 1);
+    bwd::Epi e = epi_mode(E_STATS);
+    e.stats = L.st_a;
+    e.n_ct = cdiv(T, tn);
+    Gemm g = scores_gemm(x, l, e);
+    g.out = out2(nullptr, T, Z * T, T);
+    QK_TRY(run_gemm(m, g, x.s));
+    launch_stats_combine(L.st_a, cdiv(T, tn), tn, 1, Z * T, T, lse, nullptr, nullptr, nullptr, x.s);
+    QK_TRY(probs(x, l));
+    Gemm pv{};
+    pv.A = opk(L.P, T, Z * T, T);
+    pv.A.zy = T;
+    pv.B = kv_op(L.kvh.at(l), M, nkv, d, T, nq / nkv, true, true);
+    pv.sc = sch(Z, T, d, T, RED_PREFIX);
+    pv.sc.desc_m = 1;
+    pv.epi = epi_mode(E_ACT, T);
+    pv.out = out2(L.O.at(l), nq * d, M, nq * d);
+    pv.out.zq = nq;
+    pv.out.zrow = T;
+    pv.out.zcol = d;
+    return run_gemm(m, pv, x.s);
+}
 
 // ------------------------------------------------------------------ layer forward
-// From x_in [M, H]: u1, qkv, qr, kr, lse_a, P, O, x_mid, u2, gu, h of the layout; with
-// x_out, also x_out = x_mid + W_d h.
+// x_out = layer l (x_in); keeps the layer's activations (u1, qkv, qr, kvh, lse, O, x_mid,
+// u2, gu, h) for its backward.
 int layer_fwd(const Ctx& x, int l, const float* x_in, float* x_out) {
     Model& m = x.m;
     const qk_config& c = m.cfg;
     const LayerW& W = m.layers[l];
     const BwdLayout& L = x.L;
     const int H = c.hidden, d = c.head_dim, nq = c.n_q_heads, nkv = c.n_kv_heads, I = c.intermediate;
-    const int nqkv = (nq + 2 * nkv) * d, T = x.T, M = x.M, Z = x.B * nq, grp = nq / nkv;
-    const float eps = (float)c.rms_eps, sc = 1.f / sqrtf((float)d);
-    launch_rmsnorm(x_in, 1, 0, W.attn_norm, H, eps, L.u1, c.dtype, M, x.s);
-    QK_TRY(lin_fwd(x, L.u1, H, W.w_qkv, nqkv, L.qkv, E_ACT));
-    launch_qk_fwd(L.qkv, nqkv, M, T, nq, nkv, d, W.q_norm, W.k_norm, eps, m.rope_cos, m.rope_sin, L.qr,
-                  L.kr, c.dtype, x.s);
-    // S = q k^T / sqrt(d): row statistics, then P
-    const int tn = gemm_tile_n(m, T, 1);
-    Gemm g{};
-    g.A = head_op(L.qr, nq * d, M, nq, d, T, 1, false);
-    g.B = head_op(L.kr, nkv * d, M, nkv, d, T, grp, false);
-    g.sc = sch(Z, T, T, d);
-    g.sc.tri = 1;
-    g.epi = epi_mode(E_STATS, T);
-    g.epi.scale = sc;
-    g.epi.causal = 1;
-    g.epi.stats = L.st_a;
-    g.epi.n_ct = cdiv(T, tn);
-    g.out = out2(nullptr, T);
-    QK_TRY(run_gemm(m, g, x.s));
-    launch_stats_combine(L.st_a, cdiv(T, tn), tn, 1, Z * T, T, L.lse_a, nullptr, nullptr, nullptr, x.s);
-    g.epi.mode = E_SOFTMAX;
-    g.epi.lse = L.lse_a;
-    g.out = out2(L.P, T);
-    g.out.zrow = T;
-    QK_TRY(run_gemm(m, g, x.s));
-    // O = P V (keys up to the tile's last query)
-    Gemm pv{};
-    pv.A = opk(L.P, T, Z * T, T);
-    pv.A.zy = T;
-    pv.B = head_op(L.qkv, nqkv, M, nkv, d, T, grp, true, (nq + nkv) * d);
-    pv.sc = sch(Z, T, d, T, RED_PREFIX);
-    pv.sc.desc_m = 1;
-    pv.epi = epi_mode(E_ACT, T);
-    pv.out = out2(L.O, nq * d);
-    pv.out.zq = nq;
-    pv.out.zrow = T;
-    pv.out.zcol = d;
-    QK_TRY(run_gemm(m, pv, x.s));
-    QK_TRY(lin_fwd(x, L.O, nq * d, W.w_o, H, L.x_mid, E_F32, x_in));
-    launch_rmsnorm(L.x_mid, 1, 0, W.mlp_norm, H, eps, L.u2, c.dtype, M, x.s);
-    QK_TRY(lin_fwd(x, L.u2, H, W.w_gu, 2 * I, L.gu, E_ACT));
-    launch_swiglu(L.gu, L.h, c.dtype, M, I, x.s);
-    if (x_out) QK_TRY(lin_fwd(x, L.h, I, W.w_d, H, x_out, E_F32, L.x_mid));
-    return QK_OK;
+    const int nqkv = (nq + 2 * nkv) * d, T = x.T, M = x.M;
+    const float eps = (float)c.rms_eps;
+    launch_rmsnorm(x_in, 1, 0, W.attn_norm, H, eps, L.u1.at(l), c.dtype, M, x.s);
+    QK_TRY(lin_fwd(x, L.u1.at(l), H, W.w_qkv, nqkv, L.qkv.at(l), E_ACT));
+    launch_qk_fwd(L.qkv.at(l), nqkv, M, T, nq, nkv, d, W.q_norm, W.k_norm, eps, m.rope_cos, m.rope_sin,
+                  L.qr.at(l), L.kvh.at(l), c.dtype, x.s);
+    QK_TRY(attn_fwd(x, l));
+    float* x_mid = (float*)L.x_mid.at(l);
+    QK_TRY(lin_fwd(x, L.O.at(l), nq * d, W.w_o, H, x_mid, E_F32, x_in));
+    launch_rmsnorm(x_mid, 1, 0, W.mlp_norm, H, eps, L.u2.at(l), c.dtype, M, x.s);
+    QK_TRY(lin_fwd(x, L.u2.at(l), H, W.w_gu, 2 * I, L.gu.at(l), E_ACT));
+    launch_swiglu(L.gu.at(l), L.h.at(l), c.dtype, M, I, x.s);
+    return lin_fwd(x, L.h.at(l), I, W.w_d, H, x_out, E_F32, x_mid);
 }
 
 // ------------------------------------------------------------------ layer backward
@@ -291,45 +336,53 @@ int layer_bwd(const Ctx& x, int l, float* const* G, bool acc) {
     const BwdLayout& L = x.L;
     const int H = c.hidden, d = c.head_dim, nq = c.n_q_heads, nkv = c.n_kv_heads, I = c.intermediate;
     const int nqkv = (nq + 2 * nkv) * d, T = x.T, M = x.M, Z = x.B * nq, Zk = x.B * nkv, grp = nq / nkv;
-    const float eps = (float)c.rms_eps, sc = 1.f / sqrtf((float)d);
+    const float eps = (float)c.rms_eps;
     const float* x_in = L.xs + (size_t)l * M * H;
     const int nb = rms_part_rows(M);
-    QK_TRY(layer_fwd(x, l, x_in, nullptr));
+    void* u1 = L.u1.at(l);
+    void* qkv = L.qkv.at(l);
+    void* qr = L.qr.at(l);
+    void* kvh = L.kvh.at(l);
+    void* O = L.O.at(l);
+    void* u2 = L.u2.at(l);
+    void* gu = L.gu.at(l);
     // ---- MLP: x_out = x_mid + W_d h, h = silu(W_g u2) * (W_u u2)
-    QK_TRY(lin_dw(x, L.dx_act, H, H, 0, 128, H, L.h, I, I, G[10], acc, M));
+    QK_TRY(lin_dw(x, L.dx_act, H, H, 0, 128, H, L.h.at(l), I, I, G[10], acc, M));
     QK_TRY(lin_dx(x, L.dx_act, H, W.w_d, H, I, L.dh, E_F32, M));
-    launch_swiglu_bwd(L.dh, L.gu, M, I, L.dgu, c.dtype, x.s);
-    QK_TRY(lin_dw(x, L.dgu, 2 * I, 2 * I, 0, 256, I, L.u2, H, H, G[8], acc, M));
-    QK_TRY(lin_dw(x, L.dgu, 2 * I, 2 * I, 128, 256, I, L.u2, H, H, G[9], acc, M));
+    launch_swiglu_bwd(L.dh, gu, M, I, L.dgu, c.dtype, x.s);
+    QK_TRY(lin_dw(x, L.dgu, 2 * I, 2 * I, 0, 256, I, u2, H, H, G[8], acc, M));
+    QK_TRY(lin_dw(x, L.dgu, 2 * I, 2 * I, 128, 256, I, u2, H, H, G[9], acc, M));
     QK_TRY(lin_dx(x, L.dgu, 2 * I, W.w_gu, 2 * I, H, L.du, E_F32, M));
-    launch_rms_bwd(L.x_mid, W.mlp_norm, L.du, M, H, eps, 0, L.dx, L.dx_act, L.part, c.dtype, x.s);
+    launch_rms_bwd((const float*)L.x_mid.at(l), W.mlp_norm, L.du, M, H, eps, 0, L.dx, L.dx_act, L.part,
+                   c.dtype, x.s);
     launch_gain_reduce(L.part, nb, H, H, G[7], acc, x.s);
     // ---- attention output: x_mid = x_in + W_o o
-    QK_TRY(lin_dw(x, L.dx_act, H, H, 0, 128, H, L.O, nq * d, nq * d, G[6], acc, M));
+    QK_TRY(lin_dw(x, L.dx_act, H, H, 0, 128, H, O, nq * d, nq * d, G[6], acc, M));
     QK_TRY(lin_dx(x, L.dx_act, H, W.w_o, H, nq * d, L.dO, E_ACT, M));
-    launch_attn_d(L.dO, L.O, M, T, nq, d, L.Dv, c.dtype, x.s);
-    // dS = P (dO V^T - D) / sqrt(d), causal tiles only
+    launch_attn_d(L.dO, O, M, T, nq, d, L.Dv, c.dtype, x.s);
+    // P again from the stored log-sum-exp, then dS = P (dO V^T - D) / sqrt(d)
+    QK_TRY(probs(x, l));
     Gemm g{};
-    g.A = head_op(L.dO, nq * d, M, nq, d, T, 1, false);
-    g.B = head_op(L.qkv, nqkv, M, nkv, d, T, grp, false, (nq + nkv) * d);
+    g.A = head_op(L.dO, nq * d, M, nq, d, T, false);
+    g.B = kv_op(kvh, M, nkv, d, T, grp, false, true);
     g.sc = sch(Z, T, T, d);
     g.sc.tri = 1;
     g.epi = epi_mode(E_DS, T);
-    g.epi.scale = sc;
+    g.epi.scale = 1.f / sqrtf((float)d);
     g.epi.P = L.P;
     g.epi.D = L.Dv;
-    g.out = out2(L.dS, T);
+    g.out = out2(L.dS, T, Z * T, T);
     g.out.zrow = T;
     QK_TRY(run_gemm(m, g, x.s));
     // dq_rot = dS k (keys up to the tile's last query)
     Gemm gq{};
     gq.A = opk(L.dS, T, Z * T, T);
     gq.A.zy = T;
-    gq.B = head_op(L.kr, nkv * d, M, nkv, d, T, grp, true);
+    gq.B = kv_op(kvh, M, nkv, d, T, grp, true, false);
     gq.sc = sch(Z, T, d, T, RED_PREFIX);
     gq.sc.desc_m = 1;
     gq.epi = epi_mode(E_F32, T);
-    gq.out = out2(L.dqr, nq * d);
+    gq.out = out2(L.dqr, nq * d, M, nq * d);
     gq.out.zq = nq;
     gq.out.zrow = T;
     gq.out.zcol = d;
@@ -340,7 +393,7 @@ int layer_bwd(const Ctx& x, int l, float* const* G, bool acc) {
     gk.A.zy = grp * T;
     gk.A.kwrap = T;
     gk.A.kwy = T;
-    gk.B = opm(L.qr, nq * d, M, nq * d);
+    gk.B = opm(qr, nq * d, M, nq * d);
     gk.B.zq = nkv;
     gk.B.zx = grp * d;
     gk.B.zy = T;
@@ -349,7 +402,7 @@ int layer_bwd(const Ctx& x, int l, float* const* G, bool acc) {
     gk.sc = sch(Zk, T, d, grp * T, RED_SUFFIX);
     gk.sc.seg = T;
     gk.epi = epi_mode(E_F32, T);
-    gk.out = out2(L.dkr, nkv * d);
+    gk.out = out2(L.dkr, nkv * d, M, nkv * d);
     gk.out.zq = nkv;
     gk.out.zrow = T;
     gk.out.zcol = d;
@@ -358,19 +411,19 @@ int layer_bwd(const Ctx& x, int l, float* const* G, bool acc) {
     gv.A.ptr = L.P;
     gv.B.ptr = L.dO;
     gv.epi = epi_mode(E_ACT, T);
-    gv.out = out2(x.act(L.dqkv, (size_t)(nq + nkv) * d), nqkv);
+    gv.out = out2(x.act(L.dqkv, (size_t)(nq + nkv) * d), nqkv, M, nkv * d);
     gv.out.zq = nkv;
     gv.out.zrow = T;
     gv.out.zcol = d;
     QK_TRY(run_gemm(m, gv, x.s));
     // ---- QK-norm + RoPE, then the projections
-    launch_qk_bwd(L.dqr, L.dkr, L.qkv, nqkv, M, T, nq, nkv, d, W.q_norm, W.k_norm, eps, m.rope_cos,
+    launch_qk_bwd(L.dqr, L.dkr, qkv, nqkv, M, T, nq, nkv, d, W.q_norm, W.k_norm, eps, m.rope_cos,
                   m.rope_sin, L.dqkv, L.part, c.dtype, x.s);
     launch_gain_reduce(L.part, nb, d, 2 * d, G[4], acc, x.s);
     launch_gain_reduce(L.part + d, nb, d, 2 * d, G[5], acc, x.s);
-    QK_TRY(lin_dw(x, L.dqkv, nqkv, nqkv, 0, 128, nq * d, L.u1, H, H, G[1], acc, M));
-    QK_TRY(lin_dw(x, L.dqkv, nqkv, nqkv, nq * d, 128, nkv * d, L.u1, H, H, G[2], acc, M));
-    QK_TRY(lin_dw(x, L.dqkv, nqkv, nqkv, (nq + nkv) * d, 128, nkv * d, L.u1, H, H, G[3], acc, M));
+    QK_TRY(lin_dw(x, L.dqkv, nqkv, nqkv, 0, 128, nq * d, u1, H, H, G[1], acc, M));
+    QK_TRY(lin_dw(x, L.dqkv, nqkv, nqkv, nq * d, 128, nkv * d, u1, H, H, G[2], acc, M));
+    QK_TRY(lin_dw(x, L.dqkv, nqkv, nqkv, (nq + nkv) * d, 128, nkv * d, u1, H, H, G[3], acc, M));
     QK_TRY(lin_dx(x, L.dqkv, nqkv, W.w_qkv, nqkv, H, L.du, E_F32, M));
     launch_rms_bwd(x_in, W.attn_norm, L.du, M, H, eps, 0, L.dx, L.dx_act, L.part, c.dtype, x.s);
     launch_gain_reduce(L.part, nb, H, H, G[0], acc, x.s);
@@ -406,13 +459,13 @@ int backward_impl(Model& m, const int32_t* tokens, int B, int T, const float* co
         g.epi.zt = L.zt;
         g.epi.stats = L.st_h;
         g.epi.n_ct = nct;
-        g.out = out2(nullptr, V);
+        g.out = out2(nullptr, V, rows, V);
         QK_TRY(run_gemm(m, g, s));
         launch_stats_combine(L.st_h, nct, tn, 0, rows, rows, L.lse_h, L.w + r0, L.zt, L.loss_rows + r0, s);
         g.epi.mode = E_SOFTMAX;
         g.epi.lse = L.lse_h;
         g.epi.w = L.w + r0;
-        g.out = out2(L.dz, V);
+        g.out = out2(L.dz, V, rows, V);
         QK_TRY(run_gemm(m, g, s));
         QK_TRY(lin_dw(x, L.dz, V, V, 0, 128, V, hn, H, H, g_lm, acc || r0 > 0, rows));
         QK_TRY(lin_dx(x, L.dz, V, m.lm_head, V, H, L.du + (size_t)r0 * H, E_F32, rows));

@@ -368,10 +368,11 @@ void launch_attention(Model& m, const void* q, int q_ld, const void* k_cache, co
 // query rows at positions start_b .. start_b+T-1, start_b = start_dev[b] when given,
 // else start; head_dim 128.
 bool attn_prefill_supported(int d, int nq, int nkv);
+// lse (may be null): [B, nq, T] natural-log log-sum-exp of each row's scaled scores.
 int launch_attn_prefill(const bf16* q, int q_ld, const void* k_layer, int nq, int nkv,
                         int max_batch, int max_seq, int B, int T, int start,
                         const int32_t* start_dev, bf16* o, int num_sms, uint32_t* status,
-                        cudaStream_t s);
+                        cudaStream_t s, float* lse = nullptr);
 // Split tensor-core decode attention (k_attn_decode.cu); head_dim 128, G <= 8.
 void attn_decode_split(int B, int nkv, int max_seq, int num_sms, int* chunk, int* n_split);
 size_t attn_decode_scratch_bytes(int B, int nq, int nkv, int max_seq, int num_sms);
