@@ -52,6 +52,9 @@ enum Mode : int {
                     // and the target column's t (no matrix is stored)
     E_SOFTMAX = 3,  // (exp(scale * acc - lse_row) - [n == tgt_row]) * w_row; masked entries 0
     E_DS = 4,       // P * (acc - D_row) * scale, P read from a buffer laid out like C
+    E_SWIGLU_BWD = 5,  // acc = dh[m, n] of h = silu(g) u: with (g, u) read from gu (the packed
+                       // [M, 2 I] gate / up layout, row stride ldc), writes dg and du into C
+                       // (laid out like gu) at the gate and up columns of n
 };
 
 // Row vectors (lse, w, tgt, zt, D, stats) are indexed r = z * rows_per_z + m.
@@ -66,7 +69,7 @@ struct Epi {
     float* zt;         // E_STATS: t at the target column
     float2* stats;     // E_STATS: [r][n_ct]
     int n_ct;
-    const void* P;     // E_DS
+    const void* P;     // E_DS; E_SWIGLU_BWD: gu
     const float* D;    // E_DS
 };
 
@@ -94,6 +97,8 @@ __host__ __device__ __forceinline__ long long tiles_per_z(const Sched& s, int BM
     return t;
 }
 
+constexpr int kGroupM = 16;
+
 // Tile t of the launch -> (z, m tile, n tile).
 __device__ __forceinline__ void tile_at(const Sched& s, int BM, int BN, long long per, long long t,
                                         int& z, int& mt, int& nt) {
@@ -107,8 +112,15 @@ __device__ __forceinline__ void tile_at(const Sched& s, int BM, int BN, long lon
         mt = i;
         nt = (int)(r - (long long)i * (i + 1) / 2);
     } else {
-        mt = (int)(r / nn);
-        nt = (int)(r % nn);
+        // groups of kGroupM m tiles: within a group the m tile runs fastest, so a wave of
+        // concurrent tiles touches a few n tiles of B and at most kGroupM m tiles of A
+        // (both L2-resident) instead of streaming one operand from DRAM each wave
+        const long long gsz = (long long)kGroupM * nn;
+        const int g = (int)(r / gsz);
+        const long long loc = r - (long long)g * gsz;
+        const int gm = nm - g * kGroupM < kGroupM ? nm - g * kGroupM : kGroupM;
+        mt = g * kGroupM + (int)(loc % gm);
+        nt = (int)(loc / gm);
         if (s.desc_m) mt = nm - 1 - mt;
     }
 }
@@ -195,12 +207,14 @@ __device__ __forceinline__ void stat_merge(RowStat& a, float m2, float s2) {
 
 // Epilogue values of nv <= 16 consecutive outputs (z, m, n .. n + nv - 1) from the
 // accumulators v: E_STATS updates st and returns false (nothing to store); the other
-// modes fill y and return true.  VEC: nv == 16 and every address 16-byte aligned.
-template <typename act_t, bool VEC>
+// modes fill y (E_SWIGLU_BWD: y and y2, for the gate and up columns) and return true.
+// VEC: nv == 16 and every address 16-byte aligned.
+template <typename act_t, bool VEC, int MODE>
 __device__ __forceinline__ bool epi_values(const Epi& e, const Out& o, int z, int m, int n, int nv,
-                                           const float (&v)[16], RowStat& st, float (&y)[16]) {
+                                           const float (&v)[16], RowStat& st, float (&y)[16],
+                                           float (&y2)[16]) {
     const int r = z * e.rows_per_z + m;
-    if (e.mode == E_STATS) {
+    if constexpr (MODE == E_STATS) {
         float t[16];
         float cmax = -INFINITY;
         const int tg = e.tgt ? e.tgt[r] : -1;
@@ -221,10 +235,10 @@ __device__ __forceinline__ bool epi_values(const Epi& e, const Out& o, int z, in
         return false;
     }
     const size_t off = out_offset(o, z, m, n);
-    if (e.mode == E_F32 || e.mode == E_ACT) {
+    if constexpr (MODE == E_F32 || MODE == E_ACT) {
 #pragma unroll
         for (int j = 0; j < 16; ++j) y[j] = v[j];
-        if (e.mode == E_F32 && o.addend) {
+        if (MODE == E_F32 && o.addend) {
             const float* a = o.addend + off;
             if constexpr (VEC) {
 #pragma unroll
@@ -236,7 +250,7 @@ __device__ __forceinline__ bool epi_values(const Epi& e, const Out& o, int z, in
                 for (int j = 0; j < nv; ++j) y[j] += a[j];
             }
         }
-    } else if (e.mode == E_SOFTMAX) {
+    } else if constexpr (MODE == E_SOFTMAX) {
         // e^(scale acc - lse) = 2^(acc scale log2 e - lse log2 e)
         const float l2 = e.lse[r] * kLog2e, c = e.scale * kLog2e;
         const float w = e.w ? e.w[r] : 1.f;
@@ -246,6 +260,38 @@ __device__ __forceinline__ bool epi_values(const Epi& e, const Out& o, int z, in
             const bool masked = e.causal && n + j > m;
             const float p = masked ? 0.f : exp2f_fast(fmaf(v[j], c, -l2));
             y[j] = (p - (n + j == tg ? 1.f : 0.f)) * w;
+        }
+    } else if constexpr (MODE == E_SWIGLU_BWD) {
+        // gate of column n at packed column (n / 128) 256 + n % 128, up 128 further;
+        // y = dg, y2 = du
+        const size_t go = (size_t)m * o.ldc + (size_t)(n >> 7) * 256 + (n & 127);  // one batch entry
+        const act_t* G = (const act_t*)e.P + go;
+        float gv[16], uv[16];
+        if constexpr (VEC && sizeof(act_t) == 2) {
+            const uint4 q0 = *(const uint4*)G, q1 = *(const uint4*)(G + 8);
+            const uint4 u0 = *(const uint4*)(G + 128), u1 = *(const uint4*)(G + 136);
+            const bf16* a0 = (const bf16*)&q0;
+            const bf16* a1 = (const bf16*)&q1;
+            const bf16* b0 = (const bf16*)&u0;
+            const bf16* b1 = (const bf16*)&u1;
+#pragma unroll
+            for (int j = 0; j < 8; ++j) {
+                gv[j] = __bfloat162float(a0[j]), gv[j + 8] = __bfloat162float(a1[j]);
+                uv[j] = __bfloat162float(b0[j]), uv[j + 8] = __bfloat162float(b1[j]);
+            }
+        } else {
+#pragma unroll
+            for (int j = 0; j < 16; ++j) {
+                gv[j] = j < nv ? ld_act(G + j) : 0.f;
+                uv[j] = j < nv ? ld_act(G + 128 + j) : 0.f;
+            }
+        }
+#pragma unroll
+        // SwiGLU backward (h = silu(g) u, s = sigmoid(g)): dg = dh u s (1 + g (1 - s)), du = dh g s
+        for (int j = 0; j < 16; ++j) {
+            const float sg = 1.f / (1.f + __expf(-gv[j]));
+            y[j] = v[j] * uv[j] * sg * (1.f + gv[j] * (1.f - sg));
+            y2[j] = v[j] * gv[j] * sg;
         }
     } else {  // E_DS
         const float d = e.D[r];
@@ -268,18 +314,36 @@ __device__ __forceinline__ bool epi_values(const Epi& e, const Out& o, int z, in
 }
 
 // The epilogue of nv <= 16 consecutive outputs with plain stores (CUDA-core path).
-template <typename act_t>
-__device__ __forceinline__ void epi16(const Epi& e, const Out& o, int z, int m, int n, int nv,
-                                      const float (&v)[16], RowStat& st) {
-    float y[16];
-    if (!epi_values<act_t, false>(e, o, z, m, n, nv, v, st, y)) return;
+template <typename act_t, int MODE>
+__device__ __forceinline__ void epi16_mode(const Epi& e, const Out& o, int z, int m, int n, int nv,
+                                           const float (&v)[16], RowStat& st) {
+    float y[16], y2[16];
+    if (!epi_values<act_t, false, MODE>(e, o, z, m, n, nv, v, st, y, y2)) return;
+    if constexpr (MODE == E_SWIGLU_BWD) {
+        act_t* c = (act_t*)o.C + (size_t)m * o.ldc + (size_t)(n >> 7) * 256 + (n & 127);
+        for (int j = 0; j < nv; ++j) st_act(c + j, y[j]), st_act(c + 128 + j, y2[j]);
+        return;
+    }
     const size_t off = out_offset(o, z, m, n);
-    if (e.mode == E_F32) {
+    if constexpr (MODE == E_F32) {
         float* c = (float*)o.C + off;
         for (int j = 0; j < nv; ++j) c[j] = y[j];
     } else {
         act_t* c = (act_t*)o.C + off;
         for (int j = 0; j < nv; ++j) st_act(c + j, y[j]);
+    }
+}
+
+template <typename act_t>
+__device__ __forceinline__ void epi16(const Epi& e, const Out& o, int z, int m, int n, int nv,
+                                      const float (&v)[16], RowStat& st) {
+    switch (e.mode) {
+        case E_F32: epi16_mode<act_t, E_F32>(e, o, z, m, n, nv, v, st); break;
+        case E_ACT: epi16_mode<act_t, E_ACT>(e, o, z, m, n, nv, v, st); break;
+        case E_STATS: epi16_mode<act_t, E_STATS>(e, o, z, m, n, nv, v, st); break;
+        case E_SOFTMAX: epi16_mode<act_t, E_SOFTMAX>(e, o, z, m, n, nv, v, st); break;
+        case E_DS: epi16_mode<act_t, E_DS>(e, o, z, m, n, nv, v, st); break;
+        default: epi16_mode<act_t, E_SWIGLU_BWD>(e, o, z, m, n, nv, v, st); break;
     }
 }
 
@@ -325,7 +389,6 @@ void launch_qk_bwd(const float* dqr, const float* dkr, const void* qkv, int ld, 
                    const float* rs, void* dqkv, float* part, int dtype, cudaStream_t s);
 void launch_attn_d(const void* dO, const void* O, int M, int Tlen, int nq, int d, float* Dv, int dtype,
                    cudaStream_t s);
-void launch_swiglu_bwd(const float* dh, const void* gu, int M, int I, void* dgu, int dtype, cudaStream_t s);
 void launch_embed_bwd(const int32_t* tokens, const float* dx, int M, int H, int V, float* dE, cudaStream_t s);
 void launch_sum(const float* v, int n, float* out, cudaStream_t s);
 

@@ -1,8 +1,8 @@
 // Row-wise and elementwise kernels of the backward pass (gradient of the
 // token-weighted log-likelihood, Eq. sft / Eq. ppo): per-row targets and weights,
 // the per-head QK-RMSNorm + RoPE forward that keeps the raw projections, the
-// softmax-statistics combine, RMSNorm / QK-norm / RoPE / SwiGLU / embedding
-// backward, D = rowsum(dO * O) of the attention backward, and the deterministic
+// softmax-statistics combine, RMSNorm / QK-norm / RoPE / embedding backward,
+// D = rowsum(dO * O) of the attention backward, and the deterministic
 // reductions of gain gradients and of the loss.  fp32 arithmetic throughout;
 // activations are read and written in the model dtype (act_t).
 //
@@ -11,7 +11,6 @@
 //     dx = r (dy g) - (r^3 / n) x sum(dy g x),   dg = sum over rows of dy x r
 //   RoPE (rotation of the pair (a, b) = (x_j, x_{j + d/2}) by angle p w_j):
 //     (da, db) = (dy_a cos + dy_b sin, -dy_a sin + dy_b cos)
-//   SwiGLU h = silu(g) u, s = sigmoid(g):  dg = dh u s (1 + g (1 - s)),  du = dh g s
 //   embedding x_0 = E[token]:  dE[token] += dx_0
 #include <math.h>
 
@@ -293,26 +292,6 @@ __global__ void attn_d_kernel(const T* __restrict__ dO, const T* __restrict__ O,
     if (lane == 0) Dv[((size_t)(r / Tlen) * nq + h) * Tlen + r % Tlen] = s;
 }
 
-// SwiGLU backward: gu / dgu [M, 2 I] in the packed order (blocks of 128 gate columns,
-// then the matching 128 up columns); dh fp32 [M, I].
-template <typename T>
-__global__ void swiglu_bwd_kernel(const float* __restrict__ dh, const T* __restrict__ gu, int M, int I,
-                                  T* __restrict__ dgu) {
-    pdl_wait();
-    const size_t n = (size_t)M * I;
-    for (size_t e = blockIdx.x * (size_t)blockDim.x + threadIdx.x; e < n;
-         e += (size_t)gridDim.x * blockDim.x) {
-        const size_t m = e / I;
-        const int j = (int)(e % I);
-        const size_t o = m * 2 * I + (size_t)(j >> 7) * 256 + (j & 127);
-        const float g = ld_act(gu + o), u = ld_act(gu + o + 128);
-        const float s = 1.f / (1.f + expf(-g));
-        const float d = dh[e];
-        st_act(dgu + o, d * u * s * (1.f + g * (1.f - s)));
-        st_act(dgu + o + 128, d * g * s);
-    }
-}
-
 // dE[token[r]] += dx[r] (fp32 atomics: rows that share a token add in any order).
 __global__ void embed_bwd_kernel(const int32_t* __restrict__ tokens, const float* __restrict__ dx, int H,
                                  int V, float* __restrict__ dE) {
@@ -413,17 +392,6 @@ void launch_attn_d(const void* dO, const void* O, int M, int Tlen, int nq, int d
     launch_act(dtype, [&](auto* tp) {
         using A = std::remove_pointer_t<decltype(tp)>;
         launch_k(attn_d_kernel<A>, grid, dim3(256), 0, s, (const A*)dO, (const A*)O, M, Tlen, nq, d, Dv);
-    });
-    note_launch();
-}
-
-void launch_swiglu_bwd(const float* dh, const void* gu, int M, int I, void* dgu, int dtype, cudaStream_t s) {
-    const size_t n = (size_t)M * I;
-    int blocks = (int)((n + 255) / 256);
-    if (blocks > 65535) blocks = 65535;
-    launch_act(dtype, [&](auto* tp) {
-        using A = std::remove_pointer_t<decltype(tp)>;
-        launch_k(swiglu_bwd_kernel<A>, dim3(blocks), dim3(256), 0, s, dh, (const A*)gu, M, I, (A*)dgu);
     });
     note_launch();
 }

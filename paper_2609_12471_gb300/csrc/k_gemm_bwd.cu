@@ -103,7 +103,7 @@ struct TcCfg {
     static_assert(TMEM_COLS <= 512, "accumulators exceed TMEM");
 };
 
-template <int BN, bool AMN, bool BMN>
+template <int BN, bool AMN, bool BMN, int MODE>
 __global__ void __launch_bounds__(kThreads, 1)
     gemm_bwd_tc_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant__ CUtensorMap mapB,
                        const __grid_constant__ CUtensorMap mapC, const __grid_constant__ Gemm g,
@@ -276,7 +276,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         // alternating halves) and out with one TMA store.
         const int q = warp & 3, half = (warp - 2) >> 2;
         constexpr int HC = BN / 2;
-        const bool f32 = g.epi.mode == E_F32;
+        constexpr bool f32 = MODE == E_F32;
         uint8_t* stg = sOut + (warp - 2) * (2 * 32 * 16 * 4);
         int acc = 0, blk = 0;
         uint32_t acc_phase = 0;
@@ -304,15 +304,42 @@ __global__ void __launch_bounds__(kThreads, 1)
                 for (int u = 0; u < 4; ++u) {
                     const int n = n0 + c4 + 16 * u;
                     if (n >= sc.N) break;
-                    float v[16], y[16];
+                    float v[16], y[16], y2[16];
 #pragma unroll
                     for (int j = 0; j < 16; ++j) v[j] = __uint_as_float(r[u][j]);
-                    const bool store = m < sc.M && epi_values<bf16, true>(g.epi, g.out, z, m, n, 16, v, st, y);
-                    if (g.epi.mode == E_STATS) continue;
+                    const bool store =
+                        m < sc.M && epi_values<bf16, true, MODE>(g.epi, g.out, z, m, n, 16, v, st, y, y2);
+                    if constexpr (MODE == E_STATS) continue;
                     uint8_t* buf = stg + (blk & 1) * (32 * 16 * 4);
+                    if constexpr (MODE == E_SWIGLU_BWD) {
+                        // dg and du blocks (bf16) side by side in the staging buffer, two stores
+                        if (lane == 0) tc::bulk_wait_read<0>();
+                        __syncwarp();
+                        uint4 w[4];
+                        bf16* b = (bf16*)w;
+#pragma unroll
+                        for (int j = 0; j < 16; ++j)
+                            b[j] = __float2bfloat16_rn(store ? y[j] : 0.f), b[16 + j] = __float2bfloat16_rn(store ? y2[j] : 0.f);
+                        uint4* d = (uint4*)(buf + lane * 32);
+                        d[0] = w[0];
+                        d[1] = w[1];
+                        uint4* d2 = (uint4*)(buf + 1024 + lane * 32);
+                        d2[0] = w[2];
+                        d2[1] = w[3];
+                        tc::fence_proxy_async_smem();
+                        __syncwarp();
+                        if (lane == 0) {
+                            const int gc = (n >> 7) * 256 + (n & 127);
+                            tc::tma_store_2d(&mapC, gc, orow, buf);
+                            tc::tma_store_2d(&mapC, gc + 128, orow, buf + 1024);
+                            tc::bulk_commit();
+                        }
+                        ++blk;
+                        continue;
+                    }
                     if (lane == 0) tc::bulk_wait_read<1>();  // the store issued from this half two blocks ago
                     __syncwarp();
-                    if (f32) {
+                    if constexpr (f32) {
                         float4* d = (float4*)(buf + lane * 64);
 #pragma unroll
                         for (int j = 0; j < 4; ++j)
@@ -337,7 +364,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 }
             }
             const int ct = nt * 2 + half;  // statistics column tile of HC columns
-            if (g.epi.mode == E_STATS && m < sc.M && ct < g.epi.n_ct)
+            if (MODE == E_STATS && m < sc.M && ct < g.epi.n_ct)
                 g.epi.stats[(size_t)(z * g.epi.rows_per_z + m) * g.epi.n_ct + ct] = make_float2(st.mx, st.sm);
             tc::fence_before_sync();
             __syncwarp();
@@ -419,12 +446,12 @@ bool make_out_map(CUtensorMap* map, const Out& o, bool f32) {
               CU_TENSOR_MAP_L2_PROMOTION_NONE, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
-template <int BN, bool AMN, bool BMN>
-int launch_tc(Model& m, const Gemm& g, cudaStream_t s) {
+template <int BN, bool AMN, bool BMN, int MODE>
+int launch_tc_mode(Model& m, const Gemm& g, cudaStream_t s) {
     using G = TcCfg<BN>;
     static bool attr_set = false;
     if (!attr_set) {
-        if (cudaFuncSetAttribute(gemm_bwd_tc_kernel<BN, AMN, BMN>,
+        if (cudaFuncSetAttribute(gemm_bwd_tc_kernel<BN, AMN, BMN, MODE>,
                                  cudaFuncAttributeMaxDynamicSharedMemorySize, G::SMEM) != cudaSuccess)
             return set_error(QK_ECUDA, "backward GEMM: shared-memory attribute");
         attr_set = true;
@@ -441,10 +468,31 @@ int launch_tc(Model& m, const Gemm& g, cudaStream_t s) {
     const long long per = tiles_per_z(g.sc, 128, BN);
     const long long total = per * g.sc.Z;
     const int grid = total < m.num_sms ? (int)total : m.num_sms;
-    launch_k(gemm_bwd_tc_kernel<BN, AMN, BMN>, dim3(grid), dim3(kThreads), G::SMEM, s, ma, mb, mc, g,
+    launch_k(gemm_bwd_tc_kernel<BN, AMN, BMN, MODE>, dim3(grid), dim3(kThreads), G::SMEM, s, ma, mb, mc, g,
              per, total, a3, b3, m.status);
     note_launch();
     return QK_OK;
+}
+
+// The epilogue modes each operand layout is instantiated for (the ones the backward uses).
+template <int BN, bool AMN, bool BMN>
+int launch_tc(Model& m, const Gemm& g, cudaStream_t s) {
+    const int mode = g.epi.mode;
+    if (!AMN && !BMN) {
+        if (mode == E_F32) return launch_tc_mode<BN, AMN, BMN, E_F32>(m, g, s);
+        if (mode == E_ACT) return launch_tc_mode<BN, AMN, BMN, E_ACT>(m, g, s);
+        if (mode == E_STATS) return launch_tc_mode<BN, AMN, BMN, E_STATS>(m, g, s);
+        if (mode == E_SOFTMAX) return launch_tc_mode<BN, AMN, BMN, E_SOFTMAX>(m, g, s);
+        if (mode == E_DS) return launch_tc_mode<BN, AMN, BMN, E_DS>(m, g, s);
+    } else if (!AMN && BMN) {
+        if (mode == E_F32) return launch_tc_mode<BN, AMN, BMN, E_F32>(m, g, s);
+        if (mode == E_ACT) return launch_tc_mode<BN, AMN, BMN, E_ACT>(m, g, s);
+        if (mode == E_SWIGLU_BWD) return launch_tc_mode<BN, AMN, BMN, E_SWIGLU_BWD>(m, g, s);
+    } else {
+        if (mode == E_F32) return launch_tc_mode<BN, AMN, BMN, E_F32>(m, g, s);
+        if (mode == E_ACT) return launch_tc_mode<BN, AMN, BMN, E_ACT>(m, g, s);
+    }
+    return set_error(QK_EINVAL, "backward GEMM: epilogue %d is not instantiated for this operand layout", mode);
 }
 
 bool aligned16(const void* p) { return ((uintptr_t)p & 15) == 0; }

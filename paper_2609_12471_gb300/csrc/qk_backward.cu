@@ -61,7 +61,6 @@ struct BwdLayout {
     void* dz;
     float2* st_a;
     void* P;
-    float* dh;
     void* dgu;
     float* du;
     void* dO;
@@ -117,7 +116,6 @@ int bwd_layout(const Model& m, int B, int T, char* base, BwdLayout* L) {
     L->dz = take(Mc * V * es);
     L->st_a = (float2*)take(Z * T * nct_a * 8);
     L->P = take(Z * T * T * es);
-    L->dh = (float*)take(M * I * 4);
     L->dgu = take(M * 2 * I * es);
     L->du = (float*)take(M * H * 4);
     L->dO = take(M * nq * d * es);
@@ -348,8 +346,16 @@ int layer_bwd(const Ctx& x, int l, float* const* G, bool acc) {
     void* gu = L.gu.at(l);
     // ---- MLP: x_out = x_mid + W_d h, h = silu(W_g u2) * (W_u u2)
     QK_TRY(lin_dw(x, L.dx_act, H, H, 0, 128, H, L.h.at(l), I, I, G[10], acc, M));
-    QK_TRY(lin_dx(x, L.dx_act, H, W.w_d, H, I, L.dh, E_F32, M));
-    launch_swiglu_bwd(L.dh, gu, M, I, L.dgu, c.dtype, x.s);
+    {  // dh = dx W_d with the SwiGLU backward in the epilogue: dgu = (dg, du) from gu
+        Gemm g{};
+        g.A = opk(L.dx_act, H, M, H);
+        g.B = opm(W.w_d, I, H, I);
+        g.out = out2(L.dgu, 2 * I, M, 2 * I);
+        g.epi = epi_mode(E_SWIGLU_BWD);
+        g.epi.P = gu;
+        g.sc = sch(1, M, I, H);
+        QK_TRY(run_gemm(m, g, x.s));
+    }
     QK_TRY(lin_dw(x, L.dgu, 2 * I, 2 * I, 0, 256, I, u2, H, H, G[8], acc, M));
     QK_TRY(lin_dw(x, L.dgu, 2 * I, 2 * I, 128, 256, I, u2, H, H, G[9], acc, M));
     QK_TRY(lin_dx(x, L.dgu, 2 * I, W.w_gu, 2 * I, H, L.du, E_F32, M));
