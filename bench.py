@@ -318,6 +318,7 @@ def run_ours(args, world, rank, local):
     dec._ws.clear()
     torch.cuda.empty_cache()
     decode_configs = other_decode_configs(dec, dev, stream, rank)
+    backward = backward_config(dec, dev, stream, rank, world)
 
     if rank != 0:
         return
@@ -356,6 +357,7 @@ def run_ours(args, world, rank, local):
                                "peak_source": "measured (burst)" if peaks else "fallback"},
             "decode_hbm_fraction_of_8tbs": (step_bytes * N / 1e9) / ((ms_step - prefill_ms) / 1e3) / 8000.0,
             "decode_configs": decode_configs,
+            "backward": backward,
             "roofline": roofline, "clocks": clk, "gpu_launches": int(launches),
             "launches_before_timed": int(launches0),
             "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": int(seq.nbytes),
@@ -467,6 +469,74 @@ def other_decode_configs(dec, dev, stream, rank):
     if dec.check_status() != 0 or not torch.isfinite(lpb).all():
         raise RuntimeError("the batch-64 long-context decode produced invalid output")
     del kvb
+    dec._ws.clear()
+    torch.cuda.empty_cache()
+    return out
+
+
+# --------------------------------------------------------------------------- backward
+BWD_B, BWD_T = 2, 4096
+
+
+def backward_flops(B, T):
+    """Algorithmic FLOPs of one gradient of the token log-likelihood of the 36-layer model over
+    B x T tokens: 6 flops per (token, weight) for the linear layers and the lm_head (forward 2,
+    backward 4), and 3 x the causal attention forward (QK^T and PV over the T (T + 1) / 2
+    query-key pairs of each row and head; the backward is twice the forward).  The kernels
+    also run the attention probabilities and the lm_head logits a second time (not counted)."""
+    M = B * T
+    linear = 6 * M * (36 * 192937984 + 151936 * 4096)
+    attn = 36 * 3 * 2 * 2 * 128 * 32 * B * (T * (T + 1) // 2)
+    return linear + attn
+
+
+def backward_config(dec, dev, stream, rank, world):
+    """Backward pass (qk_backward_logprob, the gradient of Eq. sft; Eq. ppo through its
+    coefficients) of the 36-layer model over 2 x 4096 tokens, token-mean coefficients:
+    device-resident inputs, then end to end from pinned host buffers (tokens and
+    coefficients in, the loss out)."""
+    import torch
+    import synth
+    peaks = measured_peaks()
+    sustained = peaks["bf16_tflops_sustained"] if peaks and "bf16_tflops_sustained" in peaks else 1700.0
+    B_, T_ = BWD_B, BWD_T
+    tok_h = torch.tensor(synth.tokens((B_, T_), dec.cfg.vocab, stream=500 + rank), dtype=torch.int32)
+    coef_h = torch.full((B_, T_ - 1), 1.0 / (B_ * (T_ - 1)), dtype=torch.float32)
+    tok = tok_h.to(dev)
+    coef = coef_h.to(dev)
+    grads = dec.new_grads()
+    loss = torch.empty(1, dtype=torch.float32, device=dev)
+    f = lambda: dec.backward(tok, coef, grads, loss=loss)
+    f()
+    torch.cuda.synchronize(dev)
+    if dec.check_status() != 0 or not torch.isfinite(loss).all():
+        raise RuntimeError("the backward pass produced invalid output")
+    t = max_over_ranks(_event_time(f, 2, stream), world)
+    # end to end: pinned host tokens / coefficients in, loss out, every call
+    tok_p, coef_p = tok_h.pin_memory(), coef_h.pin_memory()
+    loss_h = torch.empty(1, dtype=torch.float32).pin_memory()
+    tok_d, coef_d = torch.empty_like(tok), torch.empty_like(coef)
+    torch.cuda.synchronize(dev)
+    t0 = time.perf_counter()
+    for _ in range(2):
+        tok_d.copy_(tok_p, non_blocking=True)
+        coef_d.copy_(coef_p, non_blocking=True)
+        dec.backward(tok_d, coef_d, grads, loss=loss)
+        loss_h.copy_(loss, non_blocking=True)
+        torch.cuda.synchronize(dev)
+    e2e = max_over_ranks((time.perf_counter() - t0) / 2, world)
+    fl = backward_flops(B_, T_)
+    out = {"workload": f"gradient of the token-mean log-likelihood, 36-layer Qwen3-8B-shaped bf16, "
+                       f"{B_} x {T_} tokens (weights, fp32 gradients and the kept activations resident)",
+           "tokens_per_s": world * B_ * T_ / t, "ms_per_call": t * 1e3,
+           "roofline": {"bound": "tensor", "flops_per_call": fl, "achieved": fl / t / 1e12,
+                        "peak": sustained, "unit": "TFLOP/s", "frac": fl / t / 1e12 / sustained,
+                        "peak_source": "measured (sustained)" if peaks else "fallback",
+                        "dominant_kernel": "gemm_bwd_tc_kernel<256, 1, 1, E_F32> (weight gradients dW = dY^T X)"},
+           "e2e": {"tokens_per_s": world * B_ * T_ / e2e, "h2d_bytes_per_call": int(tok_h.nbytes + coef_h.nbytes),
+                   "d2h_bytes_per_call": 4},
+           "loss": float(loss_h.item())}
+    del grads
     dec._ws.clear()
     torch.cuda.empty_cache()
     return out

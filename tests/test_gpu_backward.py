@@ -6,7 +6,8 @@ coefficients (qk_grpo_coef) against the fp64 oracle (oracle/backward.py, oracle/
   the tensor's largest entry, on ragged sequence lengths (37: one partial 64-tile;
   130: three tiles and a 2-row tail);
 * bf16 decoders (tcgen05 GEMMs with K- and MN-major operands): a two-layer model
-  and one layer at Qwen3-8B width (H 4096, 32/8 heads, I 12288; vocabulary 16384),
+  and one layer at Qwen3-8B width (H 4096, 32/8 heads, I 12288; vocabulary 16384) over
+  2 x 256 tokens (two causal tiles per row),
   per-tensor relative Frobenius error within the bf16 bound, and the loss;
 * the GRPO coefficients element by element, and the GRPO gradient end to end.
 """
@@ -130,7 +131,7 @@ def test_bf16_q8b_width_layer_gradients_match_oracle():
     s = synth.ModelShape("q8b_width", 1, 4096, 32, 8, 128, 12288, 16384, "bf16")
     W = synth.LazyWeights(s)
     dec, _ = decoder(s, W)
-    worst = _check_bf16(s, W, dec, 1, 128, 72)
+    worst = _check_bf16(s, W, dec, 2, 256, 72)
     dec.close()
     print("bf16 8B-width layer relative Frobenius errors:", {k: f"{v:.2e}" for k, v in worst.items()})
 
@@ -200,3 +201,25 @@ def test_grpo_gradient_end_to_end(tiny):
         g = g.cpu().numpy().astype(np.float64)
         scale = float(np.max(np.abs(ref[nm])))
         assert float(np.max(np.abs(g - ref[nm]))) <= 1e-3 * scale, nm
+
+
+def test_bf16_q8b_width_layer_4096_tokens_against_scoring():
+    """One 8B-width layer over 1 x 4096 tokens (32 causal tiles per row, dW reductions over
+    4096 tokens): the loss the backward forms equals the scoring path's mean -log p, the
+    gradients are finite, and the lm_head gradient's columns sum to ~0 over the vocabulary."""
+    import torch
+    s = synth.ModelShape("q8b_width", 1, 4096, 32, 8, 128, 12288, 16384, "bf16")
+    dec, _ = decoder(s, synth.LazyWeights(s, cache=False))
+    B, T = 1, 4096
+    tok = torch.tensor(synth.tokens((B, T), s.vocab, stream=73), dtype=torch.int32, device="cuda")
+    coef = torch.full((B, T - 1), 1.0 / (T - 1), device="cuda")
+    ref = float(-dec.score(tok).double().mean())
+    grads = dec.new_grads()
+    loss = float(dec.backward(tok, coef, grads).item())
+    torch.cuda.synchronize()
+    assert dec.check_status() == 0
+    assert loss == pytest.approx(ref, abs=2e-3)
+    assert all(bool(torch.isfinite(g).all()) for g in grads)
+    col = grads[-1].double().sum(0).abs().max().item()
+    assert col <= 1e-2 * grads[-1].double().abs().sum(0).max().item()
+    dec.close()

@@ -130,3 +130,45 @@ def test_long_trajectory_endpoint_b64_s8192(q8b):
     dec._ws.clear()
     gc.collect()
     torch.cuda.empty_cache()
+
+
+def test_backward_b2_t4096(q8b):
+    """Gradient of the token-mean log-likelihood over 2 x 4096 tokens (the benchmark's
+    backward workload).  (b) The loss the backward forms through its own forward (tcgen05
+    GEMMs + flash attention, tile log-sum-exp statistics) equals the mean -log p of the
+    scoring path (split head statistics) within the two-path bf16 bound; (a) properties of
+    the gradient that hold at any size: every entry finite; the lm_head gradient's columns
+    sum to ~0 over the vocabulary (each row's softmax minus its one-hot sums to zero); the
+    embedding rows of tokens that occur at no position < T - 1 are exactly zero, the others
+    are not; accumulate = 1 doubles it."""
+    import torch
+    s, W, dec = q8b
+    B, T = 2, 4096
+    tok = torch.tensor(synth.tokens((B, T), s.vocab, stream=500), dtype=torch.int32, device="cuda")
+    coef = torch.full((B, T - 1), 1.0 / (B * (T - 1)), device="cuda")
+    lp = dec.score(tok).double()
+    grads = dec.new_grads()
+    loss = float(dec.backward(tok, coef, grads).item())
+    torch.cuda.synchronize()
+    assert dec.check_status() == 0
+    ref = float(-lp.mean())
+    assert abs(loss - ref) <= TWO_PATH_MEAN, (loss, ref)
+    for i, g in enumerate(grads):
+        assert torch.isfinite(g).all(), i
+    g_lm = grads[-1]
+    col = g_lm.double().sum(0).abs().max().item()
+    assert col <= 1e-2 * g_lm.double().abs().sum(0).max().item(), col
+    # the last position of a row scores nothing and no later position sees it, so only the
+    # tokens at positions < T - 1 receive embedding gradient
+    present = torch.zeros(s.vocab, dtype=torch.bool, device="cuda")
+    present[tok[:, :-1].long().reshape(-1)] = True
+    assert (grads[0][~present] == 0).all()
+    assert grads[0][present].abs().sum(1).min().item() > 0
+    emb = grads[0][present].clone()
+    dec.backward(tok, coef, grads, accumulate=True)
+    torch.cuda.synchronize()
+    assert torch.allclose(grads[0][present], 2 * emb, rtol=1e-5, atol=1e-9)
+    del grads, emb
+    dec._ws.clear()
+    gc.collect()
+    torch.cuda.empty_cache()
