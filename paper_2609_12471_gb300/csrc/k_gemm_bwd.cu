@@ -92,23 +92,30 @@ constexpr int kThreads = 64 + 32 * kEpiWarps;
 constexpr int kBK = 64;
 constexpr int kBox = 64 * 128;  // one 64 x 64 bf16 box (8 KB)
 
-template <int BN>
+// BM x BN output tiles.  BM = 256 (two 128-row MMAs per k-step, one accumulator set
+// filling TMEM, three 64 KB stages) for the large full-reduction GEMMs: it halves the
+// shared-memory bytes per flop of A and lets the ring cover more load latency; BM = 128
+// keeps two accumulator sets so the epilogue of a tile overlaps the next main loop.
+template <int BN, int BM>
 struct TcCfg {
-    static constexpr int STAGES = BN == 256 ? 4 : 6;
-    static constexpr int A_BYTES = 128 * 128;
+    static constexpr int STAGES = BM == 256 ? 3 : (BN == 256 ? 4 : 6);
+    static constexpr int A_BYTES = BM * 128;
     static constexpr int B_BYTES = BN * 128;
-    static constexpr int TMEM_COLS = 2 * BN;
+    static constexpr int ACC = BM == 256 ? 1 : 2;       // accumulator sets
+    static constexpr int ACC_COLS = (BM / 128) * BN;    // TMEM columns of one set
+    static constexpr int TMEM_COLS = ACC * ACC_COLS;
     static constexpr int STAGE_OUT = kEpiWarps * 2 * 32 * 16 * 4;  // per epilogue warp: two 32 x 16 fp32 blocks
     static constexpr int SMEM = STAGES * (A_BYTES + B_BYTES) + STAGE_OUT + 1024 + 256;
     static_assert(TMEM_COLS <= 512, "accumulators exceed TMEM");
+    static_assert(SMEM <= 232448, "shared memory per CTA");
 };
 
-template <int BN, bool AMN, bool BMN, int MODE>
+template <int BN, int BM, bool AMN, bool BMN, int MODE>
 __global__ void __launch_bounds__(kThreads, 1)
     gemm_bwd_tc_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant__ CUtensorMap mapB,
                        const __grid_constant__ CUtensorMap mapC, const __grid_constant__ Gemm g,
                        long long per, long long total, int a3, int b3, uint32_t* __restrict__ status) {
-    using G = TcCfg<BN>;
+    using G = TcCfg<BN, BM>;
     constexpr int STAGES = G::STAGES;
     extern __shared__ uint8_t smem_raw[];
     uint8_t* smem = (uint8_t*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
@@ -131,7 +138,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             tc::mbar_init(&full[s], 1);
             tc::mbar_init(&empty[s], 1);
         }
-        for (int a = 0; a < 2; ++a) {
+        for (int a = 0; a < G::ACC; ++a) {
             tc::mbar_init(&tfull[a], 1);
             tc::mbar_init(&tempty[a], kEpiWarps);
         }
@@ -158,12 +165,12 @@ __global__ void __launch_bounds__(kThreads, 1)
             bool ok = true;
             for (long long t = blockIdx.x; ok && t < total; t += gridDim.x) {
                 int z, mt, nt;
-                tile_at(sc, 128, BN, per, t, z, mt, nt);
-                const int m0 = mt * 128, n0 = nt * BN;
-                const int nkb = kblocks(sc, 128, kBK, m0);
+                tile_at(sc, BM, BN, per, t, z, mt, nt);
+                const int m0 = mt * BM, n0 = nt * BN;
+                const int nkb = kblocks(sc, BM, kBK, m0);
                 for (int j = 0; j < nkb; ++j) {
                     int k0, kend;
-                    kblock_at(sc, 128, kBK, m0, j, k0, kend);
+                    kblock_at(sc, BM, kBK, m0, j, k0, kend);
                     if (!tc::mbar_wait(&empty[stage], phase ^ 1, abort_flag)) {
                         ok = false;
                         break;
@@ -172,20 +179,25 @@ __global__ void __launch_bounds__(kThreads, 1)
                     uint8_t* a_s = sA + stage * G::A_BYTES;
                     uint8_t* b_s = sB + stage * G::B_BYTES;
                     int x, y;
-                    if (AMN) {  // MN chunks of 64: one 3-D box (chunk index as the third axis) or one box each
-                        if (a3) {
-                            op_xy(g.A, z, m0, k0, x, y);
-                            tc::tma_load_3d(a_s, &mapA, 0, y, x >> 6, &full[stage]);
-                        } else {
 #pragma unroll
-                            for (int c = 0; c < 2; ++c) {
-                                op_xy(g.A, z, m0 + 64 * c, k0, x, y);
-                                tc::tma_load_2d(a_s + c * kBox, &mapA, x, y, &full[stage]);
+                    for (int h = 0; h < BM / 128; ++h) {  // 128-row blocks of A (16 KB each)
+                        uint8_t* ah = a_s + h * 16384;
+                        const int mh = m0 + 128 * h;
+                        if (AMN) {  // MN chunks of 64: one 3-D box (chunk index as the third axis) or one box each
+                            if (a3) {
+                                op_xy(g.A, z, mh, k0, x, y);
+                                tc::tma_load_3d(ah, &mapA, 0, y, x >> 6, &full[stage]);
+                            } else {
+#pragma unroll
+                                for (int c = 0; c < 2; ++c) {
+                                    op_xy(g.A, z, mh + 64 * c, k0, x, y);
+                                    tc::tma_load_2d(ah + c * kBox, &mapA, x, y, &full[stage]);
+                                }
                             }
+                        } else {
+                            op_xy(g.A, z, mh, k0, x, y);
+                            tc::tma_load_2d(ah, &mapA, x, y, &full[stage]);
                         }
-                    } else {
-                        op_xy(g.A, z, m0, k0, x, y);
-                        tc::tma_load_2d(a_s, &mapA, x, y, &full[stage]);
                     }
                     if (BMN) {
                         if (b3) {
@@ -227,14 +239,14 @@ __global__ void __launch_bounds__(kThreads, 1)
             bool ok = true, issued = false;
             for (long long t = blockIdx.x; ok && t < total; t += gridDim.x) {
                 int z, mt, nt;
-                tile_at(sc, 128, BN, per, t, z, mt, nt);
-                const int nkb = kblocks(sc, 128, kBK, mt * 128);
+                tile_at(sc, BM, BN, per, t, z, mt, nt);
+                const int nkb = kblocks(sc, BM, kBK, mt * BM);
                 if (!tc::mbar_wait(&tempty[acc], acc_phase ^ 1, abort_flag)) {
                     ok = false;
                     break;
                 }
                 tc::fence_after_sync();
-                const uint32_t d = tmem_base + (uint32_t)(acc * BN);
+                const uint32_t d = tmem_base + (uint32_t)(acc * G::ACC_COLS);
                 for (int j = 0; j < nkb; ++j) {
                     if (!tc::mbar_wait(&full[stage], phase, abort_flag)) {
                         ok = false;
@@ -245,11 +257,15 @@ __global__ void __launch_bounds__(kThreads, 1)
                     const uint32_t b0 = tc::smem_u32(sB + stage * G::B_BYTES);
 #pragma unroll
                     for (int k = 0; k < kBK / 16; ++k) {
-                        const uint64_t ad = AMN ? tc::sw128_desc_mn(a0 + k * 2048, kBox)
-                                                : tc::sw128_desc(a0 + k * 32);
                         const uint64_t bd = BMN ? tc::sw128_desc_mn(b0 + k * 2048, kBox)
                                                 : tc::sw128_desc(b0 + k * 32);
-                        tc::mma_bf16(d, ad, bd, idesc, (j || k) ? 1u : 0u);
+#pragma unroll
+                        for (int h = 0; h < BM / 128; ++h) {  // rows 128 h .. of the tile
+                            const uint32_t ah = a0 + h * 16384;
+                            const uint64_t ad = AMN ? tc::sw128_desc_mn(ah + k * 2048, kBox)
+                                                    : tc::sw128_desc(ah + k * 32);
+                            tc::mma_bf16(d + h * BN, ad, bd, idesc, (j || k) ? 1u : 0u);
+                        }
                     }
                     issued = true;
                     tc::mma_commit(&empty[stage]);
@@ -260,8 +276,10 @@ __global__ void __launch_bounds__(kThreads, 1)
                 }
                 if (!ok) break;
                 tc::mma_commit(&tfull[acc]);
-                acc ^= 1;
-                if (acc == 0) acc_phase ^= 1;
+                if (++acc == G::ACC) {
+                    acc = 0;
+                    acc_phase ^= 1;
+                }
             }
             if (!ok && issued) {
                 tc::mma_commit(drain);
@@ -274,26 +292,29 @@ __global__ void __launch_bounds__(kThreads, 1)
         // (w - 2) / 4 of the tile, four 16-column blocks per TMEM wait.  Each 32-row x
         // 16-column block of outputs goes through the warp's staging buffer (two
         // alternating halves) and out with one TMA store.
+        // BM = 256: half selects the tile's 128-row block and the warp takes every column.
         const int q = warp & 3, half = (warp - 2) >> 2;
-        constexpr int HC = BN / 2;
+        constexpr int HC = BM == 256 ? BN : BN / 2;  // columns per warp
+        const int c_lo = BM == 256 ? 0 : half * HC, r_lo = BM == 256 ? half * 128 : 0;
         constexpr bool f32 = MODE == E_F32;
         uint8_t* stg = sOut + (warp - 2) * (2 * 32 * 16 * 4);
         int acc = 0, blk = 0;
         uint32_t acc_phase = 0;
         for (long long t = blockIdx.x; t < total; t += gridDim.x) {
             int z, mt, nt;
-            tile_at(sc, 128, BN, per, t, z, mt, nt);
-            const int m0 = mt * 128, n0 = nt * BN;
+            tile_at(sc, BM, BN, per, t, z, mt, nt);
+            const int m0 = mt * BM + r_lo, n0 = nt * BN;
             bool ok = tc::mbar_wait(&tfull[acc], acc_phase, abort_flag);
             ok = __all_sync(0xffffffffu, ok);
             if (!ok) break;
             tc::fence_after_sync();
             const int m = m0 + q * 32 + lane;
-            const uint32_t tbase = tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(acc * BN);
+            const uint32_t tbase = tmem_base + ((uint32_t)(q * 32) << 16) +
+                                   (uint32_t)(acc * G::ACC_COLS + (BM == 256 ? half * BN : 0));
             const int orow = (z / g.out.zq) * g.out.zrow + m0 + q * 32;
             const int ocol = (z % g.out.zq) * g.out.zcol;
             RowStat st{-INFINITY, 0.f};
-            for (int c4 = half * HC; c4 < (half + 1) * HC; c4 += 64) {
+            for (int c4 = c_lo; c4 < c_lo + HC; c4 += 64) {
                 if (n0 + c4 >= sc.N) break;  // uniform over the warp
                 uint32_t r[4][16];
 #pragma unroll
@@ -363,14 +384,16 @@ __global__ void __launch_bounds__(kThreads, 1)
                     ++blk;
                 }
             }
-            const int ct = nt * 2 + half;  // statistics column tile of HC columns
+            const int ct = nt * 2 + half;  // statistics column tile of HC columns (BM = 128)
             if (MODE == E_STATS && m < sc.M && ct < g.epi.n_ct)
                 g.epi.stats[(size_t)(z * g.epi.rows_per_z + m) * g.epi.n_ct + ct] = make_float2(st.mx, st.sm);
             tc::fence_before_sync();
             __syncwarp();
             if (lane == 0) tc::mbar_arrive(&tempty[acc]);
-            acc ^= 1;
-            if (acc == 0) acc_phase ^= 1;
+            if (++acc == G::ACC) {
+                acc = 0;
+                acc_phase ^= 1;
+            }
         }
         if (lane == 0) tc::bulk_wait<0>();  // every store of this warp has completed
     }
@@ -446,13 +469,13 @@ bool make_out_map(CUtensorMap* map, const Out& o, bool f32) {
               CU_TENSOR_MAP_L2_PROMOTION_NONE, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
-template <int BN, bool AMN, bool BMN, int MODE>
-int launch_tc_mode(Model& m, const Gemm& g, cudaStream_t s) {
-    using G = TcCfg<BN>;
+template <int BN, int BM, bool AMN, bool BMN, int MODE>
+int launch_tc_cfg(Model& m, const Gemm& g, cudaStream_t s) {
+    using G = TcCfg<BN, BM>;
+    auto kern = gemm_bwd_tc_kernel<BN, BM, AMN, BMN, MODE>;
     static bool attr_set = false;
     if (!attr_set) {
-        if (cudaFuncSetAttribute(gemm_bwd_tc_kernel<BN, AMN, BMN, MODE>,
-                                 cudaFuncAttributeMaxDynamicSharedMemorySize, G::SMEM) != cudaSuccess)
+        if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, G::SMEM) != cudaSuccess)
             return set_error(QK_ECUDA, "backward GEMM: shared-memory attribute");
         attr_set = true;
     }
@@ -463,15 +486,27 @@ int launch_tc_mode(Model& m, const Gemm& g, cudaStream_t s) {
     if ((!a3 && !make_op_map(&ma, g.A, AMN ? 64 : 128)) || (!b3 && !make_op_map(&mb, g.B, BMN ? 64 : BN)))
         return set_error(QK_ECUDA, "backward GEMM: tensor map encoding failed");
     memset(&mc, 0, sizeof(mc));
-    if (g.epi.mode != E_STATS && !make_out_map(&mc, g.out, g.epi.mode == E_F32))
+    if (MODE != E_STATS && !make_out_map(&mc, g.out, MODE == E_F32))
         return set_error(QK_ECUDA, "backward GEMM: output tensor map encoding failed");
-    const long long per = tiles_per_z(g.sc, 128, BN);
+    const long long per = tiles_per_z(g.sc, BM, BN);
     const long long total = per * g.sc.Z;
     const int grid = total < m.num_sms ? (int)total : m.num_sms;
-    launch_k(gemm_bwd_tc_kernel<BN, AMN, BMN, MODE>, dim3(grid), dim3(kThreads), G::SMEM, s, ma, mb, mc, g,
-             per, total, a3, b3, m.status);
+    launch_k(kern, dim3(grid), dim3(kThreads), G::SMEM, s, ma, mb, mc, g, per, total, a3, b3, m.status);
     note_launch();
     return QK_OK;
+}
+
+// 256-row tiles for the large full-reduction GEMMs: whole 256-row blocks, at least one
+// tile per SM, and an epilogue light enough to run unoverlapped (not the row statistics
+// or the two-output SwiGLU backward, measured slower without a second accumulator set).
+template <int BN, bool AMN, bool BMN, int MODE>
+int launch_tc_mode(Model& m, const Gemm& g, cudaStream_t s) {
+    if constexpr (BN == 256 && MODE != E_STATS && MODE != E_SWIGLU_BWD) {
+        const long long tiles = (long long)g.sc.Z * (g.sc.M / 256) * cdiv(g.sc.N, 256);
+        if (g.sc.red == RED_FULL && !g.sc.tri && g.sc.M % 256 == 0 && tiles >= m.num_sms)
+            return launch_tc_cfg<BN, 256, AMN, BMN, MODE>(m, g, s);
+    }
+    return launch_tc_cfg<BN, 128, AMN, BMN, MODE>(m, g, s);
 }
 
 // The epilogue modes each operand layout is instantiated for (the ones the backward uses).
