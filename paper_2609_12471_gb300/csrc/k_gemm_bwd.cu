@@ -104,7 +104,7 @@ struct TcCfg {
     static constexpr int ACC = BM == 256 ? 1 : 2;       // accumulator sets
     static constexpr int ACC_COLS = (BM / 128) * BN;    // TMEM columns of one set
     static constexpr int TMEM_COLS = ACC * ACC_COLS;
-    static constexpr int STAGE_OUT = kEpiWarps * 2 * 32 * 16 * 4;  // per epilogue warp: two 32 x 16 fp32 blocks
+    static constexpr int STAGE_OUT = kEpiWarps * 4096;  // per epilogue warp: one 32 x 128-byte block
     static constexpr int SMEM = STAGES * (A_BYTES + B_BYTES) + STAGE_OUT + 1024 + 256;
     static_assert(TMEM_COLS <= 512, "accumulators exceed TMEM");
     static_assert(SMEM <= 232448, "shared memory per CTA");
@@ -289,16 +289,19 @@ __global__ void __launch_bounds__(kThreads, 1)
     } else {
         // ---------------------------------------------------- epilogue (warps 2..9)
         // Warp w reads TMEM lanes 32 (w % 4) .. + 31 (its rows) and the columns of half
-        // (w - 2) / 4 of the tile, four 16-column blocks per TMEM wait.  Each 32-row x
-        // 16-column block of outputs goes through the warp's staging buffer (two
-        // alternating halves) and out with one TMA store.
-        // BM = 256: half selects the tile's 128-row block and the warp takes every column.
+        // (w - 2) / 4 of the tile (BM = 256: half selects the 128-row block and the warp
+        // takes every column), four 16-column blocks per TMEM wait.  Outputs leave through
+        // the warp's 4 KB staging buffer, one TMA store per 32 rows x 128 bytes (64 bf16 or
+        // 32 fp32 columns), rows stored with the 128-byte swizzle so the writes of a warp hit
+        // distinct banks; the two-output SwiGLU backward stores 32 x 16 blocks instead.
         const int q = warp & 3, half = (warp - 2) >> 2;
         constexpr int HC = BM == 256 ? BN : BN / 2;  // columns per warp
         const int c_lo = BM == 256 ? 0 : half * HC, r_lo = BM == 256 ? half * 128 : 0;
         constexpr bool f32 = MODE == E_F32;
-        uint8_t* stg = sOut + (warp - 2) * (2 * 32 * 16 * 4);
-        int acc = 0, blk = 0;
+        constexpr bool staged = MODE != E_STATS && MODE != E_SWIGLU_BWD;
+        uint8_t* stg = sOut + (warp - 2) * 4096;
+        const int sw = lane & 7;
+        int acc = 0;
         uint32_t acc_phase = 0;
         for (long long t = blockIdx.x; t < total; t += gridDim.x) {
             int z, mt, nt;
@@ -321,19 +324,23 @@ __global__ void __launch_bounds__(kThreads, 1)
                 for (int u = 0; u < 4; ++u)
                     if (n0 + c4 + 16 * u < sc.N) tc::tmem_ld16(tbase + c4 + 16 * u, r[u]);
                 tc::tmem_wait_ld();
+                if constexpr (staged) {  // the previous block's store has read the buffer
+                    if (lane == 0) tc::bulk_wait_read<0>();
+                    __syncwarp();
+                }
 #pragma unroll
                 for (int u = 0; u < 4; ++u) {
                     const int n = n0 + c4 + 16 * u;
-                    if (n >= sc.N) break;
+                    const bool in = n < sc.N;
                     float v[16], y[16], y2[16];
 #pragma unroll
                     for (int j = 0; j < 16; ++j) v[j] = __uint_as_float(r[u][j]);
                     const bool store =
-                        m < sc.M && epi_values<bf16, true, MODE>(g.epi, g.out, z, m, n, 16, v, st, y, y2);
+                        in && m < sc.M && epi_values<bf16, true, MODE>(g.epi, g.out, z, m, n, 16, v, st, y, y2);
                     if constexpr (MODE == E_STATS) continue;
-                    uint8_t* buf = stg + (blk & 1) * (32 * 16 * 4);
                     if constexpr (MODE == E_SWIGLU_BWD) {
-                        // dg and du blocks (bf16) side by side in the staging buffer, two stores
+                        if (!in) break;  // uniform
+                        // dg and du blocks (bf16, 32 x 16 each) in the staging buffer, two stores
                         if (lane == 0) tc::bulk_wait_read<0>();
                         __syncwarp();
                         uint4 w[4];
@@ -341,47 +348,59 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
                         for (int j = 0; j < 16; ++j)
                             b[j] = __float2bfloat16_rn(store ? y[j] : 0.f), b[16 + j] = __float2bfloat16_rn(store ? y2[j] : 0.f);
-                        uint4* d = (uint4*)(buf + lane * 32);
+                        uint4* d = (uint4*)(stg + lane * 32);
                         d[0] = w[0];
                         d[1] = w[1];
-                        uint4* d2 = (uint4*)(buf + 1024 + lane * 32);
+                        uint4* d2 = (uint4*)(stg + 1024 + lane * 32);
                         d2[0] = w[2];
                         d2[1] = w[3];
                         tc::fence_proxy_async_smem();
                         __syncwarp();
                         if (lane == 0) {
                             const int gc = (n >> 7) * 256 + (n & 127);
-                            tc::tma_store_2d(&mapC, gc, orow, buf);
-                            tc::tma_store_2d(&mapC, gc + 128, orow, buf + 1024);
+                            tc::tma_store_2d(&mapC, gc, orow, stg);
+                            tc::tma_store_2d(&mapC, gc + 128, orow, stg + 1024);
                             tc::bulk_commit();
                         }
-                        ++blk;
                         continue;
                     }
-                    if (lane == 0) tc::bulk_wait_read<1>();  // the store issued from this half two blocks ago
-                    __syncwarp();
+                    uint4* row = (uint4*)(stg + lane * 128);  // this lane's output row, 8 granules of 16 B
                     if constexpr (f32) {
-                        float4* d = (float4*)(buf + lane * 64);
+                        const int ub = u & 1;  // chunk within the 32-column block
 #pragma unroll
-                        for (int j = 0; j < 4; ++j)
-                            d[j] = store ? make_float4(y[4 * j], y[4 * j + 1], y[4 * j + 2], y[4 * j + 3])
-                                         : make_float4(0.f, 0.f, 0.f, 0.f);
+                        for (int j = 0; j < 4; ++j) {
+                            const float4 f = store ? make_float4(y[4 * j], y[4 * j + 1], y[4 * j + 2], y[4 * j + 3])
+                                                   : make_float4(0.f, 0.f, 0.f, 0.f);
+                            row[(ub * 4 + j) ^ sw] = *reinterpret_cast<const uint4*>(&f);
+                        }
+                        if (ub == 1) {  // 32 columns staged: store them
+                            tc::fence_proxy_async_smem();
+                            __syncwarp();
+                            if (lane == 0) {
+                                tc::tma_store_2d(&mapC, ocol + n0 + c4 + 32 * (u >> 1), orow, stg);
+                                tc::bulk_commit();
+                            }
+                            if (u == 1) {
+                                if (lane == 0) tc::bulk_wait_read<0>();
+                                __syncwarp();
+                            }
+                        }
                     } else {
                         uint4 w[2];
                         bf16* b = (bf16*)w;
 #pragma unroll
                         for (int j = 0; j < 16; ++j) b[j] = __float2bfloat16_rn(store ? y[j] : 0.f);
-                        uint4* d = (uint4*)(buf + lane * 32);
-                        d[0] = w[0];
-                        d[1] = w[1];
+                        row[(2 * u) ^ sw] = w[0];
+                        row[(2 * u + 1) ^ sw] = w[1];
                     }
+                }
+                if constexpr (staged && !f32) {  // 64 columns staged: store them
                     tc::fence_proxy_async_smem();
                     __syncwarp();
                     if (lane == 0) {
-                        tc::tma_store_2d(&mapC, ocol + n, orow, buf);
+                        tc::tma_store_2d(&mapC, ocol + n0 + c4, orow, stg);
                         tc::bulk_commit();
                     }
-                    ++blk;
                 }
             }
             const int ct = nt * 2 + half;  // statistics column tile of HC columns (BM = 128)
@@ -455,18 +474,20 @@ bool make_op_map3(CUtensorMap* map, const Op& o, int nch) {
               CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
-// Output map: fp32 or bf16 over C [rows, cols], box 16 columns x 32 rows, no swizzle.
-bool make_out_map(CUtensorMap* map, const Out& o, bool f32) {
+// Output map over C [rows, cols]: box 32 rows x 128 bytes (64 bf16 / 32 fp32 columns) with
+// the 128-byte swizzle, or (narrow) 32 rows x 16 columns unswizzled.
+bool make_out_map(CUtensorMap* map, const Out& o, bool f32, bool narrow) {
     EncodeTiledFn fn = encode_fn();
     if (!fn) return false;
     const size_t es = f32 ? 4 : 2;
     cuuint64_t dims[2] = {(cuuint64_t)o.cols, (cuuint64_t)o.rows};
     cuuint64_t strides[1] = {(cuuint64_t)o.ldc * es};
-    cuuint32_t box[2] = {16, 32};
+    cuuint32_t box[2] = {narrow ? 16u : (cuuint32_t)(128 / es), 32};
     cuuint32_t estr[2] = {1, 1};
     return fn(map, f32 ? CU_TENSOR_MAP_DATA_TYPE_FLOAT32 : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, o.C, dims,
-              strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE,
-              CU_TENSOR_MAP_L2_PROMOTION_NONE, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+              strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
+              narrow ? CU_TENSOR_MAP_SWIZZLE_NONE : CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_NONE,
+              CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
 template <int BN, int BM, bool AMN, bool BMN, int MODE>
@@ -486,7 +507,7 @@ int launch_tc_cfg(Model& m, const Gemm& g, cudaStream_t s) {
     if ((!a3 && !make_op_map(&ma, g.A, AMN ? 64 : 128)) || (!b3 && !make_op_map(&mb, g.B, BMN ? 64 : BN)))
         return set_error(QK_ECUDA, "backward GEMM: tensor map encoding failed");
     memset(&mc, 0, sizeof(mc));
-    if (MODE != E_STATS && !make_out_map(&mc, g.out, MODE == E_F32))
+    if (MODE != E_STATS && !make_out_map(&mc, g.out, MODE == E_F32, MODE == E_SWIGLU_BWD))
         return set_error(QK_ECUDA, "backward GEMM: output tensor map encoding failed");
     const long long per = tiles_per_z(g.sc, BM, BN);
     const long long total = per * g.sc.Z;
@@ -565,8 +586,10 @@ int run_gemm(Model& m, const Gemm& g, cudaStream_t s) {
     ok = ok && (sc.red != RED_SUFFIX || (sc.seg % kBK == 0 && sc.seg > 0 && sc.K % sc.seg == 0));
     ok = ok && (!g.A.kwrap || g.A.kwrap % kBK == 0) && (!g.B.kwrap || g.B.kwrap % kBK == 0);
     ok = ok && g.B.pitch == 128 && g.A.pitch % 64 == 0 && (!sc.tri || (BN == 128 && sc.M == sc.N));
-    // output tiles are whole 128-row blocks of a batch entry, or clipped at the buffer's last row
+    // output tiles are whole 128-row blocks of a batch entry, or clipped at the buffer's last row;
+    // stores of 64 (bf16) or 32 (fp32) columns stay inside N, or are clipped at the last column
     ok = ok && (sc.M % 128 == 0 || (sc.Z == 1 && g.out.rows == sc.M)) && g.out.rows > 0 && g.out.cols > 0;
+    ok = ok && (sc.N % 64 == 0 || (sc.Z == 1 && g.out.cols == sc.N));
     if (!ok) return set_error(QK_ESHAPE, "backward GEMM: shape or alignment outside the tcgen05 path");
     const bool amn = g.A.mn != 0, bmn = g.B.mn != 0;
     if (BN == 256) {
