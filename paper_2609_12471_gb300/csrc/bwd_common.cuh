@@ -375,7 +375,7 @@ void launch_qk_fwd(const void* qkv, int ld, int M, int Tlen, int nq, int nkv, in
 // tiles at or left of the diagonal of row r % rows_per_z); loss_rows (may be null).
 void launch_stats_combine(const float2* st, int n_ct, int ct_w, int causal, int R, int rows_per_z,
                           float* lse, const float* w, const float* zt, float* loss_rows, cudaStream_t s);
-// RMSNorm backward (fp32 x, g, dy [M, H]): dres (+)= dx, dres_act = act(dres); gain partials
+// RMSNorm backward (fp32 x, g, dy [M, H], H % 4 == 0): dres (+)= dx, dres_act = act(dres); gain partials
 // part [rms_part_rows(M)][H].
 int rms_part_rows(int M);
 void launch_rms_bwd(const float* x, const float* g, const float* dy, int M, int H, float eps, int init,
@@ -390,6 +390,8 @@ void launch_qk_bwd(const float* dqr, const float* dkr, const void* qkv, int ld, 
 void launch_attn_d(const void* dO, const void* O, int M, int Tlen, int nq, int d, float* Dv, int dtype,
                    cudaStream_t s);
 void launch_embed_bwd(const int32_t* tokens, const float* dx, int M, int H, int V, float* dE, cudaStream_t s);
+// h [M, I] = silu(gate) * up from the packed gate / up product gu [M, 2 I] (I % 128 == 0).
+void launch_swiglu_fwd(const void* gu, int M, int I, void* h, int dtype, cudaStream_t s);
 void launch_sum(const float* v, int n, float* out, cudaStream_t s);
 
 }  // namespace bwd

@@ -150,10 +150,10 @@ __global__ void stats_combine_kernel(const float2* __restrict__ st, int n_ct, in
     }
 }
 
-// RMSNorm backward over rows [16 b, 16 b + 16) of CTA b (256 threads, H / 256 columns
-// each): dres = (init ? 0 : dres) + dx, dres_act = act(dres), part[b][c] = sum over the
-// CTA's rows of dy x r (column c).
-constexpr int kRmsRows = 16;
+// RMSNorm backward over rows [8 b, 8 b + 8) of CTA b (256 threads; H % 4 == 0: thread i
+// owns the float4 column groups i, i + 256, ...): dres = (init ? 0 : dres) + dx,
+// dres_act = act(dres), part[b][c] = sum over the CTA's rows of dy x r (column c).
+constexpr int kRmsRows = 8;
 
 template <typename T>
 __global__ void __launch_bounds__(256)
@@ -163,43 +163,67 @@ __global__ void __launch_bounds__(256)
     extern __shared__ float dgs[];
     __shared__ float2 red[8];
     pdl_wait();
+    const int H4 = H >> 2;
     for (int c = threadIdx.x; c < H; c += 256) dgs[c] = 0.f;
+    const float4* g4 = (const float4*)g;
     const int r0 = blockIdx.x * kRmsRows;
     for (int r = r0; r < r0 + kRmsRows && r < M; ++r) {
-        const float* xr = x + (size_t)r * H;
-        const float* dr = dy + (size_t)r * H;
+        const float4* xr = (const float4*)(x + (size_t)r * H);
+        const float4* dr = (const float4*)(dy + (size_t)r * H);
         float ss = 0.f, sa = 0.f;
-        for (int c = threadIdx.x; c < H; c += 256) {
-            const float xv = xr[c];
-            ss += xv * xv;
-            sa += dr[c] * g[c] * xv;
+        for (int c = threadIdx.x; c < H4; c += 256) {
+            const float4 xv = xr[c], dv = dr[c], gv = g4[c];
+            ss += xv.x * xv.x + xv.y * xv.y + xv.z * xv.z + xv.w * xv.w;
+            sa += dv.x * gv.x * xv.x + dv.y * gv.y * xv.y + dv.z * gv.z * xv.z + dv.w * gv.w * xv.w;
         }
         const float2 t = block_sum2(ss, sa, red);
         const float rr = rsqrtf(t.x / (float)H + eps);
         const float k3 = rr * rr * rr / (float)H * t.y;
-        for (int c = threadIdx.x; c < H; c += 256) {
-            const float xv = xr[c], dv = dr[c];
-            const float dx = rr * dv * g[c] - k3 * xv;
-            const size_t o = (size_t)r * H + c;
-            const float nv = init ? dx : dres[o] + dx;
-            dres[o] = nv;
-            st_act(dres_act + o, nv);
-            dgs[c] += dv * xv * rr;
+        float4* d4 = (float4*)(dres + (size_t)r * H);
+        T* da = dres_act + (size_t)r * H;
+        for (int c = threadIdx.x; c < H4; c += 256) {
+            const float4 xv = xr[c], dv = dr[c], gv = g4[c];
+            float4 o = init ? make_float4(0.f, 0.f, 0.f, 0.f) : d4[c];
+            o.x += rr * dv.x * gv.x - k3 * xv.x;
+            o.y += rr * dv.y * gv.y - k3 * xv.y;
+            o.z += rr * dv.z * gv.z - k3 * xv.z;
+            o.w += rr * dv.w * gv.w - k3 * xv.w;
+            d4[c] = o;
+            st_act(da + 4 * c, o.x);
+            st_act(da + 4 * c + 1, o.y);
+            st_act(da + 4 * c + 2, o.z);
+            st_act(da + 4 * c + 3, o.w);
+            dgs[4 * c] += dv.x * xv.x * rr;
+            dgs[4 * c + 1] += dv.y * xv.y * rr;
+            dgs[4 * c + 2] += dv.z * xv.z * rr;
+            dgs[4 * c + 3] += dv.w * xv.w * rr;
         }
     }
     __syncthreads();
     for (int c = threadIdx.x; c < H; c += 256) part[(size_t)blockIdx.x * H + c] = dgs[c];
 }
 
-// out[c] (+)= sum over nb partial rows of part[.][c], in row order.
-__global__ void gain_reduce_kernel(const float* __restrict__ part, int nb, int n, int stride,
-                                   float* __restrict__ out, int accumulate) {
+// out[c] (+)= sum over the nb partial rows of part[.][c] (row stride `stride`): CTA
+// b takes columns 32 b .. 32 b + 31, warp w the rows w, w + 8, ... (lane = column),
+// then the eight warp sums are added in warp order (a fixed order).
+__global__ void __launch_bounds__(256)
+    gain_reduce_kernel(const float* __restrict__ part, int nb, int n, int stride, float* __restrict__ out,
+                       int accumulate) {
+    __shared__ float red[8][32];
     pdl_wait();
-    const int c = blockIdx.x * blockDim.x + threadIdx.x;
-    if (c >= n) return;
+    const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
+    const int c = blockIdx.x * 32 + lane;
     float s = 0.f;
-    for (int b = 0; b < nb; ++b) s += part[(size_t)b * stride + c];
-    out[c] = accumulate ? out[c] + s : s;
+    if (c < n)
+        for (int b = w; b < nb; b += 8) s += part[(size_t)b * stride + c];
+    red[w][lane] = s;
+    __syncthreads();
+    if (w == 0 && c < n) {
+        float t = 0.f;
+#pragma unroll
+        for (int i = 0; i < 8; ++i) t += red[i][lane];
+        out[c] = accumulate ? out[c] + t : t;
+    }
 }
 
 // QK-norm + RoPE backward.  CTA b (8 warps) takes token rows [16 b, 16 b + 16); a warp
@@ -292,6 +316,32 @@ __global__ void attn_d_kernel(const T* __restrict__ dO, const T* __restrict__ O,
     if (lane == 0) Dv[((size_t)(r / Tlen) * nq + h) * Tlen + r % Tlen] = s;
 }
 
+// h = silu(g) u from gu [M, 2 I] in the packed order (blocks of 128 gate columns, then
+// the matching 128 up columns); thread e takes 8 consecutive columns (one 16-byte load of
+// gate, one of up, one 16-byte store of h).  I % 128 == 0.
+template <typename T>
+__global__ void swiglu_fwd_kernel(const T* __restrict__ gu, int M, int I, T* __restrict__ h) {
+    constexpr int V = 16 / sizeof(T);
+    pdl_wait();
+    const size_t n = (size_t)M * I / V;
+    for (size_t e = blockIdx.x * (size_t)blockDim.x + threadIdx.x; e < n; e += (size_t)gridDim.x * blockDim.x) {
+        const size_t j0 = e * V;
+        const size_t m = j0 / I;
+        const int j = (int)(j0 - m * I);
+        const T* gp = gu + m * 2 * I + (size_t)(j >> 7) * 256 + (j & 127);
+        uint4 gq = *(const uint4*)gp, uq = *(const uint4*)(gp + 128), hq;
+        const T* ga = (const T*)&gq;
+        const T* ua = (const T*)&uq;
+        T* ha = (T*)&hq;
+#pragma unroll
+        for (int k = 0; k < V; ++k) {
+            const float gv = ld_act(ga + k);
+            st_act(ha + k, gv / (1.f + __expf(-gv)) * ld_act(ua + k));
+        }
+        *(uint4*)(h + j0) = hq;
+    }
+}
+
 // dE[token[r]] += dx[r] (fp32 atomics: rows that share a token add in any order).
 __global__ void embed_bwd_kernel(const int32_t* __restrict__ tokens, const float* __restrict__ dx, int H,
                                  int V, float* __restrict__ dE) {
@@ -365,7 +415,7 @@ void launch_rms_bwd(const float* x, const float* g, const float* dy, int M, int 
 
 void launch_gain_reduce(const float* part, int nb, int n, int stride, float* out, int accumulate,
                         cudaStream_t s) {
-    launch_k(gain_reduce_kernel, dim3(cdiv(n, 256)), dim3(256), 0, s, part, nb, n, stride, out, accumulate);
+    launch_k(gain_reduce_kernel, dim3(cdiv(n, 32)), dim3(256), 0, s, part, nb, n, stride, out, accumulate);
     note_launch();
 }
 
@@ -392,6 +442,16 @@ void launch_attn_d(const void* dO, const void* O, int M, int Tlen, int nq, int d
     launch_act(dtype, [&](auto* tp) {
         using A = std::remove_pointer_t<decltype(tp)>;
         launch_k(attn_d_kernel<A>, grid, dim3(256), 0, s, (const A*)dO, (const A*)O, M, Tlen, nq, d, Dv);
+    });
+    note_launch();
+}
+
+void launch_swiglu_fwd(const void* gu, int M, int I, void* h, int dtype, cudaStream_t s) {
+    const size_t n = (size_t)M * I / (dtype == QK_DTYPE_BF16 ? 8 : 4);
+    const int blocks = (int)(n / 256 + 1 < 152 * 16 ? n / 256 + 1 : 152 * 16);
+    launch_act(dtype, [&](auto* tp) {
+        using A = std::remove_pointer_t<decltype(tp)>;
+        launch_k(swiglu_fwd_kernel<A>, dim3(blocks), dim3(256), 0, s, (const A*)gu, M, I, (A*)h);
     });
     note_launch();
 }

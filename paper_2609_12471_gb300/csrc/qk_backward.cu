@@ -320,7 +320,7 @@ int layer_fwd(const Ctx& x, int l, const float* x_in, float* x_out) {
     QK_TRY(lin_fwd(x, L.O.at(l), nq * d, W.w_o, H, x_mid, E_F32, x_in));
     launch_rmsnorm(x_mid, 1, 0, W.mlp_norm, H, eps, L.u2.at(l), c.dtype, M, x.s);
     QK_TRY(lin_fwd(x, L.u2.at(l), H, W.w_gu, 2 * I, L.gu.at(l), E_ACT));
-    launch_swiglu(L.gu.at(l), L.h.at(l), c.dtype, M, I, x.s);
+    launch_swiglu_fwd(L.gu.at(l), M, I, L.h.at(l), c.dtype, x.s);
     return lin_fwd(x, L.h.at(l), I, W.w_d, H, x_out, E_F32, x_mid);
 }
 
