@@ -55,6 +55,8 @@ enum Mode : int {
     E_SWIGLU_BWD = 5,  // acc = dh[m, n] of h = silu(g) u: with (g, u) read from gu (the packed
                        // [M, 2 I] gate / up layout, row stride ldc), writes dg and du into C
                        // (laid out like gu) at the gate and up columns of n
+    E_SWIGLU_FWD = 6,  // acc = [gate | up] of a 256-column tile of the packed gate / up product:
+                       // C[m, 128 t + c] = bf16(silu(gate c) up c)  (tensor-core path, 256-row tiles)
 };
 
 // Row vectors (lse, w, tgt, zt, D, stats) are indexed r = z * rows_per_z + m.
@@ -357,6 +359,13 @@ struct Gemm {
 
 // Runs g on the model's path: tcgen05 for bf16 models, CUDA cores for fp32 models.
 int run_gemm(Model& m, const Gemm& g, cudaStream_t s);
+// bf16 linear C = A W^T for M >= 256 rows through this GEMM's 256 x 256 tiles (the forward
+// pass's prefill / scoring linears): epi EPI_STORE_ACT, EPI_STORE_F32, EPI_RESID_F32 or
+// EPI_SWIGLU (N = I, W the packed gate / up rows).  Returns false (nothing launched) when
+// the shape or alignment does not fit those tiles; the caller then uses its other kernels.
+bool linear_large(Model& m, const void* A, int lda, const void* W, void* C, int ldc, int M, int N,
+                  int K, int epi, cudaStream_t s);
+
 // Column width of the E_STATS partials of the kernel run_gemm picks for N columns
 // (half its N tile on the tensor-core path, its tile on the CUDA-core path).
 int gemm_tile_n(const Model& m, int N, int tri);

@@ -1,11 +1,12 @@
 // Kernel selection for the linear layers and attention of one forward call.
-#include "qk_internal.cuh"
+#include "bwd_common.cuh"
 
 namespace qk {
 
 // bf16: up to kGemvMaxRows token rows stream the weights through the CUDA-core
-// GEMV (bound by reading W), more rows go to the tcgen05 GEMM.  fp32: CUDA-core
-// GEMM (no TF32).
+// GEMV (bound by reading W); 256 or more rows whose shape fills the SMs with 256 x 256
+// tiles go to the batched tcgen05 GEMM of k_gemm_bwd.cu; other row counts to the
+// swap-AB tcgen05 GEMM of k_gemm_tc.cu.  fp32: CUDA-core GEMM (no TF32).
 void linear(Model& m, const void* A, int lda, const void* W, void* C, int ldc, int M, int N,
             int K, int epi, void* gu, cudaStream_t s) {
     const int dt = m.cfg.dtype;
@@ -13,6 +14,9 @@ void linear(Model& m, const void* A, int lda, const void* W, void* C, int ldc, i
         launch_gemv_bf16((const bf16*)A, lda, (const bf16*)W, C, ldc, M, N, K, epi, s);
         return;
     }
+    // 256 or more rows (prefill / scoring): 256 x 256 tensor-core tiles when they fit
+    if (dt == QK_DTYPE_BF16 && m.test_wait_cycles == 0 && bwd::linear_large(m, A, lda, W, C, ldc, M, N, K, epi, s))
+        return;
     if (dt == QK_DTYPE_BF16 && gemm_tc_supported(A, lda, N, K)) {
         const long long test_wait = m.test_wait_cycles;  // one launch only
         m.test_wait_cycles = 0;

@@ -298,7 +298,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         constexpr int HC = BM == 256 ? BN : BN / 2;  // columns per warp
         const int c_lo = BM == 256 ? 0 : half * HC, r_lo = BM == 256 ? half * 128 : 0;
         constexpr bool f32 = MODE == E_F32;
-        constexpr bool staged = MODE != E_STATS && MODE != E_SWIGLU_BWD;
+        constexpr bool staged = MODE != E_STATS && MODE != E_SWIGLU_BWD && MODE != E_SWIGLU_FWD;
         uint8_t* stg = sOut + (warp - 2) * 4096;
         const int sw = lane & 7;
         int acc = 0;
@@ -317,7 +317,44 @@ __global__ void __launch_bounds__(kThreads, 1)
             const int orow = (z / g.out.zq) * g.out.zrow + m0 + q * 32;
             const int ocol = (z % g.out.zq) * g.out.zcol;
             RowStat st{-INFINITY, 0.f};
-            for (int c4 = c_lo; c4 < c_lo + HC; c4 += 64) {
+            if constexpr (MODE == E_SWIGLU_FWD) {
+                // BM = 256: the warp holds all 256 columns of its rows, gate c at TMEM column
+                // c and up c at c + 128 (the packed gate / up rows); 64 outputs per store
+                for (int c = 0; c < 128; c += 64) {
+                    if (lane == 0) tc::bulk_wait_read<0>();
+                    __syncwarp();
+                    uint4* row = (uint4*)(stg + lane * 128);
+#pragma unroll
+                    for (int hh = 0; hh < 2; ++hh) {
+                        const int cc = c + 32 * hh;
+                        uint32_t gr[2][16], ur[2][16];
+                        tc::tmem_ld16(tbase + cc, gr[0]);
+                        tc::tmem_ld16(tbase + cc + 16, gr[1]);
+                        tc::tmem_ld16(tbase + 128 + cc, ur[0]);
+                        tc::tmem_ld16(tbase + 128 + cc + 16, ur[1]);
+                        tc::tmem_wait_ld();
+#pragma unroll
+                        for (int w2 = 0; w2 < 2; ++w2) {
+                            uint4 wv[2];
+                            bf16* b = (bf16*)wv;
+#pragma unroll
+                            for (int j = 0; j < 16; ++j) {
+                                const float gv = __uint_as_float(gr[w2][j]), uv = __uint_as_float(ur[w2][j]);
+                                b[j] = __float2bfloat16_rn(m < sc.M ? gv / (1.f + __expf(-gv)) * uv : 0.f);
+                            }
+                            row[(hh * 4 + w2 * 2) ^ sw] = wv[0];
+                            row[(hh * 4 + w2 * 2 + 1) ^ sw] = wv[1];
+                        }
+                    }
+                    tc::fence_proxy_async_smem();
+                    __syncwarp();
+                    if (lane == 0) {
+                        tc::tma_store_2d(&mapC, ocol + nt * 128 + c, orow, stg);
+                        tc::bulk_commit();
+                    }
+                }
+            }
+            for (int c4 = c_lo; c4 < c_lo + HC && MODE != E_SWIGLU_FWD; c4 += 64) {
                 if (n0 + c4 >= sc.N) break;  // uniform over the warp
                 uint32_t r[4][16];
 #pragma unroll
@@ -517,17 +554,24 @@ int launch_tc_cfg(Model& m, const Gemm& g, cudaStream_t s) {
     return QK_OK;
 }
 
+bool big_tiles(const Model& m, const Gemm& g) {
+    const long long tiles = (long long)g.sc.Z * (g.sc.M / 256) * cdiv(g.sc.N, 256);
+    return g.sc.red == RED_FULL && !g.sc.tri && g.sc.M % 256 == 0 && tiles >= m.num_sms;
+}
+
 // 256-row tiles for the large full-reduction GEMMs: whole 256-row blocks, at least one
 // tile per SM, and an epilogue light enough to run unoverlapped (not the row statistics
 // or the two-output SwiGLU backward, measured slower without a second accumulator set).
 template <int BN, bool AMN, bool BMN, int MODE>
 int launch_tc_mode(Model& m, const Gemm& g, cudaStream_t s) {
     if constexpr (BN == 256 && MODE != E_STATS && MODE != E_SWIGLU_BWD) {
-        const long long tiles = (long long)g.sc.Z * (g.sc.M / 256) * cdiv(g.sc.N, 256);
-        if (g.sc.red == RED_FULL && !g.sc.tri && g.sc.M % 256 == 0 && tiles >= m.num_sms)
-            return launch_tc_cfg<BN, 256, AMN, BMN, MODE>(m, g, s);
+        if (big_tiles(m, g)) return launch_tc_cfg<BN, 256, AMN, BMN, MODE>(m, g, s);
     }
-    return launch_tc_cfg<BN, 128, AMN, BMN, MODE>(m, g, s);
+    if constexpr (MODE == E_SWIGLU_FWD) {
+        return set_error(QK_ESHAPE, "SwiGLU forward epilogue needs 256 x 256 tiles");
+    } else {
+        return launch_tc_cfg<BN, 128, AMN, BMN, MODE>(m, g, s);
+    }
 }
 
 // The epilogue modes each operand layout is instantiated for (the ones the backward uses).
@@ -535,6 +579,7 @@ template <int BN, bool AMN, bool BMN>
 int launch_tc(Model& m, const Gemm& g, cudaStream_t s) {
     const int mode = g.epi.mode;
     if (!AMN && !BMN) {
+        if (mode == E_SWIGLU_FWD) return launch_tc_mode<BN, AMN, BMN, E_SWIGLU_FWD>(m, g, s);
         if (mode == E_F32) return launch_tc_mode<BN, AMN, BMN, E_F32>(m, g, s);
         if (mode == E_ACT) return launch_tc_mode<BN, AMN, BMN, E_ACT>(m, g, s);
         if (mode == E_STATS) return launch_tc_mode<BN, AMN, BMN, E_STATS>(m, g, s);
@@ -563,6 +608,31 @@ static int tile_bn(const Model& m, int N, int tri) {
 
 int gemm_tile_n(const Model& m, int N, int tri) {
     return m.cfg.dtype != QK_DTYPE_BF16 ? kSimtTile : tile_bn(m, N, tri) / 2;
+}
+
+bool linear_large(Model& m, const void* A, int lda, const void* W, void* C, int ldc, int M, int N,
+                  int K, int epi, cudaStream_t s) {
+    if (m.cfg.dtype != QK_DTYPE_BF16 || M < 256) return false;
+    const bool swiglu = epi == EPI_SWIGLU;
+    const int n_gemm = swiglu ? 2 * N : N;
+    Gemm g{};
+    g.A = Op{A, lda, M, K, 0, 0, 0, 1, 1, 0, 0, 0, 0, 0, 128};
+    g.B = Op{W, K, n_gemm, K, 0, 0, 0, 1, 1, 0, 0, 0, 0, 0, 128};
+    g.out = Out{C, ldc, M, N, 1, 0, 0, nullptr};
+    g.epi = Epi{};
+    g.epi.scale = 1.f;
+    g.sc = Sched{1, M, n_gemm, K, RED_FULL, 0, 0, 0};
+    if (epi == EPI_STORE_ACT) g.epi.mode = E_ACT;
+    else if (epi == EPI_STORE_F32) g.epi.mode = E_F32;
+    else if (epi == EPI_RESID_F32) g.epi.mode = E_F32, g.out.addend = (const float*)C;
+    else if (swiglu) g.epi.mode = E_SWIGLU_FWD;
+    else return false;
+    if (!big_tiles(m, g) || n_gemm % 256 || K % 64 || lda % 8 || ((uintptr_t)A & 15) || ((uintptr_t)W & 15) ||
+        ((uintptr_t)C & 15) || (g.epi.mode == E_F32 ? ldc % 4 : ldc % 8) || ldc < N)
+        return false;
+    const int rc = run_gemm(m, g, s);
+    if (rc != QK_OK && !m.deferred_error) m.deferred_error = rc;
+    return true;
 }
 
 int run_gemm(Model& m, const Gemm& g, cudaStream_t s) {
