@@ -66,11 +66,13 @@ int qk_op_linear(qk_model* m, const void* A, int lda, const void* W, void* C, in
  * another CTA is bounded: when one expires the kernel sets QK_STATUS_TIMEOUT,
  * waits (bounded) for its own copies in flight, frees its tensor memory and
  * returns, so the context stays usable.  After this call, the next plain
- * tensor-core linear launched for the model (qk_op_linear on a bf16 model with
- * M > 4 rows, or a prefill / scoring linear) lets its first CTA wait at most
- * wait_cycles SM cycles and issues no copy for that CTA's first k-block, so that
- * CTA's wait for it expires: its output is undefined, QK_STATUS_TIMEOUT is set
- * and qk_check_status returns QK_ETIMEOUT.  The hook disarms at that launch.
+ * tensor-core GEMM launched for the model (qk_op_linear on a bf16 model with
+ * M > 4 rows, a prefill / scoring linear, which then runs on the swap-AB kernel,
+ * or a GEMM of qk_backward_logprob) lets its first CTA wait at most wait_cycles
+ * SM cycles and issues no copy for that CTA's first k-block, so that CTA's wait
+ * for it expires: its output (and what the call computes from it) is undefined,
+ * QK_STATUS_TIMEOUT is set and qk_check_status returns QK_ETIMEOUT.  The hook
+ * disarms at that launch.
  * wait_cycles in [1, 2^31]; QK_EINVAL otherwise. */
 int qk_debug_expire_next_wait(qk_model* m, long long wait_cycles);
 

@@ -14,7 +14,9 @@
 // m/n elements by the leading byte offset (8 KB) and 8 k rows by the stride byte
 // offset (1 KB).  Two TMEM accumulators alternate so the epilogue of one tile
 // overlaps the main loop of the next.  Every mbarrier wait is bounded; on a timeout
-// the CTA raises QK_STATUS_TIMEOUT, drains its copies and MMAs and exits.
+// the CTA raises QK_STATUS_TIMEOUT, drains its copies and MMAs and exits.  A launch
+// armed by qk_debug_expire_next_wait exercises that path: CTA 0 issues no copy for
+// its first k-block and its waits give up after the armed limit.
 #include <cuda.h>
 #include <math.h>
 #include <string.h>
@@ -114,7 +116,8 @@ template <int BN, int BM, bool AMN, bool BMN, int MODE>
 __global__ void __launch_bounds__(kThreads, 1)
     gemm_bwd_tc_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant__ CUtensorMap mapB,
                        const __grid_constant__ CUtensorMap mapC, const __grid_constant__ Gemm g,
-                       long long per, long long total, int a3, int b3, uint32_t* __restrict__ status) {
+                       long long per, long long total, int a3, int b3, uint32_t* __restrict__ status,
+                       long long test_wait) {
     using G = TcCfg<BN, BM>;
     constexpr int STAGES = G::STAGES;
     extern __shared__ uint8_t smem_raw[];
@@ -132,6 +135,10 @@ __global__ void __launch_bounds__(kThreads, 1)
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const Sched& sc = g.sc;
+    // bounded-wait test (qk_debug_expire_next_wait): CTA 0 issues no copy for its first
+    // k-block and its waits give up after test_wait cycles
+    const bool test_skip = test_wait > 0 && blockIdx.x == 0;
+    const long long wlim = test_skip ? test_wait : tc::kWaitCycles;
 
     if (threadIdx.x == 0) {
         for (int s = 0; s < STAGES; ++s) {
@@ -162,7 +169,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             uint32_t phase = 0;
             int armed[STAGES];
             for (int s = 0; s < STAGES; ++s) armed[s] = -1;
-            bool ok = true;
+            bool ok = true, skip_next = test_skip;
             for (long long t = blockIdx.x; ok && t < total; t += gridDim.x) {
                 int z, mt, nt;
                 tile_at(sc, BM, BN, per, t, z, mt, nt);
@@ -171,9 +178,17 @@ __global__ void __launch_bounds__(kThreads, 1)
                 for (int j = 0; j < nkb; ++j) {
                     int k0, kend;
                     kblock_at(sc, BM, kBK, m0, j, k0, kend);
-                    if (!tc::mbar_wait(&empty[stage], phase ^ 1, abort_flag)) {
+                    if (!tc::mbar_wait(&empty[stage], phase ^ 1, abort_flag, wlim)) {
                         ok = false;
                         break;
+                    }
+                    if (skip_next) {  // bounded-wait test: this stage's copy is never issued
+                        skip_next = false;
+                        if (++stage == STAGES) {
+                            stage = 0;
+                            phase ^= 1;
+                        }
+                        continue;
                     }
                     tc::mbar_expect_tx(&full[stage], G::A_BYTES + G::B_BYTES);
                     uint8_t* a_s = sA + stage * G::A_BYTES;
@@ -241,14 +256,14 @@ __global__ void __launch_bounds__(kThreads, 1)
                 int z, mt, nt;
                 tile_at(sc, BM, BN, per, t, z, mt, nt);
                 const int nkb = kblocks(sc, BM, kBK, mt * BM);
-                if (!tc::mbar_wait(&tempty[acc], acc_phase ^ 1, abort_flag)) {
+                if (!tc::mbar_wait(&tempty[acc], acc_phase ^ 1, abort_flag, wlim)) {
                     ok = false;
                     break;
                 }
                 tc::fence_after_sync();
                 const uint32_t d = tmem_base + (uint32_t)(acc * G::ACC_COLS);
                 for (int j = 0; j < nkb; ++j) {
-                    if (!tc::mbar_wait(&full[stage], phase, abort_flag)) {
+                    if (!tc::mbar_wait(&full[stage], phase, abort_flag, wlim)) {
                         ok = false;
                         break;
                     }
@@ -307,7 +322,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             int z, mt, nt;
             tile_at(sc, BM, BN, per, t, z, mt, nt);
             const int m0 = mt * BM + r_lo, n0 = nt * BN;
-            bool ok = tc::mbar_wait(&tfull[acc], acc_phase, abort_flag);
+            bool ok = tc::mbar_wait(&tfull[acc], acc_phase, abort_flag, wlim);
             ok = __all_sync(0xffffffffu, ok);
             if (!ok) break;
             tc::fence_after_sync();
@@ -549,7 +564,10 @@ int launch_tc_cfg(Model& m, const Gemm& g, cudaStream_t s) {
     const long long per = tiles_per_z(g.sc, BM, BN);
     const long long total = per * g.sc.Z;
     const int grid = total < m.num_sms ? (int)total : m.num_sms;
-    launch_k(kern, dim3(grid), dim3(kThreads), G::SMEM, s, ma, mb, mc, g, per, total, a3, b3, m.status);
+    const long long test_wait = m.test_wait_cycles;  // one launch only
+    m.test_wait_cycles = 0;
+    launch_k(kern, dim3(grid), dim3(kThreads), G::SMEM, s, ma, mb, mc, g, per, total, a3, b3, m.status,
+             test_wait);
     note_launch();
     return QK_OK;
 }

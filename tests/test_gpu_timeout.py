@@ -63,3 +63,35 @@ def test_expired_wait_sets_timeout_and_context_stays_usable(bf16_model):
     again = _linear(dec, Ad, Wd, M, N, K).cpu().numpy()
     assert dec.check_status() == 0
     assert np.abs(again - ref).max() <= tol
+
+
+def test_expired_wait_in_the_backward_gemm():
+    """The same hook arms the next launch of the backward pass's batched tcgen05 GEMM (the
+    first layer's QKV projection of the forward it runs): the status word reports the
+    expired wait, and the next backward call on the same context gives the gradients of a
+    clean run again."""
+    import torch
+    import paper_2609_12471_gb300 as qk
+    s = synth.ModelShape("bwd_bf16", 2, 512, 4, 2, 128, 256, 1024, "bf16")
+    dec, _ = decoder(s)
+    B, T = 2, 256
+    tok = torch.tensor(synth.tokens((B, T), s.vocab, stream=77), dtype=torch.int32, device="cuda")
+    coef = torch.full((B, T - 1), 1.0 / (B * (T - 1)), device="cuda")
+    g0 = dec.new_grads()
+    dec.backward(tok, coef, g0)
+    torch.cuda.synchronize()
+    assert dec.check_status() == 0
+    g1 = dec.new_grads()
+    qk.qk_debug_expire_next_wait(dec.handle, 1 << 20)
+    dec.backward(tok, coef, g1)
+    torch.cuda.synchronize()
+    flags = qk.qk_check_status(dec.handle)
+    assert flags & qk.QK_STATUS_TIMEOUT, flags
+    dec.backward(tok, coef, g1)
+    torch.cuda.synchronize()
+    assert dec.check_status() == 0
+    for i, (a, b) in enumerate(zip(g0, g1)):
+        # bit-identical except the embedding rows, whose repeated tokens add in any order
+        tol = 1e-6 * float(a.abs().max()) if i == 0 else 0.0
+        assert float((a - b).abs().max()) <= tol, i
+    dec.close()
