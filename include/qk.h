@@ -260,8 +260,12 @@ int qk_grpo_coef(const float* lp, const float* lp_old, const float* lp_ref, int 
  * [1] or NULL receives the loss.  workspace: qk_workspace_bytes(QK_CALL_BACKWARD,
  * B, T, 0), 256-byte aligned (it keeps every layer's forward activations, about
  * 1.1 GB per layer per 8192 tokens at Qwen3-8B size, the attention probabilities of
- * one layer and a [min(B T, 4096), V] block of logit gradients).  bf16 models need T % 128 == 0, head_dim 128 and vocab % 64 == 0
- * (QK_ESHAPE otherwise); fp32 models take any shape.  Activations are rounded to
+ * one layer and a [min(B T, 4096), V] block of logit gradients).  bf16 models
+ * need head_dim 128 and vocab, hidden % 64 == 0 (QK_ESHAPE otherwise) and run each
+ * row padded to a multiple of 128 positions inside the workspace (zero
+ * coefficients after the row's end: causal attention keeps the padding invisible
+ * to the real positions, so the result is that of the unpadded rows); fp32 models
+ * take any shape.  Activations are rounded to
  * the model dtype where the forward pass rounds them (and the logit and attention
  * gradients, which are tensor-core operands, likewise); accumulation, norms,
  * softmax statistics, the residual gradient and every weight gradient are fp32.

@@ -402,6 +402,10 @@ void launch_embed_bwd(const int32_t* tokens, const float* dx, int M, int H, int 
 // h [M, I] = silu(gate) * up from the packed gate / up product gu [M, 2 I] (I % 128 == 0).
 void launch_swiglu_fwd(const void* gu, int M, int I, void* h, int dtype, cudaStream_t s);
 void launch_sum(const float* v, int n, float* out, cudaStream_t s);
+// tok_p [B, Tp] / coef_p [B, Tp - 1]: the rows of tok [B, T] / coef [B, T - 1] followed by
+// token 0 and coefficient 0 up to Tp positions.
+void launch_pad_rows(const int32_t* tok, const float* coef, int B, int T, int Tp, int32_t* tok_p, float* coef_p,
+                     cudaStream_t s);
 
 }  // namespace bwd
 }  // namespace qk

@@ -352,6 +352,17 @@ __global__ void embed_bwd_kernel(const int32_t* __restrict__ tokens, const float
     for (int c = threadIdx.x; c < H; c += blockDim.x) atomicAdd(dE + (size_t)id * H + c, dx[(size_t)r * H + c]);
 }
 
+// Rows padded from T to Tp positions: tokens id 0 and coefficients 0 past the row's end.
+__global__ void pad_rows_kernel(const int32_t* __restrict__ tok, const float* __restrict__ coef, int B, int T,
+                                int Tp, int32_t* __restrict__ tok_p, float* __restrict__ coef_p) {
+    pdl_wait();
+    const long long i = (long long)blockIdx.x * blockDim.x + threadIdx.x;
+    if (i >= (long long)B * Tp) return;
+    const int b = (int)(i / Tp), t = (int)(i % Tp);
+    tok_p[i] = t < T ? tok[(size_t)b * T + t] : 0;
+    if (t < Tp - 1) coef_p[(size_t)b * (Tp - 1) + t] = t < T - 1 ? coef[(size_t)b * (T - 1) + t] : 0.f;
+}
+
 // *out = sum of v[0 .. n) in a fixed order (one CTA of 256 threads).
 __global__ void sum_kernel(const float* __restrict__ v, int n, float* __restrict__ out) {
     __shared__ float2 red[8];
@@ -458,6 +469,13 @@ void launch_swiglu_fwd(const void* gu, int M, int I, void* h, int dtype, cudaStr
 
 void launch_embed_bwd(const int32_t* tokens, const float* dx, int M, int H, int V, float* dE, cudaStream_t s) {
     launch_k(embed_bwd_kernel, dim3(M), dim3(256), 0, s, tokens, dx, H, V, dE);
+    note_launch();
+}
+
+void launch_pad_rows(const int32_t* tok, const float* coef, int B, int T, int Tp, int32_t* tok_p, float* coef_p,
+                     cudaStream_t s) {
+    const long long n = (long long)B * Tp;
+    launch_k(pad_rows_kernel, dim3((unsigned)((n + 255) / 256)), dim3(256), 0, s, tok, coef, B, T, Tp, tok_p, coef_p);
     note_launch();
 }
 

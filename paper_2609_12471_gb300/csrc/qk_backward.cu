@@ -490,12 +490,28 @@ int backward_impl(Model& m, const int32_t* tokens, int B, int T, const float* co
 
 }  // namespace
 
+// Rows of a bf16 call are padded to a multiple of 128 positions (the tensor-core tiles'
+// granularity): the padding follows every real position, so under causal attention no
+// real position sees it, and its coefficients are zero, so it adds nothing to the loss
+// and receives no gradient.
+static int padded_len(const Model& m, int T) {
+    return m.cfg.dtype == QK_DTYPE_BF16 && T % 128 ? (T + 127) / 128 * 128 : T;
+}
+
+// Workspace: the layout for the padded length, then (when padding) the padded tokens
+// [B, Tp] and coefficients [B, Tp - 1].
+static size_t pad_bytes(int B, int T, int Tp) {
+    if (Tp == T) return 0;
+    return align256((size_t)B * Tp * 4) + align256((size_t)B * (Tp - 1) * 4);
+}
+
 int backward_workspace_bytes(const Model& m, int B, int T, size_t* bytes) {
     if (B < 1 || T < 2) return set_error(QK_ESHAPE, "backward needs B >= 1 and T >= 2");
-    if ((size_t)B * T > ((size_t)1 << 24)) return set_error(QK_ESHAPE, "too many tokens in one call");
+    const int Tp = padded_len(m, T);
+    if ((size_t)B * Tp > ((size_t)1 << 24)) return set_error(QK_ESHAPE, "too many tokens in one call");
     BwdLayout L;
-    QK_TRY(bwd_layout(m, B, T, nullptr, &L));
-    *bytes = L.total;
+    QK_TRY(bwd_layout(m, B, Tp, nullptr, &L));
+    *bytes = L.total + pad_bytes(B, T, Tp);
     return QK_OK;
 }
 
@@ -516,15 +532,26 @@ extern "C" int qk_backward_logprob(qk_model* mh, const int32_t* tokens, int B, i
             return set_error(QK_EINVAL, "gradient buffer %d is NULL or not 16-byte aligned", i);
     size_t need = 0;
     QK_TRY(backward_workspace_bytes(m, B, T, &need));
-    if (T > c.max_positions) return set_error(QK_ESHAPE, "T %d exceeds max_positions %d", T, c.max_positions);
+    const int Tp = padded_len(m, T);
+    if (Tp > c.max_positions)
+        return set_error(QK_ESHAPE, "T %d (%d padded) exceeds max_positions %d", T, Tp, c.max_positions);
     if (c.dtype == QK_DTYPE_BF16 &&
-        (T % 128 || c.head_dim != 128 || c.vocab % 64 || c.hidden % 64 || ((uintptr_t)tokens & 3)))
-        return set_error(QK_ESHAPE,
-                         "bf16 backward needs T %% 128 == 0, head_dim 128 and vocab, hidden %% 64 == 0");
+        (c.head_dim != 128 || c.vocab % 64 || c.hidden % 64 || ((uintptr_t)tokens & 3) || ((uintptr_t)coef & 3)))
+        return set_error(QK_ESHAPE, "bf16 backward needs head_dim 128 and vocab, hidden %% 64 == 0");
     if (!workspace || ((uintptr_t)workspace & 255)) return set_error(QK_EINVAL, "workspace NULL or not 256-byte aligned");
     if (ws_bytes < need) return set_error(QK_ENOSPACE, "workspace has %zu bytes, needs %zu", ws_bytes, need);
     cudaGetLastError();
-    int rc = backward_impl(m, tokens, B, T, coef, grads, accumulate != 0, loss, workspace, (cudaStream_t)stream);
+    cudaStream_t s = (cudaStream_t)stream;
+    if (Tp != T) {  // padded copies of the rows after the layout's buffers
+        BwdLayout L;
+        QK_TRY(bwd_layout(m, B, Tp, nullptr, &L));
+        int32_t* tok_p = (int32_t*)((char*)workspace + L.total);
+        float* coef_p = (float*)((char*)tok_p + align256((size_t)B * Tp * 4));
+        launch_pad_rows(tokens, coef, B, T, Tp, tok_p, coef_p, s);
+        tokens = tok_p;
+        coef = coef_p;
+    }
+    int rc = backward_impl(m, tokens, B, Tp, coef, grads, accumulate != 0, loss, workspace, s);
     if (rc != QK_OK) return rc;
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return cuda_error(e, "backward launches");

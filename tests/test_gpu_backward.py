@@ -6,6 +6,7 @@ coefficients (qk_grpo_coef) against the fp64 oracle (oracle/backward.py, oracle/
   the tensor's largest entry, on ragged sequence lengths (37: one partial 64-tile;
   130: three tiles and a 2-row tail);
 * bf16 decoders (tcgen05 GEMMs with K- and MN-major operands): a two-layer model
+  (also on ragged rows of 200 positions, padded inside the call)
   and one layer at Qwen3-8B width (H 4096, 32/8 heads, I 12288; vocabulary 16384) over
   2 x 256 tokens (two causal tiles per row),
   per-tensor relative Frobenius error within the bf16 bound, and the loss;
@@ -125,6 +126,17 @@ def test_bf16_two_layer_gradients_match_oracle():
     worst = _check_bf16(s, W, dec, 2, 256, 71)
     dec.close()
     print("bf16 two-layer relative Frobenius errors:", {k: f"{v:.2e}" for k, v in worst.items()})
+
+
+def test_bf16_ragged_rows_match_oracle():
+    """T = 200 (one full 128-position tile and a 72-position tail): the call pads the rows to
+    256 positions internally; gradients and loss are those of the unpadded rows."""
+    s = synth.ModelShape("bwd_bf16", 2, 512, 4, 2, 128, 256, 1024, "bf16")
+    W = synth.LazyWeights(s)
+    dec, _ = decoder(s, W)
+    worst = _check_bf16(s, W, dec, 2, 200, 74)
+    dec.close()
+    print("bf16 ragged (T 200) relative Frobenius errors:", {k: f"{v:.2e}" for k, v in worst.items()})
 
 
 def test_bf16_q8b_width_layer_gradients_match_oracle():
