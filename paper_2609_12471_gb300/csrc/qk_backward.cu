@@ -14,11 +14,13 @@
 //      statistics + combine), then dz = coef (softmax - onehot) in the activation
 //      type from a second pass over the logits, dW_lm (+)= dz^T hn, d hn = dz W_lm;
 //      final-norm backward;
-//   3. per layer, last to first: the backward of the MLP and of W_o, then the
-//      attention probabilities P of the layer again from its log-sum-exp (causal tiles
-//      only, one [T, T] block per (row, head)), dS = P (dP - D), dQ = dS K, dK and dV
-//      summed over each GQA group, then QK-norm and RoPE, W_qkv and the input norm,
-//      adding into the running residual gradient;
+//   3. per layer, last to first: the backward of the MLP and of W_o, then of the
+//      attention (bf16, head_dim 128: one fused tcgen05 kernel that forms P and
+//      dS = P (dP - D) on chip and accumulates dV, dK per key tile and dQ by TMA
+//      reduce-add; otherwise P again from the stored log-sum-exp as [T, T] blocks
+//      (causal tiles only), dS, dQ = dS K, dK and dV summed over each GQA group as
+//      batched GEMMs), then QK-norm and RoPE, W_qkv and the input norm, adding into
+//      the running residual gradient;
 //   4. embedding gradient (scatter-add of the residual gradient).
 // Every product is a bwd::Gemm (k_gemm_bwd.cu): tcgen05 for bf16 models, CUDA cores
 // for fp32 models.  Gain gradients are reduced in a fixed order; the embedding
@@ -73,6 +75,11 @@ struct BwdLayout {
     size_t total;
 };
 
+bool fused_attn_bwd(const Model& m, int T) {
+    const qk_config& c = m.cfg;
+    return c.dtype == QK_DTYPE_BF16 && attn_bwd_supported(c.head_dim, c.n_q_heads, c.n_kv_heads, T);
+}
+
 int bwd_layout(const Model& m, int B, int T, char* base, BwdLayout* L) {
     const qk_config& c = m.cfg;
     const size_t es = m.es, M = (size_t)B * T, H = c.hidden, d = c.head_dim, nq = c.n_q_heads,
@@ -114,13 +121,15 @@ int bwd_layout(const Model& m, int B, int T, char* base, BwdLayout* L) {
     L->lse_h = (float*)take(Mc * 4);
     L->zt = (float*)take(Mc * 4);
     L->dz = take(Mc * V * es);
+    // the bf16 head_dim-128 path runs the fused attention backward: no [T, T] blocks
+    const bool fused_attn = fused_attn_bwd(m, T);
     L->st_a = (float2*)take(Z * T * nct_a * 8);
-    L->P = take(Z * T * T * es);
+    L->P = fused_attn ? nullptr : take(Z * T * T * es);
     L->dgu = take(M * 2 * I * es);
     L->du = (float*)take(M * H * 4);
     L->dO = take(M * nq * d * es);
     L->Dv = (float*)take(Z * T * 4);
-    L->dS = take(Z * T * T * es);
+    L->dS = fused_attn ? nullptr : take(Z * T * T * es);
     L->dqr = (float*)take(M * nq * d * 4);
     L->dkr = (float*)take(M * nkv * d * 4);
     L->dqkv = take(M * nqkv * es);
@@ -366,6 +375,13 @@ int layer_bwd(const Ctx& x, int l, float* const* G, bool acc) {
     QK_TRY(lin_dw(x, L.dx_act, H, H, 0, 128, H, O, nq * d, nq * d, G[6], acc, M));
     QK_TRY(lin_dx(x, L.dx_act, H, W.w_o, H, nq * d, L.dO, E_ACT, M));
     launch_attn_d(L.dO, O, M, T, nq, d, L.Dv, c.dtype, x.s);
+    if (fused_attn_bwd(m, T)) {  // P and dS stay on chip (k_attn_bwd.cu)
+        QK_TRY_CUDA(cudaMemsetAsync(L.dqr, 0, (size_t)M * nq * d * 4, x.s));
+        const int rc = launch_attn_bwd((const bf16*)qr, (const bf16*)L.dO, (const bf16*)kvh,
+                                       (const float*)L.lse_a.at(l), L.Dv, L.dqr, L.dkr, (bf16*)L.dqkv, nqkv,
+                                       (nq + nkv) * d, x.B, T, nq, nkv, m.num_sms, m.status, x.s);
+        if (rc != QK_OK) return set_error(rc, "fused attention backward launch");
+    } else {
     // P again from the stored log-sum-exp, then dS = P (dO V^T - D) / sqrt(d)
     QK_TRY(probs(x, l));
     Gemm g{};
@@ -422,6 +438,7 @@ int layer_bwd(const Ctx& x, int l, float* const* G, bool acc) {
     gv.out.zrow = T;
     gv.out.zcol = d;
     QK_TRY(run_gemm(m, gv, x.s));
+    }
     // ---- QK-norm + RoPE, then the projections
     launch_qk_bwd(L.dqr, L.dkr, qkv, nqkv, M, T, nq, nkv, d, W.q_norm, W.k_norm, eps, m.rope_cos,
                   m.rope_sin, L.dqkv, L.part, c.dtype, x.s);

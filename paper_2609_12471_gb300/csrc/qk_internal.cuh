@@ -373,6 +373,14 @@ int launch_attn_prefill(const bf16* q, int q_ld, const void* k_layer, int nq, in
                         int max_batch, int max_seq, int B, int T, int start,
                         const int32_t* start_dev, bf16* o, int num_sms, uint32_t* status,
                         cudaStream_t s, float* lse = nullptr);
+// Fused causal attention backward on tcgen05 (k_attn_bwd.cu): head_dim 128, T % 128 == 0.
+// q, dO [B T, nq d] bf16; kvh [2][B][nkv][T][d] bf16 (K then V); lse, D [B nq T] fp32;
+// dq [B T, nq d] fp32 (zero on entry: added into); dk [B T, nkv d] fp32; dv at columns
+// dv_col0 .. of dv_base [B T, dv_ld] bf16.
+bool attn_bwd_supported(int d, int nq, int nkv, int T);
+int launch_attn_bwd(const bf16* q, const bf16* dO, const bf16* kvh, const float* lse, const float* D,
+                    float* dq, float* dk, bf16* dv_base, int dv_ld, int dv_col0, int B, int T, int nq, int nkv,
+                    int num_sms, uint32_t* status, cudaStream_t s);
 // Split tensor-core decode attention (k_attn_decode.cu); head_dim 128, G <= 8.
 void attn_decode_split(int B, int nkv, int max_seq, int num_sms, int* chunk, int* n_split);
 size_t attn_decode_scratch_bytes(int B, int nq, int nkv, int max_seq, int num_sms);
