@@ -162,11 +162,16 @@ __global__ void __launch_bounds__(kThreads, 1)
                             break;
                         }
                         const int qrow = b * a.T + i * kT, qcol = (g * G + h) * kD;
-                        tc::mbar_expect_tx(qd_full, 2 * kTile);
+                        const size_t r0 = ((size_t)b * a.nq + g * G + h) * a.T + (size_t)i * kT;
+                        tc::mbar_expect_tx(qd_full, 2 * kTile + 2 * 128 * 4);
                         tc::tma_load_2d(sQ, &mQ, qcol, qrow, qd_full);
                         tc::tma_load_2d(sQ + 16384, &mQ, qcol + 64, qrow, qd_full);
                         tc::tma_load_2d(sDO, &mDO, qcol, qrow, qd_full);
                         tc::tma_load_2d(sDO + 16384, &mDO, qcol + 64, qrow, qd_full);
+                        // the step's log-sum-exp and D rows (read by the epilogue before
+                        // the stage is released again)
+                        tc::bulk_load(sLse, a.lse + r0, 128 * 4, qd_full);
+                        tc::bulk_load(sD, a.D + r0, 128 * 4, qd_full);
                         qd_armed = st & 1;
                     }
                 }
@@ -227,9 +232,11 @@ __global__ void __launch_bounds__(kThreads, 1)
                             const uint32_t acc = (e > 0 || kk > 0) ? 1u : 0u;
                             tc::mma_bf16(tmem + 256, km(aP, kk), mn(aDO, kk), id_km, acc);   // dV += P^T dO
                             tc::mma_bf16(tmem + 384, km(aDS, kk), mn(aQ, kk), id_km, acc);   // dK += dS^T Q
-                            tc::mma_bf16(tmem + 0, mn(aDS, kk), mn(aK, kk), id_mm, kk ? 1u : 0u);  // dQ = dS K
                         }
-                        tc::mma_commit(qd_empty);
+                        tc::mma_commit(qd_empty);  // Q and dO read: the next step's copies may start
+#pragma unroll
+                        for (int kk = 0; kk < kT / 16; ++kk)
+                            tc::mma_bf16(tmem + 0, mn(aDS, kk), mn(aK, kk), id_mm, kk ? 1u : 0u);  // dQ = dS K
                         tc::mma_commit(mm2_done);
                     }
                 }
@@ -245,7 +252,6 @@ __global__ void __launch_bounds__(kThreads, 1)
     } else {
         // ---------------------------------------------------- epilogue (warps 2..5)
         const int q = warp & 3;
-        const int et = threadIdx.x - 64;  // 0..127
         const int row = q * 32 + lane;    // key row (steps 1-2, dV / dK) or query row (dQ)
         const uint32_t lane_off = (uint32_t)(q * 32) << 16;
         uint8_t* stg = smem + kOffStage + q * 4096;
@@ -259,12 +265,10 @@ __global__ void __launch_bounds__(kThreads, 1)
             for (int h = 0; ok && h < G; ++h) {
                 const int hq = g * G + h;
                 for (int i = j; i < a.nt; ++i, ++st) {
-                    // the step's log-sum-exp (base 2) and D of its 128 queries
-                    const size_t r0 = ((size_t)b * a.nq + hq) * a.T + (size_t)i * kT;
-                    sLse[et] = a.lse[r0 + et] * kLog2e;
-                    sD[et] = a.D[r0 + et];
-                    tc::bar128();
-                    ok = tc::mbar_wait(sp_full, (uint32_t)(st & 1), abort_flag);
+                    // S^T and dP^T in TMEM; the step's log-sum-exp and D rows in shared
+                    // memory (copied with Q and dO)
+                    ok = tc::mbar_wait(sp_full, (uint32_t)(st & 1), abort_flag) &&
+                         tc::mbar_wait(qd_full, (uint32_t)(st & 1), abort_flag);
                     ok = tc::bar128_and(ok);
                     if (!ok) break;
                     tc::fence_after_sync();
@@ -272,22 +276,23 @@ __global__ void __launch_bounds__(kThreads, 1)
                     const bool diag = i == j;
                     uint8_t* prow = sP + (row >> 3) * 1024 + (row & 7) * 128;
                     uint8_t* drow = sDS + (row >> 3) * 1024 + (row & 7) * 128;
+#pragma unroll 1
+                    for (int c0 = 0; c0 < kT; c0 += 64) {  // 64 queries per TMEM wait
+                        uint32_t sr[4][16], dr[4][16];
 #pragma unroll
-                    for (int c0 = 0; c0 < kT; c0 += 32) {
-                        uint32_t sr[2][16], dr[2][16];
-                        tc::tmem_ld16(tmem + lane_off + c0, sr[0]);
-                        tc::tmem_ld16(tmem + lane_off + c0 + 16, sr[1]);
-                        tc::tmem_ld16(tmem + lane_off + 128 + c0, dr[0]);
-                        tc::tmem_ld16(tmem + lane_off + 128 + c0 + 16, dr[1]);
+                        for (int u = 0; u < 4; ++u) {
+                            tc::tmem_ld16(tmem + lane_off + c0 + 16 * u, sr[u]);
+                            tc::tmem_ld16(tmem + lane_off + 128 + c0 + 16 * u, dr[u]);
+                        }
                         tc::tmem_wait_ld();
-                        uint32_t pw[16], dw[16];
+                        uint32_t pw[32], dw[32];
 #pragma unroll
-                        for (int u = 0; u < 2; ++u) {
+                        for (int u = 0; u < 4; ++u) {
 #pragma unroll
                             for (int k2 = 0; k2 < 16; k2 += 2) {
                                 const int qc = c0 + 16 * u + k2;  // query column within the tile
-                                float p0 = ex2(fmaf(__uint_as_float(sr[u][k2]), c2, -sLse[qc]));
-                                float p1 = ex2(fmaf(__uint_as_float(sr[u][k2 + 1]), c2, -sLse[qc + 1]));
+                                float p0 = ex2(fmaf(__uint_as_float(sr[u][k2]), c2, -sLse[qc] * kLog2e));
+                                float p1 = ex2(fmaf(__uint_as_float(sr[u][k2 + 1]), c2, -sLse[qc + 1] * kLog2e));
                                 if (diag) {  // key after the query: masked
                                     if (qc < row) p0 = 0.f;
                                     if (qc + 1 < row) p1 = 0.f;
@@ -298,11 +303,11 @@ __global__ void __launch_bounds__(kThreads, 1)
                                 dw[u * 8 + k2 / 2] = pack2(d0, d1);
                             }
                         }
-                        // 32 queries = 4 granules of 16 B in box (c0 / 64), granules (c0 % 64) / 8 ..
-                        const int box = c0 >> 6, g0 = (c0 & 63) >> 3;
+                        // 64 queries = the 8 granules of box c0 / 64
+                        const int box = c0 >> 6;
 #pragma unroll
-                        for (int gi = 0; gi < 4; ++gi) {
-                            const int pos = ((g0 + gi) ^ (row & 7)) << 4;
+                        for (int gi = 0; gi < 8; ++gi) {
+                            const int pos = (gi ^ (row & 7)) << 4;
                             *reinterpret_cast<uint4*>(prow + box * 16384 + pos) =
                                 make_uint4(pw[4 * gi], pw[4 * gi + 1], pw[4 * gi + 2], pw[4 * gi + 3]);
                             *reinterpret_cast<uint4*>(drow + box * 16384 + pos) =
@@ -311,7 +316,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                     }
                     tc::fence_proxy_async_smem();
                     tc::fence_before_sync();
-                    tc::bar128();  // every row written; sLse / sD reads done
+                    __syncwarp();  // this warp's rows written and its sLse / sD reads done
                     if (lane == 0) tc::mbar_arrive(pds_ready);
                     // dQ of the step: TMEM columns [0, 128), one query row per thread
                     ok = tc::mbar_wait(mm2_done, (uint32_t)(st & 1), abort_flag);
@@ -319,30 +324,32 @@ __global__ void __launch_bounds__(kThreads, 1)
                     if (!ok) break;
                     tc::fence_after_sync();
                     const int qrow = b * a.T + i * kT + q * 32;
+                    {
+                        uint32_t r[8][16];  // the row's 128 dQ columns, one TMEM wait
 #pragma unroll
-                    for (int c0 = 0; c0 < kD; c0 += 32) {
-                        uint32_t r[2][16];
-                        tc::tmem_ld16(tmem + lane_off + c0, r[0]);
-                        tc::tmem_ld16(tmem + lane_off + c0 + 16, r[1]);
+                        for (int u = 0; u < 8; ++u) tc::tmem_ld16(tmem + lane_off + 16 * u, r[u]);
                         tc::tmem_wait_ld();
-                        if (lane == 0) tc::bulk_wait_read<0>();
+                        tc::fence_before_sync();
                         __syncwarp();
-                        uint4* srow = (uint4*)(stg + lane * 128);
+                        if (lane == 0) tc::mbar_arrive(s_free);  // TMEM columns [0, 128) free
 #pragma unroll
-                        for (int gi = 0; gi < 8; ++gi) {
-                            const uint32_t* w = &r[gi >> 2][(gi & 3) * 4];
-                            srow[gi ^ sw] = make_uint4(w[0], w[1], w[2], w[3]);
-                        }
-                        tc::fence_proxy_async_smem();
-                        __syncwarp();
-                        if (lane == 0) {
-                            tma_reduce_add_2d(&mDQ, hq * kD + c0, qrow, stg);
-                            tc::bulk_commit();
+                        for (int c = 0; c < 4; ++c) {  // 32 fp32 columns per reduction
+                            if (lane == 0) tc::bulk_wait_read<0>();
+                            __syncwarp();
+                            uint4* srow = (uint4*)(stg + lane * 128);
+#pragma unroll
+                            for (int gi = 0; gi < 8; ++gi) {
+                                const uint32_t* w = &r[2 * c + (gi >> 2)][(gi & 3) * 4];
+                                srow[gi ^ sw] = make_uint4(w[0], w[1], w[2], w[3]);
+                            }
+                            tc::fence_proxy_async_smem();
+                            __syncwarp();
+                            if (lane == 0) {
+                                tma_reduce_add_2d(&mDQ, hq * kD + 32 * c, qrow, stg);
+                                tc::bulk_commit();
+                            }
                         }
                     }
-                    tc::fence_before_sync();
-                    __syncwarp();
-                    if (lane == 0) tc::mbar_arrive(s_free);
                 }
             }
             if (!ok) break;
