@@ -270,7 +270,10 @@ int qk_grpo_coef(const float* lp, const float* lp_old, const float* lp_ref, int 
  * gradients, which are tensor-core operands, likewise); accumulation, norms,
  * softmax statistics, the residual gradient and every weight gradient are fp32.
  * Gain gradients sum in a fixed order; embedding rows that share a token are
- * added with fp32 atomics (order-dependent rounding only).  A token id outside
+ * added with fp32 atomics, and on bf16 models the attention's query gradient is
+ * summed over key tiles by reductions in memory: both round in an order that can
+ * differ between calls (a few 1e-3 of a gradient's norm after bf16 operands relay
+ * it).  A token id outside
  * [0, V) sets QK_STATUS_BAD_TOKEN and counts as 0. */
 int qk_backward_logprob(qk_model* m, const int32_t* tokens, int B, int T, const float* coef,
                         float* const* grads, int n_grads, int accumulate, float* loss,

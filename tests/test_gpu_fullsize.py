@@ -140,7 +140,7 @@ def test_backward_b2_t4096(q8b):
     the gradient that hold at any size: every entry finite; the lm_head gradient's columns
     sum to ~0 over the vocabulary (each row's softmax minus its one-hot sums to zero); the
     embedding rows of tokens that occur at no position < T - 1 are exactly zero, the others
-    are not; accumulate = 1 doubles it."""
+    are not; accumulate = 1 adds the same gradient again (to rounding order)."""
     import torch
     s, W, dec = q8b
     B, T = 2, 4096
@@ -167,7 +167,10 @@ def test_backward_b2_t4096(q8b):
     emb = grads[0][present].clone()
     dec.backward(tok, coef, grads, accumulate=True)
     torch.cuda.synchronize()
-    assert torch.allclose(grads[0][present], 2 * emb, rtol=1e-5, atol=1e-9)
+    # the second call adds the same gradient up to the order-dependent rounding of the
+    # dQ reduction and the embedding atomics (relayed through bf16 operands downstream)
+    second = grads[0][present] - emb
+    assert float((second - emb).norm() / emb.norm()) <= 1e-2
     del grads, emb
     dec._ws.clear()
     gc.collect()

@@ -69,7 +69,7 @@ def test_expired_wait_in_the_backward_gemm():
     """The same hook arms the next launch of the backward pass's batched tcgen05 GEMM (the
     first layer's QKV projection of the forward it runs): the status word reports the
     expired wait, and the next backward call on the same context gives the gradients of a
-    clean run again."""
+    clean run again (to rounding order)."""
     import torch
     import paper_2609_12471_gb300 as qk
     s = synth.ModelShape("bwd_bf16", 2, 512, 4, 2, 128, 256, 1024, "bf16")
@@ -91,7 +91,8 @@ def test_expired_wait_in_the_backward_gemm():
     torch.cuda.synchronize()
     assert dec.check_status() == 0
     for i, (a, b) in enumerate(zip(g0, g1)):
-        # bit-identical except the embedding rows, whose repeated tokens add in any order
-        tol = 1e-6 * float(a.abs().max()) if i == 0 else 0.0
-        assert float((a - b).abs().max()) <= tol, i
+        # equal up to the order-dependent rounding of the attention dQ reduction and the
+        # embedding atomics (bf16 operands downstream relay it); a gradient computed from
+        # the timed-out launch's undefined output would differ by O(1)
+        assert float((a - b).norm() / a.norm()) <= 1e-2, i
     dec.close()
