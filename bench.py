@@ -532,7 +532,7 @@ def backward_config(dec, dev, stream, rank, world):
            "roofline": {"bound": "tensor", "flops_per_call": fl, "achieved": fl / t / 1e12,
                         "peak": sustained, "unit": "TFLOP/s", "frac": fl / t / 1e12 / sustained,
                         "peak_source": "measured (sustained)" if peaks else "fallback",
-                        "dominant_kernel": "gemm_bwd_tc_kernel<256, 1, 1, E_F32> (weight gradients dW = dY^T X)"},
+                        "dominant_kernel": "gemm_bwd_tc_kernel<256, 256, 1, 1, E_F32> (weight gradients dW = dY^T X)"},
            "e2e": {"tokens_per_s": world * B_ * T_ / e2e, "h2d_bytes_per_call": int(tok_h.nbytes + coef_h.nbytes),
                    "d2h_bytes_per_call": 4},
            "loss": float(loss_h.item())}

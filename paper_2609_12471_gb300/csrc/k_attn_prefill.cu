@@ -7,9 +7,13 @@
 // kernel for positions >= start, by earlier calls below start).
 //
 // Persistent: one CTA per SM walks the work items (b, kv head, 128-query tile,
-// query head of the group) it, it + grid, ...; the query heads of a group are
-// adjacent in that order (so their CTAs stream the same K/V tiles from L2 at
-// about the same time) and the longer query tiles of a group come first.  The
+// query head of the group).  The (b, kv head) groups are taken in chunks small
+// enough for the chunk's K/V to stay in L2; inside a chunk the longest query tile
+// comes first, every (group, query head) pair of one tile before the next, the
+// query heads of a group adjacent (their CTAs stream the same K/V tiles from L2 at
+// about the same time).  The items are dealt to the CTAs in rounds of one item per
+// CTA, the CTA order reversed every other round, so the CTAs' sums of work even out
+// (work falls with the item index inside a chunk).  The
 // rings, TMEM buffers and barrier phases run on across items, so the next item's
 // Q and K/V copies overlap the current item's last tiles.  192 threads:
 //   warp 0, one lane : TMA producer: the Q tile of each item, then 128-key K and
@@ -38,6 +42,7 @@
 // Every mbarrier wait is bounded; on a timeout the CTA records
 // QK_STATUS_TIMEOUT, waits (bounded) for its copies and MMAs and exits without
 // writing.
+#include <algorithm>
 #include <cuda.h>
 
 #include "qk_internal.cuh"
@@ -69,20 +74,32 @@ __device__ __forceinline__ uint32_t pack2(float lo, float hi) {
     return *reinterpret_cast<uint32_t*>(&v);
 }
 
-// Work item `it` of a launch: (b, kv head) groups in order; inside a group the
-// longest query tile first, the group's query heads innermost.
+// Work item `it` of a launch: chunks of `chunk` (b, kv head) groups (the last one
+// may be shorter) in order; inside a chunk the query tiles longest first, inside a
+// tile the chunk's groups in order, the group's query heads innermost.
 struct Item {
     int b, g, h, q0;
 };
-__device__ __forceinline__ Item item_at(int it, int n_qt, int G, int nkv) {
-    const int per_bg = n_qt * G;
-    const int bg = it / per_bg, rem = it % per_bg;
+__device__ __forceinline__ Item item_at(int it, int n_qt, int G, int nkv, int n_groups, int chunk) {
+    const int per_chunk = chunk * n_qt * G;
+    const int g0 = (it / per_chunk) * chunk, rem = it % per_chunk;
+    const int per_tile = min(chunk, n_groups - g0) * G;
+    const int k = rem % per_tile;
+    const int bg = g0 + k / G;
     Item w;
     w.b = bg / nkv;
     w.g = bg % nkv;
-    w.h = w.g * G + rem % G;
-    w.q0 = (n_qt - 1 - rem / G) * kQT;
+    w.h = w.g * G + k % G;
+    w.q0 = (n_qt - 1 - rem / per_tile) * kQT;
     return w;
+}
+
+// This CTA's item in round r (one item per CTA per round, the CTA order reversed on
+// odd rounds), or -1 past the last item.
+__device__ __forceinline__ int item_of(int r, int n_work) {
+    const int c = (r & 1) ? (int)gridDim.x - 1 - (int)blockIdx.x : (int)blockIdx.x;
+    const int it = r * (int)gridDim.x + c;
+    return it < n_work ? it : -1;
 }
 
 // First position of row b (clamped into the cache; the cache-write kernel flags it).
@@ -100,7 +117,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     attn_prefill_kernel(const __grid_constant__ CUtensorMap tmQ,
                         const __grid_constant__ CUtensorMap tmKV, int nq, int nkv,
                         int max_batch, int max_seq, int start_all,
-                        const int32_t* __restrict__ start_dev, int T, int n_work,
+                        const int32_t* __restrict__ start_dev, int T, int n_work, int chunk,
                         bf16* __restrict__ o, float* __restrict__ lse, uint32_t* __restrict__ status) {
     extern __shared__ uint8_t smem_raw[];
     uint8_t* smem = (uint8_t*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
@@ -124,6 +141,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int G = nq / nkv;
     const int n_qt = (T + kQT - 1) / kQT;
+    const int n_groups = n_work / (n_qt * G);
 
     if (threadIdx.x == 0) {
         tc::mbar_init(q_full, 1);
@@ -183,8 +201,8 @@ __global__ void __launch_bounds__(kThreads, 1)
                 v_armed[st] = (g / kStages) & 1;
                 return true;
             };
-            for (int it = blockIdx.x; ok && it < n_work; it += gridDim.x, ++n) {
-                const Item w = item_at(it, n_qt, G, nkv);
+            for (int it; ok && (it = item_of(n, n_work)) >= 0; ++n) {
+                const Item w = item_at(it, n_qt, G, nkv, n_groups, chunk);
                 const int start = row_start(start_dev, start_all, w.b, max_seq, T);
                 const int n_kt = tiles_of(start, w.q0, T);
                 const int row0 = (w.b * nkv + w.g) * max_seq;
@@ -225,8 +243,8 @@ __global__ void __launch_bounds__(kThreads, 1)
             const uint32_t q_s = tc::smem_u32(sQ);
             bool ok = true, issued = false;
             int gt = 0, n = 0;
-            for (int it = blockIdx.x; ok && it < n_work; it += gridDim.x, ++n) {
-                const Item w = item_at(it, n_qt, G, nkv);
+            for (int it; ok && (it = item_of(n, n_work)) >= 0; ++n) {
+                const Item w = item_at(it, n_qt, G, nkv, n_groups, chunk);
                 const int n_kt = tiles_of(row_start(start_dev, start_all, w.b, max_seq, T), w.q0, T);
                 if (!tc::mbar_wait(q_full, (uint32_t)(n & 1), abort_flag)) {
                     ok = false;
@@ -291,8 +309,8 @@ __global__ void __launch_bounds__(kThreads, 1)
         const float c = rsqrtf((float)kD) * 1.4426950408889634f;  // 1/sqrt(d) in base 2
         bool ok = true;
         int gt = 0;
-        for (int it = blockIdx.x; ok && it < n_work; it += gridDim.x) {
-            const Item w = item_at(it, n_qt, G, nkv);
+        for (int r = 0, it; ok && (it = item_of(r, n_work)) >= 0; ++r) {
+            const Item w = item_at(it, n_qt, G, nkv, n_groups, chunk);
             const int start = row_start(start_dev, start_all, w.b, max_seq, T);
             const int n_kt = tiles_of(start, w.q0, T);
             const int kv_len = start + T;  // cache positions 0 .. kv_len-1 are written
@@ -508,8 +526,13 @@ int launch_attn_prefill(const bf16* q, int q_ld, const void* k_layer, int nq, in
     const int n_qt = (T + kQT - 1) / kQT;
     const int n_work = B * nq * n_qt;
     const int grid = n_work < num_sms ? n_work : num_sms;
+    // groups per chunk: a chunk's K and V (cache positions 0 .. start + T - 1, every
+    // position when the rows' starts are on the device) within 32 MB of L2
+    const size_t kv_len = start_dev ? (size_t)max_seq : (size_t)std::min(max_seq, start + T);
+    const size_t group_bytes = 2 * kv_len * kD * sizeof(bf16);
+    const int chunk = (int)std::min<size_t>((size_t)B * nkv, std::max<size_t>(1, ((size_t)32 << 20) / group_bytes));
     launch_k(attn_prefill_kernel, dim3(grid), dim3(kThreads), kSmem, s, mq, mkv, nq, nkv, max_batch,
-             max_seq, start, start_dev, T, n_work, o, lse, status);
+             max_seq, start, start_dev, T, n_work, chunk, o, lse, status);
     note_launch();
     return QK_OK;
 }
