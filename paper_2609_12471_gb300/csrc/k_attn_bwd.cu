@@ -8,9 +8,11 @@
 // dV and dK summed over the query heads of each GQA group.
 //
 // Work item = (row b, kv head g, 128-key tile j), heaviest (smallest j) first, dealt
-// to the CTAs in rounds whose CTA order reverses every round; one persistent CTA per SM, 192 threads: warp 0 lane 0 the TMA producer, warp 1 the
-// TMEM owner whose lane 0 issues the MMAs, warps 2..5 the epilogue (one key row, or
-// for dQ one query row, per thread).  Per item K_j and V_j are loaded once; per
+// to the CTAs in rounds whose CTA order reverses every round.  One persistent CTA per
+// SM, 320 threads: warp 0 lane 0 the TMA producer, warp 1 the TMEM owner whose lane 0
+// issues the MMAs, warps 2..9 the epilogue, two warps per TMEM lane quadrant (one key
+// row, or for dQ one query row, per thread; each warp of a pair takes half of the
+// columns).  Per item K_j and V_j are loaded once; per
 // step (query head h of the group, 128-query tile i >= j) Q and dO are loaded and
 //   1. S^T = K Q^T and dP^T = V dO^T (M 128 keys, N 128 queries, K = d) into TMEM
 //      columns [0, 128) and [128, 256);
@@ -36,10 +38,11 @@ namespace qk {
 namespace {
 
 constexpr int kD = 128, kT = 128;
-constexpr int kThreads = 192;
+constexpr int kThreads = 320;
+constexpr int kEpiWarps = 8;
 constexpr int kTile = 2 * 16384;  // 128 rows x 128 bf16 as two 64-column boxes
 constexpr int kOffK = 0, kOffV = kTile, kOffQ = 2 * kTile, kOffDO = 3 * kTile, kOffP = 4 * kTile,
-              kOffDS = 5 * kTile, kOffStage = 6 * kTile, kOffLse = kOffStage + 4 * 4096,
+              kOffDS = 5 * kTile, kOffStage = 6 * kTile, kOffLse = kOffStage + kEpiWarps * 4096,
               kOffBar = kOffLse + 2 * 128 * 4;
 constexpr int kSmem = kOffBar + 256 + 1024;
 static_assert(kSmem <= 232448, "shared memory per CTA");
@@ -59,6 +62,22 @@ __device__ __forceinline__ void tma_reduce_add_2d(const CUtensorMap* map, int x,
                      map),
                  "r"(x), "r"(y), "r"(tc::smem_u32(src))
                  : "memory");
+}
+
+// Named barrier 1 over the epilogue warps; returns whether `pred` held in all of them.
+__device__ __forceinline__ bool epi_bar_and(bool pred) {
+    uint32_t r;
+    asm volatile(
+        "{\n"
+        ".reg .pred p, q;\n"
+        "setp.ne.u32 p, %1, 0;\n"
+        "bar.red.and.pred q, 1, %2, p;\n"
+        "selp.u32 %0, 1, 0, q;\n"
+        "}\n"
+        : "=r"(r)
+        : "r"((uint32_t)pred), "n"(kEpiWarps * 32)
+        : "memory");
+    return r != 0;
 }
 
 struct Args {
@@ -125,11 +144,11 @@ __global__ void __launch_bounds__(kThreads, 1)
         tc::mbar_init(qd_full, 1);
         tc::mbar_init(qd_empty, 1);
         tc::mbar_init(sp_full, 1);
-        tc::mbar_init(pds_ready, 4);
+        tc::mbar_init(pds_ready, kEpiWarps);
         tc::mbar_init(mm2_done, 1);
-        tc::mbar_init(s_free, 4);
+        tc::mbar_init(s_free, kEpiWarps);
         tc::mbar_init(acc_full, 1);
-        tc::mbar_init(acc_free, 4);
+        tc::mbar_init(acc_free, kEpiWarps);
         tc::mbar_init(drain, 1);
         *abort_flag = 0;
         tc::fence_mbar_init();
@@ -260,11 +279,12 @@ __global__ void __launch_bounds__(kThreads, 1)
             }
         }
     } else {
-        // ---------------------------------------------------- epilogue (warps 2..5)
-        const int q = warp & 3;
+        // ---------------------------------------------------- epilogue (warps 2..9)
+        const int q = warp & 3;           // TMEM lane quadrant
+        const int half = (warp - 2) >> 2;  // columns [64 half, 64 half + 64) of each tile
         const int row = q * 32 + lane;    // key row (steps 1-2, dV / dK) or query row (dQ)
         const uint32_t lane_off = (uint32_t)(q * 32) << 16;
-        uint8_t* stg = smem + kOffStage + q * 4096;
+        uint8_t* stg = smem + kOffStage + (warp - 2) * 4096;
         const int sw = lane & 7;
         const float c2 = a.scale * kLog2e;
         bool ok = true;
@@ -279,25 +299,26 @@ __global__ void __launch_bounds__(kThreads, 1)
                     // memory (copied with Q and dO)
                     ok = tc::mbar_wait(sp_full, (uint32_t)(st & 1), abort_flag) &&
                          tc::mbar_wait(qd_full, (uint32_t)(st & 1), abort_flag);
-                    ok = tc::bar128_and(ok);
+                    ok = epi_bar_and(ok);
                     if (!ok) break;
                     tc::fence_after_sync();
-                    // 2. P^T and dS^T of this key row, 32 queries at a time
+                    // 2. P^T and dS^T of this key row and the warp's 64 queries (the box
+                    // `half` of the tile), 32 queries per TMEM wait
                     const bool diag = i == j;
-                    uint8_t* prow = sP + (row >> 3) * 1024 + (row & 7) * 128;
-                    uint8_t* drow = sDS + (row >> 3) * 1024 + (row & 7) * 128;
+                    uint8_t* prow = sP + half * 16384 + (row >> 3) * 1024 + (row & 7) * 128;
+                    uint8_t* drow = sDS + half * 16384 + (row >> 3) * 1024 + (row & 7) * 128;
 #pragma unroll 1
-                    for (int c0 = 0; c0 < kT; c0 += 64) {  // 64 queries per TMEM wait
-                        uint32_t sr[4][16], dr[4][16];
+                    for (int c0 = half * 64; c0 < half * 64 + 64; c0 += 32) {
+                        uint32_t sr[2][16], dr[2][16];
 #pragma unroll
-                        for (int u = 0; u < 4; ++u) {
+                        for (int u = 0; u < 2; ++u) {
                             tc::tmem_ld16(tmem + lane_off + c0 + 16 * u, sr[u]);
                             tc::tmem_ld16(tmem + lane_off + 128 + c0 + 16 * u, dr[u]);
                         }
                         tc::tmem_wait_ld();
-                        uint32_t pw[32], dw[32];
+                        uint32_t pw[16], dw[16];
 #pragma unroll
-                        for (int u = 0; u < 4; ++u) {
+                        for (int u = 0; u < 2; ++u) {
 #pragma unroll
                             for (int k2 = 0; k2 < 16; k2 += 2) {
                                 const int qc = c0 + 16 * u + k2;  // query column within the tile
@@ -313,14 +334,13 @@ __global__ void __launch_bounds__(kThreads, 1)
                                 dw[u * 8 + k2 / 2] = pack2(d0, d1);
                             }
                         }
-                        // 64 queries = the 8 granules of box c0 / 64
-                        const int box = c0 >> 6;
+                        // 32 queries = granules (c0 % 64) / 8 .. + 3 of the row in box `half`
 #pragma unroll
-                        for (int gi = 0; gi < 8; ++gi) {
-                            const int pos = (gi ^ (row & 7)) << 4;
-                            *reinterpret_cast<uint4*>(prow + box * 16384 + pos) =
+                        for (int gi = 0; gi < 4; ++gi) {
+                            const int pos = ((((c0 & 63) >> 3) + gi) ^ (row & 7)) << 4;
+                            *reinterpret_cast<uint4*>(prow + pos) =
                                 make_uint4(pw[4 * gi], pw[4 * gi + 1], pw[4 * gi + 2], pw[4 * gi + 3]);
-                            *reinterpret_cast<uint4*>(drow + box * 16384 + pos) =
+                            *reinterpret_cast<uint4*>(drow + pos) =
                                 make_uint4(dw[4 * gi], dw[4 * gi + 1], dw[4 * gi + 2], dw[4 * gi + 3]);
                         }
                     }
@@ -328,22 +348,23 @@ __global__ void __launch_bounds__(kThreads, 1)
                     tc::fence_before_sync();
                     __syncwarp();  // this warp's rows written and its sLse / sD reads done
                     if (lane == 0) tc::mbar_arrive(pds_ready);
-                    // dQ of the step: TMEM columns [0, 128), one query row per thread
+                    // dQ of the step: TMEM columns [0, 128), one query row per thread, the
+                    // warp's 64 columns
                     ok = tc::mbar_wait(mm2_done, (uint32_t)(st & 1), abort_flag);
                     ok = __all_sync(0xffffffffu, ok);
                     if (!ok) break;
                     tc::fence_after_sync();
                     const int qrow = b * a.T + i * kT + q * 32;
                     {
-                        uint32_t r[8][16];  // the row's 128 dQ columns, one TMEM wait
+                        uint32_t r[4][16];  // the row's 64 dQ columns, one TMEM wait
 #pragma unroll
-                        for (int u = 0; u < 8; ++u) tc::tmem_ld16(tmem + lane_off + 16 * u, r[u]);
+                        for (int u = 0; u < 4; ++u) tc::tmem_ld16(tmem + lane_off + half * 64 + 16 * u, r[u]);
                         tc::tmem_wait_ld();
                         tc::fence_before_sync();
                         __syncwarp();
                         if (lane == 0) tc::mbar_arrive(s_free);  // TMEM columns [0, 128) free
 #pragma unroll
-                        for (int c = 0; c < 4; ++c) {  // 32 fp32 columns per reduction
+                        for (int c = 0; c < 2; ++c) {  // 32 fp32 columns per reduction
                             if (lane == 0) tc::bulk_wait_read<0>();
                             __syncwarp();
                             uint4* srow = (uint4*)(stg + lane * 128);
@@ -355,7 +376,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                             tc::fence_proxy_async_smem();
                             __syncwarp();
                             if (lane == 0) {
-                                tma_reduce_add_2d(&mDQ, hq * kD + 32 * c, qrow, stg);
+                                tma_reduce_add_2d(&mDQ, hq * kD + half * 64 + 32 * c, qrow, stg);
                                 tc::bulk_commit();
                             }
                         }
@@ -369,8 +390,8 @@ __global__ void __launch_bounds__(kThreads, 1)
             if (!ok) break;
             tc::fence_after_sync();
             const int krow = b * a.T + j * kT + q * 32;
-#pragma unroll
-            for (int c0 = 0; c0 < kD; c0 += 64) {  // dV: 64 bf16 columns per store
+            {  // dV: the warp's 64 bf16 columns, one store
+                const int c0 = half * 64;
                 uint32_t r[4][16];
 #pragma unroll
                 for (int u = 0; u < 4; ++u) tc::tmem_ld16(tmem + lane_off + 256 + c0 + 16 * u, r[u]);
@@ -394,7 +415,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 }
             }
 #pragma unroll
-            for (int c0 = 0; c0 < kD; c0 += 32) {  // dK: 32 fp32 columns per store
+            for (int c0 = half * 64; c0 < half * 64 + 64; c0 += 32) {  // dK: 32 fp32 columns per store
                 uint32_t r[2][16];
                 tc::tmem_ld16(tmem + lane_off + 384 + c0, r[0]);
                 tc::tmem_ld16(tmem + lane_off + 384 + c0 + 16, r[1]);
