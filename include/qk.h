@@ -64,6 +64,8 @@ extern "C" {
                                      drawable token: non-finite logits); 0 was used */
 #define QK_STATUS_BAD_POS 2u      /* position outside [0, max_seq); it was clamped */
 #define QK_STATUS_TIMEOUT 4u      /* a bounded device wait gave up                 */
+#define QK_STATUS_BAD_PAGE 8u     /* page-table entry outside [0, n_pages); page 0  */
+                                  /* was used in its place                         */
 
 /* Kinds of call for qk_workspace_bytes. */
 #define QK_CALL_DECODE 0   /* qk_decode_step / qk_decode_layer: B tokens          */
@@ -191,6 +193,52 @@ int qk_decode_layer(qk_model* m, int layer, void* kv, int max_batch, int max_seq
 int qk_prefill_rows(qk_model* m, void* kv, int max_batch, int max_seq, const int32_t* tokens,
                     int B, int T, const int32_t* start, const int32_t* len, float* last_logits,
                     void* workspace, size_t ws_bytes, void* stream);
+
+/* Paged KV cache.  The rollouts of one RL batch (Sec. "Execution-Aware
+ * Reinforcement Learning": G = 8 rollouts per prompt) and their appended turns
+ * (Sec. "Multi-Turn On-Policy Reflection") end at different lengths, so a
+ * dense cache that reserves max_seq positions for every row holds mostly
+ * unused positions.  A paged cache holds, per layer, a K pool then a V pool of
+ * n_pages pages, each [n_kv, page_size, d] in the model dtype (per layer
+ * 2 x n_pages x n_kv x page_size x d elements, layers contiguous: the bytes of
+ * qk_kv_bytes with max_batch = n_pages, max_seq = page_size; qk_kv_pages_bytes
+ * returns them).  Position p of row b lives at offset p % page_size of page
+ * table[b * per_row + p / page_size].  table: dev int32 [B, per_row], owned by
+ * the caller, read by every paged call and never written; an entry a call
+ * reaches (row b's pages up to its last position) must lie in [0, n_pages):
+ * one outside sets QK_STATUS_BAD_PAGE and page 0 is used in its place; entries
+ * beyond a row's last position are not read.  Rows may share a page that
+ * holds a common prefix (its positions written once, through one row), as long
+ * as no call writes positions of that page through another row.  A row holds per_row x page_size positions,
+ * which plays the part of max_seq (<= max_positions; workspace sizes:
+ * qk_workspace_bytes with max_seq = per_row x page_size).  page_size is a
+ * multiple of 128 (one tensor-core key tile never straddles two pages).  (A
+ * memory layout of this library; the paper does not describe cache memory.) */
+typedef struct qk_kv_pages {
+    const int32_t* table; /* dev int32 [B, per_row] page ids                  */
+    int per_row;          /* table entries per row                            */
+    int n_pages;          /* pages in each layer's K pool (and in its V pool) */
+    int page_size;        /* positions per page, a multiple of 128            */
+} qk_kv_pages;
+
+/* Bytes of a paged cache of n_pages pages of page_size positions (all layers).
+ * QK_ESHAPE unless n_pages >= 1 and page_size is a positive multiple of 128. */
+int qk_kv_pages_bytes(const qk_model* m, int n_pages, int page_size, size_t* bytes);
+
+/* qk_decode_step over a paged cache (same tokens, pos, outputs and workspace as
+ * qk_decode_step with max_seq = per_row x page_size; pos[b] < per_row x
+ * page_size, else QK_STATUS_BAD_POS and clamping). */
+int qk_decode_step_paged(qk_model* m, void* kv, const qk_kv_pages* pages, const int32_t* tokens,
+                         const int32_t* pos, int B, float* logits, const int32_t* targets,
+                         float* logprobs, int32_t* argmax, void* workspace, size_t ws_bytes,
+                         void* stream);
+
+/* qk_prefill_rows over a paged cache: prompts (start[b] = 0) and appended turns
+ * at per-row positions, the same arguments and rules as qk_prefill_rows with
+ * max_seq = per_row x page_size. */
+int qk_prefill_rows_paged(qk_model* m, void* kv, const qk_kv_pages* pages, const int32_t* tokens,
+                          int B, int T, const int32_t* start, const int32_t* len, float* last_logits,
+                          void* workspace, size_t ws_bytes, void* stream);
 
 /* Teacher-forced scoring (Eq. sft / Eq. ppo inputs): tokens dev int32 [B, T],
  * T >= 2.  logprobs dev fp32 [B, T-1]: logprobs[b, t] = log p(tokens[b, t+1] |

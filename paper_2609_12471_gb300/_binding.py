@@ -16,7 +16,7 @@ _LIB_FILE = os.path.join(PKG, "libqk.so")
 QK_OK, QK_EINVAL, QK_ESHAPE, QK_EDTYPE, QK_ECUDA, QK_ETIMEOUT, QK_EDEVICE, QK_ENOSPACE = (
     0, -1, -2, -3, -4, -5, -6, -7)
 QK_DTYPE_BF16, QK_DTYPE_F32 = 0, 1
-QK_STATUS_BAD_TOKEN, QK_STATUS_BAD_POS, QK_STATUS_TIMEOUT = 1, 2, 4
+QK_STATUS_BAD_TOKEN, QK_STATUS_BAD_POS, QK_STATUS_TIMEOUT, QK_STATUS_BAD_PAGE = 1, 2, 4, 8
 QK_CALL_DECODE, QK_CALL_PREFILL, QK_CALL_SCORE, QK_CALL_ROLLOUT, QK_CALL_BACKWARD = 0, 1, 2, 3, 4
 QK_PROF_QKV, QK_PROF_O, QK_PROF_GATE_UP, QK_PROF_DOWN, QK_PROF_ATTN, QK_PROF_LM_HEAD = range(6)
 QK_EPI_STORE, QK_EPI_STORE_F32, QK_EPI_RESID_F32, QK_EPI_SWIGLU = 0, 1, 2, 3
@@ -35,7 +35,8 @@ __all__ = [
     "QK_EPI_STORE_F32", "QK_EPI_RESID_F32", "QK_EPI_SWIGLU", "qk_op_linear_swiglu_static",
     "QK_STATIC_SCRATCH_BYTES", "qk_grpo_workspace_bytes", "qk_grpo_token_loss", "qk_score_grpo",
     "qk_rollout_sampled", "qk_prefill_rows", "qk_debug_expire_next_wait", "QK_CALL_BACKWARD",
-    "qk_grpo_coef", "qk_backward_logprob",
+    "qk_grpo_coef", "qk_backward_logprob", "QK_STATUS_BAD_PAGE", "qk_kv_pages", "qk_kv_pages_bytes",
+    "qk_decode_step_paged", "qk_prefill_rows_paged",
 ]
 
 
@@ -55,6 +56,13 @@ class qk_config(ctypes.Structure):
 
     def __repr__(self):
         return "qk_config(" + ", ".join(f"{n}={getattr(self, n)}" for n, _ in self._fields_) + ")"
+
+
+class qk_kv_pages(ctypes.Structure):
+    """Paged cache layout: table (device int32 [B, per_row] page ids), per_row,
+    n_pages, page_size (a multiple of 128)."""
+    _fields_ = [("table", ctypes.c_void_p), ("per_row", ctypes.c_int32),
+                ("n_pages", ctypes.c_int32), ("page_size", ctypes.c_int32)]
 
 
 def lib_path() -> str:
@@ -92,6 +100,11 @@ _SIGS = {
     "qk_debug_expire_next_wait": ([_P, ctypes.c_longlong], _I),
     "qk_grpo_coef": ([_P, _P, _P, _I, _I, _I, _P, _I, _P, _F, _F, _F, _P, _P, _P, _P, _SZ, _P], _I),
     "qk_backward_logprob": ([_P, _P, _I, _I, _P, ctypes.POINTER(_P), _I, _I, _P, _P, _SZ, _P], _I),
+    "qk_kv_pages_bytes": ([_P, _I, _I, ctypes.POINTER(_SZ)], _I),
+    "qk_decode_step_paged": ([_P, _P, ctypes.POINTER(qk_kv_pages), _P, _P, _I, _P, _P, _P, _P, _P, _SZ,
+                              _P], _I),
+    "qk_prefill_rows_paged": ([_P, _P, ctypes.POINTER(qk_kv_pages), _P, _I, _I, _P, _P, _P, _P, _SZ, _P],
+                              _I),
 }
 
 _lib = None
@@ -280,6 +293,33 @@ def qk_prefill_rows(m, kv, max_batch, max_seq, tokens, B, T, start, length=None,
     _check(_load().qk_prefill_rows(m, _ptr(kv), max_batch, max_seq, _ptr(tokens), B, T, _ptr(start),
                                    _ptr(length), _ptr(last_logits), _ptr(workspace),
                                    _nbytes(workspace, ws_bytes), _stream(stream)))
+
+
+def _pages(table, per_row, n_pages, page_size):
+    return qk_kv_pages(_ptr(table), per_row, n_pages, page_size)
+
+
+def qk_kv_pages_bytes(m, n_pages: int, page_size: int) -> int:
+    n = _SZ()
+    _check(_load().qk_kv_pages_bytes(m, n_pages, page_size, ctypes.byref(n)))
+    return n.value
+
+
+def qk_decode_step_paged(m, kv, table, per_row, n_pages, page_size, tokens, pos, B, logits=None,
+                         targets=None, logprobs=None, argmax=None, workspace=None, ws_bytes=None,
+                         stream=None):
+    pg = _pages(table, per_row, n_pages, page_size)
+    _check(_load().qk_decode_step_paged(m, _ptr(kv), ctypes.byref(pg), _ptr(tokens), _ptr(pos), B,
+                                        _ptr(logits), _ptr(targets), _ptr(logprobs), _ptr(argmax),
+                                        _ptr(workspace), _nbytes(workspace, ws_bytes), _stream(stream)))
+
+
+def qk_prefill_rows_paged(m, kv, table, per_row, n_pages, page_size, tokens, B, T, start, length=None,
+                          last_logits=None, workspace=None, ws_bytes=None, stream=None):
+    pg = _pages(table, per_row, n_pages, page_size)
+    _check(_load().qk_prefill_rows_paged(m, _ptr(kv), ctypes.byref(pg), _ptr(tokens), B, T, _ptr(start),
+                                         _ptr(length), _ptr(last_logits), _ptr(workspace),
+                                         _nbytes(workspace, ws_bytes), _stream(stream)))
 
 
 def qk_check_status(m, stream=None) -> int:

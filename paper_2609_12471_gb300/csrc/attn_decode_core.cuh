@@ -50,7 +50,8 @@ static_assert(4 * 8 * kD * 4 + 4 * 8 * 2 * 4 <= kRingBytes, "merge buffers");
 
 struct Args {
     const bf16* q;
-    int q_ld, nq, nkv, max_batch, max_seq;
+    int q_ld, nq, nkv;
+    KvPages kp;        // cache layout (paged: page % 64 == 0, so a 64-key tile stays in its page)
     PosIndex pos;
     int chunk, n_split;
     float* part_o;     // [B nq][n_split][128]
@@ -66,9 +67,10 @@ __device__ __forceinline__ uint32_t tile_addr(uint32_t tile, int key, int c) {
 }
 
 // Runs item (split, b, kvh) on 128 threads with thread index tid (0..127) and
-// warp = tid / 32.  ring: kRingBytes of 1024-aligned shared memory; full: its
+// warp = tid / 32.  PAGED: the cache is paged (a.kp.table set); else dense.  ring: kRingBytes of 1024-aligned shared memory; full: its
 // kStages mbarriers (count 1); tmKV: 3-D map of the caches ({128, rows, layers},
 // K rows first, then V rows), z: the layer.  *last_s: a shared int.
+template <bool PAGED>
 __device__ __forceinline__ int decode_item(const Args& a, const CUtensorMap* tmKV, int z, int split,
                                             int b, int kvh, uint8_t* ring, uint64_t* full,
                                             int& tiles, volatile int* abort_flag, int* last_s,
@@ -77,7 +79,7 @@ __device__ __forceinline__ int decode_item(const Args& a, const CUtensorMap* tmK
     using ms::ldsm_x4_t;
     using ms::mma16816;
     using ms::pack_bf16;
-    const int nq = a.nq, nkv = a.nkv, max_seq = a.max_seq;
+    const int nq = a.nq, nkv = a.nkv, cap = a.kp.cap();
     const int G = nq / nkv;
     const int warp = tid >> 5, lane = tid & 31;
     const int g = lane >> 2, tig = lane & 3;
@@ -85,7 +87,7 @@ __device__ __forceinline__ int decode_item(const Args& a, const CUtensorMap* tmK
     float* red_ml = red + 4 * 8 * kD;    // [4 warps][8 rows][2]
 
     int p = a.pos.pos_dev ? a.pos.pos_dev[b] : a.pos.start;
-    if (p < 0 || p >= max_seq) p = p < 0 ? 0 : max_seq - 1;  // flagged by the cache-write kernel
+    if (p < 0 || p >= cap) p = p < 0 ? 0 : cap - 1;  // flagged by the cache-write kernel
     // The row's key tiles 0 .. p/64 are cut into n_split equal runs at this row's own
     // position; `chunk` caps a run at the cost model's length.
     const int n_tiles_b = p / kTileKeys + 1;
@@ -95,15 +97,17 @@ __device__ __forceinline__ int decode_item(const Args& a, const CUtensorMap* tmK
     if (split >= n_valid) return 0;  // nothing to attend in this split; the merge skips it
     const int k_end = min(k_begin + per * kTileKeys, p + 1);
     const int n_tiles = (k_end - k_begin + kTileKeys - 1) / kTileKeys;
-    // Row of key 0 of (b, kvh) in the 2-D view of a layer's K (V follows after max_batch*nkv*max_seq rows).
-    const int row0 = (b * nkv + kvh) * max_seq;
-    const int v_off = a.max_batch * nkv * max_seq;
+    // V's pool follows K's in the 2-D view of a layer's cache; a dense cache's row b is
+    // its page b, so the row of key k of (b, kvh) is row0 + k
+    const int v_off = a.kp.n_pages * nkv * a.kp.page;
+    const int row0 = (b * nkv + kvh) * a.kp.page;
 
     tc::bar128();  // the ring (and the previous item's merge buffers) is free
     auto issue = [&](int t) {
         const int st = (tiles + t) % kStages;
         uint8_t* base = ring + st * kStageBytes;
-        const int r = row0 + k_begin + t * kTileKeys;
+        const int r = PAGED ? kv_row(a.kp, nkv, b, kvh, k_begin + t * kTileKeys, a.status)
+                            : row0 + k_begin + t * kTileKeys;  // the tile's first key
         tc::mbar_expect_tx(&full[st], kStageBytes);
         tc::tma_load_3d(base, tmKV, 0, r, z, &full[st]);
         tc::tma_load_3d(base + kHalfBytes, tmKV, 64, r, z, &full[st]);

@@ -13,6 +13,8 @@ using attn::kD;
 using attn::kTileKeys;
 constexpr int kSmem = attn::kRingBytes + 1024 + 256;
 
+// PAGED: the cache is paged (one instance each, so the dense one pays no page lookup)
+template <bool PAGED>
 __global__ void __launch_bounds__(128)
     attn_decode_kernel(const __grid_constant__ CUtensorMap tmKV, const __grid_constant__ attn::Args a) {
     extern __shared__ uint8_t smem_raw[];
@@ -31,8 +33,8 @@ __global__ void __launch_bounds__(128)
     }
     __syncthreads();
     int tiles = 0;
-    attn::decode_item(a, &tmKV, 0, blockIdx.x, blockIdx.y / a.nkv, blockIdx.y % a.nkv, smem, full,
-                      tiles, abort_flag, last_s, threadIdx.x);
+    attn::decode_item<PAGED>(a, &tmKV, 0, blockIdx.x, blockIdx.y / a.nkv, blockIdx.y % a.nkv, smem, full,
+                             tiles, abort_flag, last_s, threadIdx.x);
 }
 
 typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*,
@@ -93,15 +95,15 @@ void attn_scratch_parts(void* scratch, int B, int nq, int nkv, int max_seq, int 
 // 3-D map over the K / V caches of `layers` layers (layer stride layer_bytes): rows of
 // 128 bf16 elements, K rows of a layer first, then its V rows; 64 x 64-row boxes,
 // 128-byte swizzle.
-bool make_kv_map(CUtensorMap* map, const void* k_layer0, int max_batch, int nkv, int max_seq,
-                 int layers, size_t layer_bytes) {
+bool make_kv_map(CUtensorMap* map, const void* k_layer0, const KvPages& kp, int nkv, int layers,
+                 size_t layer_bytes) {
     void* fn = nullptr;
     cudaDriverEntryPointQueryResult qr;
     if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000, cudaEnableDefault,
                                          &qr) != cudaSuccess ||
         qr != cudaDriverEntryPointSuccess)
         return false;
-    const size_t rows = 2 * (size_t)max_batch * nkv * max_seq;
+    const size_t rows = 2 * (size_t)kp.n_pages * nkv * kp.page;
     if (rows >= ((size_t)1 << 31)) return false;
     if (layers < 1) return false;
     if (layers == 1) layer_bytes = rows * kD * 2;
@@ -118,32 +120,37 @@ bool make_kv_map(CUtensorMap* map, const void* k_layer0, int max_batch, int nkv,
 bool attn_decode_supported(int d, int nq, int nkv) { return d == kD && nq / nkv <= 8; }
 
 int launch_attn_decode(const bf16* q, int q_ld, const void* k_layer, int nq, int nkv,
-                       int max_batch, int max_seq, int B, PosIndex pos, void* scratch,
+                       const KvPages& kp, int B, PosIndex pos, void* scratch,
                        bf16* o, int num_sms, uint32_t* status, cudaStream_t s) {
     static bool attr_set = false;
     if (!attr_set) {
-        if (cudaFuncSetAttribute(attn_decode_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+        if (cudaFuncSetAttribute(attn_decode_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 kSmem) != cudaSuccess ||
+            cudaFuncSetAttribute(attn_decode_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                  kSmem) != cudaSuccess)
             return QK_ECUDA;
         attr_set = true;
     }
     CUtensorMap map;
-    if (!make_kv_map(&map, k_layer, max_batch, nkv, max_seq, 1, 0)) return QK_ECUDA;
+    if (kp.table && kp.page % kTileKeys) return QK_ESHAPE;  // a paged tile must not cross a page
+    if (!make_kv_map(&map, k_layer, kp, nkv, 1, 0)) return QK_ECUDA;
     attn::Args a;
     a.q = q;
     a.q_ld = q_ld;
     a.nq = nq;
     a.nkv = nkv;
-    a.max_batch = max_batch;
-    a.max_seq = max_seq;
+    a.kp = kp;
     a.pos = pos;
-    attn_decode_split(B, nkv, max_seq, num_sms, &a.chunk, &a.n_split);
-    attn_scratch_parts(scratch, B, nq, nkv, max_seq, num_sms, a.n_split, &a.part_o, &a.part_ml,
+    attn_decode_split(B, nkv, kp.cap(), num_sms, &a.chunk, &a.n_split);
+    attn_scratch_parts(scratch, B, nq, nkv, kp.cap(), num_sms, a.n_split, &a.part_o, &a.part_ml,
                        &a.tickets);
     a.out = o;
     a.status = status;
     dim3 grid(a.n_split, B * nkv);
-    launch_k(attn_decode_kernel, grid, dim3(128), kSmem, s, map, a);
+    if (kp.table)
+        launch_k(attn_decode_kernel<true>, grid, dim3(128), kSmem, s, map, a);
+    else
+        launch_k(attn_decode_kernel<false>, grid, dim3(128), kSmem, s, map, a);
     note_launch(1);
     return QK_OK;
 }

@@ -116,7 +116,7 @@ __device__ __forceinline__ int tiles_of(int start, int q0, int T) {
 __global__ void __launch_bounds__(kThreads, 1)
     attn_prefill_kernel(const __grid_constant__ CUtensorMap tmQ,
                         const __grid_constant__ CUtensorMap tmKV, int nq, int nkv,
-                        int max_batch, int max_seq, int start_all,
+                        KvPages kp, int start_all,
                         const int32_t* __restrict__ start_dev, int T, int n_work, int chunk,
                         bf16* __restrict__ o, float* __restrict__ lse, uint32_t* __restrict__ status) {
     extern __shared__ uint8_t smem_raw[];
@@ -170,7 +170,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     tc::fence_after_sync();
     const uint32_t tmem_base = *tmem_slot;
     pdl_wait();  // q, K, V and the row starts come from the previous kernels
-    const int v_off = max_batch * nkv * max_seq;
+    const int v_off = kp.n_pages * nkv * kp.page;  // V's pool follows K's
+    const int max_seq = kp.cap();                  // positions a row holds
 
     if (warp == 0) {
         if (lane == 0) {
@@ -205,7 +206,9 @@ __global__ void __launch_bounds__(kThreads, 1)
                 const Item w = item_at(it, n_qt, G, nkv, n_groups, chunk);
                 const int start = row_start(start_dev, start_all, w.b, max_seq, T);
                 const int n_kt = tiles_of(start, w.q0, T);
-                const int row0 = (w.b * nkv + w.g) * max_seq;
+                // the row (in the cache view) of key tile j (paged: page % 128 == 0, so the
+                // tile lies in one page; dense: the rows past the row's end are masked)
+                auto tile_row = [&](int j) { return kv_row(kp, nkv, w.b, w.g, j * kKT, status); };
                 // the Q buffer is free once every S MMA of the previous item has completed
                 if (n > 0 && !tc::mbar_wait(q_empty, (uint32_t)((n - 1) & 1), abort_flag)) {
                     ok = false;
@@ -216,11 +219,11 @@ __global__ void __launch_bounds__(kThreads, 1)
                 tc::tma_load_2d(sQ + kBox, &tmQ, w.h * kD + 64, w.b * T + w.q0, q_full);
                 q_armed = n & 1;
                 for (int j = 0; j <= n_kt; ++j) {
-                    if (j < n_kt && !load_k(gt + j, row0 + j * kKT)) {
+                    if (j < n_kt && !load_k(gt + j, tile_row(j))) {
                         ok = false;
                         break;
                     }
-                    if (j >= 1 && !load_v(gt + j - 1, row0 + (j - 1) * kKT)) {
+                    if (j >= 1 && !load_v(gt + j - 1, tile_row(j - 1))) {
                         ok = false;
                         break;
                     }
@@ -499,7 +502,7 @@ bool make_map128(EncodeTiledFn fn, CUtensorMap* map, const void* base, size_t in
 bool attn_prefill_supported(int d, int nq, int nkv) { return d == kD && nq % nkv == 0; }
 
 int launch_attn_prefill(const bf16* q, int q_ld, const void* k_layer, int nq, int nkv,
-                        int max_batch, int max_seq, int B, int T, int start,
+                        const KvPages& kp, int B, int T, int start,
                         const int32_t* start_dev, bf16* o, int num_sms,
                         uint32_t* status, cudaStream_t s, float* lse) {
     static bool attr_set = false;
@@ -515,7 +518,9 @@ int launch_attn_prefill(const bf16* q, int q_ld, const void* k_layer, int nq, in
                                          &qr) != cudaSuccess ||
         qr != cudaDriverEntryPointSuccess)
         return QK_ECUDA;
-    const size_t rows = 2 * (size_t)max_batch * nkv * max_seq;
+    if (kp.table && kp.page % kKT) return QK_ESHAPE;  // a paged tile must not cross a page
+    const int max_seq = kp.cap();
+    const size_t rows = 2 * (size_t)kp.n_pages * nkv * kp.page;
     if (rows >= ((size_t)1 << 31) || (size_t)B * T >= ((size_t)1 << 31)) return QK_ESHAPE;
     // q rows are 16-byte aligned (q_ld % 8 == 0) and every box starts at a multiple of 64
     if (q_ld % 8 || ((uintptr_t)q & 15)) return QK_EINVAL;
@@ -531,8 +536,8 @@ int launch_attn_prefill(const bf16* q, int q_ld, const void* k_layer, int nq, in
     const size_t kv_len = start_dev ? (size_t)max_seq : (size_t)std::min(max_seq, start + T);
     const size_t group_bytes = 2 * kv_len * kD * sizeof(bf16);
     const int chunk = (int)std::min<size_t>((size_t)B * nkv, std::max<size_t>(1, ((size_t)32 << 20) / group_bytes));
-    launch_k(attn_prefill_kernel, dim3(grid), dim3(kThreads), kSmem, s, mq, mkv, nq, nkv, max_batch,
-             max_seq, start, start_dev, T, n_work, chunk, o, lse, status);
+    launch_k(attn_prefill_kernel, dim3(grid), dim3(kThreads), kSmem, s, mq, mkv, nq, nkv, kp, start,
+             start_dev, T, n_work, chunk, o, lse, status);
     note_launch();
     return QK_OK;
 }

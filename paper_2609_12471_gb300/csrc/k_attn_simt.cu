@@ -38,7 +38,7 @@ __device__ __forceinline__ float row_dot(const T* __restrict__ row, const float*
 
 template <typename T, int D>
 __global__ void attention_simt_kernel(const T* __restrict__ q, int q_ld, const T* __restrict__ kc,
-                                      const T* __restrict__ vc, int nq, int nkv, int max_seq,
+                                      const T* __restrict__ vc, int nq, int nkv, KvPages kp,
                                       PosIndex pos, T* __restrict__ o, uint32_t* status) {
     constexpr int E = D / 32;
     extern __shared__ float qs[];  // [warps][D]
@@ -48,9 +48,10 @@ __global__ void attention_simt_kernel(const T* __restrict__ q, int q_ld, const T
     int r = blockIdx.x, kvh = blockIdx.y, h = kvh * group + warp;
     int b = r / pos.T, t = r % pos.T;
     int p = pos.pos_dev ? pos.pos_dev[b] + t : pos.start + t;
-    if (p < 0 || p >= max_seq) {
+    const int cap = kp.cap();
+    if (p < 0 || p >= cap) {
         if (lane == 0) atomicOr(status, QK_STATUS_BAD_POS);
-        p = p < 0 ? 0 : max_seq - 1;
+        p = p < 0 ? 0 : cap - 1;
     }
     float* qw = qs + warp * D;
     const T* qrow = q + (size_t)r * q_ld + (size_t)h * D;
@@ -58,14 +59,15 @@ __global__ void attention_simt_kernel(const T* __restrict__ q, int q_ld, const T
 #pragma unroll
     for (int i = 0; i < E; ++i) qw[lane + 32 * i] = to_f(qrow[lane + 32 * i]) * scale;
     __syncwarp();
-    const T* K = kc + ((size_t)b * nkv + kvh) * max_seq * D;
-    const T* Vv = vc + ((size_t)b * nkv + kvh) * max_seq * D;
+    // row of key position j in the K and V views
+    auto krow = [&](int j) { return (size_t)kv_row(kp, nkv, b, kvh, j, status) * D; };
     float m = -INFINITY, l = 0.f, acc[E];
 #pragma unroll
     for (int i = 0; i < E; ++i) acc[i] = 0.f;
     for (int kb = 0; kb <= p; kb += 32) {
         int j = kb + lane;
-        float s = j <= p ? row_dot<T, D>(K + (size_t)j * D, qw) : -INFINITY;
+        const size_t jr = j <= p ? krow(j) : 0;  // this lane's key's row in K and in V
+        float s = j <= p ? row_dot<T, D>(kc + jr, qw) : -INFINITY;
         float mb = s;
 #pragma unroll
         for (int off = 16; off > 0; off >>= 1) mb = fmaxf(mb, __shfl_xor_sync(0xffffffffu, mb, off));
@@ -81,7 +83,7 @@ __global__ void attention_simt_kernel(const T* __restrict__ q, int q_ld, const T
         int nk = p - kb + 1 < 32 ? p - kb + 1 : 32;
         for (int jj = 0; jj < nk; ++jj) {
             float w = __shfl_sync(0xffffffffu, pj, jj);
-            const T* vr = Vv + (size_t)(kb + jj) * D;
+            const T* vr = vc + __shfl_sync(0xffffffffu, jr, jj);
 #pragma unroll
             for (int i = 0; i < E; ++i) acc[i] += w * to_f(vr[lane + 32 * i]);
         }
@@ -96,7 +98,7 @@ __global__ void attention_simt_kernel(const T* __restrict__ q, int q_ld, const T
 }  // namespace
 
 void launch_attention_simt(const void* q, int q_ld, const void* k_cache, const void* v_cache,
-                           int dtype, int M, int nq, int nkv, int d, int max_seq, PosIndex pos,
+                           int dtype, int M, int nq, int nkv, int d, const KvPages& kp, PosIndex pos,
                            void* o, uint32_t* status, cudaStream_t s) {
     note_launch();
     if (M <= 0) return;
@@ -106,7 +108,7 @@ void launch_attention_simt(const void* q, int q_ld, const void* k_cache, const v
     size_t smem = (size_t)group * d * sizeof(float);
 #define QK_ATT(T, D)                                                                           \
     launch_k(attention_simt_kernel<T, D>, grid, dim3(threads), smem, s, (const T*)q, q_ld,    \
-             (const T*)k_cache, (const T*)v_cache, nq, nkv, max_seq, pos, (T*)o, status)
+             (const T*)k_cache, (const T*)v_cache, nq, nkv, kp, pos, (T*)o, status)
     if (dtype == QK_DTYPE_BF16) {
         if (d == 128) QK_ATT(bf16, 128); else QK_ATT(bf16, 64);
     } else {

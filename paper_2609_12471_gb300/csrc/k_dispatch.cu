@@ -34,31 +34,29 @@ void linear(Model& m, const void* A, int lda, const void* W, void* C, int ldc, i
 }
 
 void launch_attention(Model& m, const void* q, int q_ld, const void* k_cache, const void* v_cache,
-                      int M, int max_batch, int max_seq, PosIndex pos, void* o, void* scratch,
+                      int M, const KvPages& kp, PosIndex pos, void* o, void* scratch,
                       cudaStream_t s) {
     const qk_config& c = m.cfg;
+    // the tensor-core kernels address V as the rows after K's pool
+    const bool v_follows = (const char*)v_cache == (const char*)k_cache + (size_t)kp.n_pages * c.n_kv_heads *
+                                                                         kp.page * c.head_dim * 2;
     if (c.dtype == QK_DTYPE_BF16 && pos.T == 1 && scratch &&
-        attn_decode_supported(c.head_dim, c.n_q_heads, c.n_kv_heads) &&
-        (const char*)v_cache == (const char*)k_cache + (size_t)max_batch * c.n_kv_heads * max_seq *
-                                                            c.head_dim * 2) {
+        attn_decode_supported(c.head_dim, c.n_q_heads, c.n_kv_heads) && v_follows) {
         int rc = launch_attn_decode((const bf16*)q, q_ld, k_cache, c.n_q_heads, c.n_kv_heads,
-                                    max_batch, max_seq, M, pos, scratch, (bf16*)o, m.num_sms,
-                                    m.status, s);
+                                    kp, M, pos, scratch, (bf16*)o, m.num_sms, m.status, s);
         if (rc != QK_OK && !m.deferred_error) m.deferred_error = rc;
         return;
     }
     if (c.dtype == QK_DTYPE_BF16 && pos.T > 1 &&
-        attn_prefill_supported(c.head_dim, c.n_q_heads, c.n_kv_heads) &&
-        (const char*)v_cache == (const char*)k_cache + (size_t)max_batch * c.n_kv_heads * max_seq *
-                                                            c.head_dim * 2) {
+        attn_prefill_supported(c.head_dim, c.n_q_heads, c.n_kv_heads) && v_follows) {
         int rc = launch_attn_prefill((const bf16*)q, q_ld, k_cache, c.n_q_heads, c.n_kv_heads,
-                                     max_batch, max_seq, M / pos.T, pos.T, pos.start, pos.pos_dev,
+                                     kp, M / pos.T, pos.T, pos.start, pos.pos_dev,
                                      (bf16*)o, m.num_sms, m.status, s);
         if (rc != QK_OK && !m.deferred_error) m.deferred_error = rc;
         return;
     }
     launch_attention_simt(q, q_ld, k_cache, v_cache, c.dtype, M, c.n_q_heads, c.n_kv_heads,
-                          c.head_dim, max_seq, pos, o, m.status, s);
+                          c.head_dim, kp, pos, o, m.status, s);
 }
 
 }  // namespace qk

@@ -61,9 +61,9 @@ struct Cfg {
     static constexpr int ACC_COLS = SWIGLU ? 2 * BN : BN;
     static constexpr int TMEM_COLS = pow2_at_least(2 * ACC_COLS);
     // fused epilogue scratch (floats): s_row[64], p_row[64] (int), red[4][64], xch[BN][128],
-    // cos / sin [2][BN][64], flag
+    // cos / sin [2][BN][64], flag, c_row[64] (int)
     // plain GEMM: the EPI_LSE transpose buffer [16 tokens][128 features] and the tile's targets
-    static constexpr int FUSE_FLOATS = FUSED ? 64 + 64 + 4 * 64 + 128 * BN + 128 * BN + 4
+    static constexpr int FUSE_FLOATS = FUSED ? 64 + 64 + 4 * 64 + 128 * BN + 128 * BN + 4 + 64
                                              : 16 * 128 + (BN > 16 ? BN : 16);
     static constexpr int SMEM =
         STAGES * (A_BYTES + B_BYTES) + 1024 /*align*/ + 256 /*barriers*/ + FUSE_FLOATS * 4;
@@ -181,6 +181,7 @@ __device__ __forceinline__ bool fused_epilogue(const Fuse& fz, float* C, int ldc
     float* rope_c = xch + 128 * BN;       // [BN][64] cos / sin at each token's position (QKV)
     float* rope_s = rope_c + 64 * BN;
     volatile int* flag = (volatile int*)(rope_s + 64 * BN);
+    int* c_row = (int*)(rope_s + 64 * BN + 4);  // [64] cache row of kv head 0 per token (QKV)
     constexpr int kParts = 128 / BN;
     {
         // s_row[j] = rsqrt(sum_i ssq_in[i][j] / H + eps): 128 / BN threads per token
@@ -193,7 +194,7 @@ __device__ __forceinline__ bool fused_epilogue(const Fuse& fz, float* C, int ldc
             for (int i = part; i < fz.n_ssq; i += kParts) t += fz.ssq_in[(size_t)i * M + j];
         xch[part * BN + j] = t;
         if (fz.op == FUSE_QKV && e < BN) {
-            const int lim = fz.max_seq < fz.max_positions ? fz.max_seq : fz.max_positions;
+            const int lim = fz.kv.cap() < fz.max_positions ? fz.kv.cap() : fz.max_positions;
             int p = 0;
             if (e < M) {
                 p = fz.pos.pos_dev ? fz.pos.pos_dev[e] : fz.pos.start;
@@ -203,6 +204,8 @@ __device__ __forceinline__ bool fused_epilogue(const Fuse& fz, float* C, int ldc
                 }
             }
             p_row[e] = p;
+            // kv head g of the token sits g x page rows further: (page id x nkv + g) x page + offset
+            c_row[e] = e < M ? kv_row(fz.kv, fz.nkv, e, 0, p, fz.status) : 0;
         }
         epi_bar();
         if (e < BN) {
@@ -353,7 +356,7 @@ __device__ __forceinline__ bool fused_epilogue(const Fuse& fz, float* C, int ldc
                         if (hh < nq)
                             fz.q_out[(size_t)j * fz.q_ld + (size_t)hh * 128 + row] = __float2bfloat16_rn(o);
                         else
-                            fz.k_cache[(((size_t)j * nkv + (hh - nq)) * fz.max_seq + p_row[j]) * 128 + row] =
+                            fz.k_cache[(size_t)(c_row[j] + (hh - nq) * fz.kv.page) * 128 + row] =
                                 __float2bfloat16_rn(o);
                     }
                 }
@@ -361,7 +364,7 @@ __device__ __forceinline__ bool fused_epilogue(const Fuse& fz, float* C, int ldc
 #pragma unroll
                 for (int j = 0; j < BN; ++j)
                     if (j < M)
-                        fz.v_cache[(((size_t)j * nkv + (hh - nq - nkv)) * fz.max_seq + p_row[j]) * 128 + row] =
+                        fz.v_cache[(size_t)(c_row[j] + (hh - nq - nkv) * fz.kv.page) * 128 + row] =
                             __float2bfloat16_rn(v[j]);
             }
         } else if (fz.op == FUSE_RESID) {

@@ -149,7 +149,7 @@ __global__ void qk_norm_rope_kernel(T* __restrict__ qkv, int nq, int nkv, const 
                                     const float* __restrict__ gk, float eps,
                                     const float* __restrict__ rc, const float* __restrict__ rs,
                                     int max_positions, PosIndex pos, T* __restrict__ kc,
-                                    T* __restrict__ vc, int max_seq, uint32_t* status) {
+                                    T* __restrict__ vc, KvPages kp, uint32_t* status) {
     constexpr int E = D / 32, HALF = D / 2;
     pdl_wait();
     pdl_trigger();  // short kernel: let the next one launch and prefetch now
@@ -160,7 +160,7 @@ __global__ void qk_norm_rope_kernel(T* __restrict__ qkv, int nq, int nkv, const 
     int r = blockIdx.x;
     int b = r / pos.T, t = r % pos.T;
     int p = pos.pos_dev ? pos.pos_dev[b] + t : pos.start + t;
-    int lim = max_seq < max_positions ? max_seq : max_positions;
+    int lim = kp.cap() < max_positions ? kp.cap() : max_positions;
     if (p < 0 || p >= lim) {
         if (lane == 0) atomicOr(status, QK_STATUS_BAD_POS);
         p = p < 0 ? 0 : lim - 1;
@@ -171,7 +171,7 @@ __global__ void qk_norm_rope_kernel(T* __restrict__ qkv, int nq, int nkv, const 
     for (int i = 0; i < E; ++i) e[i] = to_f(src[lane + 32 * i]);
     if (hh >= nq + nkv) {  // value head: straight to the cache
         int kvh = hh - nq - nkv;
-        T* dst = vc + (((size_t)b * nkv + kvh) * max_seq + p) * D;
+        T* dst = vc + (size_t)kv_row(kp, nkv, b, kvh, p, lane == 0 ? status : nullptr) * D;
 #pragma unroll
         for (int i = 0; i < E; ++i) dst[lane + 32 * i] = src[lane + 32 * i];
         return;
@@ -199,7 +199,7 @@ __global__ void qk_norm_rope_kernel(T* __restrict__ qkv, int nq, int nkv, const 
         dst = src;
     } else {
         int kvh = hh - nq;
-        dst = kc + (((size_t)b * nkv + kvh) * max_seq + p) * D;
+        dst = kc + (size_t)kv_row(kp, nkv, b, kvh, p, lane == 0 ? status : nullptr) * D;
     }
 #pragma unroll
     for (int i = 0; i < E; ++i) dst[lane + 32 * i] = from_f<T>(e[i]);
@@ -208,13 +208,13 @@ __global__ void qk_norm_rope_kernel(T* __restrict__ qkv, int nq, int nkv, const 
 void launch_qk_norm_rope(void* qkv, int dtype, int M, int nq, int nkv, int d, const float* gq,
                          const float* gk, float eps, const float* rope_cos, const float* rope_sin,
                          int max_positions, PosIndex pos, void* k_cache, void* v_cache,
-                         int max_seq, uint32_t* status, cudaStream_t s) {
+                         const KvPages& kp, uint32_t* status, cudaStream_t s) {
     note_launch();
     if (M <= 0) return;
     dim3 grid(M, (nq + 2 * nkv + 7) / 8);
 #define QK_NR(T, D)                                                                          \
     launch_k(qk_norm_rope_kernel<T, D>, grid, dim3(256), 0, s, (T*)qkv, nq, nkv, gq, gk, eps,  \
-             rope_cos, rope_sin, max_positions, pos, (T*)k_cache, (T*)v_cache, max_seq, status)
+             rope_cos, rope_sin, max_positions, pos, (T*)k_cache, (T*)v_cache, kp, status)
     if (dtype == QK_DTYPE_BF16) {
         if (d == 128) QK_NR(bf16, 128); else QK_NR(bf16, 64);
     } else {

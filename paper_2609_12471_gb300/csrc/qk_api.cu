@@ -221,7 +221,7 @@ struct KVView {
     char* base;        // layer 0's K
     size_t layer_bytes;  // bytes from one layer's K to the next layer's K (0: shared scratch)
     size_t half_bytes;   // bytes from a layer's K to its V
-    int max_batch, max_seq;
+    KvPages kp;          // where a row's positions sit inside a layer's K (and V)
     void* k(int l) const { return base + (size_t)l * layer_bytes; }
     void* v(int l) const { return base + (size_t)l * layer_bytes + half_bytes; }
 };
@@ -229,7 +229,14 @@ struct KVView {
 static KVView cache_view(const Model& m, void* kv, int max_batch, int max_seq) {
     const qk_config& c = m.cfg;
     size_t half = (size_t)max_batch * c.n_kv_heads * max_seq * c.head_dim * m.es;
-    return KVView{(char*)kv, 2 * half, half, max_batch, max_seq};
+    return KVView{(char*)kv, 2 * half, half, KvPages::dense(max_batch, max_seq)};
+}
+
+// A paged cache: per layer a K pool then a V pool of n_pages pages.
+static KVView paged_view(const Model& m, void* kv, const qk_kv_pages& pg) {
+    const qk_config& c = m.cfg;
+    size_t half = (size_t)pg.n_pages * c.n_kv_heads * pg.page_size * c.head_dim * m.es;
+    return KVView{(char*)kv, 2 * half, half, KvPages{pg.table, pg.per_row, pg.n_pages, pg.page_size}};
 }
 
 static void run_layer(Model& m, int l, const Workspace& w, int M, PosIndex pos,
@@ -245,10 +252,10 @@ static void run_layer(Model& m, int l, const Workspace& w, int M, PosIndex pos,
     linear(m, w.u, H, L.w_qkv, w.qkv, nqkv, M, nqkv, H, EPI_STORE_ACT, w.gu, s);
     prof_close(m, pr, s);
     launch_qk_norm_rope(w.qkv, c.dtype, M, nq, nkv, d, L.q_norm, L.k_norm, eps, m.rope_cos,
-                        m.rope_sin, c.max_positions, pos, kv.k(l), kv.v(l), kv.max_seq, m.status,
+                        m.rope_sin, c.max_positions, pos, kv.k(l), kv.v(l), kv.kp, m.status,
                         s);
     pr = prof_open(m, QK_PROF_ATTN, s);
-    launch_attention(m, w.qkv, nqkv, kv.k(l), kv.v(l), M, kv.max_batch, kv.max_seq, pos, w.o,
+    launch_attention(m, w.qkv, nqkv, kv.k(l), kv.v(l), M, kv.kp, pos, w.o,
                      w.attn, s);
     prof_close(m, pr, s);
     pr = prof_open(m, QK_PROF_O, s);
@@ -300,12 +307,12 @@ static void run_layer_fused(Model& m, int l, const Workspace& w, int M, PosIndex
     fq.q_ld = nqkv;
     fq.k_cache = (bf16*)kv.k(l);
     fq.v_cache = (bf16*)kv.v(l);
-    fq.max_seq = kv.max_seq;
+    fq.kv = kv.kp;
     pr = prof_open(m, QK_PROF_QKV, s);
     gemm(w.xg, H, L.w_qkv, nqkv, H, fq);
     prof_close(m, pr, s);
     pr = prof_open(m, QK_PROF_ATTN, s);
-    launch_attention(m, w.qkv, nqkv, kv.k(l), kv.v(l), M, kv.max_batch, kv.max_seq, pos, w.o,
+    launch_attention(m, w.qkv, nqkv, kv.k(l), kv.v(l), M, kv.kp, pos, w.o,
                      w.attn, s);
     prof_close(m, pr, s);
     Fuse fo = f;
@@ -394,6 +401,25 @@ static int get_ws(const Model& m, int kind, int B, int T, int max_seq, void* ws,
     if (ws_bytes < w->total)
         return set_error(QK_ENOSPACE, "workspace has %zu bytes, needs %zu", ws_bytes, w->total);
     return workspace_layout(m, kind, B, T, max_seq, w, (char*)ws);
+}
+
+// A paged cache: the pool and table shapes (the table's contents are checked on the
+// device: an entry outside [0, n_pages) sets QK_STATUS_BAD_PAGE).
+static int check_pages(const Model& m, void* kv, const qk_kv_pages* pg, int B) {
+    if (!kv || !pg || !pg->table) return set_error(QK_EINVAL, "kv cache, pages or page table is NULL");
+    if (((uintptr_t)kv & 255) != 0) return set_error(QK_EINVAL, "kv cache must be 256-byte aligned");
+    if (((uintptr_t)pg->table & 3) != 0) return set_error(QK_EINVAL, "page table must be 4-byte aligned");
+    if (pg->n_pages < 1 || pg->per_row < 1 || pg->page_size < 128 || pg->page_size % 128)
+        return set_error(QK_ESHAPE, "n_pages %d, per_row %d, page_size %d (>= 1, >= 1, a multiple of 128)",
+                         pg->n_pages, pg->per_row, pg->page_size);
+    const long long cap = (long long)pg->per_row * pg->page_size;
+    if (cap > m.cfg.max_positions)
+        return set_error(QK_ESHAPE, "per_row x page_size = %lld exceeds the RoPE table (%d positions)", cap,
+                         m.cfg.max_positions);
+    if (2 * (long long)pg->n_pages * m.cfg.n_kv_heads * pg->page_size >= (1ll << 31))
+        return set_error(QK_ESHAPE, "a layer's pools exceed 2^31 rows of head_dim");
+    if (B < 1) return set_error(QK_ESHAPE, "batch %d < 1", B);
+    return QK_OK;
 }
 
 static int check_cache(const Model& m, void* kv, int max_batch, int max_seq, int B) {
@@ -630,6 +656,14 @@ int qk_kv_bytes(const qk_model* mh, int max_batch, int max_seq, size_t* bytes) {
     return QK_OK;
 }
 
+int qk_kv_pages_bytes(const qk_model* mh, int n_pages, int page_size, size_t* bytes) {
+    if (!mh || !bytes) return set_error(QK_EINVAL, "null argument");
+    if (n_pages < 1 || page_size < 128 || page_size % 128)
+        return set_error(QK_ESHAPE, "n_pages %d >= 1 and page_size %d a multiple of 128 are required", n_pages,
+                         page_size);
+    return qk_kv_bytes(mh, n_pages, page_size, bytes);  // the same bytes as n_pages rows of page_size
+}
+
 int qk_workspace_bytes(const qk_model* mh, int kind, int B, int T, int max_seq, size_t* bytes) {
     if (!mh || !bytes) return set_error(QK_EINVAL, "null argument");
     const Model& m = *(const Model*)mh;
@@ -651,14 +685,13 @@ int qk_workspace_bytes(const qk_model* mh, int kind, int B, int T, int max_seq, 
 
 // start_dev (dev [B] or null): per-row first positions instead of start_pos; row_len
 // (dev [B] or null): the head reads row b's token row_len[b] - 1 instead of T - 1.
-static int prefill_impl(Model& m, void* kv, int max_batch, int max_seq, TokIndex tok, int B, int T,
+static int prefill_impl(Model& m, const KVView& view, TokIndex tok, int B, int T,
                         int start_pos, float* last_logits, OutIndex oi, float* lp, int32_t* am,
                         void* ws, size_t ws_bytes, cudaStream_t s,
                         const int32_t* start_dev = nullptr, const int32_t* row_len = nullptr) {
     Workspace w;
-    QK_TRY(get_ws(m, QK_CALL_PREFILL, B, T, max_seq, ws, ws_bytes, &w));
+    QK_TRY(get_ws(m, QK_CALL_PREFILL, B, T, view.kp.cap(), ws, ws_bytes, &w));
     int M = B * T;
-    KVView view = cache_view(m, kv, max_batch, max_seq);
     launch_embed(m.embed, m.cfg.dtype, m.cfg.vocab, m.cfg.hidden, tok, M, w.x, m.status, s);
     PosIndex pos{start_dev, start_pos, T};
     for (int l = 0; l < m.cfg.n_layers; ++l) run_layer(m, l, w, M, pos, view, s);
@@ -679,8 +712,9 @@ int qk_prefill(qk_model* mh, void* kv, int max_batch, int max_seq, const int32_t
                          start_pos + T, max_seq);
     if (logprobs && !targets) return set_error(QK_EINVAL, "logprobs requested without targets");
     OutIndex oi{1, 1, 1, 0, targets, 1, 0, 0};
-    return prefill_impl(m, kv, max_batch, max_seq, TokIndex{tokens, T, T, 0}, B, T, start_pos,
-                        last_logits, oi, logprobs, argmax, workspace, ws_bytes, (cudaStream_t)stream);
+    return prefill_impl(m, cache_view(m, kv, max_batch, max_seq), TokIndex{tokens, T, T, 0}, B, T,
+                        start_pos, last_logits, oi, logprobs, argmax, workspace, ws_bytes,
+                        (cudaStream_t)stream);
 }
 
 int qk_prefill_rows(qk_model* mh, void* kv, int max_batch, int max_seq, const int32_t* tokens, int B,
@@ -691,17 +725,30 @@ int qk_prefill_rows(qk_model* mh, void* kv, int max_batch, int max_seq, const in
     QK_TRY(check_cache(m, kv, max_batch, max_seq, B));
     if (T < 1 || T > max_seq) return set_error(QK_ESHAPE, "T %d outside 1 .. max_seq %d", T, max_seq);
     OutIndex oi{1, 1, 1, 0, nullptr, 1, 0, 0};
-    return prefill_impl(m, kv, max_batch, max_seq, TokIndex{tokens, T, T, 0}, B, T, 0, last_logits,
-                        oi, nullptr, nullptr, workspace, ws_bytes, (cudaStream_t)stream, start, len);
+    return prefill_impl(m, cache_view(m, kv, max_batch, max_seq), TokIndex{tokens, T, T, 0}, B, T, 0,
+                        last_logits, oi, nullptr, nullptr, workspace, ws_bytes, (cudaStream_t)stream,
+                        start, len);
 }
 
-static int decode_impl(Model& m, void* kv, int max_batch, int max_seq, TokIndex tok, PosIndex pos,
+int qk_prefill_rows_paged(qk_model* mh, void* kv, const qk_kv_pages* pages, const int32_t* tokens,
+                          int B, int T, const int32_t* start, const int32_t* len, float* last_logits,
+                          void* workspace, size_t ws_bytes, void* stream) {
+    if (!mh || !tokens || !start) return set_error(QK_EINVAL, "null argument");
+    Model& m = *(Model*)mh;
+    QK_TRY(check_pages(m, kv, pages, B));
+    const int cap = pages->per_row * pages->page_size;
+    if (T < 1 || T > cap) return set_error(QK_ESHAPE, "T %d outside 1 .. per_row x page_size %d", T, cap);
+    OutIndex oi{1, 1, 1, 0, nullptr, 1, 0, 0};
+    return prefill_impl(m, paged_view(m, kv, *pages), TokIndex{tokens, T, T, 0}, B, T, 0, last_logits, oi,
+                        nullptr, nullptr, workspace, ws_bytes, (cudaStream_t)stream, start, len);
+}
+
+static int decode_impl(Model& m, const KVView& view, TokIndex tok, PosIndex pos,
                        int B, float* logits, OutIndex oi, float* lp, int32_t* am, void* ws,
                        size_t ws_bytes, cudaStream_t s) {
     Workspace w;
-    QK_TRY(get_ws(m, QK_CALL_DECODE, B, 1, max_seq, ws, ws_bytes, &w));
-    KVView view = cache_view(m, kv, max_batch, max_seq);
-    QK_TRY(clear_attn_tickets(m, w, B, max_seq, s));
+    QK_TRY(get_ws(m, QK_CALL_DECODE, B, 1, view.kp.cap(), ws, ws_bytes, &w));
+    QK_TRY(clear_attn_tickets(m, w, B, view.kp.cap(), s));
     m.in_decode = true;
     if (w.part) {
         const qk_config& c = m.cfg;
@@ -750,7 +797,21 @@ int qk_decode_step(qk_model* mh, void* kv, int max_batch, int max_seq, const int
     QK_TRY(check_cache(m, kv, max_batch, max_seq, B));
     if (logprobs && !targets) return set_error(QK_EINVAL, "logprobs requested without targets");
     OutIndex oi{1, 1, 1, 0, targets, 1, 0, 0};
-    return decode_impl(m, kv, max_batch, max_seq, TokIndex{tokens, 1, 1, 0}, PosIndex{pos, 0, 1}, B,
+    return decode_impl(m, cache_view(m, kv, max_batch, max_seq), TokIndex{tokens, 1, 1, 0},
+                       PosIndex{pos, 0, 1}, B, logits, oi, logprobs, argmax, workspace, ws_bytes,
+                       (cudaStream_t)stream);
+}
+
+int qk_decode_step_paged(qk_model* mh, void* kv, const qk_kv_pages* pages, const int32_t* tokens,
+                         const int32_t* pos, int B, float* logits, const int32_t* targets,
+                         float* logprobs, int32_t* argmax, void* workspace, size_t ws_bytes,
+                         void* stream) {
+    if (!mh || !tokens || !pos) return set_error(QK_EINVAL, "null argument");
+    Model& m = *(Model*)mh;
+    QK_TRY(check_pages(m, kv, pages, B));
+    if (logprobs && !targets) return set_error(QK_EINVAL, "logprobs requested without targets");
+    OutIndex oi{1, 1, 1, 0, targets, 1, 0, 0};
+    return decode_impl(m, paged_view(m, kv, *pages), TokIndex{tokens, 1, 1, 0}, PosIndex{pos, 0, 1}, B,
                        logits, oi, logprobs, argmax, workspace, ws_bytes, (cudaStream_t)stream);
 }
 
@@ -790,7 +851,7 @@ static int score_impl(Model& m, const int32_t* tokens, int B, int T, float* logp
     // One layer's K and V live in scratch shaped like a cache of B rows x T positions;
     // every layer reuses it (layer stride 0).
     size_t half = (size_t)B * m.cfg.n_kv_heads * T * m.cfg.head_dim * m.es;
-    KVView view{(char*)w.skv, 0, half, B, T};
+    KVView view{(char*)w.skv, 0, half, KvPages::dense(B, T)};
     launch_embed(m.embed, m.cfg.dtype, m.cfg.vocab, m.cfg.hidden, TokIndex{tokens, T, T, 0}, M, w.x,
                  m.status, s);
     PosIndex pos{nullptr, 0, T};
@@ -940,8 +1001,9 @@ static int rollout_impl(Model& m, qk_model* mh, void* kv, int max_batch, int max
     } scope(m, sampled);
     const int L = sampled ? P : P + N + 1;  // row length of seq
     OutIndex oi{1, 1, N + 1, 0, sampled ? nullptr : seq, L, P, 0};
-    QK_TRY(prefill_impl(m, kv, max_batch, max_seq, TokIndex{seq, P, L, 0}, B, P, 0, nullptr, oi,
-                        logprobs, argmax, workspace, ws_bytes, s));
+    const KVView view = cache_view(m, kv, max_batch, max_seq);
+    QK_TRY(prefill_impl(m, view, TokIndex{seq, P, L, 0}, B, P, 0, nullptr, oi, logprobs, argmax, workspace,
+                        ws_bytes, s));
     if (N == 0) return QK_OK;
     // cursor slots
     const size_t slot = align256((size_t)B * 4);
@@ -961,8 +1023,8 @@ static int rollout_impl(Model& m, qk_model* mh, void* kv, int max_batch, int max
     };
     auto one_step = [&]() -> int {
         prepare(s);
-        return decode_impl(m, kv, max_batch, max_seq, TokIndex{tok, 1, 1, 0}, PosIndex{pos, 0, 1},
-                           B, nullptr, od, logprobs, argmax, workspace, ws_bytes, s);
+        return decode_impl(m, view, TokIndex{tok, 1, 1, 0}, PosIndex{pos, 0, 1}, B, nullptr, od, logprobs,
+                           argmax, workspace, ws_bytes, s);
     };
     // Step 0 runs directly (it also performs any one-time kernel set-up).
     QK_TRY(one_step());
@@ -996,8 +1058,8 @@ static int rollout_impl(Model& m, qk_model* mh, void* kv, int max_batch, int max
         QK_TRY_CUDA(cudaStreamBeginCapture(cs_stream, cudaStreamCaptureModeThreadLocal));
         const uint64_t before = g_launches.load();
         prepare(cs_stream);
-        int rc = decode_impl(m, kv, max_batch, max_seq, TokIndex{tok, 1, 1, 0}, PosIndex{pos, 0, 1},
-                             B, nullptr, od, logprobs, argmax, workspace, ws_bytes, cs_stream);
+        int rc = decode_impl(m, view, TokIndex{tok, 1, 1, 0}, PosIndex{pos, 0, 1}, B, nullptr, od, logprobs,
+                             argmax, workspace, ws_bytes, cs_stream);
         kernels = (int)(g_launches.load() - before);
         g_launches.fetch_sub((uint64_t)kernels);  // counted again below, once per replay
         cudaGraph_t graph = nullptr;

@@ -284,8 +284,8 @@ int attn_fwd(const Ctx& x, int l) {
     const BwdLayout& L = x.L;
     float* lse = (float*)L.lse_a.at(l);
     if (c.dtype == QK_DTYPE_BF16 && attn_prefill_supported(d, nq, nkv))
-        return launch_attn_prefill((const bf16*)L.qr.at(l), nq * d, L.kvh.at(l), nq, nkv, x.B, T, x.B, T, 0,
-                                   nullptr, (bf16*)L.O.at(l), m.num_sms, m.status, x.s, lse);
+        return launch_attn_prefill((const bf16*)L.qr.at(l), nq * d, L.kvh.at(l), nq, nkv, KvPages::dense(x.B, T),
+                                   x.B, T, 0, nullptr, (bf16*)L.O.at(l), m.num_sms, m.status, x.s, lse);
     const int tn = gemm_tile_n(m, T, 1);
     bwd::Epi e = epi_mode(E_STATS);
     e.stats = L.st_a;

@@ -171,6 +171,37 @@ struct PosIndex {
     int start, T;
 };
 
+// Where a layer's cache keeps the keys and values of row b's positions.  Each of a
+// layer's K and V is a pool of n_pages pages, [n_pages, nkv, page, d]; position p of
+// row b sits at offset p % page of page table[b * per_row + p / page].  A dense cache
+// [max_batch, nkv, max_seq, d] is the same with one page per row: table null, page b,
+// page = max_seq, per_row = 1.  A row holds per_row * page positions (cap()).
+struct KvPages {
+    const int32_t* table;  // device [rows, per_row] page ids, or null (dense)
+    int per_row;
+    int n_pages;
+    int page;
+    __host__ __device__ int cap() const { return per_row * page; }
+    static KvPages dense(int max_batch, int max_seq) { return KvPages{nullptr, 1, max_batch, max_seq}; }
+};
+
+// Row index, in the 2-D view [n_pages nkv page, d] of a layer's K (or V), of position
+// p of (row b, kv head g).  A page id outside [0, n_pages) sets QK_STATUS_BAD_PAGE (when
+// status is given) and reads page 0.
+__device__ __forceinline__ int kv_row(const KvPages& kp, int nkv, int b, int g, int p,
+                                      uint32_t* status) {
+    int pg = b, off = p;
+    if (kp.table) {
+        pg = kp.table[(size_t)b * kp.per_row + p / kp.page];
+        off = p % kp.page;
+        if ((unsigned)pg >= (unsigned)kp.n_pages) {
+            if (status) atomicOr(status, QK_STATUS_BAD_PAGE);
+            pg = 0;
+        }
+    }
+    return (pg * nkv + g) * kp.page + off;
+}
+
 // Where the log-prob / argmax of flattened logits row r goes.  b = r / T, t = r % T;
 // the row is skipped when t >= out_lim; target = tgt[b * tgt_ld + tgt_off + t];
 // outputs at index b * out_ld + out_off + t.
@@ -194,7 +225,7 @@ void launch_rmsnorm(const float* x, int in_step, int in_off, const float* g, int
 void launch_qk_norm_rope(void* qkv, int dtype, int M, int nq, int nkv, int d, const float* gq,
                          const float* gk, float eps, const float* rope_cos, const float* rope_sin,
                          int max_positions, PosIndex pos, void* k_cache, void* v_cache,
-                         int max_seq, uint32_t* status, cudaStream_t s);
+                         const KvPages& kp, uint32_t* status, cudaStream_t s);
 void launch_swiglu(const void* gu, void* h, int dtype, int M, int I, cudaStream_t s);
 // GRPO token loss (Sec. "GRPO Optimization"): inputs and output of Eq. ppo for the
 // tokens whose log-prob a kernel forms; loss_tok == nullptr disables it.
@@ -258,10 +289,10 @@ void launch_rope_table(float* cos_t, float* sin_t, int max_positions, int d, dou
 void launch_widen_gain(const void* src, int dtype, float* dst, int n, cudaStream_t s);
 
 // Attention.  q rows of q_ld elements holding nq heads of d (row r = b * T + t),
-// caches [B_max, nkv, max_seq, d] of one layer; row r attends cache positions
-// 0 .. pos(r) inclusive; o [M, nq * d].
+// one layer's caches laid out as kp says; row r attends cache positions 0 .. pos(r)
+// inclusive; o [M, nq * d].
 void launch_attention_simt(const void* q, int q_ld, const void* k_cache, const void* v_cache,
-                           int dtype, int M, int nq, int nkv, int d, int max_seq, PosIndex pos,
+                           int dtype, int M, int nq, int nkv, int d, const KvPages& kp, PosIndex pos,
                            void* o, uint32_t* status, cudaStream_t s);
 
 // GEMMs: C[M, N] = A[M, K] * W[N, K]^T with an epilogue (see Epi).
@@ -320,7 +351,7 @@ struct Fuse {
     int q_ld;
     bf16* k_cache;
     bf16* v_cache;
-    int max_seq;
+    KvPages kv;
     uint32_t* status;
     // FUSE_RESID
     float* x;
@@ -362,7 +393,7 @@ void linear(Model& m, const void* A, int lda, const void* W, void* C, int ldc, i
 // whose partials use `scratch` (attn_decode_scratch_bytes); other cases run the
 // SIMT kernel.
 void launch_attention(Model& m, const void* q, int q_ld, const void* k_cache, const void* v_cache,
-                      int M, int max_batch, int max_seq, PosIndex pos, void* o, void* scratch,
+                      int M, const KvPages& kp, PosIndex pos, void* o, void* scratch,
                       cudaStream_t s);
 // Causal tensor-core attention for prefill / scoring (k_attn_prefill.cu): M = B x T
 // query rows at positions start_b .. start_b+T-1, start_b = start_dev[b] when given,
@@ -370,7 +401,7 @@ void launch_attention(Model& m, const void* q, int q_ld, const void* k_cache, co
 bool attn_prefill_supported(int d, int nq, int nkv);
 // lse (may be null): [B, nq, T] natural-log log-sum-exp of each row's scaled scores.
 int launch_attn_prefill(const bf16* q, int q_ld, const void* k_layer, int nq, int nkv,
-                        int max_batch, int max_seq, int B, int T, int start,
+                        const KvPages& kp, int B, int T, int start,
                         const int32_t* start_dev, bf16* o, int num_sms, uint32_t* status,
                         cudaStream_t s, float* lse = nullptr);
 // Fused causal attention backward on tcgen05 (k_attn_bwd.cu): head_dim 128, T % 128 == 0.
@@ -390,12 +421,12 @@ int* attn_decode_tickets(void* scratch, int B, int nq, int nkv, int max_seq, int
 void attn_scratch_parts(void* scratch, int B, int nq, int nkv, int max_seq, int num_sms, int n_split,
                         float** part_o, float2** part_ml, int** tickets);
 // 3-D TMA map over `layers` layers' K / V caches (k_layer0 = layer 0's K, layer stride
-// layer_bytes; ignored for one layer).
-bool make_kv_map(CUtensorMap* map, const void* k_layer0, int max_batch, int nkv, int max_seq,
-                 int layers, size_t layer_bytes);
+// layer_bytes; ignored for one layer), each layer's K then V pools laid out as kp says.
+bool make_kv_map(CUtensorMap* map, const void* k_layer0, const KvPages& kp, int nkv, int layers,
+                 size_t layer_bytes);
 bool attn_decode_supported(int d, int nq, int nkv);
 int launch_attn_decode(const bf16* q, int q_ld, const void* k_layer, int nq, int nkv,
-                       int max_batch, int max_seq, int B, PosIndex pos, void* scratch, bf16* o,
+                       const KvPages& kp, int B, PosIndex pos, void* scratch, bf16* o,
                        int num_sms, uint32_t* status, cudaStream_t s);
 
 }  // namespace qk

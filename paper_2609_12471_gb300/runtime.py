@@ -171,6 +171,33 @@ class Decoder:
                                     argmax, ws)
         return logprobs
 
+    # ------------------------------------------------------------ paged cache
+    def new_kv_pages(self, n_pages: int, page_size: int) -> torch.Tensor:
+        """A paged cache of n_pages pages of page_size positions (per layer a K pool then a
+        V pool, each [n_pages, n_kv, page_size, d])."""
+        return torch.empty(B.qk_kv_pages_bytes(self.handle, n_pages, page_size), dtype=torch.uint8,
+                           device=self.device)
+
+    def decode_step_paged(self, kv, table, n_pages, page_size, tokens, pos, logits=None, targets=None,
+                          logprobs=None, argmax=None):
+        """decode_step over a paged cache; table: device int32 [B, per_row] page ids."""
+        Bn, per_row = table.shape
+        assert table.dtype == torch.int32 and table.is_contiguous()
+        ws = self.workspace(B.QK_CALL_DECODE, tokens.shape[0], 1, per_row * page_size)
+        B.qk_decode_step_paged(self.handle, kv, table, per_row, n_pages, page_size, tokens, pos,
+                               tokens.shape[0], logits, targets, logprobs, argmax, ws)
+
+    def prefill_rows_paged(self, kv, table, n_pages, page_size, tokens, start, length=None,
+                           last_logits=None):
+        """prefill_rows over a paged cache; table: device int32 [B, per_row] page ids."""
+        Bn, T = tokens.shape
+        assert table.dtype == torch.int32 and table.is_contiguous()
+        per_row = table.shape[1]
+        ws = self.workspace(B.QK_CALL_PREFILL, Bn, T, per_row * page_size)
+        B.qk_prefill_rows_paged(self.handle, kv, table, per_row, n_pages, page_size, tokens, Bn, T, start,
+                                length, last_logits, ws)
+        return last_logits
+
     def check_status(self) -> int:
         return B.qk_check_status(self.handle)
 

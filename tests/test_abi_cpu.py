@@ -141,3 +141,19 @@ def test_debug_hook_validates_on_the_host():
     with pytest.raises(qk.QKError) as e:
         qk.qk_debug_expire_next_wait(None, 1000)
     assert e.value.code == qk.QK_EINVAL
+
+
+def test_paged_entry_points_validate_on_the_host(lib):
+    """The paged-cache calls reject a missing model or pages before any device work, and
+    the binding's qk_kv_pages has the header's layout (pointer, three int32)."""
+    import paper_2609_12471_gb300 as qk
+    assert ctypes.sizeof(qk.qk_kv_pages) == 24
+    assert [f for f, _ in qk.qk_kv_pages._fields_] == ["table", "per_row", "n_pages", "page_size"]
+    P = 256
+    for call in (lambda: qk.qk_kv_pages_bytes(None, 4, 128),
+                 lambda: qk.qk_decode_step_paged(None, P, P, 2, 4, 128, P, P, 2, ws_bytes=0, stream=0),
+                 lambda: qk.qk_prefill_rows_paged(None, P, P, 2, 4, 128, P, 2, 8, P, ws_bytes=0, stream=0)):
+        with pytest.raises(qk.QKError) as e:
+            call()
+        assert e.value.code == qk.QK_EINVAL
+    assert qk.QK_STATUS_BAD_PAGE == 8
