@@ -31,8 +31,8 @@
  *    has launched nothing.  Data-dependent faults found on the device (a token
  *    id outside [0, vocab), a position outside the cache, a bounded wait that
  *    expired) set bits of the model's device status word instead; the kernels
- *    then substitute a safe value (token 0, position clamped) rather than read
- *    out of bounds.  qk_check_status() reads and clears that word.
+ *    then substitute a safe value (token 0, position clamped, page 0 for a page
+ *    id outside the pool) rather than read out of bounds.  qk_check_status() reads and clears that word.
  *  - dtype.  QK_DTYPE_BF16 models keep weights, activations and KV cache in
  *    bf16 with fp32 accumulation, an fp32 residual stream and fp32 softmax /
  *    log-softmax statistics.  QK_DTYPE_F32 models are fp32 end to end (no TF32).
@@ -239,6 +239,17 @@ int qk_decode_step_paged(qk_model* m, void* kv, const qk_kv_pages* pages, const 
 int qk_prefill_rows_paged(qk_model* m, void* kv, const qk_kv_pages* pages, const int32_t* tokens,
                           int B, int T, const int32_t* start, const int32_t* len, float* last_logits,
                           void* workspace, size_t ws_bytes, void* stream);
+
+/* qk_rollout_teacher_forced and qk_rollout_sampled over a paged cache: the same
+ * arguments, outputs, workspace (max_seq = per_row x page_size) and graph replay
+ * (the replayed graph is cached per cache base, page layout, table pointer and
+ * the call's buffers).  P + N <= per_row x page_size. */
+int qk_rollout_teacher_forced_paged(qk_model* m, void* kv, const qk_kv_pages* pages,
+                                    const int32_t* seq, int B, int P, int N, float* logprobs,
+                                    int32_t* argmax, void* workspace, size_t ws_bytes, void* stream);
+int qk_rollout_sampled_paged(qk_model* m, void* kv, const qk_kv_pages* pages, const int32_t* prompt,
+                             int B, int P, int N, float tau, uint64_t seed, int32_t* tokens,
+                             float* logprobs, void* workspace, size_t ws_bytes, void* stream);
 
 /* Teacher-forced scoring (Eq. sft / Eq. ppo inputs): tokens dev int32 [B, T],
  * T >= 2.  logprobs dev fp32 [B, T-1]: logprobs[b, t] = log p(tokens[b, t+1] |

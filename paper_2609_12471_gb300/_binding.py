@@ -36,7 +36,8 @@ __all__ = [
     "QK_STATIC_SCRATCH_BYTES", "qk_grpo_workspace_bytes", "qk_grpo_token_loss", "qk_score_grpo",
     "qk_rollout_sampled", "qk_prefill_rows", "qk_debug_expire_next_wait", "QK_CALL_BACKWARD",
     "qk_grpo_coef", "qk_backward_logprob", "QK_STATUS_BAD_PAGE", "qk_kv_pages", "qk_kv_pages_bytes",
-    "qk_decode_step_paged", "qk_prefill_rows_paged",
+    "qk_decode_step_paged", "qk_prefill_rows_paged", "qk_rollout_teacher_forced_paged",
+    "qk_rollout_sampled_paged",
 ]
 
 
@@ -101,6 +102,10 @@ _SIGS = {
     "qk_grpo_coef": ([_P, _P, _P, _I, _I, _I, _P, _I, _P, _F, _F, _F, _P, _P, _P, _P, _SZ, _P], _I),
     "qk_backward_logprob": ([_P, _P, _I, _I, _P, ctypes.POINTER(_P), _I, _I, _P, _P, _SZ, _P], _I),
     "qk_kv_pages_bytes": ([_P, _I, _I, ctypes.POINTER(_SZ)], _I),
+    "qk_rollout_teacher_forced_paged": ([_P, _P, ctypes.POINTER(qk_kv_pages), _P, _I, _I, _I, _P, _P, _P,
+                                         _SZ, _P], _I),
+    "qk_rollout_sampled_paged": ([_P, _P, ctypes.POINTER(qk_kv_pages), _P, _I, _I, _I, _F, ctypes.c_uint64,
+                                  _P, _P, _P, _SZ, _P], _I),
     "qk_decode_step_paged": ([_P, _P, ctypes.POINTER(qk_kv_pages), _P, _P, _I, _P, _P, _P, _P, _P, _SZ,
                               _P], _I),
     "qk_prefill_rows_paged": ([_P, _P, ctypes.POINTER(qk_kv_pages), _P, _I, _I, _P, _P, _P, _P, _SZ, _P],
@@ -320,6 +325,22 @@ def qk_prefill_rows_paged(m, kv, table, per_row, n_pages, page_size, tokens, B, 
     _check(_load().qk_prefill_rows_paged(m, _ptr(kv), ctypes.byref(pg), _ptr(tokens), B, T, _ptr(start),
                                          _ptr(length), _ptr(last_logits), _ptr(workspace),
                                          _nbytes(workspace, ws_bytes), _stream(stream)))
+
+
+def qk_rollout_teacher_forced_paged(m, kv, table, per_row, n_pages, page_size, seq, B, P, N, logprobs,
+                                    argmax=None, workspace=None, ws_bytes=None, stream=None):
+    pg = _pages(table, per_row, n_pages, page_size)
+    _check(_load().qk_rollout_teacher_forced_paged(m, _ptr(kv), ctypes.byref(pg), _ptr(seq), B, P, N,
+                                                   _ptr(logprobs), _ptr(argmax), _ptr(workspace),
+                                                   _nbytes(workspace, ws_bytes), _stream(stream)))
+
+
+def qk_rollout_sampled_paged(m, kv, table, per_row, n_pages, page_size, prompt, B, P, N, tau, seed, tokens,
+                             logprobs, workspace=None, ws_bytes=None, stream=None):
+    pg = _pages(table, per_row, n_pages, page_size)
+    _check(_load().qk_rollout_sampled_paged(m, _ptr(kv), ctypes.byref(pg), _ptr(prompt), B, P, N, tau, seed,
+                                            _ptr(tokens), _ptr(logprobs), _ptr(workspace),
+                                            _nbytes(workspace, ws_bytes), _stream(stream)))
 
 
 def qk_check_status(m, stream=None) -> int:

@@ -983,11 +983,11 @@ int qk_score_grpo(qk_model* mh, const int32_t* tokens, int B, int T, const float
 // every input token and target.  Sampling: seq is the prompt [B, P]; the head of
 // each step draws the next token into sampled [B, N+1] (m.sampling), and the next
 // step reads it from there.
-static int rollout_impl(Model& m, qk_model* mh, void* kv, int max_batch, int max_seq,
-                        const int32_t* seq, int B, int P, int N, float* logprobs, int32_t* argmax,
-                        const SampleArgs* sampled, void* workspace, size_t ws_bytes,
-                        cudaStream_t s) {
-    QK_TRY(check_cache(m, kv, max_batch, max_seq, B));
+// The cache (dense or paged) was checked by the caller.
+static int rollout_impl(Model& m, qk_model* mh, const KVView& view, const int32_t* seq, int B, int P,
+                        int N, float* logprobs, int32_t* argmax, const SampleArgs* sampled,
+                        void* workspace, size_t ws_bytes, cudaStream_t s) {
+    const int max_seq = view.kp.cap();
     if (P < 1 || N < 0 || (long)P + N > max_seq)
         return set_error(QK_ESHAPE, "prompt %d + steps %d exceed the cache of %d", P, N, max_seq);
     size_t need;
@@ -1001,7 +1001,6 @@ static int rollout_impl(Model& m, qk_model* mh, void* kv, int max_batch, int max
     } scope(m, sampled);
     const int L = sampled ? P : P + N + 1;  // row length of seq
     OutIndex oi{1, 1, N + 1, 0, sampled ? nullptr : seq, L, P, 0};
-    const KVView view = cache_view(m, kv, max_batch, max_seq);
     QK_TRY(prefill_impl(m, view, TokIndex{seq, P, L, 0}, B, P, 0, nullptr, oi, logprobs, argmax, workspace,
                         ws_bytes, s));
     if (N == 0) return QK_OK;
@@ -1037,11 +1036,12 @@ static int rollout_impl(Model& m, qk_model* mh, void* kv, int max_batch, int max
     }
     uint32_t inv_tau_bits = 0;
     if (sampled) memcpy(&inv_tau_bits, &sampled->inv_tau, 4);
-    const uint64_t key[15] = {(uint64_t)(uintptr_t)kv, (uint64_t)max_batch, (uint64_t)max_seq,
-                              (uint64_t)(uintptr_t)seq, (uint64_t)B, (uint64_t)P, (uint64_t)N,
-                              (uint64_t)(uintptr_t)logprobs, (uint64_t)(uintptr_t)argmax,
-                              (uint64_t)(uintptr_t)workspace, (uint64_t)ws_bytes,
-                              sampled ? 1ull : 0ull,
+    const uint64_t key[17] = {(uint64_t)(uintptr_t)view.base, (uint64_t)view.kp.n_pages,
+                              (uint64_t)view.kp.page, (uint64_t)(uintptr_t)view.kp.table,
+                              (uint64_t)view.kp.per_row, (uint64_t)(uintptr_t)seq, (uint64_t)B,
+                              (uint64_t)P, (uint64_t)N, (uint64_t)(uintptr_t)logprobs,
+                              (uint64_t)(uintptr_t)argmax, (uint64_t)(uintptr_t)workspace,
+                              (uint64_t)ws_bytes, sampled ? 1ull : 0ull,
                               sampled ? (uint64_t)(uintptr_t)sampled->out_tokens : 0ull,
                               sampled ? (uint64_t)sampled->seed : 0ull, (uint64_t)inv_tau_bits};
     cudaGraphExec_t exec = nullptr;
@@ -1093,20 +1093,52 @@ int qk_rollout_teacher_forced(qk_model* mh, void* kv, int max_batch, int max_seq
                               const int32_t* seq, int B, int P, int N, float* logprobs,
                               int32_t* argmax, void* workspace, size_t ws_bytes, void* stream) {
     if (!mh || !seq || !logprobs) return set_error(QK_EINVAL, "null argument");
-    return rollout_impl(*(Model*)mh, mh, kv, max_batch, max_seq, seq, B, P, N, logprobs, argmax,
+    Model& m = *(Model*)mh;
+    QK_TRY(check_cache(m, kv, max_batch, max_seq, B));
+    return rollout_impl(m, mh, cache_view(m, kv, max_batch, max_seq), seq, B, P, N, logprobs, argmax,
                         nullptr, workspace, ws_bytes, (cudaStream_t)stream);
+}
+
+int qk_rollout_teacher_forced_paged(qk_model* mh, void* kv, const qk_kv_pages* pages, const int32_t* seq,
+                                    int B, int P, int N, float* logprobs, int32_t* argmax, void* workspace,
+                                    size_t ws_bytes, void* stream) {
+    if (!mh || !seq || !logprobs) return set_error(QK_EINVAL, "null argument");
+    Model& m = *(Model*)mh;
+    QK_TRY(check_pages(m, kv, pages, B));
+    return rollout_impl(m, mh, paged_view(m, kv, *pages), seq, B, P, N, logprobs, argmax, nullptr,
+                        workspace, ws_bytes, (cudaStream_t)stream);
+}
+
+static int sampled_args(qk_model* mh, const int32_t* prompt, int B, int N, float tau, uint64_t seed,
+                        int32_t* tokens, const float* logprobs, SampleArgs* sa) {
+    if (!mh || !prompt || !tokens || !logprobs) return set_error(QK_EINVAL, "null argument");
+    if (!(tau > 0.f) || !(1.f / tau < 3.0e38f)) return set_error(QK_EINVAL, "temperature must be > 0");
+    if (B >= (1 << 24) || N + 1 >= (1 << 22) || ((Model*)mh)->cfg.vocab > (1 << 18))
+        return set_error(QK_ESHAPE, "sampling counters need B < 2^24, N < 2^22, vocab <= 2^18");
+    *sa = SampleArgs{(unsigned long long)seed, 1.f / tau, tokens};
+    return QK_OK;
 }
 
 int qk_rollout_sampled(qk_model* mh, void* kv, int max_batch, int max_seq, const int32_t* prompt,
                        int B, int P, int N, float tau, uint64_t seed, int32_t* tokens,
                        float* logprobs, void* workspace, size_t ws_bytes, void* stream) {
-    if (!mh || !prompt || !tokens || !logprobs) return set_error(QK_EINVAL, "null argument");
-    if (!(tau > 0.f) || !(1.f / tau < 3.0e38f)) return set_error(QK_EINVAL, "temperature must be > 0");
-    if (B >= (1 << 24) || N + 1 >= (1 << 22) || ((Model*)mh)->cfg.vocab > (1 << 18))
-        return set_error(QK_ESHAPE, "sampling counters need B < 2^24, N < 2^22, vocab <= 2^18");
-    const SampleArgs sa{(unsigned long long)seed, 1.f / tau, tokens};
-    return rollout_impl(*(Model*)mh, mh, kv, max_batch, max_seq, prompt, B, P, N, logprobs, nullptr,
+    SampleArgs sa;
+    QK_TRY(sampled_args(mh, prompt, B, N, tau, seed, tokens, logprobs, &sa));
+    Model& m = *(Model*)mh;
+    QK_TRY(check_cache(m, kv, max_batch, max_seq, B));
+    return rollout_impl(m, mh, cache_view(m, kv, max_batch, max_seq), prompt, B, P, N, logprobs, nullptr,
                         &sa, workspace, ws_bytes, (cudaStream_t)stream);
+}
+
+int qk_rollout_sampled_paged(qk_model* mh, void* kv, const qk_kv_pages* pages, const int32_t* prompt, int B,
+                             int P, int N, float tau, uint64_t seed, int32_t* tokens, float* logprobs,
+                             void* workspace, size_t ws_bytes, void* stream) {
+    SampleArgs sa;
+    QK_TRY(sampled_args(mh, prompt, B, N, tau, seed, tokens, logprobs, &sa));
+    Model& m = *(Model*)mh;
+    QK_TRY(check_pages(m, kv, pages, B));
+    return rollout_impl(m, mh, paged_view(m, kv, *pages), prompt, B, P, N, logprobs, nullptr, &sa,
+                        workspace, ws_bytes, (cudaStream_t)stream);
 }
 
 int qk_check_status(qk_model* mh, void* stream, uint32_t* flags) {

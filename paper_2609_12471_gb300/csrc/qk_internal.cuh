@@ -113,7 +113,7 @@ struct Model {
     // Instantiated decode-step graphs of qk_rollout_teacher_forced, keyed by the call's
     // pointers and sizes (every kernel parameter of a step is fixed by them).
     struct StepGraph {
-        uint64_t key[15];
+        uint64_t key[17];
         cudaGraphExec_t exec;
         int kernels;  // kernel nodes of one step (for the launch counter)
     };

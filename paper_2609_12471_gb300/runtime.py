@@ -198,6 +198,31 @@ class Decoder:
                                 length, last_logits, ws)
         return last_logits
 
+    def rollout_paged(self, kv, table, n_pages, page_size, seq, P, logprobs=None, argmax=None):
+        """rollout over a paged cache; table: device int32 [B, per_row] page ids."""
+        Bn, L = seq.shape
+        N = L - P - 1
+        per_row = table.shape[1]
+        assert table.dtype == torch.int32 and table.is_contiguous()
+        if logprobs is None:
+            logprobs = torch.empty(Bn, N + 1, dtype=torch.float32, device=self.device)
+        ws = self.workspace(B.QK_CALL_ROLLOUT, Bn, P, per_row * page_size)
+        B.qk_rollout_teacher_forced_paged(self.handle, kv, table, per_row, n_pages, page_size, seq, Bn, P, N,
+                                          logprobs, argmax, ws)
+        return logprobs
+
+    def rollout_sampled_paged(self, kv, table, n_pages, page_size, prompt, N, tau=1.0, seed=0):
+        """rollout_sampled over a paged cache; table: device int32 [B, per_row] page ids."""
+        Bn, P = prompt.shape
+        per_row = table.shape[1]
+        assert table.dtype == torch.int32 and table.is_contiguous()
+        tokens = torch.empty(Bn, N + 1, dtype=torch.int32, device=self.device)
+        logprobs = torch.empty(Bn, N + 1, dtype=torch.float32, device=self.device)
+        ws = self.workspace(B.QK_CALL_ROLLOUT, Bn, P, per_row * page_size)
+        B.qk_rollout_sampled_paged(self.handle, kv, table, per_row, n_pages, page_size, prompt, Bn, P, N, tau,
+                                   seed, tokens, logprobs, ws)
+        return tokens, logprobs
+
     def check_status(self) -> int:
         return B.qk_check_status(self.handle)
 

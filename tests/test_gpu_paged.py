@@ -187,3 +187,39 @@ def test_paged_arguments_are_checked_on_the_host():
         qk.qk_kv_pages_bytes(h, 4, 96)
     assert e.value.code == qk.QK_ESHAPE
     assert qk.qk_kv_pages_bytes(h, 4, PAGE) == qk.qk_kv_bytes(h, 4, PAGE)
+
+
+@pytest.mark.parametrize("dtype", ["fp32", "bf16"])
+def test_paged_rollouts_equal_dense(dtype):
+    """Whole rollouts (the prompt prefill, then decode steps replayed from a captured
+    graph) over a paged cache: the teacher-forced log-probs and arg-maxes, and at a
+    fixed seed the sampled tokens and their log-probs, bit-identical to the dense
+    cache's.  P + N crosses into each row's second page."""
+    import torch
+    if dtype == "fp32":
+        s = synth.shape("tiny_fp32")
+    else:
+        s = synth.ModelShape("attn_bf16", 2, 512, 4, 2, 128, 256, 1024, "bf16")
+    dec, _ = decoder(s, synth.LazyWeights(s))
+    B, P, N, per_row = 6, 70, 80, 2
+    max_seq = per_row * PAGE
+    seq = _cu(synth.tokens((B, P + N + 1), s.vocab, stream=440))
+    prompt = seq[:, :P].contiguous()
+    kv = dec.new_kv(B, max_seq)
+    am_d = torch.empty(B, N + 1, dtype=torch.int32, device="cuda")
+    lp_d = dec.rollout(kv, B, max_seq, seq, P, argmax=am_d)
+    tok_d, slp_d = dec.rollout_sampled(kv, B, max_seq, prompt, N, tau=1.0, seed=7)
+    assert dec.check_status() == 0
+    del kv
+    n_pages = B * per_row + 3
+    rng = np.random.default_rng(441)
+    tab = _cu(rng.permutation(n_pages)[:B * per_row].reshape(B, per_row))
+    pool = dec.new_kv_pages(n_pages, PAGE)
+    pool.fill_(0xFF)
+    am_p = torch.empty(B, N + 1, dtype=torch.int32, device="cuda")
+    lp_p = dec.rollout_paged(pool, tab, n_pages, PAGE, seq, P, argmax=am_p)
+    tok_p, slp_p = dec.rollout_sampled_paged(pool, tab, n_pages, PAGE, prompt, N, tau=1.0, seed=7)
+    assert dec.check_status() == 0
+    assert torch.equal(lp_d, lp_p) and torch.equal(am_d, am_p)
+    assert torch.equal(tok_d, tok_p) and torch.equal(slp_d, slp_p)
+    assert bool(torch.isfinite(lp_p).all()) and bool(torch.isfinite(slp_p).all())
